@@ -1,0 +1,159 @@
+"""Model-level pins of the oracle (no GPU): the float64 brute-force model, the
+causal invariant, search invariants and exhaustive beam search on a tiny vocab.
+
+Model: App. A (encoder-decoder Transformer), Sec. 3.3 / Fig. 5 (quantisation
+points), App. D (pre-LN, shared vocabulary, greedy search).
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+
+from oracle import bruteforce as BF
+from oracle import oracle as O
+from paper_2306_04235_gb300 import synth
+
+MINI = {
+    "pre": synth.ModelConfig(2, 2, 64, 2, 128, 300, 64, 1, 1, max_pos=64),
+    "post": synth.ModelConfig(2, 1, 64, 4, 96, 300, 64, 0, 1, max_pos=64),
+    "fact": synth.ModelConfig(3, 2, 64, 2, 128, 300, 32, 1, 0, max_pos=64),
+}
+
+
+def _blob(kind, seed=11, gamma=None, out_bias=None):
+    return synth.build_blob(MINI[kind], seed, gamma_range=gamma, out_bias=out_bias)
+
+
+def _src(cfg, B, lo, hi, seed):
+    return synth.source_batch(cfg.vocab, B, lo, hi, seed)
+
+
+@pytest.mark.parametrize("kind", ["pre", "post", "fact"])
+def test_encoder_matches_float64_bruteforce(kind):
+    cfg = MINI[kind]
+    blob = _blob(kind, gamma=(0.5, 1.5))
+    ids, lens = _src(cfg, 3, 5, 20, 3)
+    model = BF.Model(blob)
+    total = agree = 0
+    for b in range(3):
+        enc, ck, cv = O.encode(blob, ids[b], lens[b], cfg)
+        benc, bck, bcv = model.encode(ids[b], lens[b])
+        for got, ref in [(enc, benc), (ck, bck), (cv, bcv)]:
+            diff = np.abs(got.astype(np.int64) - ref.astype(np.int64))
+            assert diff.max() <= 2
+            total += diff.size
+            agree += int((diff == 0).sum())
+    assert agree / total > 0.99
+
+
+@pytest.mark.parametrize("kind", ["pre", "post", "fact"])
+def test_decoder_logits_match_float64_bruteforce(kind):
+    cfg = MINI[kind]
+    blob = _blob(kind, gamma=(0.5, 1.5))
+    ids, lens = _src(cfg, 1, 12, 12, 4)
+    tgt = np.concatenate([[cfg.bos_id], synth.Stream(5, "t").randint(3, cfg.vocab - 1, 9)]).astype(np.int32)
+    logits, _ = O.decode_trace(blob, ids[0], lens[0], tgt, cfg)
+    ref = BF.Model(blob).decode_forced(ids[0], lens[0], tgt)
+    err = np.abs(logits - ref) / (np.abs(ref).max(axis=1, keepdims=True))
+    # int8 codes may differ by one step near rounding ties; logits stay within 2%
+    assert np.median(err) < 1e-4 and err.max() < 2e-2
+
+
+@pytest.mark.parametrize("kind", ["pre", "post", "fact"])
+def test_incremental_decoder_equals_masked_full_sequence(kind):
+    cfg = MINI[kind]
+    blob = _blob(kind, gamma=(0.5, 1.5))
+    ids, lens = _src(cfg, 1, 7, 7, 6)
+    tgt = np.concatenate([[cfg.bos_id], synth.Stream(6, "t").randint(3, cfg.vocab - 1, 15)]).astype(np.int32)
+    inc, _ = O.decode_trace(blob, ids[0], lens[0], tgt, cfg)
+    full = O.decode_forced(blob, ids[0], lens[0], tgt, cfg)
+    assert np.array_equal(inc, full)
+
+
+def test_greedy_tokens_are_argmax_of_their_own_trace():
+    cfg = MINI["pre"]
+    blob = _blob("pre")
+    ids, lens = _src(cfg, 2, 4, 30, 8)
+    out, olen, _ = O.translate(blob, ids, lens, 1, 20)
+    for b in range(2):
+        n = int(olen[b])
+        tgt = np.concatenate([[cfg.bos_id], out[b, :n - 1]]).astype(np.int32)
+        logits, _ = O.decode_trace(blob, ids[b, :lens[b]], lens[b], tgt, cfg)
+        assert np.array_equal(np.argmax(logits, axis=1), out[b, :n])   # first max = lowest id
+        assert np.all(out[b, n:] == cfg.pad_id)
+
+
+def test_padding_does_not_change_a_sentence():
+    cfg = MINI["fact"]
+    blob = _blob("fact")
+    ids, lens = _src(cfg, 4, 3, 25, 9)
+    out, olen, _ = O.translate(blob, ids, lens, 1, 12, n_threads=2)
+    for b in range(4):
+        alone, al, _ = O.translate(blob, ids[b:b + 1, :lens[b]], lens[b:b + 1], 1, 12)
+        assert np.array_equal(alone[0], out[b]) and al[0] == olen[b]
+
+
+@pytest.mark.parametrize("beam", [1, 3])
+def test_forced_eos_terminates_immediately(beam):
+    cfg = MINI["pre"]
+    blob = _blob("pre", out_bias={cfg.eos_id: 1000.0})
+    ids, lens = _src(cfg, 2, 5, 9, 10)
+    out, olen, _ = O.translate(blob, ids, lens, beam, 10)
+    assert np.all(olen == 1) and np.all(out[:, 0] == cfg.eos_id) and np.all(out[:, 1:] == cfg.pad_id)
+
+
+def test_beam_of_one_equals_greedy_up_to_logprob_ties():
+    cfg = MINI["post"]
+    blob = _blob("post")
+    ids, lens = _src(cfg, 6, 4, 20, 12)
+    g, gl, _ = O.translate(blob, ids, lens, 1, 16)
+    bb, bl, _ = O.translate(blob, ids, lens, -1, 16)     # beam search of width 1
+    for b in range(6):
+        if np.array_equal(bb[b], g[b]):
+            continue
+        # a mismatch is only allowed where rounding of the log-probabilities ties two logits
+        first = next(t for t in range(16) if bb[b, t] != g[b, t])
+        tgt = np.concatenate([[cfg.bos_id], g[b, :first]]).astype(np.int32)
+        logits, _ = O.decode_trace(blob, ids[b, :lens[b]], lens[b], tgt, cfg)
+        lp = O.log_softmax(logits[first])
+        assert lp[bb[b, first]] == lp[g[b, first]]
+
+
+def test_beam_search_is_exhaustive_on_a_four_token_vocabulary():
+    """With k = 64 >= 4^3 no hypothesis is ever dropped, so the best beam must be
+    the best of all continuations, scored step by step with the oracle's own
+    log-softmax and fp32 accumulation."""
+    cfg = synth.ModelConfig(1, 1, 16, 1, 32, 4, 16, 1, 1, max_pos=8)
+    T = 3
+    for seed in range(4):
+        blob = synth.build_blob(cfg, 50 + seed)
+        src = np.array([[3, 3, 0, 3, 3]], np.int32)
+        lens = np.array([5], np.int32)
+        ids, olen, score = O.translate(blob, src, lens, 64, T)
+        scored = {}
+        for seq in itertools.product(range(4), repeat=T):
+            cut = next((i + 1 for i, y in enumerate(seq) if y == cfg.eos_id), T)
+            seq = seq[:cut]
+            if seq in scored:
+                continue
+            tgt = np.array([cfg.bos_id] + list(seq[:-1]), np.int32)
+            logits = O.decode_forced(blob, src[0], 5, tgt, cfg)
+            cum = np.float32(0.0)
+            for t, y in enumerate(seq):
+                cum = np.float32(cum + O.log_softmax(logits[t])[y])
+            scored[seq] = cum
+        ranked = sorted(scored.items(), key=lambda kv: -kv[1])
+        (seq, cum), runner = ranked[0], ranked[1]
+        assert cum > runner[1]
+        assert score[0] == cum
+        assert list(ids[0, :len(seq)]) == list(seq) and olen[0] == len(seq)
+
+
+def test_malformed_blobs_are_rejected():
+    blob = _blob("pre")
+    assert O.check_blob(blob)[0] == O.OK
+    assert O.check_blob(blob[:-16])[0] == O.EFORMAT
+    assert O.check_blob(blob + b"\0" * 16)[0] == O.EFORMAT
+    assert O.check_blob(b"XNMT" + blob[4:])[0] == O.EFORMAT
+    assert O.check_blob(blob[:40])[0] == O.EFORMAT

@@ -1,0 +1,234 @@
+"""Pins of the oracle's building blocks against closed forms, library routines
+and float64 brute force (no GPU).
+
+Quantiser: App. B (Eq. 3/4) with zero point 0, symmetric clamp, ties to even.
+Linear: Sec. 3.3 / Fig. 5 (int8 x int8 -> int32, full-precision bias).
+LayerNorm: App. A / App. D.  Attention: Eq. 1/2.
+"""
+import math
+import struct
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2306_04235_gb300 import synth
+
+
+def f32(x):
+    return struct.unpack("<f", struct.pack("<f", x))[0]
+
+
+def ulp32(x):
+    x = abs(f32(x))
+    if x == 0.0:
+        return 2.0 ** -149
+    e = math.frexp(x)[1]
+    return 2.0 ** (e - 24)
+
+
+# ----------------------------------------------------------------- quantiser
+@pytest.mark.parametrize("x,code", [
+    (0.5, 0), (1.5, 2), (2.5, 2), (-0.5, 0), (-1.5, -2), (-2.5, -2),
+    (126.5, 126), (127.5, 127), (127.49, 127), (128.0, 127), (1e9, 127),
+    (-126.5, -126), (-127.5, -127), (-128.0, -127), (-1e9, -127), (0.49999997, 0),
+])
+def test_q8_table(x, code):
+    assert O.q8(x, 1.0) == code
+
+
+def test_q8_never_minus_128_and_scale_roundtrip():
+    for s in [f32(0.01), f32(4.0 / 127), f32(0.3), f32(1e-3)]:
+        inv = f32(1.0 / s)
+        for q in range(-127, 128):
+            assert O.q8(f32(q * s), inv) == q
+    assert O.q8(-3e38, 1.0) == -127
+
+
+# -------------------------------------------------------------- integer GEMM
+def test_gemm_matches_int64_matmul():
+    rng = np.random.default_rng(0)
+    for M, N, K in [(1, 7, 16), (5, 33, 256), (3, 4, 2048)]:
+        A = rng.integers(-127, 128, (M, K), dtype=np.int64).astype(np.int8)
+        W = rng.integers(-127, 128, (N, K), dtype=np.int64).astype(np.int8)
+        ref = A.astype(np.int64) @ W.astype(np.int64).T
+        assert np.array_equal(O.gemm_i32(A, W).astype(np.int64), ref)
+
+
+def test_gemm_extremes_and_row_sums():
+    K = 2048
+    A = np.full((2, K), 127, np.int8); A[1] = -127
+    W = np.full((3, K), -127, np.int8); W[1] = 127; W[2, ::2] = 1
+    C = O.gemm_i32(A, W)
+    assert C[0, 0] == -127 * 127 * K and C[1, 0] == 127 * 127 * K   # |acc| < 2^31
+    ones = np.ones((1, 300), np.int8)
+    W = synth.uniform_int8(3, "w", (9, 300))
+    assert np.array_equal(O.gemm_i32(ones, W)[0], W.astype(np.int64).sum(axis=1))
+
+
+# ------------------------------------------------------------------ epilogues
+def _linear_case(seed, M=4, N=40, K=96):
+    A = synth.uniform_int8(seed, "a", (M, K))
+    W = synth.uniform_int8(seed, "w", (N, K))
+    s_w = synth.uniform_f32(seed, "sw", (N,), 1e-4, 3e-4)
+    b = synth.uniform_f32(seed, "b", (N,), -0.05, 0.05)
+    return A, W, s_w, b
+
+
+def test_linear_f32_vs_float64():
+    A, W, s_w, b = _linear_case(1)
+    s_x = f32(0.031)
+    y = O.linear(A, W, s_w, b, s_x, O.MODE_F32)
+    acc = A.astype(np.float64) @ W.astype(np.float64).T
+    y64 = acc * (np.float64(s_x) * s_w.astype(np.float64)) + b
+    tol = 4 * 2.0 ** -24 * (np.abs(acc * s_x * s_w) + np.abs(b)) + 1e-30
+    assert np.all(np.abs(y - y64) <= tol)
+
+
+def test_linear_q8_relu_and_residual_vs_float64():
+    A, W, s_w, b = _linear_case(2)
+    s_x, s_o = f32(0.031), f32(0.05)
+    inv = f32(1.0 / s_o)
+    acc = A.astype(np.float64) @ W.astype(np.float64).T
+    y64 = acc * (np.float64(s_x) * s_w.astype(np.float64)) + b
+    for mode, pre in [(O.MODE_Q8, y64), (O.MODE_RELU_Q8, np.maximum(y64, 0.0))]:
+        q = O.linear(A, W, s_w, b, s_x, mode, inv_out=inv).astype(np.int64)
+        ref = np.clip(np.rint(pre / s_o), -127, 127)
+        frac = np.abs(pre / s_o - np.trunc(pre / s_o))
+        near_half = np.abs(frac - 0.5) < 1e-4
+        assert np.all(np.abs(q - ref) <= near_half), "codes differ away from a rounding tie"
+        if mode == O.MODE_RELU_Q8:
+            assert np.all(q[y64 < -1e-3] == 0)
+    r0 = synth.uniform_f32(5, "r", y64.shape, -3, 3)
+    g = f32(0.75)
+    r1 = O.linear(A, W, s_w, b, s_x, O.MODE_RESID, gamma=g, resid=r0)
+    ref = g * r0.astype(np.float64) + y64
+    assert np.allclose(r1, ref, rtol=1e-6, atol=1e-6)
+
+
+# ------------------------------------------------------------------ LayerNorm
+def _ln64(x, g, b):
+    x = x.astype(np.float64)
+    mu = x.mean(axis=-1, keepdims=True)
+    var = ((x - mu) ** 2).mean(axis=-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + 1e-5) * g + b
+
+
+def test_layernorm_constant_row_gives_beta():
+    d = 256
+    g = synth.uniform_f32(1, "g", (d,), 0.5, 1.5)
+    b = synth.uniform_f32(1, "b", (d,), -1, 1)
+    r = np.full((3, d), 7.25, np.float32); r[1] = -700.5; r[2] = 0.0
+    out, _ = O.layernorm(r, g, b)
+    assert np.array_equal(out, np.broadcast_to(b, out.shape))
+
+
+@pytest.mark.parametrize("d,scale", [(128, 1.0), (256, 30.0), (512, 700.0), (384, 1e-3), (2048, 1e6)])
+def test_layernorm_vs_float64(d, scale):
+    r = (synth.Stream(d, "r").normal(5 * d).reshape(5, d) * scale + scale * 0.3).astype(np.float32)
+    g = synth.uniform_f32(d, "g", (d,), 0.5, 1.5)
+    b = synth.uniform_f32(d, "b", (d,), -0.2, 0.2)
+    out, codes = O.layernorm(r, g, b, inv=f32(127 / 4.0))
+    ref = _ln64(r, g, b)
+    # a few fp32 roundings of O(1) values; var/(d-1) or another epsilon is far outside this
+    assert np.all(np.abs(out - ref) <= 1e-6 + 1e-6 * np.abs(ref))
+    assert np.array_equal(codes, np.array([[O.q8(v, f32(127 / 4.0)) for v in row] for row in out]))
+
+
+def test_layernorm_permutation_invariant_and_overflow():
+    d = 256
+    r = (synth.Stream(9, "r").normal(d) * 5).astype(np.float32)[None]
+    g = np.ones(d, np.float32); b = np.zeros(d, np.float32)
+    perm = np.argsort(synth.Stream(9, "p").uniform(d))
+    out, _ = O.layernorm(r, g, b)
+    out_p, _ = O.layernorm(r[:, perm], g, b)
+    assert np.array_equal(out[:, perm], out_p)          # same mean and rstd bit for bit
+    bad = r.copy(); bad[0, 3] = 2.0 ** 32
+    with pytest.raises(O.OracleError):
+        O.layernorm(bad, g, b)
+
+
+# ------------------------------------------------------------------ exp / log
+def test_exp_own_within_2ulp_on_a_grid():
+    xs = np.concatenate([-np.linspace(0, 87.0, 40001, dtype=np.float32),
+                         -np.logspace(-8, 0, 2001, dtype=np.float32),
+                         np.float32([-0.34657359, -0.34657358, -0.6931472, -17.328680])])
+    for x in xs:
+        x = float(x)
+        e = O.exp_own(x)
+        assert abs(e - math.exp(x)) <= 2 * ulp32(math.exp(x)), x
+    assert O.exp_own(0.0) == 1.0
+    assert O.exp_own(-87.5) == 0.0 and O.exp_own(-1e30) == 0.0
+
+
+def test_log_own_relative_error():
+    rng = np.random.default_rng(7)
+    zs = list(range(1, 2000)) + [2.0 ** k for k in range(0, 45)] + \
+         list(np.exp(rng.uniform(0, 30, 3000)))
+    for z in zs:
+        z = float(z)
+        ref = math.log(z)
+        got = O.log_own(z)
+        if z == 1.0:
+            assert got == 0.0
+        else:
+            assert abs(got - ref) <= 1e-15 * abs(ref) + 1e-300, z
+
+
+# ------------------------------------------------------------------ attention
+def _att_inputs(seed, n, dh=64, lo=-127, hi=127):
+    q = synth.uniform_int8(seed, "q", (dh,), lo, hi)
+    K = synth.uniform_int8(seed, "k", (n, dh), lo, hi)
+    V = synth.uniform_int8(seed, "v", (n, dh), lo, hi)
+    return q, K, V
+
+
+def _attend(q, K, V, sigma, rho):
+    n, dh = K.shape
+    Kc = K[None, None]; Vc = V[None, None]
+    return O.attention_decode(q[None, None], Kc, Vc, np.array([n], np.int32), sigma, rho)[0, 0]
+
+
+def test_attention_single_key_returns_value():
+    q, K, V = _att_inputs(1, 1)
+    out = _attend(q, K, V, f32(0.01), 1.0)
+    assert np.array_equal(out, V[0])
+    rho = f32(0.6)
+    out = _attend(q, K, V, f32(0.01), rho)
+    assert np.array_equal(out, np.array([O.q8(float(v), rho) for v in V[0]], np.int8))
+
+
+def test_attention_equal_scores_average_values():
+    n, dh = 12, 64
+    q, K, V = _att_inputs(2, n)
+    K = np.broadcast_to(K[0], (n, dh)).copy()             # every key identical
+    out = _attend(q, K, V, f32(0.02), 1.0)
+    mean = V.astype(np.float64).mean(axis=0)
+    assert np.array_equal(out, np.clip(np.rint(mean), -127, 127).astype(np.int8))
+
+
+def test_attention_dominant_key_is_one_hot():
+    n, dh = 40, 64
+    q, K, V = _att_inputs(3, n, lo=-20, hi=20)
+    K[17] = np.sign(q) * 127                                # far larger score than the rest
+    out = _attend(q, K, V, f32(0.1), 1.0)
+    assert np.array_equal(out, V[17])
+
+
+@pytest.mark.parametrize("n,sigma", [(5, 0.001), (64, 0.0005), (300, 0.0002), (512, 0.0001)])
+def test_attention_vs_float64_softmax(n, sigma):
+    q, K, V = _att_inputs(n, n)
+    sigma = f32(sigma); rho = f32(0.9)
+    s = (K.astype(np.float64) @ q.astype(np.float64)) * sigma
+    p = np.exp(s - s.max()); p /= p.sum()
+    P = O.attention_probs(q, K, sigma)
+    assert np.max(np.abs(P - p)) < 2e-6                     # 2^-24 fixed-point weights
+    ctx64 = (p @ V.astype(np.float64)) * rho
+    out = _attend(q, K, V, sigma, rho).astype(np.float64)
+    assert np.all(np.abs(out - np.clip(np.rint(ctx64), -127, 127)) <= 1)
+    assert np.mean(out == np.clip(np.rint(ctx64), -127, 127)) > 0.95
+
+
+def test_sigma_definition():
+    assert O.sigma(f32(0.03), f32(0.05), 64) == f32(0.03 * 0.05 / 8.0) or \
+        abs(O.sigma(f32(0.03), f32(0.05), 64) - f32(0.03) * f32(0.05) / 8.0) <= ulp32(0.03 * 0.05 / 8)
