@@ -1,0 +1,226 @@
+/*
+ * mnmt.h -- C ABI of the GB300 (sm_103a) full-INT8 encoder-decoder translation
+ * path of MobileNMT (arXiv 2306.04235).
+ *
+ * The paper states the problem as: translate a batch of source token ids with
+ * an INT8 Transformer encoder-decoder whose weights, activations and embedding
+ * are 8-bit (Sec. 3.3, Table 5 "8-8-8"), decoding step by step with greedy
+ * search (App. D) or beam search (Table 6).  The calls below follow that
+ * statement: load quantised weights and scales, encode a source batch, run
+ * decode steps, or translate end to end.
+ *
+ * Conventions shared by every call
+ *   - Return value: MNMT_OK (0) or a negative MNMT_E* code; nothing throws or
+ *     traps across the ABI.  mnmt_last_error() returns a thread-local message
+ *     describing the last failure on the calling thread.
+ *   - A session whose device work failed (a CUDA error or a device-side status
+ *     such as MNMT_EOVERFLOW) is poisoned: every later call on it returns the
+ *     same code.  Free it and create a new one.
+ *   - Ownership: blob and input arrays are borrowed for the duration of the call
+ *     (the blob is copied to the device); output arrays are owned by the caller.
+ *   - Streams: a model is bound to one CUDA stream (cudaStream_t passed as
+ *     void*, NULL = legacy default stream); all its sessions' work is issued on
+ *     it.  Models and sessions are not thread-safe.
+ *   - Token ids are in [0, vocab); PAD = 0, BOS = 1 (decoder start), EOS = 2
+ *     (the ids the blob header carries).
+ *
+ * MNMT v1 weight blob (little endian).  64-byte header: char magic[4] = "MNMT",
+ * uint32 version = 1, int32 config[13] in mnmt_config field order, zero padding.
+ * Then the arrays below in this order, each starting at a 16-byte aligned
+ * offset (zero padding between arrays), the blob ending right after the last
+ * array's padding.  A "linear" is {int8 W[N][K] (row n = output channel,
+ * K contiguous), f32 s_w[N] (per-output-channel weight scale), f32 b[N]}.
+ * d = d_model, F = d_ffn, V = vocab, E = d_embed.
+ *     int8 emb_q[V][E], f32 emb_s[V]            shared src/tgt embedding codes and row scales
+ *     if E != d: linear proj (N = d, K = E)     factorised embedding E -> d
+ *     f32 globals[4] = {emb_scale, s_enc, s_dout, 0}
+ *     f32 pe[max_pos][d]                        positional table
+ *     n_enc x { self-attention block, FFN block }
+ *     if pre_ln: f32 enc_ln_g[d], enc_ln_b[d]   final encoder LayerNorm
+ *     n_dec x { self-attention block, cross-attention block, FFN block }
+ *     if pre_ln: f32 dec_ln_g[d], dec_ln_b[d]   final decoder LayerNorm
+ *     if !tied_output: int8 out_w[V][d], f32 out_s[V]
+ *     f32 out_b[V]
+ *   self-attention block:  f32 ln_g[d], ln_b[d];
+ *                          f32 s[8] = {s_in, s_q, s_k, s_v, s_ctx, gamma, 0, 0};
+ *                          linear qkv (N = 3d, rows q | k | v, K = d); linear o (N = d, K = d)
+ *   cross-attention block: f32 ln_g[d], ln_b[d]; f32 s[8] (as above; s_k, s_v
+ *                          quantise the cross keys/values); linear q (d x d);
+ *                          linear kv (N = 2d, rows k | v, K = d; input is the
+ *                          quantised encoder output at scale s_enc); linear o (d x d)
+ *   FFN block:             f32 ln_g[d], ln_b[d]; f32 s[4] = {s_in, s_h, gamma, 0};
+ *                          linear w1 (N = F, K = d); linear w2 (N = d, K = F)
+ *   With tied_output the output projection is emb_q / emb_s (requires E = d).
+ *   Scales s_* are the per-tensor activation scales of the quantisation points
+ *   of Fig. 5; pre_ln = 0 selects post-LN sublayers (LayerNorm after the
+ *   residual add, no final LayerNorm).  Constraints checked at load: d, F, E
+ *   multiples of 16 (64 where a dimension is a GEMM K), d_model / n_heads in
+ *   {32, 64, 128}, d <= 2048, vocab >= 4.
+ */
+#ifndef MNMT_H
+#define MNMT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    MNMT_OK = 0,
+    MNMT_EINVAL = -1,    /* bad argument (size, id, pointer, flag) */
+    MNMT_ENOMEM = -2,    /* device or host allocation failed */
+    MNMT_ECUDA = -3,     /* a CUDA runtime call failed */
+    MNMT_ETIMEOUT = -4,  /* a bounded device wait gave up */
+    MNMT_EFORMAT = -5,   /* malformed weight blob */
+    MNMT_EOVERFLOW = -6  /* a LayerNorm input left the fixed-point domain (|x| >= 2^32) */
+};
+
+/* flags of mnmt_encode / mnmt_translate */
+#define MNMT_DEVICE_PTRS 1 /* id/length inputs and translate outputs are device pointers */
+
+typedef struct {
+    int32_t n_enc, n_dec, d_model, n_heads, d_ffn, vocab, d_embed, pre_ln, tied_output, max_pos,
+        pad_id, bos_id, eos_id;
+} mnmt_config;
+
+typedef struct mnmt_model mnmt_model;     /* owns the device copy of the weights */
+typedef struct mnmt_session mnmt_session; /* owns caches, workspace and search state */
+
+/* Host-only validation of a blob (no CUDA call).  Fills *cfg_out on success.
+ * Returns MNMT_EFORMAT for a malformed blob. */
+int mnmt_blob_check(const void *blob, size_t bytes, mnmt_config *cfg_out);
+
+/* Quantised weights and scales (Sec. 3.3, Fig. 5): validates the blob, copies
+ * it to the device and derives the per-column requantisation constants.
+ * cuda_stream: cudaStream_t the model and its sessions run on.
+ * *out receives the model on success. */
+int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stream, mnmt_model **out);
+void mnmt_model_free(mnmt_model *model);
+int mnmt_model_config(const mnmt_model *model, mnmt_config *cfg_out);
+
+/* A session sized for up to max_batch sentences of up to max_src_len tokens,
+ * beam width `beam` (1 = greedy, 2..16 = beam search) and up to max_len decode
+ * steps (max_len <= max_pos).  Allocates all device memory the session uses;
+ * no later call allocates. */
+int mnmt_session_create(mnmt_model *model, int32_t max_batch, int32_t max_src_len, int32_t beam,
+                        int32_t max_len, mnmt_session **out);
+void mnmt_session_free(mnmt_session *s);
+
+/* Encoder (App. A): src_ids [B][S_pad] right-padded with PAD, src_lens [B]
+ * (1 <= len <= S_pad).  Runs the encoder stack and the cross-attention key /
+ * value projections of every decoder layer, then resets the search state
+ * (every hypothesis starts from BOS at step 0).  Asynchronous on the model's
+ * stream. */
+int mnmt_encode(mnmt_session *s, const int32_t *src_ids, const int32_t *src_lens, int32_t B,
+                int32_t S_pad, int32_t flags);
+
+/* One incremental decoder step for every hypothesis (greedy or beam), then
+ * synchronises.  Host outputs, each NULL to skip: tokens [B*beam] (token
+ * chosen at this step per hypothesis), parents [B*beam] (beam index within the
+ * sentence it extends), scores [B*beam] (cumulative log-probability; 0 for
+ * greedy); *all_done = 1 once every sentence has finished.  Returns
+ * MNMT_EINVAL after max_len steps. */
+int mnmt_decode_step(mnmt_session *s, int32_t *tokens, int32_t *parents, float *scores,
+                     int32_t *all_done);
+
+/* encode + decode until every sentence has emitted EOS or max_len steps ran.
+ * out_ids [B][max_len]: tokens of the best hypothesis, EOS included, PAD after;
+ * out_lens [B]: number of tokens up to and including EOS (max_len if none);
+ * out_scores [B]: cumulative log-probability of the best beam (0 for greedy).
+ * With MNMT_DEVICE_PTRS all five arrays are device pointers and the call is
+ * asynchronous apart from the periodic completion check; otherwise they are
+ * host pointers and the call returns after the results are copied back. */
+int mnmt_translate(mnmt_session *s, const int32_t *src_ids, const int32_t *src_lens, int32_t B,
+                   int32_t S_pad, int32_t max_len, int32_t flags, int32_t *out_ids,
+                   int32_t *out_lens, float *out_scores);
+
+/* Copies an intermediate tensor of the last encode / decode step to host
+ * memory for parity checks.  Returns MNMT_EINVAL if `bytes` differs from the
+ * tap's size (query the size with host_dst = NULL: the size is returned as
+ * a positive value).
+ *   MNMT_TAP_ENC_OUT    int8  [B][S_pad][d]       quantised encoder output
+ *   MNMT_TAP_CROSS_K/V  int8  [B][H][S_pad][dh]   cross keys/values of decoder layer `layer`
+ *   MNMT_TAP_SELF_K/V   int8  [B*beam][H][max_len][dh] self-attention cache of layer `layer`
+ *                             (rows are physical cache rows; beam search reads them
+ *                              through MNMT_TAP_ANCESTRY)
+ *   MNMT_TAP_DEC_OUT    int8  [B*beam][d]         quantised decoder output of the last step
+ *   MNMT_TAP_LOGITS     f32   [B*beam][vocab]     logits of the last step (beam search only)
+ *   MNMT_TAP_RESID      f32   [rows][d]           residual stream (encoder rows after encode,
+ *                                                  decoder rows after a step)
+ *   MNMT_TAP_HISTORY    int32 [max_len][B*beam]   token chosen per step and hypothesis
+ *   MNMT_TAP_PARENTS    int32 [max_len][B*beam]   parent beam per step and hypothesis
+ *   MNMT_TAP_ANCESTRY   int32 [B*beam][max_len]   physical cache row holding each position */
+enum {
+    MNMT_TAP_ENC_OUT = 1,
+    MNMT_TAP_CROSS_K = 2,
+    MNMT_TAP_CROSS_V = 3,
+    MNMT_TAP_SELF_K = 4,
+    MNMT_TAP_SELF_V = 5,
+    MNMT_TAP_DEC_OUT = 6,
+    MNMT_TAP_LOGITS = 7,
+    MNMT_TAP_RESID = 8,
+    MNMT_TAP_HISTORY = 9,
+    MNMT_TAP_PARENTS = 10,
+    MNMT_TAP_ANCESTRY = 11
+};
+int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, void *host_dst, size_t bytes);
+
+/* Thread-local description of the last error on this thread ("" if none). */
+const char *mnmt_last_error(void);
+
+/* ---------------------------------------------------------------------------
+ * Kernel-level entry points (microbenchmarks and per-kernel parity).  All
+ * pointers are device pointers; work is queued on `cuda_stream` and the call
+ * returns without synchronising.  They allocate nothing.
+ * ------------------------------------------------------------------------- */
+
+/* Quantised linear with a fused epilogue (Sec. 3.3, Fig. 5; Eq. 3):
+ *   acc[m][n] = sum_k A[m][k] W[n][k]  (int8 x int8 -> exact int32)
+ *   y = fl(fl(acc * fl(s_x * s_w[n])) + bias[n])
+ *   mode MNMT_EPI_Q8:      out_q[m][n] = q8(y, inv_out[n])
+ *        MNMT_EPI_RELU_Q8: out_q[m][n] = q8(max(y, 0), inv_out[n])
+ *        MNMT_EPI_RESID:   out_f[m][n] = fl(fl(gamma * out_f[m][n]) + y)
+ *        MNMT_EPI_F32:     out_f[m][n] = y
+ * q8(x, inv) = clamp(round_half_even(fl(x * inv)), -127, 127).
+ * A [M][K], W [N][K] row-major int8 with K a multiple of 64 (16 when M <= 16),
+ * both 16-byte aligned; s_w, bias, inv_out [N] fp32; out_q int8 / out_f fp32
+ * [M][N]. */
+enum { MNMT_EPI_Q8 = 0, MNMT_EPI_RELU_Q8 = 1, MNMT_EPI_RESID = 2, MNMT_EPI_F32 = 3 };
+int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
+                const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
+                int8_t *out_q, float *out_f, void *cuda_stream);
+
+/* Output-vocabulary projection fused with greedy selection (App. D): for each
+ * row m, keys[m] = max over n of pack(y[m][n], n) with y as in mnmt_linear and
+ * pack(y, n) = (ord(y) << 32) | (0xFFFFFFFF - n), where ord maps fp32 to uint32
+ * monotonically (-0 as +0).  The winning id is 0xFFFFFFFF - (keys[m] & 0xFFFFFFFF):
+ * the largest logit, ties to the lowest id.  keys [M] (uint64) must hold 0
+ * before the call (the kernel combines with atomicMax).  A [M][K], W [N][K] as
+ * in mnmt_linear. */
+int mnmt_linear_argmax(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
+                       int32_t M, int32_t N, int32_t K, uint64_t *keys, void *cuda_stream);
+
+/* Incremental attention (Eq. 1/2 per head) of R query rows over per-row
+ * caches: q [R][H][dh], Kc/Vc [R][H][T][dh] int8; row r attends keys
+ * j < n_keys[r] (1 <= n_keys[r] <= T <= 1024).  Scores acc_j = q.k_j (int32),
+ * s_j = fl(acc_j * sigma); weights E_j = rne(exp(fl(s_j - max)) 2^24);
+ * ctx[r][h][e] = q8(fl32((sum_j E_j v_j[e]) / (sum_j E_j)), rho), with the
+ * sums exact integers.  dh in {32, 64, 128}. */
+int mnmt_attention_decode(const int8_t *q, const int8_t *Kc, const int8_t *Vc, const int32_t *n_keys,
+                          int32_t R, int32_t H, int32_t dh, int32_t T, float sigma, float rho,
+                          int8_t *ctx, void *cuda_stream);
+
+/* LayerNorm of M rows of length d (App. A / App. D) with optional fp32 output
+ * out_f [M][d] and int8 output out_q = q8(LN(r), inv) (either may be NULL).
+ * Mean and biased variance are exact fixed-point sums on a grid set by each
+ * row's largest magnitude; eps = 1e-5.  *status (device int, may be NULL)
+ * receives MNMT_EOVERFLOW if a row holds |x| >= 2^32. */
+int mnmt_layernorm(const float *r, const float *g, const float *b, int32_t M, int32_t d, float inv,
+                   float *out_f, int8_t *out_q, int32_t *status, void *cuda_stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MNMT_H */

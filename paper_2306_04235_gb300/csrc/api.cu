@@ -1,0 +1,1211 @@
+// api.cu -- host runtime and C ABI of libmnmt (include/mnmt.h).
+//
+// Model: the MNMT v1 blob is validated on the host, copied to the device once
+// (every array keeps its 16-byte aligned blob offset, so int8 weight rows stay
+// K-contiguous in HBM) and the per-column requantisation constants
+// inv_out[n] = fl(1 / s_out) and the attention constants sigma, rho are derived
+// on the host.
+//
+// Session: one device arena holds the residual stream, int8 activations, the
+// int8 self- and cross-attention caches and the search state; nothing is
+// allocated after mnmt_session_create.  The decoder step (embedding, every
+// decoder layer, the vocabulary projection and the search update) is captured
+// once per (batch, padded source length) as a CUDA graph and replayed; every
+// kernel of a step reads the step counter from device memory and returns at
+// once when the search is done, so extra replays are cheap.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+
+using namespace mnmt;
+
+// ---------------------------------------------------------------------------
+// errors
+// ---------------------------------------------------------------------------
+static thread_local std::string g_err;
+
+static int fail(int code, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+#define CK(call)                                                                                  \
+    do {                                                                                          \
+        cudaError_t e_ = (call);                                                                  \
+        if (e_ != cudaSuccess)                                                                    \
+            return fail(MNMT_ECUDA, "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, \
+                        __LINE__);                                                                \
+    } while (0)
+
+static std::once_flag g_init_once;
+static cudaError_t g_init_err = cudaSuccess;
+
+static int lib_init() {
+    std::call_once(g_init_once, [] {
+        g_init_err = linear_init();
+        if (g_init_err == cudaSuccess) g_init_err = attention_init();
+        if (g_init_err == cudaSuccess) g_init_err = rows_init();
+    });
+    if (g_init_err != cudaSuccess)
+        return fail(MNMT_ECUDA, "kernel set-up failed: %s", cudaGetErrorString(g_init_err));
+    return MNMT_OK;
+}
+
+// ---------------------------------------------------------------------------
+// blob layout (host walk over the documented MNMT v1 order)
+// ---------------------------------------------------------------------------
+namespace {
+
+struct LinOff {
+    size_t w, s, b;
+    int n, k;
+};
+struct SelfOff {
+    size_t ln_g, ln_b, sc;
+    LinOff qkv, o;
+};
+struct CrossOff {
+    size_t ln_g, ln_b, sc;
+    LinOff q, kv, o;
+};
+struct FfnOff {
+    size_t ln_g, ln_b, sc;
+    LinOff w1, w2;
+};
+struct Layout {
+    mnmt_config c;
+    size_t emb_q, emb_s, globals, pe, enc_ln_g, enc_ln_b, dec_ln_g, dec_ln_b, out_w, out_s, out_b;
+    LinOff proj;
+    std::vector<SelfOff> enc_self, dec_self;
+    std::vector<FfnOff> enc_ffn, dec_ffn;
+    std::vector<CrossOff> dec_cross;
+};
+
+struct Walker {
+    size_t off, size;
+    bool bad;
+    size_t take(size_t n) {
+        if (bad || n > size || off > size - n) {
+            bad = true;
+            return 0;
+        }
+        size_t at = off;
+        off = (off + n + 15) & ~(size_t)15;
+        if (off > size) off = size;
+        return at;
+    }
+    LinOff lin(int n, int k) {
+        LinOff l;
+        l.n = n;
+        l.k = k;
+        l.w = take((size_t)n * k);
+        l.s = take((size_t)n * 4);
+        l.b = take((size_t)n * 4);
+        return l;
+    }
+};
+
+bool pow2_in(int v, int lo, int hi) { return v >= lo && v <= hi && (v & (v - 1)) == 0; }
+
+int parse_layout(const void *blob, size_t bytes, Layout *L) {
+    if (!blob || bytes < 64) return fail(MNMT_EFORMAT, "blob shorter than its 64-byte header");
+    const uint8_t *p = static_cast<const uint8_t *>(blob);
+    if (std::memcmp(p, "MNMT", 4) != 0) return fail(MNMT_EFORMAT, "bad magic");
+    uint32_t ver;
+    std::memcpy(&ver, p + 4, 4);
+    if (ver != 1) return fail(MNMT_EFORMAT, "unsupported blob version %u", ver);
+    int32_t h[13];
+    std::memcpy(h, p + 8, sizeof(h));
+    mnmt_config &c = L->c;
+    c.n_enc = h[0]; c.n_dec = h[1]; c.d_model = h[2]; c.n_heads = h[3]; c.d_ffn = h[4];
+    c.vocab = h[5]; c.d_embed = h[6]; c.pre_ln = h[7]; c.tied_output = h[8]; c.max_pos = h[9];
+    c.pad_id = h[10]; c.bos_id = h[11]; c.eos_id = h[12];
+    const int d = c.d_model, F = c.d_ffn, V = c.vocab, E = c.d_embed;
+    if (c.n_enc < 1 || c.n_enc > 64 || c.n_dec < 1 || c.n_dec > 64) return fail(MNMT_EFORMAT, "layer counts out of range");
+    if (d < 64 || d > 2048 || d % 64 || c.n_heads < 1 || d % c.n_heads) return fail(MNMT_EFORMAT, "d_model %d / heads %d unsupported", d, c.n_heads);
+    if (!pow2_in(d / c.n_heads, 32, 128)) return fail(MNMT_EFORMAT, "head dim %d not in {32,64,128}", d / c.n_heads);
+    if (c.n_heads > 16) return fail(MNMT_EFORMAT, "more than 16 heads");
+    if (F < 64 || F % 64 || F > 8192) return fail(MNMT_EFORMAT, "d_ffn %d unsupported", F);
+    if (V < 4 || E < 16 || E % 16 || E > d) return fail(MNMT_EFORMAT, "vocab / d_embed out of range");
+    if (c.tied_output && E != d) return fail(MNMT_EFORMAT, "tied output needs d_embed == d_model");
+    if (c.max_pos < 1 || c.max_pos > 1024) return fail(MNMT_EFORMAT, "max_pos out of range");
+    for (int id : {c.pad_id, c.bos_id, c.eos_id})
+        if (id < 0 || id >= V) return fail(MNMT_EFORMAT, "special id out of range");
+    Walker w{64, bytes, false};
+    L->emb_q = w.take((size_t)V * E);
+    L->emb_s = w.take((size_t)V * 4);
+    if (E != d) L->proj = w.lin(d, E);
+    L->globals = w.take(16);
+    L->pe = w.take((size_t)c.max_pos * d * 4);
+    auto self_blk = [&]() {
+        SelfOff s;
+        s.ln_g = w.take((size_t)d * 4);
+        s.ln_b = w.take((size_t)d * 4);
+        s.sc = w.take(32);
+        s.qkv = w.lin(3 * d, d);
+        s.o = w.lin(d, d);
+        return s;
+    };
+    auto ffn_blk = [&]() {
+        FfnOff f;
+        f.ln_g = w.take((size_t)d * 4);
+        f.ln_b = w.take((size_t)d * 4);
+        f.sc = w.take(16);
+        f.w1 = w.lin(F, d);
+        f.w2 = w.lin(d, F);
+        return f;
+    };
+    for (int l = 0; l < c.n_enc; l++) {
+        L->enc_self.push_back(self_blk());
+        L->enc_ffn.push_back(ffn_blk());
+    }
+    if (c.pre_ln) {
+        L->enc_ln_g = w.take((size_t)d * 4);
+        L->enc_ln_b = w.take((size_t)d * 4);
+    }
+    for (int l = 0; l < c.n_dec; l++) {
+        L->dec_self.push_back(self_blk());
+        CrossOff x;
+        x.ln_g = w.take((size_t)d * 4);
+        x.ln_b = w.take((size_t)d * 4);
+        x.sc = w.take(32);
+        x.q = w.lin(d, d);
+        x.kv = w.lin(2 * d, d);
+        x.o = w.lin(d, d);
+        L->dec_cross.push_back(x);
+        L->dec_ffn.push_back(ffn_blk());
+    }
+    if (c.pre_ln) {
+        L->dec_ln_g = w.take((size_t)d * 4);
+        L->dec_ln_b = w.take((size_t)d * 4);
+    }
+    if (!c.tied_output) {
+        L->out_w = w.take((size_t)V * d);
+        L->out_s = w.take((size_t)V * 4);
+    } else {
+        L->out_w = L->emb_q;
+        L->out_s = L->emb_s;
+    }
+    L->out_b = w.take((size_t)V * 4);
+    if (w.bad || w.off != bytes) return fail(MNMT_EFORMAT, "blob size does not match its config");
+    return MNMT_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// model
+// ---------------------------------------------------------------------------
+namespace {
+struct Lin {
+    const int8_t *w;
+    const float *s, *b;
+    int n, k;
+};
+struct LnP {
+    const float *g, *b;
+};
+struct SelfBlk {
+    LnP ln;
+    float s_in, s_q, s_k, s_v, s_ctx, gamma, sigma, rho;
+    Lin qkv, o;
+    const float *inv_qkv;
+};
+struct CrossBlk {
+    LnP ln;
+    float s_in, s_q, s_k, s_v, s_ctx, gamma, sigma, rho;
+    Lin q, kv, o;
+    const float *inv_q, *inv_kv;
+};
+struct FfnBlk {
+    LnP ln;
+    float s_in, s_h, gamma;
+    Lin w1, w2;
+    const float *inv_h;
+};
+}  // namespace
+
+struct mnmt_model {
+    mnmt_config c;
+    cudaStream_t stream;
+    bool own_stream;
+    uint8_t *d_blob;
+    float *d_aux;
+    size_t bytes;
+    const int8_t *emb_q;
+    const float *emb_s;
+    bool factorised;
+    Lin proj;
+    float emb_scale, s_enc, s_dout;
+    const float *pe;
+    std::vector<SelfBlk> enc_self, dec_self;
+    std::vector<CrossBlk> dec_cross;
+    std::vector<FfnBlk> enc_ffn, dec_ffn;
+    LnP enc_final, dec_final;
+    Lin out;
+};
+
+static float host_sigma(float s_q, float s_k, int dh) {
+    return (float)((double)s_q * (double)s_k / std::sqrt((double)dh));
+}
+
+extern "C" int mnmt_blob_check(const void *blob, size_t bytes, mnmt_config *cfg_out) {
+    Layout L;
+    int st = parse_layout(blob, bytes, &L);
+    if (st) return st;
+    if (cfg_out) *cfg_out = L.c;
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_model_config(const mnmt_model *m, mnmt_config *cfg_out) {
+    if (!m || !cfg_out) return fail(MNMT_EINVAL, "null argument");
+    *cfg_out = m->c;
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stream, mnmt_model **out) {
+    if (!out) return fail(MNMT_EINVAL, "out is null");
+    *out = nullptr;
+    Layout L;
+    int st = parse_layout(blob, bytes, &L);
+    if (st) return st;
+    if ((st = lib_init())) return st;
+    mnmt_model *m = new (std::nothrow) mnmt_model();
+    if (!m) return fail(MNMT_ENOMEM, "host allocation failed");
+    m->c = L.c;
+    m->bytes = bytes;
+    if (cuda_stream) {
+        m->stream = static_cast<cudaStream_t>(cuda_stream);
+        m->own_stream = false;
+    } else {
+        // the legacy default stream cannot be captured into a graph: use a
+        // blocking stream of our own, ordered with the legacy stream
+        if (cudaStreamCreate(&m->stream) != cudaSuccess) {
+            delete m;
+            return fail(MNMT_ECUDA, "cudaStreamCreate failed");
+        }
+        m->own_stream = true;
+    }
+    const uint8_t *hb = static_cast<const uint8_t *>(blob);
+    const mnmt_config &c = m->c;
+    const int d = c.d_model, F = c.d_ffn, dh = d / c.n_heads;
+    if (cudaMalloc(&m->d_blob, bytes) != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ENOMEM, "cudaMalloc of %zu weight bytes failed", bytes);
+    }
+    if (cudaMemcpyAsync(m->d_blob, blob, bytes, cudaMemcpyHostToDevice, m->stream) != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ECUDA, "weight upload failed");
+    }
+    auto hf = [&](size_t off, int i) {
+        float v;
+        std::memcpy(&v, hb + off + 4 * i, 4);
+        return v;
+    };
+    auto dlin = [&](const LinOff &o) {
+        Lin l;
+        l.w = reinterpret_cast<const int8_t *>(m->d_blob + o.w);
+        l.s = reinterpret_cast<const float *>(m->d_blob + o.s);
+        l.b = reinterpret_cast<const float *>(m->d_blob + o.b);
+        l.n = o.n;
+        l.k = o.k;
+        return l;
+    };
+    auto dln = [&](size_t g, size_t b) {
+        return LnP{reinterpret_cast<const float *>(m->d_blob + g), reinterpret_cast<const float *>(m->d_blob + b)};
+    };
+    // derived per-column requantisation constants: inv = fl(1 / s)
+    std::vector<float> aux;
+    std::vector<size_t> aux_at;
+    auto push_inv = [&](std::initializer_list<std::pair<float, int>> segs) {
+        aux_at.push_back(aux.size());
+        for (auto &sg : segs)
+            for (int i = 0; i < sg.second; i++) aux.push_back(1.0f / sg.first);
+        while (aux.size() % 4) aux.push_back(0.0f);
+        return aux_at.size() - 1;
+    };
+    struct Pend {
+        const float **dst;
+        size_t idx;
+    };
+    std::vector<Pend> pend;
+    m->emb_q = reinterpret_cast<const int8_t *>(m->d_blob + L.emb_q);
+    m->emb_s = reinterpret_cast<const float *>(m->d_blob + L.emb_s);
+    m->factorised = c.d_embed != d;
+    if (m->factorised) m->proj = dlin(L.proj);
+    m->emb_scale = hf(L.globals, 0);
+    m->s_enc = hf(L.globals, 1);
+    m->s_dout = hf(L.globals, 2);
+    m->pe = reinterpret_cast<const float *>(m->d_blob + L.pe);
+    auto mk_self = [&](const SelfOff &o) {
+        SelfBlk s;
+        s.ln = dln(o.ln_g, o.ln_b);
+        s.s_in = hf(o.sc, 0); s.s_q = hf(o.sc, 1); s.s_k = hf(o.sc, 2); s.s_v = hf(o.sc, 3);
+        s.s_ctx = hf(o.sc, 4); s.gamma = hf(o.sc, 5);
+        s.sigma = host_sigma(s.s_q, s.s_k, dh);
+        s.rho = s.s_v / s.s_ctx;
+        s.qkv = dlin(o.qkv);
+        s.o = dlin(o.o);
+        s.inv_qkv = nullptr;
+        return s;
+    };
+    auto mk_ffn = [&](const FfnOff &o) {
+        FfnBlk f;
+        f.ln = dln(o.ln_g, o.ln_b);
+        f.s_in = hf(o.sc, 0); f.s_h = hf(o.sc, 1); f.gamma = hf(o.sc, 2);
+        f.w1 = dlin(o.w1);
+        f.w2 = dlin(o.w2);
+        f.inv_h = nullptr;
+        return f;
+    };
+    for (int l = 0; l < c.n_enc; l++) {
+        m->enc_self.push_back(mk_self(L.enc_self[l]));
+        m->enc_ffn.push_back(mk_ffn(L.enc_ffn[l]));
+    }
+    for (int l = 0; l < c.n_dec; l++) {
+        m->dec_self.push_back(mk_self(L.dec_self[l]));
+        const CrossOff &o = L.dec_cross[l];
+        CrossBlk x;
+        x.ln = dln(o.ln_g, o.ln_b);
+        x.s_in = hf(o.sc, 0); x.s_q = hf(o.sc, 1); x.s_k = hf(o.sc, 2); x.s_v = hf(o.sc, 3);
+        x.s_ctx = hf(o.sc, 4); x.gamma = hf(o.sc, 5);
+        x.sigma = host_sigma(x.s_q, x.s_k, dh);
+        x.rho = x.s_v / x.s_ctx;
+        x.q = dlin(o.q);
+        x.kv = dlin(o.kv);
+        x.o = dlin(o.o);
+        m->dec_cross.push_back(x);
+        m->dec_ffn.push_back(mk_ffn(L.dec_ffn[l]));
+    }
+    // vectors are final now: record pointer slots to patch after the aux upload
+    for (auto &s : m->enc_self) pend.push_back({&s.inv_qkv, push_inv({{s.s_q, d}, {s.s_k, d}, {s.s_v, d}})});
+    for (auto &s : m->dec_self) pend.push_back({&s.inv_qkv, push_inv({{s.s_q, d}, {s.s_k, d}, {s.s_v, d}})});
+    for (auto &f : m->enc_ffn) pend.push_back({&f.inv_h, push_inv({{f.s_h, F}})});
+    for (auto &f : m->dec_ffn) pend.push_back({&f.inv_h, push_inv({{f.s_h, F}})});
+    for (auto &x : m->dec_cross) {
+        pend.push_back({&x.inv_q, push_inv({{x.s_q, d}})});
+        pend.push_back({&x.inv_kv, push_inv({{x.s_k, d}, {x.s_v, d}})});
+    }
+    if (c.pre_ln) {
+        m->enc_final = dln(L.enc_ln_g, L.enc_ln_b);
+        m->dec_final = dln(L.dec_ln_g, L.dec_ln_b);
+    }
+    m->out.w = reinterpret_cast<const int8_t *>(m->d_blob + L.out_w);
+    m->out.s = reinterpret_cast<const float *>(m->d_blob + L.out_s);
+    m->out.b = reinterpret_cast<const float *>(m->d_blob + L.out_b);
+    m->out.n = c.vocab;
+    m->out.k = d;
+    if (cudaMalloc(&m->d_aux, aux.size() * 4) != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ENOMEM, "cudaMalloc of derived constants failed");
+    }
+    if (cudaMemcpyAsync(m->d_aux, aux.data(), aux.size() * 4, cudaMemcpyHostToDevice, m->stream) != cudaSuccess ||
+        cudaStreamSynchronize(m->stream) != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ECUDA, "upload of derived constants failed");
+    }
+    for (auto &pd : pend) *pd.dst = m->d_aux + aux_at[pd.idx];
+    *out = m;
+    return MNMT_OK;
+}
+
+extern "C" void mnmt_model_free(mnmt_model *m) {
+    if (!m) return;
+    if (m->stream) cudaStreamSynchronize(m->stream);
+    if (m->d_blob) cudaFree(m->d_blob);
+    if (m->d_aux) cudaFree(m->d_aux);
+    if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);
+    delete m;
+}
+
+// ---------------------------------------------------------------------------
+// session
+// ---------------------------------------------------------------------------
+enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_STATUS = 5, ST_N = 8 };
+
+struct mnmt_session {
+    mnmt_model *m;
+    int Bmax, Smax, k, Tcap;
+    int B = 0, S = 0, max_len = 0;
+    int steps = 0;      // decode steps launched since the last encode
+    int poisoned = 0;
+    uint8_t *arena = nullptr;
+    size_t arena_bytes = 0;
+    float *resid, *cum, *logits;
+    int8_t *act, *qkv, *ctx, *hid, *qbuf, *enc_q, *ck, *cv, *sk, *sv;
+    int32_t *src_ids, *src_lens, *tok, *fin, *hist, *parents, *anc, *out_ids, *out_lens;
+    float *out_scores;
+    unsigned long long *keys, *cand;
+    int *state;
+    int *h_state = nullptr;  // pinned mirror of state
+    size_t ck_layer, sk_layer;  // per-layer strides of the caches (elements)
+    cudaGraphExec_t gexec = nullptr;
+    int graph_B = -1, graph_S = -1;
+};
+
+static int poison(mnmt_session *s, int code) {
+    if (!s->poisoned) s->poisoned = code;
+    return code;
+}
+
+extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max_src_len, int32_t beam,
+                                   int32_t max_len, mnmt_session **out) {
+    if (!out) return fail(MNMT_EINVAL, "out is null");
+    *out = nullptr;
+    if (!m) return fail(MNMT_EINVAL, "model is null");
+    const mnmt_config &c = m->c;
+    if (max_batch < 1 || max_src_len < 1 || max_src_len > 512 || max_src_len > c.max_pos || beam < 1 ||
+        beam > 16 || beam > c.vocab || max_len < 1 || max_len > c.max_pos || max_len > 1024)
+        return fail(MNMT_EINVAL, "session sizes out of range (batch %d, src %d, beam %d, len %d)", max_batch,
+                    max_src_len, beam, max_len);
+    mnmt_session *s = new (std::nothrow) mnmt_session();
+    if (!s) return fail(MNMT_ENOMEM, "host allocation failed");
+    s->m = m;
+    s->Bmax = max_batch;
+    s->Smax = max_src_len;
+    s->k = beam;
+    s->Tcap = max_len;
+    const size_t d = c.d_model, F = c.d_ffn, V = c.vocab, L = c.n_dec;
+    const size_t R = (size_t)max_batch * beam, ME = (size_t)max_batch * max_src_len;
+    const size_t rows = ME > R ? ME : R;
+    s->ck_layer = (size_t)max_batch * max_src_len * d;
+    s->sk_layer = R * max_len * d;
+    // arena layout (256-byte aligned pieces)
+    size_t off = 0;
+    auto piece = [&](size_t bytes) {
+        size_t at = off;
+        off += (bytes + 255) & ~(size_t)255;
+        return at;
+    };
+    size_t o_resid = piece(rows * d * 4), o_act = piece(rows * (d > F ? d : F)), o_qkv = piece(ME * 3 * d),
+           o_ctx = piece(rows * d), o_hid = piece(rows * F), o_qbuf = piece(R * d), o_encq = piece(ME * d),
+           o_ck = piece(L * s->ck_layer), o_cv = piece(L * s->ck_layer), o_sk = piece(L * s->sk_layer),
+           o_sv = piece(L * s->sk_layer), o_ids = piece(ME * 4), o_lens = piece((size_t)max_batch * 4),
+           o_tok = piece(R * 4), o_fin = piece(R * 4), o_cum = piece(R * 4),
+           o_hist = piece((size_t)max_len * R * 4), o_par = piece((size_t)max_len * R * 4),
+           o_anc = piece(R * max_len * 4), o_keys = piece(R * 8), o_cand = piece(R * beam * 8),
+           o_logits = piece(beam > 1 ? R * V * 4 : 256), o_outids = piece((size_t)max_batch * max_len * 4),
+           o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
+           o_state = piece(ST_N * 4);
+    s->arena_bytes = off;
+    if (cudaMalloc(&s->arena, off) != cudaSuccess) {
+        delete s;
+        return fail(MNMT_ENOMEM, "cudaMalloc of %zu session bytes failed", off);
+    }
+    if (cudaMallocHost(&s->h_state, ST_N * 4) != cudaSuccess) {
+        cudaFree(s->arena);
+        delete s;
+        return fail(MNMT_ENOMEM, "pinned host allocation failed");
+    }
+    uint8_t *a = s->arena;
+    s->resid = reinterpret_cast<float *>(a + o_resid);
+    s->act = reinterpret_cast<int8_t *>(a + o_act);
+    s->qkv = reinterpret_cast<int8_t *>(a + o_qkv);
+    s->ctx = reinterpret_cast<int8_t *>(a + o_ctx);
+    s->hid = reinterpret_cast<int8_t *>(a + o_hid);
+    s->qbuf = reinterpret_cast<int8_t *>(a + o_qbuf);
+    s->enc_q = reinterpret_cast<int8_t *>(a + o_encq);
+    s->ck = reinterpret_cast<int8_t *>(a + o_ck);
+    s->cv = reinterpret_cast<int8_t *>(a + o_cv);
+    s->sk = reinterpret_cast<int8_t *>(a + o_sk);
+    s->sv = reinterpret_cast<int8_t *>(a + o_sv);
+    s->src_ids = reinterpret_cast<int32_t *>(a + o_ids);
+    s->src_lens = reinterpret_cast<int32_t *>(a + o_lens);
+    s->tok = reinterpret_cast<int32_t *>(a + o_tok);
+    s->fin = reinterpret_cast<int32_t *>(a + o_fin);
+    s->cum = reinterpret_cast<float *>(a + o_cum);
+    s->hist = reinterpret_cast<int32_t *>(a + o_hist);
+    s->parents = reinterpret_cast<int32_t *>(a + o_par);
+    s->anc = reinterpret_cast<int32_t *>(a + o_anc);
+    s->keys = reinterpret_cast<unsigned long long *>(a + o_keys);
+    s->cand = reinterpret_cast<unsigned long long *>(a + o_cand);
+    s->logits = reinterpret_cast<float *>(a + o_logits);
+    s->out_ids = reinterpret_cast<int32_t *>(a + o_outids);
+    s->out_lens = reinterpret_cast<int32_t *>(a + o_outlens);
+    s->out_scores = reinterpret_cast<float *>(a + o_outsc);
+    s->state = reinterpret_cast<int *>(a + o_state);
+    if (cudaMemsetAsync(s->arena, 0, off, m->stream) != cudaSuccess ||
+        cudaStreamSynchronize(m->stream) != cudaSuccess) {
+        mnmt_session_free(s);
+        return fail(MNMT_ECUDA, "arena initialisation failed");
+    }
+    *out = s;
+    return MNMT_OK;
+}
+
+extern "C" void mnmt_session_free(mnmt_session *s) {
+    if (!s) return;
+    if (s->m && s->m->stream) cudaStreamSynchronize(s->m->stream);
+    if (s->gexec) cudaGraphExecDestroy(s->gexec);
+    if (s->arena) cudaFree(s->arena);
+    if (s->h_state) cudaFreeHost(s->h_state);
+    delete s;
+}
+
+// ---------------------------------------------------------------------------
+// launch sequences
+// ---------------------------------------------------------------------------
+namespace {
+
+Epi base_epi(int mode, float s_x, const Lin &l) {
+    Epi e;
+    std::memset(&e, 0, sizeof(e));
+    e.mode = mode;
+    e.s_x = s_x;
+    e.s_w = l.s;
+    e.bias = l.b;
+    return e;
+}
+
+#define LK(call)                                                                                   \
+    do {                                                                                           \
+        cudaError_t e_ = (call);                                                                   \
+        if (e_ != cudaSuccess) return fail(MNMT_ECUDA, "%s: %s", #call, cudaGetErrorString(e_));   \
+    } while (0)
+
+// LayerNorm after a residual update.  Pre-LN: q8(LN_next(r)) into act (r kept).
+// Post-LN: r = LN_this(r) in place, act = q8(r).
+int ln_after_residual(mnmt_session *s, int M, const LnP &ln_pre_next, const LnP &ln_post_this, float s_next,
+                      int8_t *act_out, const int *skip) {
+    mnmt_model *m = s->m;
+    LnArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.r = s->resid;
+    a.M = M;
+    a.d = m->c.d_model;
+    a.inv = 1.0f / s_next;
+    a.out_q = act_out;
+    a.status = s->state + ST_STATUS;
+    a.skip = skip;
+    if (m->c.pre_ln) {
+        a.g = ln_pre_next.g;
+        a.b = ln_pre_next.b;
+    } else {
+        a.g = ln_post_this.g;
+        a.b = ln_post_this.b;
+        a.out_f = s->resid;
+    }
+    LK(launch_layernorm(a, m->stream));
+    return MNMT_OK;
+}
+
+int run_encoder(mnmt_session *s, int B, int S) {
+    mnmt_model *m = s->m;
+    const mnmt_config &c = m->c;
+    const int d = c.d_model, F = c.d_ffn, H = c.n_heads, dh = d / H, M = B * S;
+    cudaStream_t st = m->stream;
+    int *status = s->state + ST_STATUS;
+    {
+        EmbedArgs e;
+        std::memset(&e, 0, sizeof(e));
+        e.ids = s->src_ids;
+        e.S = S;
+        e.emb_q = m->emb_q;
+        e.emb_s = m->emb_s;
+        if (m->factorised) {
+            e.proj_w = m->proj.w;
+            e.proj_s = m->proj.s;
+            e.proj_b = m->proj.b;
+        }
+        e.emb_scale = m->emb_scale;
+        e.pe = m->pe;
+        e.M = M;
+        e.d = d;
+        e.E = c.d_embed;
+        e.V = c.vocab;
+        e.r = s->resid;
+        e.out_q = s->act;
+        if (c.pre_ln) {
+            e.ln_g = m->enc_self[0].ln.g;
+            e.ln_b = m->enc_self[0].ln.b;
+        }
+        e.inv = 1.0f / m->enc_self[0].s_in;
+        e.status = status;
+        LK(launch_embed(e, st));
+    }
+    for (int l = 0; l < c.n_enc; l++) {
+        const SelfBlk &A = m->enc_self[l];
+        const FfnBlk &Fb = m->enc_ffn[l];
+        Epi e = base_epi(EPI_Q8, A.s_in, A.qkv);
+        e.inv_out = A.inv_qkv;
+        e.out = s->qkv;
+        e.ldo = 3 * d;
+        LK(launch_linear(s->act, d, A.qkv.w, M, 3 * d, d, e, st));
+        AttnEncArgs at;
+        at.qkv = s->qkv;
+        at.ctx = s->ctx;
+        at.len = s->src_lens;
+        at.B = B;
+        at.S = S;
+        at.H = H;
+        at.dh = dh;
+        at.d = d;
+        at.sigma = A.sigma;
+        at.rho = A.rho;
+        LK(launch_attention_encoder(at, st));
+        e = base_epi(EPI_RESID, A.s_ctx, A.o);
+        e.f32 = s->resid;
+        e.ldf = d;
+        e.gamma = A.gamma;
+        LK(launch_linear(s->ctx, d, A.o.w, M, d, d, e, st));
+        int rc = ln_after_residual(s, M, Fb.ln, A.ln, Fb.s_in, s->act, nullptr);
+        if (rc) return rc;
+        e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
+        e.inv_out = Fb.inv_h;
+        e.out = s->hid;
+        e.ldo = F;
+        LK(launch_linear(s->act, d, Fb.w1.w, M, F, d, e, st));
+        e = base_epi(EPI_RESID, Fb.s_h, Fb.w2);
+        e.f32 = s->resid;
+        e.ldf = d;
+        e.gamma = Fb.gamma;
+        LK(launch_linear(s->hid, F, Fb.w2.w, M, d, F, e, st));
+        if (l + 1 < c.n_enc) {
+            const SelfBlk &An = m->enc_self[l + 1];
+            rc = ln_after_residual(s, M, An.ln, Fb.ln, An.s_in, s->act, nullptr);
+        } else {
+            rc = ln_after_residual(s, M, m->enc_final, Fb.ln, m->s_enc, s->enc_q, nullptr);
+        }
+        if (rc) return rc;
+    }
+    for (int l = 0; l < c.n_dec; l++) {
+        const CrossBlk &X = m->dec_cross[l];
+        Epi e = base_epi(EPI_KV_CROSS, m->s_enc, X.kv);
+        e.inv_out = X.inv_kv;
+        e.kc = s->ck + l * s->ck_layer;
+        e.vc = s->cv + l * s->ck_layer;
+        e.d = d;
+        e.H = H;
+        e.dh = dh;
+        e.S = S;
+        LK(launch_linear(s->enc_q, d, X.kv.w, M, 2 * d, d, e, st));
+    }
+    return MNMT_OK;
+}
+
+// one decoder step for all B*k hypotheses (captured into a graph)
+int issue_decode_step(mnmt_session *s) {
+    mnmt_model *m = s->m;
+    const mnmt_config &c = m->c;
+    const int d = c.d_model, F = c.d_ffn, H = c.n_heads, dh = d / H;
+    const int R = s->B * s->k;
+    cudaStream_t st = m->stream;
+    const int *done = s->state + ST_DONE;
+    int *t_ptr = s->state + ST_T;
+    int *status = s->state + ST_STATUS;
+    {
+        EmbedArgs e;
+        std::memset(&e, 0, sizeof(e));
+        e.tok = s->tok;
+        e.t_ptr = t_ptr;
+        e.emb_q = m->emb_q;
+        e.emb_s = m->emb_s;
+        if (m->factorised) {
+            e.proj_w = m->proj.w;
+            e.proj_s = m->proj.s;
+            e.proj_b = m->proj.b;
+        }
+        e.emb_scale = m->emb_scale;
+        e.pe = m->pe;
+        e.M = R;
+        e.d = d;
+        e.E = c.d_embed;
+        e.V = c.vocab;
+        e.r = s->resid;
+        e.out_q = s->act;
+        if (c.pre_ln) {
+            e.ln_g = m->dec_self[0].ln.g;
+            e.ln_b = m->dec_self[0].ln.b;
+        }
+        e.inv = 1.0f / m->dec_self[0].s_in;
+        e.status = status;
+        e.skip = done;
+        LK(launch_embed(e, st));
+    }
+    for (int l = 0; l < c.n_dec; l++) {
+        const SelfBlk &A = m->dec_self[l];
+        const CrossBlk &X = m->dec_cross[l];
+        const FfnBlk &Fb = m->dec_ffn[l];
+        Epi e = base_epi(EPI_QKV_DEC, A.s_in, A.qkv);
+        e.inv_out = A.inv_qkv;
+        e.out = s->qbuf;
+        e.ldo = d;
+        e.kc = s->sk + l * s->sk_layer;
+        e.vc = s->sv + l * s->sk_layer;
+        e.t_ptr = t_ptr;
+        e.d = d;
+        e.H = H;
+        e.dh = dh;
+        e.T = s->Tcap;
+        e.skip = done;
+        LK(launch_linear(s->act, d, A.qkv.w, R, 3 * d, d, e, st));
+        AttnDecArgs at;
+        std::memset(&at, 0, sizeof(at));
+        at.q = s->qbuf;
+        at.kc = s->sk + l * s->sk_layer;
+        at.vc = s->sv + l * s->sk_layer;
+        at.ctx = s->ctx;
+        at.R = R;
+        at.H = H;
+        at.dh = dh;
+        at.T = s->Tcap;
+        at.cross = 0;
+        at.beam = s->k;
+        at.t_ptr = t_ptr;
+        at.anc = s->k > 1 ? s->anc : nullptr;
+        at.sigma = A.sigma;
+        at.rho = A.rho;
+        at.skip = done;
+        LK(launch_attention_decode(at, st));
+        e = base_epi(EPI_RESID, A.s_ctx, A.o);
+        e.f32 = s->resid;
+        e.ldf = d;
+        e.gamma = A.gamma;
+        e.skip = done;
+        LK(launch_linear(s->ctx, d, A.o.w, R, d, d, e, st));
+        int rc = ln_after_residual(s, R, X.ln, A.ln, X.s_in, s->act, done);
+        if (rc) return rc;
+        e = base_epi(EPI_Q8, X.s_in, X.q);
+        e.inv_out = X.inv_q;
+        e.out = s->qbuf;
+        e.ldo = d;
+        e.skip = done;
+        LK(launch_linear(s->act, d, X.q.w, R, d, d, e, st));
+        at.kc = s->ck + l * s->ck_layer;
+        at.vc = s->cv + l * s->ck_layer;
+        at.T = s->S;
+        at.cross = 1;
+        at.src_len = s->src_lens;
+        at.anc = nullptr;
+        at.sigma = X.sigma;
+        at.rho = X.rho;
+        LK(launch_attention_decode(at, st));
+        e = base_epi(EPI_RESID, X.s_ctx, X.o);
+        e.f32 = s->resid;
+        e.ldf = d;
+        e.gamma = X.gamma;
+        e.skip = done;
+        LK(launch_linear(s->ctx, d, X.o.w, R, d, d, e, st));
+        rc = ln_after_residual(s, R, Fb.ln, X.ln, Fb.s_in, s->act, done);
+        if (rc) return rc;
+        e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
+        e.inv_out = Fb.inv_h;
+        e.out = s->hid;
+        e.ldo = F;
+        e.skip = done;
+        LK(launch_linear(s->act, d, Fb.w1.w, R, F, d, e, st));
+        e = base_epi(EPI_RESID, Fb.s_h, Fb.w2);
+        e.f32 = s->resid;
+        e.ldf = d;
+        e.gamma = Fb.gamma;
+        e.skip = done;
+        LK(launch_linear(s->hid, F, Fb.w2.w, R, d, F, e, st));
+        if (l + 1 < c.n_dec) {
+            const SelfBlk &An = m->dec_self[l + 1];
+            rc = ln_after_residual(s, R, An.ln, Fb.ln, An.s_in, s->act, done);
+        } else {
+            rc = ln_after_residual(s, R, m->dec_final, Fb.ln, m->s_dout, s->act, done);
+        }
+        if (rc) return rc;
+    }
+    if (s->k == 1) {
+        Epi e = base_epi(EPI_ARGMAX, m->s_dout, m->out);
+        e.keys = s->keys;
+        e.skip = done;
+        LK(launch_linear(s->act, d, m->out.w, R, c.vocab, d, e, st));
+        GreedyArgs g;
+        g.keys = s->keys;
+        g.tok = s->tok;
+        g.fin = s->fin;
+        g.hist = s->hist;
+        g.t_ptr = t_ptr;
+        g.done = s->state + ST_DONE;
+        g.tmax_ptr = s->state + ST_TMAX;
+        g.R = R;
+        g.T = s->Tcap;
+        g.eos = c.eos_id;
+        g.pad = c.pad_id;
+        LK(launch_greedy_update(g, st));
+    } else {
+        Epi e = base_epi(EPI_F32, m->s_dout, m->out);
+        e.f32 = s->logits;
+        e.ldf = c.vocab;
+        e.skip = done;
+        LK(launch_linear(s->act, d, m->out.w, R, c.vocab, d, e, st));
+        BeamArgs b;
+        b.logits = s->logits;
+        b.tok = s->tok;
+        b.fin = s->fin;
+        b.cum = s->cum;
+        b.hist = s->hist;
+        b.parents = s->parents;
+        b.anc = s->anc;
+        b.cand = s->cand;
+        b.t_ptr = t_ptr;
+        b.done = s->state + ST_DONE;
+        b.ticket = s->state + ST_TICKET;
+        b.tmax_ptr = s->state + ST_TMAX;
+        b.B = s->B;
+        b.k = s->k;
+        b.V = c.vocab;
+        b.T = s->Tcap;
+        b.eos = c.eos_id;
+        b.pad = c.pad_id;
+        b.status = status;
+        LK(launch_beam_step(b, st));
+    }
+    return MNMT_OK;
+}
+
+int ensure_graph(mnmt_session *s) {
+    if (s->gexec && s->graph_B == s->B && s->graph_S == s->S) return MNMT_OK;
+    if (s->gexec) {
+        cudaGraphExecDestroy(s->gexec);
+        s->gexec = nullptr;
+    }
+    cudaStream_t st = s->m->stream;
+    cudaGraph_t g = nullptr;
+    CK(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
+    int rc = issue_decode_step(s);
+    cudaError_t ce = cudaStreamEndCapture(st, &g);
+    if (rc) {
+        if (g) cudaGraphDestroy(g);
+        return rc;
+    }
+    if (ce != cudaSuccess) return fail(MNMT_ECUDA, "graph capture failed: %s", cudaGetErrorString(ce));
+    ce = cudaGraphInstantiate(&s->gexec, g, 0);
+    cudaGraphDestroy(g);
+    if (ce != cudaSuccess) {
+        s->gexec = nullptr;
+        return fail(MNMT_ECUDA, "graph instantiation failed: %s", cudaGetErrorString(ce));
+    }
+    s->graph_B = s->B;
+    s->graph_S = s->S;
+    return MNMT_OK;
+}
+
+int check_device_status(mnmt_session *s) {
+    // called after a synchronisation that covered a copy of state into h_state
+    int code = s->h_state[ST_STATUS];
+    if (code) return poison(s, fail(code, "device reported status %d", code));
+    return MNMT_OK;
+}
+
+int sync_state(mnmt_session *s) {
+    cudaStream_t st = s->m->stream;
+    cudaError_t e = cudaMemcpyAsync(s->h_state, s->state, ST_N * 4, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return poison(s, fail(MNMT_ECUDA, "device work failed: %s", cudaGetErrorString(e)));
+    return check_device_status(s);
+}
+
+}  // namespace
+
+extern "C" int mnmt_encode(mnmt_session *s, const int32_t *src_ids, const int32_t *src_lens, int32_t B,
+                           int32_t S_pad, int32_t flags) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    if (s->poisoned) return fail(s->poisoned, "session poisoned by an earlier failure");
+    if (!src_ids || !src_lens || B < 1 || B > s->Bmax || S_pad < 1 || S_pad > s->Smax)
+        return fail(MNMT_EINVAL, "encode: bad batch %d / padded length %d (capacity %d / %d)", B, S_pad, s->Bmax,
+                    s->Smax);
+    mnmt_model *m = s->m;
+    cudaStream_t st = m->stream;
+    const bool dev = flags & MNMT_DEVICE_PTRS;
+    if (!dev) {
+        for (int b = 0; b < B; b++)
+            if (src_lens[b] < 1 || src_lens[b] > S_pad) return fail(MNMT_EINVAL, "source length %d out of range", src_lens[b]);
+        for (long i = 0; i < (long)B * S_pad; i++)
+            if (src_ids[i] < 0 || src_ids[i] >= m->c.vocab) return fail(MNMT_EINVAL, "source id out of range");
+    }
+    cudaMemcpyKind kind = dev ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    CK(cudaMemcpyAsync(s->src_ids, src_ids, (size_t)B * S_pad * 4, kind, st));
+    CK(cudaMemcpyAsync(s->src_lens, src_lens, (size_t)B * 4, kind, st));
+    s->B = B;
+    s->S = S_pad;
+    int rc = run_encoder(s, B, S_pad);
+    if (rc) return poison(s, rc);
+    InitArgs ia;
+    ia.tok = s->tok;
+    ia.fin = s->fin;
+    ia.anc = s->anc;
+    ia.hist = s->hist;
+    ia.parents = s->parents;
+    ia.cum = s->cum;
+    ia.keys = s->keys;
+    ia.t_ptr = s->state + ST_T;
+    ia.done = s->state + ST_DONE;
+    ia.ticket = s->state + ST_TICKET;
+    ia.R = B * s->k;
+    ia.k = s->k;
+    ia.T = s->Tcap;
+    ia.bos = m->c.bos_id;
+    ia.pad = m->c.pad_id;
+    CK(launch_search_init(ia, st));
+    s->max_len = s->Tcap;
+    s->h_state[ST_TMAX] = s->Tcap;
+    CK(cudaMemcpyAsync(s->state + ST_TMAX, s->h_state + ST_TMAX, 4, cudaMemcpyHostToDevice, st));
+    s->steps = 0;
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_decode_step(mnmt_session *s, int32_t *tokens, int32_t *parents, float *scores,
+                                int32_t *all_done) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    if (s->poisoned) return fail(s->poisoned, "session poisoned by an earlier failure");
+    if (s->B < 1) return fail(MNMT_EINVAL, "decode_step before encode");
+    if (s->steps >= s->max_len) return fail(MNMT_EINVAL, "all %d steps already ran", s->max_len);
+    int rc = ensure_graph(s);
+    if (rc) return poison(s, rc);
+    cudaStream_t st = s->m->stream;
+    CK(cudaGraphLaunch(s->gexec, st));
+    const int t = s->steps++;
+    const int R = s->B * s->k;
+    if (tokens) CK(cudaMemcpyAsync(tokens, s->hist + (size_t)t * R, R * 4, cudaMemcpyDeviceToHost, st));
+    if (parents) CK(cudaMemcpyAsync(parents, s->parents + (size_t)t * R, R * 4, cudaMemcpyDeviceToHost, st));
+    if (scores) CK(cudaMemcpyAsync(scores, s->cum, R * 4, cudaMemcpyDeviceToHost, st));
+    if ((rc = sync_state(s))) return rc;
+    if (scores && s->k == 1)
+        for (int i = 0; i < R; i++) scores[i] = 0.0f;
+    if (all_done) *all_done = s->h_state[ST_DONE];
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_translate(mnmt_session *s, const int32_t *src_ids, const int32_t *src_lens, int32_t B,
+                              int32_t S_pad, int32_t max_len, int32_t flags, int32_t *out_ids,
+                              int32_t *out_lens, float *out_scores) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    if (max_len < 1 || max_len > s->Tcap) return fail(MNMT_EINVAL, "max_len %d outside [1, %d]", max_len, s->Tcap);
+    if (!out_ids || !out_lens || !out_scores) return fail(MNMT_EINVAL, "null output");
+    int rc = mnmt_encode(s, src_ids, src_lens, B, S_pad, flags);
+    if (rc) return rc;
+    cudaStream_t st = s->m->stream;
+    s->max_len = max_len;
+    s->h_state[ST_TMAX] = max_len;
+    CK(cudaMemcpyAsync(s->state + ST_TMAX, s->h_state + ST_TMAX, 4, cudaMemcpyHostToDevice, st));
+    if ((rc = ensure_graph(s))) return poison(s, rc);
+    const int CHECK = 16;
+    int steps = 0;
+    while (steps < max_len) {
+        int n = max_len - steps < CHECK ? max_len - steps : CHECK;
+        for (int i = 0; i < n; i++) CK(cudaGraphLaunch(s->gexec, st));
+        steps += n;
+        if (steps < max_len) {
+            if ((rc = sync_state(s))) return rc;
+            if (s->h_state[ST_DONE]) break;
+        }
+    }
+    s->steps = steps;
+    const bool dev = flags & MNMT_DEVICE_PTRS;
+    FinalArgs fa;
+    fa.hist = s->hist;
+    fa.parents = s->parents;
+    fa.cum = s->cum;
+    fa.t_ptr = s->state + ST_T;
+    fa.out_ids = dev ? out_ids : s->out_ids;
+    fa.out_lens = dev ? out_lens : s->out_lens;
+    fa.out_scores = dev ? out_scores : s->out_scores;
+    fa.B = B;
+    fa.k = s->k;
+    fa.T = s->Tcap;
+    fa.max_len = max_len;
+    fa.eos = s->m->c.eos_id;
+    fa.pad = s->m->c.pad_id;
+    CK(launch_finalize(fa, st));
+    if (!dev) {
+        CK(cudaMemcpyAsync(out_ids, s->out_ids, (size_t)B * max_len * 4, cudaMemcpyDeviceToHost, st));
+        CK(cudaMemcpyAsync(out_lens, s->out_lens, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
+        CK(cudaMemcpyAsync(out_scores, s->out_scores, (size_t)B * 4, cudaMemcpyDeviceToHost, st));
+        return sync_state(s);
+    }
+    // device outputs: report asynchronous failures at the next synchronising call
+    cudaError_t e = cudaMemcpyAsync(s->h_state, s->state, ST_N * 4, cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return poison(s, fail(MNMT_ECUDA, "state copy failed: %s", cudaGetErrorString(e)));
+    return MNMT_OK;
+}
+
+extern "C" int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, void *host_dst, size_t bytes) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    const mnmt_config &c = s->m->c;
+    const size_t d = c.d_model, H = c.n_heads, dh = d / H, R = (size_t)s->B * s->k;
+    const void *src = nullptr;
+    size_t n = 0;
+    auto need_layer = [&]() { return layer >= 0 && layer < c.n_dec; };
+    switch (tap) {
+        case MNMT_TAP_ENC_OUT:
+            src = s->enc_q;
+            n = (size_t)s->B * s->S * d;
+            break;
+        case MNMT_TAP_CROSS_K:
+        case MNMT_TAP_CROSS_V:
+            if (!need_layer()) return fail(MNMT_EINVAL, "layer out of range");
+            src = (tap == MNMT_TAP_CROSS_K ? s->ck : s->cv) + layer * s->ck_layer;
+            n = (size_t)s->B * H * s->S * dh;
+            break;
+        case MNMT_TAP_SELF_K:
+        case MNMT_TAP_SELF_V:
+            if (!need_layer()) return fail(MNMT_EINVAL, "layer out of range");
+            src = (tap == MNMT_TAP_SELF_K ? s->sk : s->sv) + layer * s->sk_layer;
+            n = R * H * s->Tcap * dh;
+            break;
+        case MNMT_TAP_DEC_OUT:
+            src = s->act;
+            n = R * d;
+            break;
+        case MNMT_TAP_LOGITS:
+            if (s->k == 1) return fail(MNMT_EINVAL, "logits are kept only for beam search");
+            src = s->logits;
+            n = R * c.vocab * 4;
+            break;
+        case MNMT_TAP_RESID:
+            src = s->resid;
+            n = (s->steps > 0 ? R : (size_t)s->B * s->S) * d * 4;
+            break;
+        case MNMT_TAP_HISTORY:
+            src = s->hist;
+            n = (size_t)s->Tcap * R * 4;
+            break;
+        case MNMT_TAP_PARENTS:
+            src = s->parents;
+            n = (size_t)s->Tcap * R * 4;
+            break;
+        case MNMT_TAP_ANCESTRY:
+            src = s->anc;
+            n = R * s->Tcap * 4;
+            break;
+        default:
+            return fail(MNMT_EINVAL, "unknown tap %d", tap);
+    }
+    if (!host_dst) return (int64_t)n;
+    if (bytes != n) return fail(MNMT_EINVAL, "tap %d holds %zu bytes, not %zu", tap, n, bytes);
+    cudaStream_t st = s->m->stream;
+    CK(cudaMemcpyAsync(host_dst, src, n, cudaMemcpyDeviceToHost, st));
+    CK(cudaStreamSynchronize(st));
+    return MNMT_OK;
+}
+
+extern "C" const char *mnmt_last_error(void) { return g_err.c_str(); }
+
+// ---------------------------------------------------------------------------
+// kernel-level entry points
+// ---------------------------------------------------------------------------
+extern "C" int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
+                           const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
+                           int8_t *out_q, float *out_f, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!A || !W || !s_w || !bias || M < 1 || N < 1 || K < 16 || K % 16 || (M > 16 && K % 64))
+        return fail(MNMT_EINVAL, "linear: bad shape M=%d N=%d K=%d", M, N, K);
+    if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15)
+        return fail(MNMT_EINVAL, "linear: A and W must be 16-byte aligned");
+    if (M <= 16 && K > 2048) return fail(MNMT_EINVAL, "linear: K > 2048 at M <= 16");
+    Epi e;
+    std::memset(&e, 0, sizeof(e));
+    e.s_x = s_x;
+    e.s_w = s_w;
+    e.bias = bias;
+    switch (mode) {
+        case MNMT_EPI_Q8:
+        case MNMT_EPI_RELU_Q8:
+            if (!out_q || !inv_out) return fail(MNMT_EINVAL, "linear: int8 output needs out_q and inv_out");
+            e.mode = mode == MNMT_EPI_Q8 ? EPI_Q8 : EPI_RELU_Q8;
+            e.out = out_q;
+            e.ldo = N;
+            e.inv_out = inv_out;
+            break;
+        case MNMT_EPI_RESID:
+        case MNMT_EPI_F32:
+            if (!out_f) return fail(MNMT_EINVAL, "linear: fp32 output needs out_f");
+            e.mode = mode == MNMT_EPI_RESID ? EPI_RESID : EPI_F32;
+            e.f32 = out_f;
+            e.ldf = N;
+            e.gamma = gamma;
+            break;
+        default:
+            return fail(MNMT_EINVAL, "linear: unknown mode %d", mode);
+    }
+    cudaError_t err = launch_linear(A, K, W, M, N, K, e, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_linear_argmax(const int8_t *A, const int8_t *W, const float *s_w, const float *bias,
+                                  float s_x, int32_t M, int32_t N, int32_t K, uint64_t *keys, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!A || !W || !s_w || !bias || !keys || M < 1 || N < 1 || K < 16 || K % 16 || (M > 16 && K % 64) ||
+        (M <= 16 && K > 2048))
+        return fail(MNMT_EINVAL, "linear_argmax: bad shape M=%d N=%d K=%d", M, N, K);
+    if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(W)) & 15)
+        return fail(MNMT_EINVAL, "linear_argmax: A and W must be 16-byte aligned");
+    Epi e;
+    std::memset(&e, 0, sizeof(e));
+    e.mode = EPI_ARGMAX;
+    e.s_x = s_x;
+    e.s_w = s_w;
+    e.bias = bias;
+    e.keys = reinterpret_cast<unsigned long long *>(keys);
+    cudaError_t err = launch_linear(A, K, W, M, N, K, e, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear_argmax launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_attention_decode(const int8_t *q, const int8_t *Kc, const int8_t *Vc, const int32_t *n_keys,
+                                     int32_t R, int32_t H, int32_t dh, int32_t T, float sigma, float rho,
+                                     int8_t *ctx, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!q || !Kc || !Vc || !n_keys || !ctx || R < 1 || H < 1 || H > 16 || T < 1 || T > 1024 ||
+        (dh != 32 && dh != 64 && dh != 128))
+        return fail(MNMT_EINVAL, "attention: bad shape R=%d H=%d dh=%d T=%d", R, H, dh, T);
+    AttnDecArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.q = q;
+    a.kc = Kc;
+    a.vc = Vc;
+    a.ctx = ctx;
+    a.R = R;
+    a.H = H;
+    a.dh = dh;
+    a.T = T;
+    a.beam = 1;
+    a.n_keys = n_keys;
+    a.sigma = sigma;
+    a.rho = rho;
+    cudaError_t err = launch_attention_decode(a, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "attention launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_layernorm(const float *r, const float *g, const float *b, int32_t M, int32_t d, float inv,
+                              float *out_f, int8_t *out_q, int32_t *status, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!r || !g || !b || M < 1 || d < 1 || d > 2048) return fail(MNMT_EINVAL, "layernorm: bad shape");
+    LnArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.r = r;
+    a.g = g;
+    a.b = b;
+    a.M = M;
+    a.d = d;
+    a.inv = inv;
+    a.out_f = out_f;
+    a.out_q = out_q;
+    a.status = status;
+    cudaError_t err = launch_layernorm(a, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "layernorm launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}

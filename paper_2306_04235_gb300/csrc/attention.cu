@@ -1,0 +1,267 @@
+// attention.cu -- scaled dot-product attention of the INT8 encoder-decoder
+// (App. A, Eq. 1/2) per head, with the quantisation points of Fig. 5b: int8 Q,
+// K, V and context; the softmax in full precision.
+//
+// Per head and query row: scores acc_j = q . k_j (exact int32, dp4a),
+// s_j = fl(acc_j * sigma), m = max_j s_j, weights E_j = rne(exp(fl(s_j - m)) 2^24)
+// (an integer in [0, 2^24]), context N_e = sum_j E_j v_j[e] and Z = sum_j E_j as
+// exact integer sums (so any summation order gives the same bits), then
+// ctx_e = q8(fl32(N_e / Z), rho).  N_e is accumulated in two int32 halves,
+// E_j = Eh 2^12 + El, which cannot overflow for up to 1024 keys.
+//
+// Kernels:
+//   attn_decode  one warp per (row, head): the incremental step of the decoder
+//                over the self-attention cache (keys 0..t, through the beam
+//                ancestry table when hypotheses were reordered) or over the
+//                cross-attention keys of the row's sentence.  Bound by the
+//                cache bytes it streams.
+//   attn_encoder one block per (sentence, head, 32-query chunk): K and V of
+//                the head staged in shared memory, keys masked past the
+//                source length.
+#include "common.cuh"
+#include "internal.h"
+
+namespace mnmt {
+
+constexpr int DEC_MAX_KEYS = 1024;
+
+template <int DH>
+__global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
+    if (a.skip && *a.skip) return;
+    extern __shared__ int dsm[];
+    const int r = blockIdx.x;
+    const int h = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int n, t = 0;
+    if (a.cross) {
+        n = a.src_len[r / a.beam];
+        n = n < 1 ? 1 : (n > a.T ? a.T : n);  // lengths are validated on the host path; clamp on the device path
+    } else if (a.n_keys) {
+        n = a.n_keys[r];
+        t = n - 1;
+    } else {
+        t = *a.t_ptr;
+        n = t + 1;
+    }
+    // physical row of every key position (shared by the heads of this row)
+    const int cap = a.T;                  // key capacity: cache length / padded source length
+    int *prow = dsm;                      // [cap]
+    int *sc = dsm + cap + h * cap;        // per head [cap]: scores, then weights
+    for (int j = threadIdx.x; j < n; j += blockDim.x) {
+        int p;
+        if (a.cross) p = r / a.beam;
+        else p = (a.anc && j < t) ? a.anc[(size_t)r * a.T + j] : r;
+        prow[j] = p;
+    }
+    __syncthreads();
+    if (h >= a.H) return;
+
+    constexpr int QC = DH / 16;
+    int4 qv[QC];
+    const int4 *qp = reinterpret_cast<const int4 *>(a.q + (size_t)r * a.H * DH + h * DH);
+#pragma unroll
+    for (int c = 0; c < QC; c++) qv[c] = qp[c];
+
+    float mx = -INFINITY;
+    for (int j = lane; j < n; j += 32) {
+        const int4 *kr = reinterpret_cast<const int4 *>(a.kc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH);
+        int acc = 0;
+#pragma unroll
+        for (int c = 0; c < QC; c++) acc = dot16(qv[c], kr[c], acc);
+        float s = __fmul_rn(__int2float_rn(acc), a.sigma);
+        sc[j] = __float_as_int(s);
+        mx = fmaxf(mx, s);
+    }
+    mx = warp_max_f(mx);
+    long long Z = 0;
+    for (int j = lane; j < n; j += 32) {
+        int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
+        sc[j] = E;
+        Z += E;
+    }
+    Z = warp_sum_ll(Z);
+    __syncwarp();
+
+    constexpr int EPL = DH / 32;  // context elements per lane
+    int hi[EPL], lo[EPL];
+#pragma unroll
+    for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
+    for (int j = 0; j < n; j++) {
+        int E = sc[j];
+        int Eh = E >> 12, El = E & 4095;
+        const int8_t *vr = a.vc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH + lane * EPL;
+        int v[EPL];
+        if constexpr (EPL == 1) {
+            v[0] = vr[0];
+        } else if constexpr (EPL == 2) {
+            char2 x = *reinterpret_cast<const char2 *>(vr);
+            v[0] = x.x;
+            v[1] = x.y;
+        } else {
+            char4 x = *reinterpret_cast<const char4 *>(vr);
+            v[0] = x.x;
+            v[1] = x.y;
+            v[2] = x.z;
+            v[3] = x.w;
+        }
+#pragma unroll
+        for (int u = 0; u < EPL; u++) {
+            hi[u] += Eh * v[u];
+            lo[u] += El * v[u];
+        }
+    }
+    int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + lane * EPL;
+    double dz = __ll2double_rn(Z);
+#pragma unroll
+    for (int u = 0; u < EPL; u++) {
+        long long N = (long long)hi[u] * 4096 + lo[u];
+        float c = __double2float_rn(__ddiv_rn(__ll2double_rn(N), dz));
+        out[u] = q8(c, a.rho);
+    }
+}
+
+cudaError_t launch_attention_decode(const AttnDecArgs &a, cudaStream_t st) {
+    if (a.H > 16 || a.T < 1 || a.T > DEC_MAX_KEYS) return cudaErrorInvalidValue;
+    size_t smem = (size_t)(1 + a.H) * a.T * sizeof(int);
+    dim3 block(32 * a.H);
+    switch (a.dh) {
+        case 32:
+            attn_decode<32><<<a.R, block, smem, st>>>(a);
+            break;
+        case 64:
+            attn_decode<64><<<a.R, block, smem, st>>>(a);
+            break;
+        case 128:
+            attn_decode<128><<<a.R, block, smem, st>>>(a);
+            break;
+        default:
+            return cudaErrorInvalidValue;
+    }
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// encoder self-attention
+// ---------------------------------------------------------------------------
+constexpr int ENC_WARPS = 4;
+constexpr int ENC_MAX_KEYS = 512;
+constexpr int ENC_QCHUNK = 32;
+
+template <int DH>
+__global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a) {
+    extern __shared__ __align__(16) uint8_t esm[];
+    constexpr int KS = DH + 16;  // padded key row: conflict-free 16-byte lane reads
+    const int bh = blockIdx.x;
+    const int b = bh / a.H, h = bh - b * a.H;
+    const int S = a.S;
+    int len = a.len[b];
+    len = len < 1 ? 1 : (len > S ? S : len);  // validated on the host path; clamp on the device path
+    uint8_t *Ks = esm;                         // [S][KS]
+    int8_t *Vs = reinterpret_cast<int8_t *>(esm + (size_t)S * KS);  // [S][DH]
+    int *wsm = reinterpret_cast<int *>(esm + (size_t)S * KS + (size_t)S * DH);  // [warps][S]
+    const int ld = 3 * a.d;
+    const int8_t *base = a.qkv + (size_t)b * S * ld;
+    // stage K and V of this head (valid keys only)
+    constexpr int CH = DH / 16;
+    for (int i = threadIdx.x; i < len * CH; i += blockDim.x) {
+        int j = i / CH, c = i - j * CH;
+        const int4 *src = reinterpret_cast<const int4 *>(base + (size_t)j * ld + a.d + h * DH);
+        reinterpret_cast<int4 *>(Ks + (size_t)j * KS)[c] = src[c];
+        const int4 *vsrc = reinterpret_cast<const int4 *>(base + (size_t)j * ld + 2 * a.d + h * DH);
+        reinterpret_cast<int4 *>(Vs + (size_t)j * DH)[c] = vsrc[c];
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int *sc = wsm + warp * S;
+    const int q0 = blockIdx.y * ENC_QCHUNK;
+    const int q1 = min(q0 + ENC_QCHUNK, S);
+    constexpr int EPL = DH / 32;
+    for (int qi = q0 + warp; qi < q1; qi += ENC_WARPS) {
+        int4 qv[CH];
+        const int4 *qp = reinterpret_cast<const int4 *>(base + (size_t)qi * ld + h * DH);
+#pragma unroll
+        for (int c = 0; c < CH; c++) qv[c] = qp[c];
+        float mx = -INFINITY;
+        for (int j = lane; j < len; j += 32) {
+            const int4 *kr = reinterpret_cast<const int4 *>(Ks + (size_t)j * KS);
+            int acc = 0;
+#pragma unroll
+            for (int c = 0; c < CH; c++) acc = dot16(qv[c], kr[c], acc);
+            float s = __fmul_rn(__int2float_rn(acc), a.sigma);
+            sc[j] = __float_as_int(s);
+            mx = fmaxf(mx, s);
+        }
+        mx = warp_max_f(mx);
+        long long Z = 0;
+        for (int j = lane; j < len; j += 32) {
+            int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
+            sc[j] = E;
+            Z += E;
+        }
+        Z = warp_sum_ll(Z);
+        __syncwarp();
+        int hi[EPL], lo[EPL];
+#pragma unroll
+        for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
+        for (int j = 0; j < len; j++) {
+            int E = sc[j];
+            int Eh = E >> 12, El = E & 4095;
+            const int8_t *vr = Vs + (size_t)j * DH + lane * EPL;
+#pragma unroll
+            for (int u = 0; u < EPL; u++) {
+                int v = vr[u];
+                hi[u] += Eh * v;
+                lo[u] += El * v;
+            }
+        }
+        double dz = __ll2double_rn(Z);
+        int8_t *out = a.ctx + ((size_t)b * S + qi) * a.d + h * DH + lane * EPL;
+#pragma unroll
+        for (int u = 0; u < EPL; u++) {
+            long long N = (long long)hi[u] * 4096 + lo[u];
+            out[u] = q8(__double2float_rn(__ddiv_rn(__ll2double_rn(N), dz)), a.rho);
+        }
+        __syncwarp();
+    }
+}
+
+template <int DH>
+static cudaError_t launch_enc(const AttnEncArgs &a, cudaStream_t st) {
+    size_t smem = (size_t)a.S * (DH + 16) + (size_t)a.S * DH + (size_t)ENC_WARPS * a.S * sizeof(int);
+    auto k = attn_encoder<DH>;
+    dim3 grid(a.B * a.H, (a.S + ENC_QCHUNK - 1) / ENC_QCHUNK);
+    k<<<grid, 32 * ENC_WARPS, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_attention_encoder(const AttnEncArgs &a, cudaStream_t st) {
+    if (a.S < 1 || a.S > ENC_MAX_KEYS) return cudaErrorInvalidValue;
+    switch (a.dh) {
+        case 32:
+            return launch_enc<32>(a, st);
+        case 64:
+            return launch_enc<64>(a, st);
+        case 128:
+            return launch_enc<128>(a, st);
+        default:
+            return cudaErrorInvalidValue;
+    }
+}
+
+}  // namespace mnmt
+
+namespace mnmt {
+// Opt the attention kernels into the shared memory their largest shapes use
+// (called once per process before any launch or stream capture).
+cudaError_t attention_init() {
+    cudaError_t err = cudaSuccess;
+    int dec = (1 + 16) * DEC_MAX_KEYS * (int)sizeof(int);
+    if (!err) err = cudaFuncSetAttribute(attn_decode<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, dec);
+    if (!err) err = cudaFuncSetAttribute(attn_decode<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, dec);
+    if (!err) err = cudaFuncSetAttribute(attn_decode<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, dec);
+    auto enc = [](int dh) { return ENC_MAX_KEYS * (dh + 16) + ENC_MAX_KEYS * dh + ENC_WARPS * ENC_MAX_KEYS * 4; };
+    if (!err) err = cudaFuncSetAttribute(attn_encoder<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(32));
+    if (!err) err = cudaFuncSetAttribute(attn_encoder<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(64));
+    if (!err) err = cudaFuncSetAttribute(attn_encoder<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(128));
+    return err;
+}
+}  // namespace mnmt

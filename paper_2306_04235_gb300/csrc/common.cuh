@@ -1,0 +1,182 @@
+// common.cuh -- device arithmetic shared by the sm_103a kernels of libmnmt.
+//
+// Every float operation here is written with explicit round-to-nearest
+// intrinsics and the library is compiled with --fmad=false, so each a*b+c is
+// two IEEE roundings exactly as the method's arithmetic is defined (the int8
+// quantiser of App. B with zero point 0, the full-precision epilogues of Fig. 5,
+// the fixed-point LayerNorm and softmax sums).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mnmt.h"
+
+#define MNMT_DEV __device__ __forceinline__
+
+// ---------------------------------------------------------------------------
+// quantiser: q8(x, inv) = clamp(round_half_even(fl(x * inv)), -127, 127)
+// ---------------------------------------------------------------------------
+MNMT_DEV int8_t q8(float x, float inv) {
+    float t = rintf(__fmul_rn(x, inv));
+    t = fminf(fmaxf(t, -127.0f), 127.0f);
+    return (int8_t)__float2int_rz(t);
+}
+
+// dequantise + bias: y = fl(fl(acc * fl(s_x * s_w)) + b)
+MNMT_DEV float dequant_bias(int32_t acc, float s_x, float s_w, float b) {
+    float sc = __fmul_rn(s_x, s_w);
+    return __fadd_rn(__fmul_rn(__int2float_rn(acc), sc), b);
+}
+
+// ---------------------------------------------------------------------------
+// round_half_even(v * 2^shift) as int64, with integer operations only.  Equal
+// to llrint(ldexp((double)v, shift)) whenever |v| 2^shift < 2^62.
+// ---------------------------------------------------------------------------
+MNMT_DEV long long fx_scale(float v, int shift) {
+    uint32_t bits = __float_as_uint(v);
+    uint32_t ex = (bits >> 23) & 0xFFu;
+    uint32_t man = bits & 0x7FFFFFu;
+    int e;
+    if (ex == 0) {
+        e = -126 - 23;  // subnormal: value = man * 2^-149
+    } else {
+        man |= 0x800000u;
+        e = (int)ex - 127 - 23;  // value = man * 2^e
+    }
+    int s = e + shift;
+    long long q;
+    if (s >= 0) {
+        q = (long long)man << s;
+    } else if (s < -25) {
+        q = 0;  // man < 2^24: the value is below 1/2
+    } else {
+        int r = -s;
+        uint32_t qq = man >> r;
+        uint32_t rem = man & ((1u << r) - 1u);
+        uint32_t half = 1u << (r - 1);
+        if (rem > half || (rem == half && (qq & 1u))) qq++;
+        q = (long long)qq;
+    }
+    return (bits >> 31) ? -q : q;
+}
+
+// exponent e with |v| < 2^e (0 for v == 0), as frexpf
+MNMT_DEV int exp_bound(float v) {
+    int e = 0;
+    if (v != 0.0f) frexpf(v, &e);
+    return e;
+}
+
+// ---------------------------------------------------------------------------
+// e^x for x <= 0: Cody-Waite reduction with ln2 split into a 16-bit head and
+// a tail, degree-7 Taylor polynomial of e^r by Horner in fused multiply-adds,
+// scaled by 2^n through the exponent field; 0 below -87.
+// ---------------------------------------------------------------------------
+MNMT_DEV float exp_own(float x) {
+    if (x < -87.0f) return 0.0f;
+    float n = rintf(__fmul_rn(x, 0x1.715476p+0f));
+    float r = __fmaf_rn(-n, 0x1.62e4p-1f, x);
+    r = __fmaf_rn(-n, 0x1.7f7d1cp-20f, r);
+    float p = 0x1.a01a02p-13f;
+    p = __fmaf_rn(p, r, 0x1.6c16c2p-10f);
+    p = __fmaf_rn(p, r, 0x1.111112p-7f);
+    p = __fmaf_rn(p, r, 0x1.555556p-5f);
+    p = __fmaf_rn(p, r, 0x1.555556p-3f);
+    p = __fmaf_rn(p, r, 0.5f);
+    p = __fmaf_rn(p, r, 1.0f);
+    p = __fmaf_rn(p, r, 1.0f);
+    int ni = __float2int_rz(n);
+    float two_n = __uint_as_float((uint32_t)(ni + 127) << 23);
+    return __fmul_rn(p, two_n);
+}
+
+// softmax weight on the 2^-24 grid: rne(exp(x) * 2^24), x <= 0
+MNMT_DEV int32_t softmax_weight(float x) {
+    return __float2int_rn(__fmul_rn(exp_own(x), 16777216.0f));
+}
+
+// natural log in double for z >= 1: z = f 2^k, f in [sqrt(1/2), sqrt(2)),
+// ln f = 2 atanh(s), s = (f - 1)/(f + 1), odd series up to s^23.
+MNMT_DEV double log_own(double z) {
+    int k;
+    double f = frexp(z, &k);
+    if (f < 0x1.6a09e667f3bcdp-1) {
+        f = __dmul_rn(f, 2.0);
+        k = k - 1;
+    }
+    double s = __ddiv_rn(__dadd_rn(f, -1.0), __dadd_rn(f, 1.0));
+    double s2 = __dmul_rn(s, s);
+    double q = 0x1.642c8590b2164p-5;
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.8618618618618p-5);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.af286bca1af28p-5);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.e1e1e1e1e1e1ep-5);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.1111111111111p-4);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.3b13b13b13b14p-4);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.745d1745d1746p-4);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.c71c71c71c71cp-4);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.2492492492492p-3);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.999999999999ap-3);
+    q = __dadd_rn(__dmul_rn(q, s2), 0x1.5555555555555p-2);
+    q = __dadd_rn(__dmul_rn(q, s2), 1.0);
+    return __dadd_rn(__dmul_rn(__dmul_rn(2.0, s), q), __dmul_rn((double)k, 0x1.62e42fefa39efp-1));
+}
+
+// ---------------------------------------------------------------------------
+// Ordering keys: a float and an index packed so that unsigned max picks the
+// larger float, and between equal floats the lower index (-0 counts as +0).
+// ---------------------------------------------------------------------------
+MNMT_DEV uint32_t ordered_bits(float f) {
+    uint32_t u = __float_as_uint(__fadd_rn(f, 0.0f));  // -0 + 0 = +0
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+MNMT_DEV float from_ordered_bits(uint32_t o) {
+    uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+    return __uint_as_float(u);
+}
+MNMT_DEV unsigned long long pack_key(float f, uint32_t idx) {
+    return ((unsigned long long)ordered_bits(f) << 32) | (unsigned long long)(0xFFFFFFFFu - idx);
+}
+MNMT_DEV uint32_t key_index(unsigned long long k) { return 0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull); }
+MNMT_DEV float key_value(unsigned long long k) { return from_ordered_bits((uint32_t)(k >> 32)); }
+
+// ---------------------------------------------------------------------------
+// warp reductions
+// ---------------------------------------------------------------------------
+MNMT_DEV float warp_max_f(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
+    return v;
+}
+MNMT_DEV long long warp_sum_ll(long long v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+MNMT_DEV int warp_sum_i(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+MNMT_DEV unsigned long long warp_max_u64(unsigned long long v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        unsigned long long w = __shfl_xor_sync(0xFFFFFFFFu, v, o);
+        v = w > v ? w : v;
+    }
+    return v;
+}
+
+// dp4a over 16 bytes held as int4
+MNMT_DEV int dot16(int4 a, int4 b, int acc) {
+    acc = __dp4a(a.x, b.x, acc);
+    acc = __dp4a(a.y, b.y, acc);
+    acc = __dp4a(a.z, b.z, acc);
+    acc = __dp4a(a.w, b.w, acc);
+    return acc;
+}
+
+// device-side status word: first error wins
+MNMT_DEV void set_status(int *status, int code) {
+    if (status) atomicCAS(status, 0, code);
+}

@@ -1,0 +1,156 @@
+// internal.h -- types and kernel launchers shared by the translation units of
+// libmnmt (host code + sm_103a kernels).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/mnmt.h"
+
+namespace mnmt {
+
+// Epilogue of a quantised linear (Sec. 3.3, Fig. 5).  y = fl(fl(acc *
+// fl(s_x * s_w[n])) + bias[n]) then, per mode:
+enum EpiMode {
+    EPI_Q8 = 0,       // out[m*ldo + n] = q8(y, inv_out[n])
+    EPI_RELU_Q8 = 1,  // out[m*ldo + n] = q8(max(y, 0), inv_out[n])
+    EPI_RESID = 2,    // f32[m*ldf + n] = fl(fl(gamma * f32) + y)
+    EPI_F32 = 3,      // f32[m*ldf + n] = y
+    EPI_QKV_DEC = 4,  // n < d: out[m*ldo + n] = q8(y); n >= d: K / V cache at position *t_ptr
+    EPI_KV_CROSS = 5, // row m = b*S + s: K / V -> cross cache [b][H][S][dh]
+    EPI_ARGMAX = 6,   // keys[m] = max over n of pack_key(y, n)   (greedy vocabulary projection)
+};
+
+struct Epi {
+    int mode;
+    float s_x;
+    const float *s_w;
+    const float *bias;
+    const float *inv_out;
+    int8_t *out;
+    int ldo;
+    float *f32;
+    int ldf;
+    float gamma;
+    // caches (EPI_QKV_DEC: [R][H][T][dh]; EPI_KV_CROSS: [B][H][S][dh])
+    int8_t *kc, *vc;
+    const int *t_ptr;
+    int d, H, dh, T, S;
+    unsigned long long *keys;
+    const int *skip;  // if non-null and *skip != 0, the kernel does nothing
+};
+
+// ---- one-time kernel attribute set-up (before any launch or capture) ----
+cudaError_t linear_init();
+cudaError_t attention_init();
+cudaError_t rows_init();
+
+// ---- launchers (stream-ordered, no synchronisation) ----
+cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int N, int K, const Epi &e,
+                          cudaStream_t st);
+
+struct LnArgs {
+    const float *r;   // [M][d] input rows (row stride d)
+    float *out_f;     // optional fp32 output (may alias r)
+    int8_t *out_q;    // optional int8 output
+    const float *g, *b;
+    float inv;
+    int M, d;
+    int *status;
+    const int *skip;
+};
+cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st);
+
+struct EmbedArgs {
+    const int32_t *ids;   // [M] token ids, or nullptr to use tok (decoder)
+    const int32_t *tok;   // decoder tokens [M]
+    int S;                // encoder: row m is position m % S; decoder: position *t_ptr
+    const int *t_ptr;
+    const int8_t *emb_q;
+    const float *emb_s;
+    const int8_t *proj_w;  // factorised E -> d (nullptr if E == d)
+    const float *proj_s, *proj_b;
+    float emb_scale;
+    const float *pe;
+    int M, d, E, V;
+    float *r;              // fp32 [M][d] residual out
+    int8_t *out_q;         // int8 sublayer input out
+    const float *ln_g, *ln_b;  // if non-null: out_q = q8(LN(x), inv) else q8(x, inv)
+    float inv;
+    int *status;
+    const int *skip;
+};
+cudaError_t launch_embed(const EmbedArgs &a, cudaStream_t st);
+
+struct AttnDecArgs {
+    const int8_t *q;        // [R][d] (head h at h*dh)
+    const int8_t *kc, *vc;  // self: [R][H][T][dh]; cross: [B][H][S][dh]
+    int8_t *ctx;            // [R][d]
+    int R, H, dh, T;        // T = cache capacity (self) or S_pad (cross)
+    int cross;              // 0 = self (keys 0..t), 1 = cross (keys < src_len[r / beam])
+    int beam;
+    const int *t_ptr;       // self: current step (keys 0..t)
+    const int *n_keys;      // kernel-level entry: keys per row (overrides t_ptr)
+    const int *src_len;     // cross
+    const int *anc;         // self, beam > 1: [R][T] physical row of each position (or null)
+    float sigma, rho;
+    const int *skip;
+};
+cudaError_t launch_attention_decode(const AttnDecArgs &a, cudaStream_t st);
+
+struct AttnEncArgs {
+    const int8_t *qkv;  // [B*S][3d]: q | k | v
+    int8_t *ctx;        // [B*S][d]
+    const int *len;     // [B]
+    int B, S, H, dh, d;
+    float sigma, rho;
+};
+cudaError_t launch_attention_encoder(const AttnEncArgs &a, cudaStream_t st);
+
+// greedy: consume argmax keys, write history / next tokens / finished / done
+struct GreedyArgs {
+    unsigned long long *keys;  // [R], reset to 0 after reading
+    int32_t *tok;              // [R] next input token
+    int32_t *fin;              // [R]
+    int32_t *hist;             // [T][R]
+    int *t_ptr, *done;
+    const int *tmax_ptr;       // steps of this translation (device)
+    int R, T, eos, pad;
+};
+cudaError_t launch_greedy_update(const GreedyArgs &a, cudaStream_t st);
+
+// beam search: per-row log-softmax + top-k, then per-sentence selection
+struct BeamArgs {
+    const float *logits;       // [R][V]
+    int32_t *tok, *fin;        // [R]
+    float *cum;                // [R]
+    int32_t *hist, *parents;   // [T][R]
+    int32_t *anc;              // [R][T]
+    unsigned long long *cand;  // [R][k] row candidates
+    int *t_ptr, *done, *ticket;   // ticket[0..1]: arrival and running counters
+    const int *tmax_ptr;          // steps of this translation (device)
+    int B, k, V, T, eos, pad;     // T: cache / history capacity
+    int *status;
+};
+cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st);
+
+struct InitArgs {
+    int32_t *tok, *fin, *anc, *hist, *parents;
+    float *cum;
+    unsigned long long *keys;
+    int *t_ptr, *done, *ticket;
+    int R, k, T, bos, pad;
+};
+cudaError_t launch_search_init(const InitArgs &a, cudaStream_t st);
+
+struct FinalArgs {
+    const int32_t *hist, *parents;
+    const float *cum;
+    const int *t_ptr;
+    int32_t *out_ids, *out_lens;
+    float *out_scores;
+    int B, k, T, max_len, eos, pad;
+};
+cudaError_t launch_finalize(const FinalArgs &a, cudaStream_t st);
+
+}  // namespace mnmt

@@ -1,0 +1,468 @@
+// rows.cu -- row-wise kernels of the INT8 encoder-decoder: embedding gather
+// (+ factorised projection), LayerNorm + requantisation, and the search steps
+// (greedy argmax bookkeeping, beam log-softmax / top-k / reorder, init and
+// final backtracking).
+//
+// LayerNorm (App. A / App. D) keeps the mean and the biased variance as exact
+// fixed-point sums: each row's largest magnitude (an order-free maximum) sets a
+// power-of-two grid on which every term r_i 2^(52-ea) or c_i^2 2^(52-2eb) is an
+// integer below 2^52, accumulated in int64.  Any reduction tree therefore gives
+// the same mean and rstd bits.
+#include "common.cuh"
+#include "internal.h"
+
+namespace mnmt {
+
+// ---------------------------------------------------------------------------
+// warp LayerNorm over a row held as VPL values per lane (element u*32 + lane)
+// ---------------------------------------------------------------------------
+template <int VPL>
+MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restrict__ g,
+                             const float *__restrict__ b, float (&out)[VPL], int lane) {
+    float amax = 0.0f;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) amax = fmaxf(amax, fabsf(x[u]));
+    amax = warp_max_f(amax);
+    if (!(amax < 0x1p32f)) return false;
+    const int ea = exp_bound(amax);
+    long long s1 = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
+    s1 = warp_sum_ll(s1);
+    const float mu = __double2float_rn(__ddiv_rn(ldexp(__ll2double_rn(s1), ea - 52), (double)d));
+    float c[VPL];
+    float bmax = 0.0f;
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        c[u] = __fsub_rn(x[u], mu);
+        if (u * 32 + lane < d) bmax = fmaxf(bmax, fabsf(c[u]));
+    }
+    bmax = warp_max_f(bmax);
+    const int eb = exp_bound(bmax);
+    long long s2 = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
+    s2 = warp_sum_ll(s2);
+    const double var = __ddiv_rn(ldexp(__ll2double_rn(s2), 2 * eb - 52), (double)d);
+    const float rstd = __double2float_rn(__ddiv_rn(1.0, __dsqrt_rn(__dadd_rn(var, 1e-5))));
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        int i = u * 32 + lane;
+        if (i < d) out[u] = __fadd_rn(__fmul_rn(__fmul_rn(c[u], rstd), g[i]), b[i]);
+    }
+    return true;
+}
+
+// ---------------------------------------------------------------------------
+// LayerNorm kernel: one warp per row
+// ---------------------------------------------------------------------------
+template <int VPL>
+__global__ void __launch_bounds__(256) layernorm_kernel(LnArgs a) {
+    if (a.skip && *a.skip) return;
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= a.M) return;
+    const float *r = a.r + (size_t)row * a.d;
+    float x[VPL], y[VPL];
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        int i = u * 32 + lane;
+        x[u] = i < a.d ? r[i] : 0.0f;
+    }
+    if (!warp_layernorm<VPL>(x, a.d, a.g, a.b, y, lane)) {
+        if (lane == 0) set_status(a.status, MNMT_EOVERFLOW);
+        return;
+    }
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        int i = u * 32 + lane;
+        if (i < a.d) {
+            if (a.out_f) a.out_f[(size_t)row * a.d + i] = y[u];
+            if (a.out_q) a.out_q[(size_t)row * a.d + i] = q8(y[u], a.inv);
+        }
+    }
+}
+
+cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
+    if (a.M <= 0) return cudaSuccess;
+    dim3 grid((a.M + 7) / 8), block(256);
+    int vpl = (a.d + 31) / 32;
+    if (vpl <= 4) layernorm_kernel<4><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 8) layernorm_kernel<8><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 16) layernorm_kernel<16><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 32) layernorm_kernel<32><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 64) layernorm_kernel<64><<<grid, block, 0, st>>>(a);
+    else return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// embedding: one warp per row.  x = fl(fl(dequant(Eq[id]) * emb_scale) + PE[pos])
+// (factorised: the E-dim int8 row feeds the E -> d linear, its row scale folded
+// into the dequantisation), then r = x and the first sublayer's input
+// q8(LN(x)) (pre-LN) or q8(x) (post-LN).
+// ---------------------------------------------------------------------------
+template <int VPL>
+__global__ void __launch_bounds__(256) embed_kernel(EmbedArgs a) {
+    if (a.skip && *a.skip) return;
+    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= a.M) return;
+    int id = a.ids ? a.ids[row] : a.tok[row];
+    const int pos = a.ids ? row % a.S : *a.t_ptr;
+    if (id < 0 || id >= a.V) {
+        if (lane == 0) set_status(a.status, MNMT_EINVAL);
+        id = 0;
+    }
+    const float es = a.emb_s[id];
+    const float *pe = a.pe + (size_t)pos * a.d;
+    float x[VPL];
+    if (!a.proj_w) {
+        const int8_t *q = a.emb_q + (size_t)id * a.E;
+#pragma unroll
+        for (int u = 0; u < VPL; u++) {
+            int i = u * 32 + lane;
+            if (i < a.d) {
+                float t = __fmul_rn(__fmul_rn((float)q[i], es), a.emb_scale);
+                x[u] = __fadd_rn(t, pe[i]);
+            } else {
+                x[u] = 0.0f;
+            }
+        }
+    } else {
+        const int4 *q = reinterpret_cast<const int4 *>(a.emb_q + (size_t)id * a.E);
+        const int ec = a.E / 16;
+#pragma unroll
+        for (int u = 0; u < VPL; u++) {
+            int n = u * 32 + lane;
+            x[u] = 0.0f;
+            if (n < a.d) {
+                const int4 *w = reinterpret_cast<const int4 *>(a.proj_w + (size_t)n * a.E);
+                int acc = 0;
+                for (int c = 0; c < ec; c++) acc = dot16(q[c], w[c], acc);
+                float y = dequant_bias(acc, es, a.proj_s[n], a.proj_b[n]);
+                x[u] = __fadd_rn(__fmul_rn(y, a.emb_scale), pe[n]);
+            }
+        }
+    }
+    float y[VPL];
+    bool ok = true;
+    if (a.ln_g) ok = warp_layernorm<VPL>(x, a.d, a.ln_g, a.ln_b, y, lane);
+    if (!ok) {
+        if (lane == 0) set_status(a.status, MNMT_EOVERFLOW);
+        return;
+    }
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        int i = u * 32 + lane;
+        if (i < a.d) {
+            a.r[(size_t)row * a.d + i] = x[u];
+            a.out_q[(size_t)row * a.d + i] = q8(a.ln_g ? y[u] : x[u], a.inv);
+        }
+    }
+}
+
+cudaError_t launch_embed(const EmbedArgs &a, cudaStream_t st) {
+    if (a.M <= 0) return cudaSuccess;
+    dim3 grid((a.M + 7) / 8), block(256);
+    int vpl = (a.d + 31) / 32;
+    if (vpl <= 4) embed_kernel<4><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 8) embed_kernel<8><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 16) embed_kernel<16><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 32) embed_kernel<32><<<grid, block, 0, st>>>(a);
+    else if (vpl <= 64) embed_kernel<64><<<grid, block, 0, st>>>(a);
+    else return cudaErrorInvalidValue;
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// search state
+// ---------------------------------------------------------------------------
+__global__ void search_init_kernel(InitArgs a) {
+    int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < a.R) {
+        a.tok[i] = a.bos;
+        a.fin[i] = 0;
+        a.cum[i] = (i % a.k == 0) ? 0.0f : -INFINITY;  // only beam 0 of a sentence starts live
+        a.keys[i] = 0ull;
+    }
+    for (int j = i; j < a.R * a.T; j += gridDim.x * blockDim.x) {
+        a.anc[j] = j / a.T;
+        a.hist[j] = a.pad;
+        a.parents[j] = 0;
+    }
+    if (i == 0) {
+        *a.t_ptr = 0;
+        *a.done = 0;
+        a.ticket[0] = 0;
+        a.ticket[1] = 0;
+    }
+}
+
+cudaError_t launch_search_init(const InitArgs &a, cudaStream_t st) {
+    int n = a.R * a.T;
+    int blocks = (n + 255) / 256;
+    if (blocks < 1) blocks = 1;
+    if (blocks > 1024) blocks = 1024;
+    search_init_kernel<<<blocks, 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+// greedy: argmax key -> token; after EOS a sentence emits PAD
+__global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
+    if (*a.done) return;
+    const int t = *a.t_ptr;
+    int fin_all = 1;
+    for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
+        unsigned long long k = a.keys[r];
+        a.keys[r] = 0ull;
+        int y = (int)key_index(k);
+        int f = a.fin[r];
+        int out = f ? a.pad : y;
+        a.hist[(size_t)t * a.R + r] = out;
+        a.tok[r] = out;
+        if (!f && y == a.eos) f = 1;
+        a.fin[r] = f;
+        fin_all &= f;
+    }
+    int all = __syncthreads_and(fin_all);
+    if (threadIdx.x == 0) {
+        if (all || t + 1 >= *a.tmax_ptr) *a.done = 1;
+        *a.t_ptr = t + 1;
+    }
+}
+
+cudaError_t launch_greedy_update(const GreedyArgs &a, cudaStream_t st) {
+    int threads = a.R < 1024 ? ((a.R + 31) / 32) * 32 : 1024;
+    greedy_update_kernel<<<1, threads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// beam search (width k <= 16)
+// ---------------------------------------------------------------------------
+constexpr int BEAM_MAX = 16;
+constexpr int BR_THREADS = 256;
+
+// insert key into the descending list lst[0..k) (keys are unique): the key is
+// carried down the list, swapping with every smaller entry
+template <int KM>
+MNMT_DEV void topk_insert(unsigned long long (&lst)[KM], int k, unsigned long long key) {
+#pragma unroll
+    for (int i = 0; i < KM; i++) {
+        if (i < k && key > lst[i]) {
+            unsigned long long tmp = lst[i];
+            lst[i] = key;
+            key = tmp;
+        }
+    }
+}
+
+template <int KM>
+__global__ void __launch_bounds__(BR_THREADS) beam_rows_kernel(BeamArgs a) {
+    if (*a.done) return;
+    const int r = blockIdx.x;
+    const int k = a.k;
+    const int V = a.V;
+    const int lb = r % k;  // beam index within the sentence
+    unsigned long long *out = a.cand + (size_t)r * k;
+    __shared__ float s_m;
+    __shared__ float s_lam;
+    __shared__ long long s_z[BR_THREADS / 32];
+    __shared__ float s_mx[BR_THREADS / 32];
+    __shared__ unsigned long long s_key[BR_THREADS / 32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (a.fin[r]) {
+        // a finished hypothesis offers itself once, unchanged, with token PAD
+        for (int i = threadIdx.x; i < k; i += BR_THREADS)
+            out[i] = i == 0 ? pack_key(a.cum[r], (uint32_t)(lb * V + a.pad)) : 0ull;
+        return;
+    }
+    const float *l = a.logits + (size_t)r * V;
+    float mx = -INFINITY;
+    for (int n = threadIdx.x; n < V; n += BR_THREADS) mx = fmaxf(mx, l[n]);
+    mx = warp_max_f(mx);
+    if (lane == 0) s_mx[warp] = mx;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float m = s_mx[0];
+        for (int w = 1; w < BR_THREADS / 32; w++) m = fmaxf(m, s_mx[w]);
+        s_m = m;
+    }
+    __syncthreads();
+    const float m = s_m;
+    long long z = 0;
+    for (int n = threadIdx.x; n < V; n += BR_THREADS) z += softmax_weight(__fsub_rn(l[n], m));
+    z = warp_sum_ll(z);
+    if (lane == 0) s_z[warp] = z;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        long long Z = 0;
+        for (int w = 0; w < BR_THREADS / 32; w++) Z += s_z[w];
+        // lambda = ln Z - 24 ln 2 (log of the normaliser of the 2^-24 weights)
+        s_lam = __double2float_rn(__dadd_rn(log_own(__ll2double_rn(Z)), -0x1.0a2b23f3bab73p+4));
+    }
+    __syncthreads();
+    const float lam = s_lam;
+    const float cum = a.cum[r];
+    unsigned long long lst[KM];
+#pragma unroll
+    for (int i = 0; i < KM; i++) lst[i] = 0ull;
+    for (int n = threadIdx.x; n < V; n += BR_THREADS) {
+        float lp = __fsub_rn(__fsub_rn(l[n], m), lam);
+        float sc = __fadd_rn(cum, lp);
+        topk_insert<KM>(lst, k, pack_key(sc, (uint32_t)(lb * V + n)));
+    }
+    // block-wide selection of the k best: k rounds of a max over list heads
+    int head = 0;
+    for (int i = 0; i < k; i++) {
+        unsigned long long mine = 0ull;
+#pragma unroll
+        for (int h = 0; h < KM; h++)
+            if (h == head && h < k) mine = lst[h];
+        unsigned long long w = warp_max_u64(mine);
+        if (lane == 0) s_key[warp] = w;
+        __syncthreads();
+        unsigned long long best = s_key[0];
+        for (int j = 1; j < BR_THREADS / 32; j++) best = s_key[j] > best ? s_key[j] : best;
+        if (mine == best && best != 0ull) head++;
+        if (threadIdx.x == 0) out[i] = best;
+        __syncthreads();
+    }
+}
+
+// per sentence: best k of the k*k row candidates; reorder state
+__global__ void __launch_bounds__(256) beam_select_kernel(BeamArgs a) {
+    if (*a.done) return;
+    const int b = blockIdx.x;
+    const int k = a.k, V = a.V, T = a.T;
+    const int t = *a.t_ptr;
+    __shared__ unsigned long long cand[BEAM_MAX * BEAM_MAX];
+    __shared__ unsigned long long sel[BEAM_MAX];
+    __shared__ int pfin[BEAM_MAX];
+    __shared__ int s_all;
+    extern __shared__ int anc_old[];  // [k][T]
+    const int r0 = b * k;
+    for (int i = threadIdx.x; i < k * k; i += blockDim.x) cand[i] = a.cand[(size_t)r0 * k + i];
+    for (int i = threadIdx.x; i < k; i += blockDim.x) pfin[i] = a.fin[r0 + i];
+    for (int i = threadIdx.x; i < k * t; i += blockDim.x) {
+        int rr = i / t, j = i - rr * t;
+        anc_old[rr * T + j] = a.anc[(size_t)(r0 + rr) * T + j];
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        // k rounds of selection over k*k keys (unique keys, descending)
+        for (int i = 0; i < k; i++) {
+            unsigned long long best = 0ull;
+            int bi = 0;
+            for (int j = 0; j < k * k; j++)
+                if (cand[j] > best) {
+                    best = cand[j];
+                    bi = j;
+                }
+            sel[i] = best;
+            cand[bi] = 0ull;
+        }
+        int all = 1;
+        for (int i = 0; i < k; i++) {
+            uint32_t idx = key_index(sel[i]);
+            int p = (int)(idx / (uint32_t)V), n = (int)(idx - (uint32_t)p * V);
+            int f = pfin[p] || n == a.eos;
+            all &= f;
+        }
+        s_all = all;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < k; i += blockDim.x) {
+        unsigned long long key = sel[i];
+        uint32_t idx = key_index(key);
+        int p = (int)(idx / (uint32_t)V), n = (int)(idx - (uint32_t)p * V);
+        int r = r0 + i;
+        a.cum[r] = key_value(key);
+        a.fin[r] = pfin[p] || n == a.eos;
+        a.tok[r] = n;
+        a.hist[(size_t)t * (a.B * k) + r] = n;
+        a.parents[(size_t)t * (a.B * k) + r] = p;
+    }
+    // ancestry: new row i takes parent p's positions 0..t-1 and p's own slot at t
+    for (int x = threadIdx.x; x < k * (t + 1); x += blockDim.x) {
+        int i = x / (t + 1), j = x - i * (t + 1);
+        uint32_t idx = key_index(sel[i]);
+        int p = (int)(idx / (uint32_t)V);
+        a.anc[(size_t)(r0 + i) * T + j] = (j < t) ? anc_old[p * T + j] : r0 + p;
+    }
+    // the last block to finish decides whether every sentence is done
+    __shared__ int s_last;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        if (!s_all) atomicAdd(a.ticket + 1, 1);  // sentences still running
+        int prev = atomicAdd(a.ticket, 1);
+        s_last = prev == (int)gridDim.x - 1;
+    }
+    __syncthreads();
+    if (s_last && threadIdx.x == 0) {
+        __threadfence();
+        int running = atomicAdd(a.ticket + 1, 0);
+        if (running == 0 || t + 1 >= *a.tmax_ptr) *a.done = 1;
+        a.ticket[0] = 0;
+        a.ticket[1] = 0;
+        *a.t_ptr = t + 1;
+    }
+}
+
+cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
+    if (a.k < 1 || a.k > BEAM_MAX) return cudaErrorInvalidValue;
+    int R = a.B * a.k;
+    if (a.k <= 4) beam_rows_kernel<4><<<R, BR_THREADS, 0, st>>>(a);
+    else if (a.k <= 8) beam_rows_kernel<8><<<R, BR_THREADS, 0, st>>>(a);
+    else beam_rows_kernel<16><<<R, BR_THREADS, 0, st>>>(a);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    size_t smem = (size_t)a.k * a.T * sizeof(int);
+    beam_select_kernel<<<a.B, 256, smem, st>>>(a);
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// final outputs: best hypothesis of each sentence (beam 0 after the last step),
+// backtracked through the parent pointers
+// ---------------------------------------------------------------------------
+__global__ void finalize_kernel(FinalArgs a) {
+    const int b = blockIdx.x;
+    if (threadIdx.x != 0) return;
+    const int steps = *a.t_ptr;
+    const int R = a.B * a.k;
+    int r = b * a.k;
+    // walk back from the last step, writing tokens in reverse
+    for (int t = steps - 1; t >= 0; t--) {
+        a.out_ids[(size_t)b * a.max_len + t] = a.hist[(size_t)t * R + r];
+        if (a.k > 1) r = b * a.k + a.parents[(size_t)t * R + r];
+    }
+    int n = steps;
+    for (int t = 0; t < steps; t++)
+        if (a.out_ids[(size_t)b * a.max_len + t] == a.eos) {
+            n = t + 1;
+            break;
+        }
+    for (int t = n; t < a.max_len; t++) a.out_ids[(size_t)b * a.max_len + t] = a.pad;
+    a.out_lens[b] = n;
+    a.out_scores[b] = a.k > 1 ? a.cum[b * a.k] : 0.0f;
+}
+
+// Opt the beam reorder kernel into the shared memory of its largest shape
+// (k = 16 hypotheses x 1024 positions); once per process, before any capture.
+cudaError_t rows_init() {
+    return cudaFuncSetAttribute(beam_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                BEAM_MAX * 1024 * (int)sizeof(int));
+}
+
+cudaError_t launch_finalize(const FinalArgs &a, cudaStream_t st) {
+    finalize_kernel<<<a.B, 32, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace mnmt

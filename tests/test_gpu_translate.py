@@ -1,0 +1,210 @@
+"""End-to-end parity of the translation path (C ABI, sm_103a kernels) against the
+CPU oracle: identical token sequences, lengths and beam scores, and bit-exact
+intermediate taps (encoder output, cross-attention keys/values, self-attention
+cache, decoder output), on the seeded synthetic workloads at full size (sampled
+sentences where the oracle is slow) and on small models that span the
+configuration space (pre/post-LN, factorised/tied embedding, greedy/beam)."""
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2306_04235_gb300 import mnmt, synth
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+MINI = {
+    "pre": synth.ModelConfig(2, 2, 64, 2, 128, 300, 64, 1, 1, max_pos=64),
+    "post": synth.ModelConfig(2, 1, 64, 1, 128, 300, 64, 0, 1, max_pos=64),
+    "fact": synth.ModelConfig(3, 2, 128, 4, 256, 500, 32, 1, 0, max_pos=96),
+    "wide-head": synth.ModelConfig(1, 2, 256, 2, 256, 400, 256, 1, 1, max_pos=64),
+}
+
+
+@pytest.fixture(scope="module")
+def stream():
+    return torch.cuda.Stream()
+
+
+def _gpu(blob, ids, lens, beam, max_len, stream, max_batch=None, max_src=None):
+    tr = mnmt.Translator(blob, max_batch or ids.shape[0], max_src or ids.shape[1], beam, max_len, stream)
+    try:
+        out = tr.translate(ids, lens, max_len)
+    finally:
+        tr.close()
+    return out
+
+
+@pytest.mark.parametrize("kind", list(MINI))
+@pytest.mark.parametrize("beam", [1, 3])
+def test_small_models_match_oracle(kind, beam, stream):
+    cfg = MINI[kind]
+    blob = synth.build_blob(cfg, 21, gamma_range=(0.5, 1.5))
+    ids, lens = synth.source_batch(cfg.vocab, 5, 1, 40, 22)
+    T = 24
+    g_ids, g_len, g_sc = _gpu(blob, ids, lens, beam, T, stream)
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, beam, T, n_threads=5)
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_len, o_len)
+    assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
+
+
+def test_tiny_workload_tokens_and_taps(stream):
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("tiny-b1-s16-greedy16")
+    d, H, L = cfg.d_model, cfg.n_heads, cfg.n_dec
+    dh = d // H
+    tr = mnmt.Translator(blob, 1, ids.shape[1], beam, T, stream)
+    try:
+        out, olen, _ = tr.translate(ids, lens, T)
+        S = ids.shape[1]
+        enc = mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_ENC_OUT, 0, np.int8, (1, S, d))
+        ck = [mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_CROSS_K, l, np.int8, (1, H, S, dh)) for l in range(L)]
+        cv = [mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_CROSS_V, l, np.int8, (1, H, S, dh)) for l in range(L)]
+        sk = [mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_SELF_K, l, np.int8, (1, H, T, dh)) for l in range(L)]
+        sv = [mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_SELF_V, l, np.int8, (1, H, T, dh)) for l in range(L)]
+        dec = mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_DEC_OUT, 0, np.int8, (1, d))
+    finally:
+        tr.close()
+    ref, rlen, _ = O.translate(blob, ids, lens, beam, T)
+    assert np.array_equal(out, ref) and np.array_equal(olen, rlen)
+    e_q, e_k, e_v = O.encode(blob, ids[0], lens[0], cfg)
+    assert np.array_equal(enc[0], e_q)
+    for l in range(L):
+        assert np.array_equal(ck[l][0].transpose(1, 0, 2).reshape(S, d), e_k[l])
+        assert np.array_equal(cv[l][0].transpose(1, 0, 2).reshape(S, d), e_v[l])
+    n = int(olen[0])
+    tgt = np.concatenate([[cfg.bos_id], out[0, :n - 1]]).astype(np.int32)
+    logits, dec_q, self_k, self_v = O.decode_trace(blob, ids[0], lens[0], tgt, cfg, want_cache=True)
+    assert np.array_equal(dec, dec_q[n - 1:n])
+    for l in range(L):
+        assert np.array_equal(sk[l][0, :, :n].transpose(1, 0, 2).reshape(n, d), self_k[l])
+        assert np.array_equal(sv[l][0, :, :n].transpose(1, 0, 2).reshape(n, d), self_v[l])
+
+
+def test_small_batch1_workload_matches_oracle(stream):
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("small-b1-s10to50-greedy64")
+    g = _gpu(blob, ids, lens, beam, T, stream)
+    o = O.translate(blob, ids, lens, beam, T)
+    assert np.array_equal(g[0], o[0]) and np.array_equal(g[1], o[1])
+
+
+def test_paper_shape_src30_tgt30(stream):
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("small-b1-s30-greedy30")
+    g = _gpu(blob, ids, lens, beam, T, stream)
+    o = O.translate(blob, ids, lens, beam, T)
+    assert np.array_equal(g[0], o[0]) and np.array_equal(g[1], o[1])
+
+
+def test_small_batched_beam_workload_sampled(stream):
+    """Batch 32, beam 4, 128 steps at full size; the oracle checks 4 sentences."""
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("small-b32-s10to80-beam4-t128")
+    g_ids, g_len, g_sc = _gpu(blob, ids, lens, beam, T, stream)
+    pick = [0, 9, 17, 31]
+    o_ids, o_len, o_sc = O.translate(blob, ids[pick], lens[pick], beam, T, n_threads=4)
+    assert np.array_equal(g_ids[pick], o_ids)
+    assert np.array_equal(g_len[pick], o_len)
+    assert np.array_equal(g_sc[pick].view(np.uint32), o_sc.view(np.uint32))
+
+
+def test_wide_batched_beam_workload_sampled(stream):
+    """Batch 128, beam 4, 160 steps at full size; the oracle checks 2 sentences."""
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("wide-b128-s20to128-beam4-t160")
+    g_ids, g_len, g_sc = _gpu(blob, ids, lens, beam, T, stream)
+    pick = [5, 127]
+    o_ids, o_len, o_sc = O.translate(blob, ids[pick], lens[pick], beam, T, n_threads=2)
+    assert np.array_equal(g_ids[pick], o_ids)
+    assert np.array_equal(g_len[pick], o_len)
+    assert np.array_equal(g_sc[pick].view(np.uint32), o_sc.view(np.uint32))
+
+
+def test_longest_source(stream):
+    cfg = synth.MODELS["small-12x2-d256-v32k-e128"]
+    blob = synth.build_blob(cfg, 1)
+    ids, lens = synth.source_batch(cfg.vocab, 2, 500, 512, 33)
+    ids = np.pad(ids, ((0, 0), (0, 512 - ids.shape[1])))
+    g = _gpu(blob, ids, lens, 1, 6, stream)
+    o = O.translate(blob, ids, lens, 1, 6, n_threads=2)
+    assert np.array_equal(g[0], o[0])
+
+
+@pytest.mark.parametrize("beam", [1, 4])
+def test_forced_eos_stops_at_once(beam, stream):
+    cfg = MINI["pre"]
+    blob = synth.build_blob(cfg, 3, out_bias={cfg.eos_id: 1000.0})
+    ids, lens = synth.source_batch(cfg.vocab, 3, 2, 9, 4)
+    g_ids, g_len, _ = _gpu(blob, ids, lens, beam, 20, stream)
+    assert np.all(g_len == 1) and np.all(g_ids[:, 0] == cfg.eos_id) and np.all(g_ids[:, 1:] == cfg.pad_id)
+
+
+@pytest.mark.parametrize("beam", [1, 3])
+def test_decode_step_api_matches_translate(beam, stream):
+    cfg = MINI["fact"]
+    blob = synth.build_blob(cfg, 8)
+    ids, lens = synth.source_batch(cfg.vocab, 2, 3, 20, 9)
+    T = 12
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, beam, T, n_threads=2)
+    tr = mnmt.Translator(blob, 2, ids.shape[1], beam, T, stream)
+    try:
+        mnmt.mnmt_encode(tr.session, ids, lens, 2, ids.shape[1])
+        toks, pars = [], []
+        for t in range(T):
+            tok, par, sc, done = mnmt.mnmt_decode_step(tr.session, 2 * beam)
+            toks.append(tok); pars.append(par)
+            if done:
+                break
+        with pytest.raises(mnmt.MnmtError):
+            for _ in range(T + 1):
+                mnmt.mnmt_decode_step(tr.session, 2 * beam)
+    finally:
+        tr.close()
+    # backtrack beam 0 of each sentence through the parents
+    for b in range(2):
+        r = 0
+        seq = []
+        for t in range(len(toks) - 1, -1, -1):
+            seq.append(toks[t][b * beam + r])
+            r = pars[t][b * beam + r] if beam > 1 else 0
+        seq = seq[::-1]
+        n = int(o_len[b])
+        assert seq[:n] == list(o_ids[b, :n])
+
+
+def test_device_pointer_path_equals_host_path(stream):
+    cfg = MINI["pre"]
+    blob = synth.build_blob(cfg, 5)
+    ids, lens = synth.source_batch(cfg.vocab, 4, 2, 30, 6)
+    T = 16
+    tr = mnmt.Translator(blob, 4, ids.shape[1], 2, T, stream)
+    try:
+        h = tr.translate(ids, lens, T)
+        d_ids, d_lens = torch.from_numpy(ids).cuda(), torch.from_numpy(lens).cuda()
+        o_ids = torch.zeros((4, T), dtype=torch.int32, device="cuda")
+        o_len = torch.zeros(4, dtype=torch.int32, device="cuda")
+        o_sc = torch.zeros(4, dtype=torch.float32, device="cuda")
+        torch.cuda.synchronize()
+        mnmt.mnmt_translate(tr.session, d_ids, d_lens, 4, ids.shape[1], T, mnmt.DEVICE_PTRS, o_ids, o_len, o_sc)
+        stream.synchronize()
+        assert np.array_equal(o_ids.cpu().numpy(), h[0]) and np.array_equal(o_len.cpu().numpy(), h[1])
+        assert np.array_equal(o_sc.cpu().numpy(), h[2])
+    finally:
+        tr.close()
+
+
+def test_bad_inputs_are_rejected(stream):
+    cfg = MINI["pre"]
+    blob = synth.build_blob(cfg, 5)
+    tr = mnmt.Translator(blob, 2, 10, 1, 8, stream)
+    try:
+        ids = np.full((2, 10), 5, np.int32)
+        with pytest.raises(mnmt.MnmtError) as ei:
+            tr.translate(ids, np.array([3, 11], np.int32), 8)       # length beyond S_pad
+        assert ei.value.code == mnmt.EINVAL
+        bad = ids.copy(); bad[1, 2] = cfg.vocab
+        with pytest.raises(mnmt.MnmtError):
+            tr.translate(bad, np.array([3, 4], np.int32), 8)         # id outside the vocabulary
+        with pytest.raises(mnmt.MnmtError):
+            tr.translate(np.full((3, 10), 5, np.int32), np.array([3, 4, 5], np.int32), 8)  # batch > capacity
+        out = tr.translate(ids, np.array([3, 4], np.int32), 8)      # session still usable
+        assert out[0].shape == (2, 8)
+    finally:
+        tr.close()
