@@ -202,6 +202,23 @@ int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, const float 
 int mnmt_linear_argmax(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                        int32_t M, int32_t N, int32_t K, uint64_t *keys, void *cuda_stream);
 
+/* The call above without any caller-provided scratch, for callers that cannot
+ * allocate device memory (their device memory is owned by another allocator or
+ * a fixed budget, or they run on a latency-critical thread where cudaMalloc's
+ * implicit synchronisation is not acceptable).  The paper has no counterpart:
+ * this is a deployment variant of the fused vocabulary projection + argmax.
+ * ids [M] (int32, device) receives the argmax id of each row, ties to the
+ * lowest id; A, W, s_w, bias as in mnmt_linear_argmax.  The packed keys live in
+ * a library-owned 32 KB device array (4096 rows), so M must be in [1, 4096]
+ * (MNMT_EINVAL otherwise).  Nothing is allocated: the array is part of the
+ * loaded library on every GPU that uses it, until the process exits.  The
+ * first call on a device looks up the array's address and sets up the GEMM
+ * kernels on that device; make that first call before any stream capture.
+ * Every call shares the one array: calls whose GPU work overlaps (different
+ * streams or threads without ordering) race and may return wrong ids. */
+int mnmt_linear_argmax_ids_noalloc(const int8_t *A, const int8_t *W, const float *s_w, const float *bias,
+                                   float s_x, int32_t M, int32_t N, int32_t K, int32_t *ids, void *cuda_stream);
+
 /* Incremental attention (Eq. 1/2 per head) of R query rows over per-row
  * caches: q [R][H][dh], Kc/Vc [R][H][T][dh] int8; row r attends keys
  * j < n_keys[r] (1 <= n_keys[r] <= T <= 1024).  Scores acc_j = q.k_j (int32),

@@ -1098,6 +1098,8 @@ extern "C" int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, v
 
 extern "C" const char *mnmt_last_error(void) { return g_err.c_str(); }
 
+int mnmt::set_error(int code, const char *msg) { return fail(code, "%s", msg); }
+
 // ---------------------------------------------------------------------------
 // kernel-level entry points
 // ---------------------------------------------------------------------------

@@ -40,6 +40,9 @@ struct Epi {
     const int *skip;  // if non-null and *skip != 0, the kernel does nothing
 };
 
+// records msg as the calling thread's mnmt_last_error() and returns code
+int set_error(int code, const char *msg);
+
 // ---- one-time kernel attribute set-up (before any launch or capture) ----
 cudaError_t linear_init();
 cudaError_t attention_init();

@@ -70,6 +70,8 @@ def _declare(L):
     L.mnmt_last_error.argtypes = []; L.mnmt_last_error.restype = C.c_char_p
     L.mnmt_linear.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p]
     L.mnmt_linear_argmax.argtypes = [p, p, p, p, f, i32, i32, i32, p, p]
+    L.mnmt_linear_argmax_ids_noalloc.argtypes = [p, p, p, p, f, i32, i32, i32, p, p]
+    L.mnmt_linear_argmax_ids_noalloc.restype = C.c_int
     L.mnmt_attention_decode.argtypes = [p, p, p, p, i32, i32, i32, i32, f, f, p, p]
     L.mnmt_layernorm.argtypes = [p, p, p, i32, i32, f, p, p, p, p]
     for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
@@ -174,6 +176,12 @@ def mnmt_linear(A, W, s_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_q, out_
 def mnmt_linear_argmax(A, W, s_w, bias, s_x, M, N, K, keys, stream=None):
     _chk(lib().mnmt_linear_argmax(_ptr(A), _ptr(W), _ptr(s_w), _ptr(bias), float(s_x), M, N, K, _ptr(keys),
                                   _stream_handle(stream)))
+
+
+def mnmt_linear_argmax_ids_noalloc(A, W, s_w, bias, s_x, M, N, K, ids, stream=None):
+    """Greedy vocabulary argmax into int32 ids with library-owned scratch (no allocation)."""
+    _chk(lib().mnmt_linear_argmax_ids_noalloc(_ptr(A), _ptr(W), _ptr(s_w), _ptr(bias), float(s_x), M, N, K,
+                                              _ptr(ids), _stream_handle(stream)))
 
 
 def argmax_from_keys(keys: np.ndarray) -> np.ndarray:
