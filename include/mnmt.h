@@ -167,6 +167,14 @@ enum {
 };
 int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, void *host_dst, size_t bytes);
 
+/* Which decode-step implementation the session uses for the batch encoded
+ * last: 1 = the single thread-block-cluster step (greedy batches of at most 4
+ * sentences whose shapes fit one cluster's shared memory), 0 = the multi-kernel
+ * step; negative on error.  Setting MNMT_DECODE_CLUSTER=0 in the environment
+ * before the first decode of a batch forces the multi-kernel step.  Both give
+ * bit-identical results. */
+int mnmt_session_decode_path(mnmt_session *s);
+
 /* Thread-local description of the last error on this thread ("" if none). */
 const char *mnmt_last_error(void);
 

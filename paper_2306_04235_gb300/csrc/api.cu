@@ -18,6 +18,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -58,6 +59,7 @@ static int lib_init() {
         g_init_err = linear_init();
         if (g_init_err == cudaSuccess) g_init_err = attention_init();
         if (g_init_err == cudaSuccess) g_init_err = rows_init();
+        if (g_init_err == cudaSuccess) g_init_err = decode_cluster_init();
     });
     if (g_init_err != cudaSuccess)
         return fail(MNMT_ECUDA, "kernel set-up failed: %s", cudaGetErrorString(g_init_err));
@@ -454,6 +456,11 @@ struct mnmt_session {
     size_t ck_layer, sk_layer;  // per-layer strides of the caches (elements)
     cudaGraphExec_t gexec = nullptr;
     int graph_B = -1, graph_S = -1;
+    // cluster decode step (small greedy batches)
+    DcParams *d_dc = nullptr;
+    bool use_cluster = false;
+    int dc_nc = 0;
+    size_t dc_smem = 0;
 };
 
 static int poison(mnmt_session *s, int code) {
@@ -499,7 +506,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
            o_anc = piece(R * max_len * 4), o_keys = piece(R * 8), o_cand = piece(R * beam * 8),
            o_logits = piece(beam > 1 ? R * V * 4 : 256), o_outids = piece((size_t)max_batch * max_len * 4),
            o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
-           o_state = piece(ST_N * 4);
+           o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams));
     s->arena_bytes = off;
     if (cudaMalloc(&s->arena, off) != cudaSuccess) {
         delete s;
@@ -537,6 +544,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
     s->out_lens = reinterpret_cast<int32_t *>(a + o_outlens);
     s->out_scores = reinterpret_cast<float *>(a + o_outsc);
     s->state = reinterpret_cast<int *>(a + o_state);
+    s->d_dc = reinterpret_cast<DcParams *>(a + o_dc);
     if (cudaMemsetAsync(s->arena, 0, off, m->stream) != cudaSuccess ||
         cudaStreamSynchronize(m->stream) != cudaSuccess) {
         mnmt_session_free(s);
@@ -706,6 +714,24 @@ int issue_decode_step(mnmt_session *s) {
     const int *done = s->state + ST_DONE;
     int *t_ptr = s->state + ST_T;
     int *status = s->state + ST_STATUS;
+    if (s->use_cluster) {
+        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, st));
+        GreedyArgs g;
+        g.keys = s->keys;
+        g.tok = s->tok;
+        g.fin = s->fin;
+        g.hist = s->hist;
+        g.t_ptr = t_ptr;
+        g.done = s->state + ST_DONE;
+        g.tmax_ptr = s->state + ST_TMAX;
+        g.R = R;
+        g.T = s->Tcap;
+        g.eos = c.eos_id;
+        g.pad = c.pad_id;
+        LK(launch_vocab_greedy(s->act, m->out.w, m->out.s, m->out.b, m->s_dout, R, c.vocab, d, s->keys,
+                               s->state + ST_TICKET, g, st));
+        return MNMT_OK;
+    }
     {
         EmbedArgs e;
         std::memset(&e, 0, sizeof(e));
@@ -870,6 +896,58 @@ int issue_decode_step(mnmt_session *s) {
     return MNMT_OK;
 }
 
+// Chooses the decode-step implementation for the current batch: the
+// single-cluster step for greedy batches of at most DC_RMAX sentences whose
+// shapes fit one cluster's shared memory, else the multi-kernel step.
+// MNMT_DECODE_CLUSTER=0 in the environment forces the multi-kernel step.
+int setup_cluster_step(mnmt_session *s) {
+    mnmt_model *m = s->m;
+    const mnmt_config &c = m->c;
+    s->use_cluster = false;
+    const char *env = getenv("MNMT_DECODE_CLUSTER");
+    if (env && env[0] == '0') return MNMT_OK;
+    const int d = c.d_model, F = c.d_ffn, H = c.n_heads, dh = d / H;
+    const int R = s->B * s->k;
+    const int nc = dc_cluster_size(d);
+    if (s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
+        F % (16 * nc) || (3 * d) % (16 * nc))
+        return MNMT_OK;
+    DcParams P;
+    std::memset(&P, 0, sizeof(P));
+    P.R = R; P.d = d; P.H = H; P.dh = dh; P.F = F; P.E = c.d_embed; P.V = c.vocab; P.T = s->Tcap; P.S = s->S;
+    P.n_dec = c.n_dec; P.pre_ln = c.pre_ln; P.factorised = m->factorised; P.nc = nc;
+    P.emb_q = m->emb_q; P.emb_s = m->emb_s;
+    if (m->factorised) P.proj = DcLin{m->proj.w, m->proj.s, m->proj.b};
+    P.emb_scale = m->emb_scale; P.pe = m->pe;
+    P.fin_g = m->dec_final.g; P.fin_b = m->dec_final.b; P.s_dout = m->s_dout;
+    P.tok = s->tok; P.t_ptr = s->state + ST_T; P.done = s->state + ST_DONE; P.src_len = s->src_lens;
+    P.act_out = s->act; P.resid_out = s->resid; P.status = s->state + ST_STATUS;
+    for (int l = 0; l < c.n_dec; l++) {
+        const SelfBlk &A = m->dec_self[l];
+        const CrossBlk &X = m->dec_cross[l];
+        const FfnBlk &Fb = m->dec_ffn[l];
+        DcLayer &Y = P.layer[l];
+        Y.ln1_g = A.ln.g; Y.ln1_b = A.ln.b; Y.ln2_g = X.ln.g; Y.ln2_b = X.ln.b; Y.ln3_g = Fb.ln.g; Y.ln3_b = Fb.ln.b;
+        Y.s_in1 = A.s_in; Y.s_ctx1 = A.s_ctx; Y.gamma1 = A.gamma; Y.sigma1 = A.sigma; Y.rho1 = A.rho;
+        Y.s_in2 = X.s_in; Y.s_ctx2 = X.s_ctx; Y.gamma2 = X.gamma; Y.sigma2 = X.sigma; Y.rho2 = X.rho;
+        Y.s_in3 = Fb.s_in; Y.s_h = Fb.s_h; Y.gamma3 = Fb.gamma;
+        Y.qkv = DcLin{A.qkv.w, A.qkv.s, A.qkv.b}; Y.o = DcLin{A.o.w, A.o.s, A.o.b};
+        Y.q2 = DcLin{X.q.w, X.q.s, X.q.b}; Y.o2 = DcLin{X.o.w, X.o.s, X.o.b};
+        Y.w1 = DcLin{Fb.w1.w, Fb.w1.s, Fb.w1.b}; Y.w2 = DcLin{Fb.w2.w, Fb.w2.s, Fb.w2.b};
+        Y.inv_qkv = A.inv_qkv; Y.inv_q2 = X.inv_q; Y.inv_h = Fb.inv_h;
+        Y.self_k = s->sk + l * s->sk_layer; Y.self_v = s->sv + l * s->sk_layer;
+        Y.cross_k = s->ck + l * s->ck_layer; Y.cross_v = s->cv + l * s->ck_layer;
+    }
+    size_t smem = dc_layout(P);
+    if (!decode_cluster_fits(dh, nc, smem)) return MNMT_OK;
+    CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
+    CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
+    s->use_cluster = true;
+    s->dc_nc = nc;
+    s->dc_smem = smem;
+    return MNMT_OK;
+}
+
 int ensure_graph(mnmt_session *s) {
     if (s->gexec && s->graph_B == s->B && s->graph_S == s->S) return MNMT_OK;
     if (s->gexec) {
@@ -877,6 +955,8 @@ int ensure_graph(mnmt_session *s) {
         s->gexec = nullptr;
     }
     cudaStream_t st = s->m->stream;
+    int rc0 = setup_cluster_step(s);
+    if (rc0) return rc0;
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
     int rc = issue_decode_step(s);
@@ -1097,6 +1177,14 @@ extern "C" int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, v
 }
 
 extern "C" const char *mnmt_last_error(void) { return g_err.c_str(); }
+
+extern "C" int mnmt_session_decode_path(mnmt_session *s) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    if (s->B < 1) return fail(MNMT_EINVAL, "no batch encoded yet");
+    int rc = ensure_graph(s);
+    if (rc) return rc;
+    return s->use_cluster ? 1 : 0;
+}
 
 int mnmt::set_error(int code, const char *msg) { return fail(code, "%s", msg); }
 

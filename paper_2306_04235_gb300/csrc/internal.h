@@ -156,4 +156,50 @@ struct FinalArgs {
 };
 cudaError_t launch_finalize(const FinalArgs &a, cudaStream_t st);
 
+// ---- decode step of small greedy batches on one thread-block cluster ----
+constexpr int DC_RMAX = 4;   // rows (sentences) per step
+constexpr int DC_LMAX = 16;  // decoder layers
+
+struct DcLin {
+    const int8_t *w;
+    const float *s, *b;
+};
+struct DcLayer {
+    const float *ln1_g, *ln1_b, *ln2_g, *ln2_b, *ln3_g, *ln3_b;
+    float s_in1, s_ctx1, gamma1, sigma1, rho1;
+    float s_in2, s_ctx2, gamma2, sigma2, rho2;
+    float s_in3, s_h, gamma3;
+    DcLin qkv, o, q2, o2, w1, w2;
+    const float *inv_qkv, *inv_q2, *inv_h;
+    int8_t *self_k, *self_v;          // [R][H][T][dh]
+    const int8_t *cross_k, *cross_v;  // [B][H][S][dh]
+};
+struct DcParams {
+    int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
+    const int8_t *emb_q;
+    const float *emb_s;
+    DcLin proj;
+    float emb_scale;
+    const float *pe;
+    const float *fin_g, *fin_b;
+    float s_dout;
+    const int32_t *tok;
+    const int *t_ptr, *done;
+    const int32_t *src_len;
+    int8_t *act_out;
+    float *resid_out;
+    int *status;
+    // shared-memory carve-up (bytes), filled by dc_layout
+    int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, slot_bytes, att_cap;
+    DcLayer layer[DC_LMAX];
+};
+int dc_cluster_size(int d);
+size_t dc_layout(DcParams &P);
+cudaError_t decode_cluster_init();
+bool decode_cluster_fits(int dh, int nc, size_t smem);
+cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, cudaStream_t st);
+cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
+                                int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
+                                cudaStream_t st);
+
 }  // namespace mnmt

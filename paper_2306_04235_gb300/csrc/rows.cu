@@ -14,49 +14,6 @@
 namespace mnmt {
 
 // ---------------------------------------------------------------------------
-// warp LayerNorm over a row held as VPL values per lane (element u*32 + lane)
-// ---------------------------------------------------------------------------
-template <int VPL>
-MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restrict__ g,
-                             const float *__restrict__ b, float (&out)[VPL], int lane) {
-    float amax = 0.0f;
-#pragma unroll
-    for (int u = 0; u < VPL; u++)
-        if (u * 32 + lane < d) amax = fmaxf(amax, fabsf(x[u]));
-    amax = warp_max_f(amax);
-    if (!(amax < 0x1p32f)) return false;
-    const int ea = exp_bound(amax);
-    long long s1 = 0;
-#pragma unroll
-    for (int u = 0; u < VPL; u++)
-        if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
-    s1 = warp_sum_ll(s1);
-    const float mu = __double2float_rn(__ddiv_rn(ldexp(__ll2double_rn(s1), ea - 52), (double)d));
-    float c[VPL];
-    float bmax = 0.0f;
-#pragma unroll
-    for (int u = 0; u < VPL; u++) {
-        c[u] = __fsub_rn(x[u], mu);
-        if (u * 32 + lane < d) bmax = fmaxf(bmax, fabsf(c[u]));
-    }
-    bmax = warp_max_f(bmax);
-    const int eb = exp_bound(bmax);
-    long long s2 = 0;
-#pragma unroll
-    for (int u = 0; u < VPL; u++)
-        if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
-    s2 = warp_sum_ll(s2);
-    const double var = __ddiv_rn(ldexp(__ll2double_rn(s2), 2 * eb - 52), (double)d);
-    const float rstd = __double2float_rn(__ddiv_rn(1.0, __dsqrt_rn(__dadd_rn(var, 1e-5))));
-#pragma unroll
-    for (int u = 0; u < VPL; u++) {
-        int i = u * 32 + lane;
-        if (i < d) out[u] = __fadd_rn(__fmul_rn(__fmul_rn(c[u], rstd), g[i]), b[i]);
-    }
-    return true;
-}
-
-// ---------------------------------------------------------------------------
 // LayerNorm kernel: one warp per row
 // ---------------------------------------------------------------------------
 template <int VPL>

@@ -67,6 +67,7 @@ def _declare(L):
     L.mnmt_decode_step.argtypes = [p, p, p, p, p]
     L.mnmt_translate.argtypes = [p, p, p, i32, i32, i32, i32, p, p, p]
     L.mnmt_debug_tap.argtypes = [p, i32, i32, p, sz]; L.mnmt_debug_tap.restype = C.c_int64
+    L.mnmt_session_decode_path.argtypes = [p]; L.mnmt_session_decode_path.restype = C.c_int
     L.mnmt_last_error.argtypes = []; L.mnmt_last_error.restype = C.c_char_p
     L.mnmt_linear.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p]
     L.mnmt_linear_argmax.argtypes = [p, p, p, p, f, i32, i32, i32, p, p]
@@ -166,6 +167,14 @@ def mnmt_debug_tap(session: int, tap: int, layer: int = 0, dtype=np.int8, shape=
     out = np.zeros(n // np.dtype(dtype).itemsize, dtype)
     _chk(int(lib().mnmt_debug_tap(session, tap, layer, _ptr(out), n)))
     return out.reshape(shape) if shape is not None else out
+
+
+def mnmt_session_decode_path(session: int) -> int:
+    """1 if the session's decode step runs on one thread-block cluster, 0 for the multi-kernel step."""
+    r = lib().mnmt_session_decode_path(session)
+    if r < 0:
+        raise MnmtError(r, last_error())
+    return r
 
 
 def mnmt_linear(A, W, s_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_q, out_f, stream=None):

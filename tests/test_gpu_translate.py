@@ -208,3 +208,70 @@ def test_bad_inputs_are_rejected(stream):
         assert out[0].shape == (2, 8)
     finally:
         tr.close()
+
+
+def _with_path(cluster: bool):
+    import os
+    if cluster:
+        os.environ.pop("MNMT_DECODE_CLUSTER", None)
+    else:
+        os.environ["MNMT_DECODE_CLUSTER"] = "0"
+
+
+@pytest.mark.parametrize("kind", list(MINI))
+@pytest.mark.parametrize("B", [1, 3, 4])
+def test_cluster_decode_step_matches_oracle(kind, B, stream):
+    """Greedy batches of <= 4 sentences run the single-cluster decode step."""
+    cfg = MINI[kind]
+    blob = synth.build_blob(cfg, 31, gamma_range=(0.5, 1.5))
+    ids, lens = synth.source_batch(cfg.vocab, B, 1, 40, 32)
+    T = 24
+    _with_path(True)
+    tr = mnmt.Translator(blob, B, ids.shape[1], 1, T, stream)
+    try:
+        g_ids, g_len, _ = tr.translate(ids, lens, T)
+        assert mnmt.mnmt_session_decode_path(tr.session) == 1
+    finally:
+        tr.close()
+    o_ids, o_len, _ = O.translate(blob, ids, lens, 1, T, n_threads=B)
+    assert np.array_equal(g_ids, o_ids) and np.array_equal(g_len, o_len)
+
+
+@pytest.mark.parametrize("name", ["tiny-b1-s16-greedy16", "small-b1-s10to50-greedy64"])
+def test_cluster_and_kernel_paths_bit_identical(name, stream):
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs(name)
+    d, H, L = cfg.d_model, cfg.n_heads, cfg.n_dec
+    dh = d // H
+    res = {}
+    for cluster in (True, False):
+        _with_path(cluster)
+        tr = mnmt.Translator(blob, 1, ids.shape[1], beam, T, stream)
+        try:
+            out = tr.translate(ids, lens, T)
+            assert mnmt.mnmt_session_decode_path(tr.session) == int(cluster)
+            taps = [mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_DEC_OUT, 0, np.int8),
+                    mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_RESID, 0, np.float32)]
+            for l in range(L):
+                taps.append(mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_SELF_K, l, np.int8))
+                taps.append(mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_SELF_V, l, np.int8))
+            res[cluster] = (out, taps)
+        finally:
+            tr.close()
+    _with_path(True)
+    (o1, t1), (o0, t0) = res[True], res[False]
+    assert np.array_equal(o1[0], o0[0]) and np.array_equal(o1[1], o0[1])
+    for a, b in zip(t1, t0):
+        assert np.array_equal(a.view(np.uint8), b.view(np.uint8))
+    ref = O.translate(blob, ids, lens, beam, T)
+    assert np.array_equal(o1[0], ref[0])
+
+
+def test_bench_workload_uses_cluster_step(stream):
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("small-b1-s10to50-greedy64")
+    _with_path(True)
+    tr = mnmt.Translator(blob, 1, ids.shape[1], beam, T, stream)
+    try:
+        mnmt.mnmt_encode(tr.session, ids, lens, 1, ids.shape[1])
+        assert mnmt.mnmt_session_decode_path(tr.session) == 1
+    finally:
+        tr.close()
