@@ -594,7 +594,12 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-int dc_cluster_size(int d) { return d / 16 >= 16 ? 16 : (d / 16 >= 8 ? 8 : 0); }
+// CTAs per cluster: one 16-column slice of d per CTA, at most 16 CTAs
+int dc_cluster_size(int d) {
+    int nc = d / 16;
+    if (nc > 16) nc = 16;
+    return nc >= 2 ? nc : 0;
+}
 
 size_t dc_layout(DcParams &P) {
     // shared-memory carve-up (16-byte aligned pieces)
