@@ -53,9 +53,9 @@
  *   With tied_output the output projection is emb_q / emb_s (requires E = d).
  *   Scales s_* are the per-tensor activation scales of the quantisation points
  *   of Fig. 5; pre_ln = 0 selects post-LN sublayers (LayerNorm after the
- *   residual add, no final LayerNorm).  Constraints checked at load: d, F, E
- *   multiples of 16 (64 where a dimension is a GEMM K), d_model / n_heads in
- *   {32, 64, 128}, d <= 2048, vocab >= 4.
+ *   residual add, no final LayerNorm).  Constraints checked at load: d_model a
+ *   power of two in [64, 2048], d_ffn a multiple of 64, d_embed a multiple of
+ *   16, d_model / n_heads in {32, 64, 128}, at most 16 heads, vocab >= 4.
  */
 #ifndef MNMT_H
 #define MNMT_H
@@ -231,8 +231,8 @@ int mnmt_linear_argmax_ids_noalloc(const int8_t *A, const int8_t *W, const float
  * caches: q [R][H][dh], Kc/Vc [R][H][T][dh] int8; row r attends keys
  * j < n_keys[r] (1 <= n_keys[r] <= T <= 1024).  Scores acc_j = q.k_j (int32),
  * s_j = fl(acc_j * sigma); weights E_j = rne(exp(fl(s_j - max)) 2^24);
- * ctx[r][h][e] = q8(fl32((sum_j E_j v_j[e]) / (sum_j E_j)), rho), with the
- * sums exact integers.  dh in {32, 64, 128}. */
+ * ctx[r][h][e] = q8(nearest fp32 to (sum_j E_j v_j[e]) / (sum_j E_j), rho),
+ * with the sums exact integers.  dh in {32, 64, 128}. */
 int mnmt_attention_decode(const int8_t *q, const int8_t *Kc, const int8_t *Vc, const int32_t *n_keys,
                           int32_t R, int32_t H, int32_t dh, int32_t T, float sigma, float rho,
                           int8_t *ctx, void *cuda_stream);

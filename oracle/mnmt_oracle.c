@@ -220,14 +220,33 @@ static void linear_row(const int8_t *a, float s_x, const olin *L, float *y) {
         y[n] = dequant_bias(dot_i8(a, L->w + (size_t)n * L->k, L->k), s_x, L->s[n], L->b[n]);
 }
 
+/* Nearest float (ties to even) to the exact value s 2^e / d.  The long double
+ * quotient (64-bit significand on x86, 113-bit on Arm) is exact for the
+ * power-of-two d of every model here, so the one rounding to float is the
+ * correct rounding of the exact value, subnormals included. */
+static float rn32_scaled(int64_t s, int e, int d) {
+    return (float)(ldexpl((long double)s, e) / (long double)d);
+}
+
+/* Nearest float (ties to even) to the exact quotient n / z of integers with
+ * |n| < 2^62 and 1 <= z < 2^35.  If n/z is not itself a midpoint M 2^E between
+ * two floats (M odd, < 2^26), it lies at least 2^-60 (relative) away from
+ * every midpoint, while the long double quotient is within 2^-64 of n/z; so
+ * the long double quotient rounds to float exactly as n/z does (and a
+ * midpoint quotient is computed exactly, ties going to even). */
+static float rn32_quotient(int64_t n, int64_t z) {
+    return (float)((long double)n / (long double)z);
+}
+
 /* LayerNorm (App. A / App. D).  The paper fixes neither epsilon nor the
  * arithmetic; this reading makes the mean and the (biased, divide-by-d)
  * variance exact fixed-point sums, so their value does not depend on the
- * summation order.  Each sum is taken on a grid set by the row's own largest
- * magnitude (an order-free maximum): with 2^ea > max|r_i| every term
- * r_i 2^(52-ea) is below 2^52, and with 2^eb > max|c_i| every c_i^2 2^(52-2eb)
- * is below 2^52, so d <= 2048 terms cannot overflow int64 and every term keeps
- * its leading 24+ bits.  eps = 1e-5.  |r_i| >= 2^32 is rejected. */
+ * summation order, each rounded once to fp32.  Each sum is taken on a grid
+ * set by the row's own largest magnitude (an order-free maximum): with
+ * 2^ea > max|r_i| every term r_i 2^(52-ea) is below 2^52, and with
+ * 2^eb > max|c_i| every c_i^2 2^(52-2eb) is below 2^52, so d <= 2048 terms
+ * cannot overflow int64 and every term keeps its leading 24+ bits.
+ * rstd = 1 / sqrt(var + 1e-5) in IEEE fp32.  |r_i| >= 2^32 is rejected. */
 static int layer_norm(const float *r, int d, const oln *ln, float *out) {
     float amax = 0.0f;
     for (int i = 0; i < d; i++) {
@@ -239,7 +258,7 @@ static int layer_norm(const float *r, int d, const oln *ln, float *out) {
     if (amax > 0.0f) frexpf(amax, &ea);
     int64_t s1 = 0;
     for (int i = 0; i < d; i++) s1 += llrint(ldexp((double)r[i], 52 - ea));
-    float mu = (float)(ldexp((double)s1, ea - 52) / (double)d);
+    float mu = rn32_scaled(s1, ea - 52, d);
     float bmax = 0.0f;
     for (int i = 0; i < d; i++) {
         float v = fabsf(r[i] - mu);
@@ -253,8 +272,8 @@ static int layer_norm(const float *r, int d, const oln *ln, float *out) {
         float c2 = c * c;
         s2 += llrint(ldexp((double)c2, 52 - 2 * eb));
     }
-    double var = ldexp((double)s2, 2 * eb - 52) / (double)d;
-    float rstd = (float)(1.0 / sqrt(var + 1e-5));
+    float var = rn32_scaled(s2, 2 * eb - 52, d);
+    float rstd = 1.0f / sqrtf(var + 1e-5f);
     for (int i = 0; i < d; i++) {
         float c = r[i] - mu;
         float t = c * rstd;
@@ -316,8 +335,9 @@ static double log_own(double z) {
 /* One attention head (Eq. 1/2).  Scores are int32 dot products of int8 q and
  * keys, scaled by sigma = fl32(s_q s_k / sqrt(d_h)); the softmax stays in full
  * precision as fixed-point weights E_j = rne(exp(s_j - max) * 2^24); the
- * context is the exact integer sum of E_j v_j over the exact sum of E_j, in
- * units of V's codes, then requantised with rho = fl(s_v / s_ctx). */
+ * context is the nearest float to the exact integer sum of E_j v_j over the
+ * exact sum of E_j, in units of V's codes, then requantised with
+ * rho = fl(s_v / s_ctx). */
 static void attend(const int8_t *q, const int8_t *const *keys, const int8_t *const *vals,
                    int n, int dh, float sigma, float rho, int8_t *out, float *sbuf,
                    int64_t *nbuf) {
@@ -335,7 +355,7 @@ static void attend(const int8_t *q, const int8_t *const *keys, const int8_t *con
         for (int e = 0; e < dh; e++) nbuf[e] += Ej * (int64_t)vals[j][e];
     }
     for (int e = 0; e < dh; e++) {
-        float ctx = (float)((double)nbuf[e] / (double)Z);
+        float ctx = rn32_quotient(nbuf[e], Z);
         out[e] = q8(ctx, rho);
     }
 }
@@ -891,7 +911,7 @@ int oracle_attention_probs(const int8_t *q, const int8_t *K, int n, int dh, floa
     int64_t Z = 0;
     for (int j = 0; j < n; j++) Z += (int64_t)rintf(exp_own(s[j] - m) * 16777216.0f);
     for (int j = 0; j < n; j++)
-        P[j] = (float)((double)(int64_t)rintf(exp_own(s[j] - m) * 16777216.0f) / (double)Z);
+        P[j] = rn32_quotient((int64_t)rintf(exp_own(s[j] - m) * 16777216.0f), Z);
     free(s);
     return OR_OK;
 }

@@ -137,7 +137,8 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
     c.pad_id = h[10]; c.bos_id = h[11]; c.eos_id = h[12];
     const int d = c.d_model, F = c.d_ffn, V = c.vocab, E = c.d_embed;
     if (c.n_enc < 1 || c.n_enc > 64 || c.n_dec < 1 || c.n_dec > 64) return fail(MNMT_EFORMAT, "layer counts out of range");
-    if (d < 64 || d > 2048 || d % 64 || c.n_heads < 1 || d % c.n_heads) return fail(MNMT_EFORMAT, "d_model %d / heads %d unsupported", d, c.n_heads);
+    if (!pow2_in(d, 64, 2048) || c.n_heads < 1 || d % c.n_heads)
+        return fail(MNMT_EFORMAT, "d_model %d / heads %d unsupported (d_model: a power of two in [64, 2048])", d, c.n_heads);
     if (!pow2_in(d / c.n_heads, 32, 128)) return fail(MNMT_EFORMAT, "head dim %d not in {32,64,128}", d / c.n_heads);
     if (c.n_heads > 16) return fail(MNMT_EFORMAT, "more than 16 heads");
     if (F < 64 || F % 64 || F > 8192) return fail(MNMT_EFORMAT, "d_ffn %d unsupported", F);
@@ -1283,7 +1284,8 @@ extern "C" int mnmt_layernorm(const float *r, const float *g, const float *b, in
                               float *out_f, int8_t *out_q, int32_t *status, void *cuda_stream) {
     int rc = lib_init();
     if (rc) return rc;
-    if (!r || !g || !b || M < 1 || d < 1 || d > 2048) return fail(MNMT_EINVAL, "layernorm: bad shape");
+    if (!r || !g || !b || M < 1 || d < 1 || d > 2048 || (d & (d - 1)))
+        return fail(MNMT_EINVAL, "layernorm: d must be a power of two <= 2048");
     LnArgs a;
     std::memset(&a, 0, sizeof(a));
     a.r = r;

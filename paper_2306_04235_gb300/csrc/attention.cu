@@ -6,7 +6,7 @@
 // s_j = fl(acc_j * sigma), m = max_j s_j, weights E_j = rne(exp(fl(s_j - m)) 2^24)
 // (an integer in [0, 2^24]), context N_e = sum_j E_j v_j[e] and Z = sum_j E_j as
 // exact integer sums (so any summation order gives the same bits), then
-// ctx_e = q8(fl32(N_e / Z), rho).  N_e is accumulated in two int32 halves,
+// ctx_e = q8(nearest fp32 to N_e / Z, rho).  N_e is accumulated in two int32 halves,
 // E_j = Eh 2^12 + El, which cannot overflow for up to 1024 keys.
 //
 // Kernels:
@@ -110,12 +110,10 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
         }
     }
     int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + lane * EPL;
-    double dz = __ll2double_rn(Z);
 #pragma unroll
     for (int u = 0; u < EPL; u++) {
         long long N = (long long)hi[u] * 4096 + lo[u];
-        float c = __double2float_rn(__ddiv_rn(__ll2double_rn(N), dz));
-        out[u] = q8(c, a.rho);
+        out[u] = q8(rn32_div(N, Z), a.rho);
     }
 }
 
@@ -213,12 +211,11 @@ __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a) {
                 lo[u] += El * v;
             }
         }
-        double dz = __ll2double_rn(Z);
         int8_t *out = a.ctx + ((size_t)b * S + qi) * a.d + h * DH + lane * EPL;
 #pragma unroll
         for (int u = 0; u < EPL; u++) {
             long long N = (long long)hi[u] * 4096 + lo[u];
-            out[u] = q8(__double2float_rn(__ddiv_rn(__ll2double_rn(N), dz)), a.rho);
+            out[u] = q8(rn32_div(N, Z), a.rho);
         }
         __syncwarp();
     }

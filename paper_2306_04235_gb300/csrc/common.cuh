@@ -177,11 +177,93 @@ MNMT_DEV int dot16(int4 a, int4 b, int acc) {
 }
 
 // ---------------------------------------------------------------------------
+// Exact roundings to fp32 with integer operations only (no double precision,
+// which is slow on this part).
+// ---------------------------------------------------------------------------
+// nearest float (ties to even) to S * 2^e, subnormals included
+MNMT_DEV float rn32_pow2(long long S, int e) {
+    if (S == 0) return 0.0f;
+    const unsigned long long a = S < 0 ? 0ull - (unsigned long long)S : (unsigned long long)S;
+    const int nb = 64 - __clzll(a);  // significant bits of a
+    const int E = nb - 1 + e;        // floor(log2 |value|)
+    const int p = E >= -126 ? 24 : 150 + E;  // bits the float keeps
+    const int shift = nb - p;
+    unsigned long long q;
+    if (shift <= 0) {
+        q = a << (-shift);
+    } else if (shift > 64) {
+        q = 0;
+    } else {
+        q = shift == 64 ? 0ull : (a >> shift);
+        const unsigned long long rem = shift == 64 ? a : (a & ((1ull << shift) - 1ull));
+        const unsigned long long half = 1ull << (shift - 1);
+        if (rem > half || (rem == half && (q & 1ull))) q++;
+    }
+    uint32_t bits;
+    if (E >= -126) {
+        int EE = E;
+        if (q == (1ull << 24)) {
+            q >>= 1;
+            EE++;
+        }
+        bits = EE > 127 ? 0x7F800000u : (((uint32_t)(EE + 127) << 23) | (uint32_t)(q - (1ull << 23)));
+    } else {
+        bits = (uint32_t)q;  // subnormal, or the smallest normal after a carry
+    }
+    if (S < 0) bits |= 0x80000000u;
+    return __uint_as_float(bits);
+}
+
+// sign of a - X * 2^E for a < 2^62, X < 2^63
+MNMT_DEV int cmp_scaled(unsigned long long a, unsigned long long X, int E) {
+    if (E >= 0) {
+        if (X == 0) return a > 0 ? 1 : 0;
+        if (64 - __clzll(X) + E > 62) return -1;  // X 2^E >= 2^62 > a
+        const unsigned long long v = X << E;
+        return a > v ? 1 : (a < v ? -1 : 0);
+    }
+    const int s = -E;
+    const unsigned long long qx = s >= 64 ? 0ull : (X >> s);
+    const unsigned long long rx = s >= 64 ? X : (X & ((1ull << s) - 1ull));
+    if (a > qx) return 1;
+    if (a < qx) return -1;
+    return rx ? -1 : 0;
+}
+
+// nearest float (ties to even) to the exact quotient n / z, |n| < 2^41, 1 <= z < 2^35
+MNMT_DEV float rn32_div(long long n, long long z) {
+    if (n == 0) return 0.0f;
+    const unsigned long long a = n < 0 ? 0ull - (unsigned long long)n : (unsigned long long)n;
+    float q = __fdiv_rn(__ull2float_rn(a), __ll2float_rn(z));  // within a few ulp of a / z
+    for (int it = 0; it < 8; it++) {
+        const uint32_t qb = __float_as_uint(q);
+        const unsigned long long mq = (qb & 0x7FFFFFu) | 0x800000u;  // q = mq 2^eq (normal: a/z > 2^-35)
+        const int eq = (int)((qb >> 23) & 0xFFu) - 150;
+        // midpoint above: (2 mq + 1) 2^(eq-1); below: (2 mq - 1) 2^(eq-1), or (2^25 - 1) 2^(eq-2) at a power of two
+        const int up = cmp_scaled(a, (unsigned long long)z * (2ull * mq + 1ull), eq - 1);
+        if (up > 0 || (up == 0 && (mq & 1ull))) {
+            q = __uint_as_float(qb + 1u);
+            continue;
+        }
+        const bool pow2 = mq == 0x800000ull;
+        const int dn = pow2 ? cmp_scaled(a, (unsigned long long)z * ((1ull << 25) - 1ull), eq - 2)
+                            : cmp_scaled(a, (unsigned long long)z * (2ull * mq - 1ull), eq - 1);
+        if (dn < 0 || (dn == 0 && (mq & 1ull))) {
+            q = __uint_as_float(qb - 1u);
+            continue;
+        }
+        break;
+    }
+    return n < 0 ? -q : q;
+}
+
+// ---------------------------------------------------------------------------
 // LayerNorm (App. A / App. D) of one row by one warp.  Mean and biased
 // variance are exact fixed-point sums: the row's largest magnitude (an
 // order-free maximum) sets a power-of-two grid on which every term is an
 // integer below 2^52, summed in int64, so any reduction order gives the same
-// bits; eps = 1e-5; returns false if |x| >= 2^32.
+// bits; each sum / d is rounded once to fp32 (d a power of two); rstd =
+// 1 / sqrt(var + 1e-5) in IEEE fp32; returns false if |x| >= 2^32.
 // warp LayerNorm over a row held as VPL values per lane (element u*32 + lane)
 // ---------------------------------------------------------------------------
 template <int VPL>
@@ -199,7 +281,8 @@ MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restri
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
     s1 = warp_sum_ll(s1);
-    const float mu = __double2float_rn(__ddiv_rn(ldexp(__ll2double_rn(s1), ea - 52), (double)d));
+    const int log2d = 31 - __clz(d);  // d is a power of two
+    const float mu = rn32_pow2(s1, ea - 52 - log2d);
     float c[VPL];
     float bmax = 0.0f;
 #pragma unroll
@@ -214,8 +297,8 @@ MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restri
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
     s2 = warp_sum_ll(s2);
-    const double var = __ddiv_rn(ldexp(__ll2double_rn(s2), 2 * eb - 52), (double)d);
-    const float rstd = __double2float_rn(__ddiv_rn(1.0, __dsqrt_rn(__dadd_rn(var, 1e-5))));
+    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
 #pragma unroll
     for (int u = 0; u < VPL; u++) {
         int i = u * 32 + lane;

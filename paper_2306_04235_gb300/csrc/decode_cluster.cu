@@ -51,14 +51,14 @@ MNMT_DEV int sb3(int x) { return x >> 24; }
 
 struct DcSlice {
     const int8_t *w;
-    const float *s, *b;
+    const float *s, *b, *inv;  // inv: per-column requantisation constants (or null)
     int rows, K;
 };
 
 // weight slice of phase ph for CTA c: phase 0 is the factorised embedding
 // projection (empty when not factorised), then per layer qkv, o, q2, o2, w1, w2
 MNMT_DEV DcSlice dc_slice(const DcParams &P, int ph, int c) {
-    DcSlice s{nullptr, nullptr, nullptr, 0, 0};
+    DcSlice s{nullptr, nullptr, nullptr, nullptr, 0, 0};
     const int nsd = P.d / P.nc, ns3 = 3 * P.d / P.nc, nsf = P.F / P.nc;
     const DcLin *L = nullptr;
     int n0 = 0;
@@ -72,11 +72,11 @@ MNMT_DEV DcSlice dc_slice(const DcParams &P, int ph, int c) {
         const int l = (ph - 1) / 6, k = (ph - 1) % 6;
         const DcLayer &Y = P.layer[l];
         switch (k) {
-            case 0: L = &Y.qkv; s.rows = ns3; s.K = P.d; n0 = c * ns3; break;
+            case 0: L = &Y.qkv; s.rows = ns3; s.K = P.d; n0 = c * ns3; s.inv = Y.inv_qkv + n0; break;
             case 1: L = &Y.o; s.rows = nsd; s.K = P.d; n0 = c * nsd; break;
-            case 2: L = &Y.q2; s.rows = nsd; s.K = P.d; n0 = c * nsd; break;
+            case 2: L = &Y.q2; s.rows = nsd; s.K = P.d; n0 = c * nsd; s.inv = Y.inv_q2 + n0; break;
             case 3: L = &Y.o2; s.rows = nsd; s.K = P.d; n0 = c * nsd; break;
-            case 4: L = &Y.w1; s.rows = nsf; s.K = P.d; n0 = c * nsf; break;
+            case 4: L = &Y.w1; s.rows = nsf; s.K = P.d; n0 = c * nsf; s.inv = Y.inv_h + n0; break;
             default: L = &Y.w2; s.rows = nsd; s.K = P.F; n0 = c * nsd; break;
         }
     }
@@ -86,62 +86,24 @@ MNMT_DEV DcSlice dc_slice(const DcParams &P, int ph, int c) {
     return s;
 }
 
-// ring slot layout: W rows (rows * K bytes), then s[rows], b[rows] (fp32)
+// ring slot layout: W rows (rows * K bytes), then s[rows], b[rows], inv[rows] (fp32)
 MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring, int slot_bytes, int nphase) {
     if (ph < nphase) {
         DcSlice s = dc_slice(P, ph, c);
         uint8_t *dst = ring + (size_t)(ph % DC_NB) * slot_bytes;
         const int wchunks = s.rows * s.K / 16, vchunks = s.rows * 4 / 16;
-        for (int i = threadIdx.x; i < wchunks + 2 * vchunks; i += DC_THREADS) {
+        const int nv = s.inv ? 3 : 2;
+        for (int i = threadIdx.x; i < wchunks + nv * vchunks; i += DC_THREADS) {
             if (i < wchunks) {
                 dc_cp16(dst + i * 16, s.w + (size_t)i * 16);
-            } else if (i < wchunks + vchunks) {
-                int j = i - wchunks;
-                dc_cp16(dst + wchunks * 16 + j * 16, reinterpret_cast<const uint8_t *>(s.s) + j * 16);
             } else {
-                int j = i - wchunks - vchunks;
-                dc_cp16(dst + wchunks * 16 + vchunks * 16 + j * 16, reinterpret_cast<const uint8_t *>(s.b) + j * 16);
+                const int j = i - wchunks, v = j / vchunks, k = j - v * vchunks;
+                const float *src = v == 0 ? s.s : (v == 1 ? s.b : s.inv);
+                dc_cp16(dst + wchunks * 16 + j * 16, reinterpret_cast<const uint8_t *>(src) + k * 16);
             }
         }
     }
     dc_commit();
-}
-
-// y-values of a GEMV slice held in shared memory: for each local row n (of
-// `rows`) and input row m (< R), acc = W[n] . A[m]; epi(m, n, acc, s_w, b)
-template <typename F>
-MNMT_DEV void dc_gemv(const uint8_t *slot, int rows, int K, const int8_t *A, int lda, int R, F epi) {
-    const int8_t *W = reinterpret_cast<const int8_t *>(slot);
-    const float *sw = reinterpret_cast<const float *>(slot + rows * K);
-    const float *bb = sw + rows;
-    const int kc = K / 16;
-    const int lpc = kc >= 32 ? 32 : kc;  // K >= 128 so lpc >= 8
-    const int gpw = 32 / lpc;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int grp = lane / lpc, sl = lane % lpc;
-    for (int r0 = warp * gpw; r0 < rows; r0 += DC_WARPS * gpw) {
-        const int n = r0 + grp;
-        int acc[DC_RMAX];
-#pragma unroll
-        for (int m = 0; m < DC_RMAX; m++) acc[m] = 0;
-        if (n < rows) {
-            const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)n * K);
-            for (int c = sl; c < kc; c += lpc) {
-                int4 w = wr[c];
-#pragma unroll
-                for (int m = 0; m < DC_RMAX; m++)
-                    if (m < R) acc[m] = dot16(reinterpret_cast<const int4 *>(A + (size_t)m * lda)[c], w, acc[m]);
-            }
-        }
-#pragma unroll
-        for (int m = 0; m < DC_RMAX; m++)
-            for (int o = lpc / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
-        if (sl == 0 && n < rows) {
-#pragma unroll
-            for (int m = 0; m < DC_RMAX; m++)
-                if (m < R) epi(m, n, acc[m], sw[n], bb[n]);
-        }
-    }
 }
 
 // copy stage [R][row_bytes] into every CTA's full buffer at column offset
@@ -158,53 +120,103 @@ MNMT_DEV void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int r
     }
 }
 
-// LayerNorm of the R rows of r (one warp per row), q8 into a (and, when
-// write_back, the normalised fp32 row back into r)
-MNMT_DEV void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv, int8_t *a,
-                           bool write_back, int *status) {
+// Block-wide LayerNorm of the R rows of r: 8/R' warps per row (R' = R rounded
+// up to a power of two), partial maxima and exact int64 sums combined through
+// shared memory.  q8(LN(r), inv) goes to a; with write_back the normalised row
+// also replaces r.  Same arithmetic as warp_layernorm.
+__device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
+                                          int8_t *a, int write_back, int *status, float *red_f,
+                                          long long *red_l) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (warp < R) {
-        float x[16], y[16];
-#pragma unroll
-        for (int u = 0; u < 16; u++) {
-            int i = u * 32 + lane;
-            x[u] = i < d ? r[(size_t)warp * d + i] : 0.0f;
+    const int rp = R <= 1 ? 1 : (R <= 2 ? 2 : 4);
+    const int wpr = DC_WARPS / rp;          // warps per row
+    const int m = warp / wpr, wi = warp - m * wpr;
+    const bool active = m < R;
+    const int chunk = d / wpr;              // elements of the row this warp owns
+    const int i0 = wi * chunk;
+    const int log2d = 31 - __clz(d);
+    float *row = r + (size_t)m * d;
+    // max |x|
+    float amax = 0.0f;
+    if (active)
+        for (int i = i0 + lane; i < i0 + chunk; i += 32) amax = fmaxf(amax, fabsf(row[i]));
+    amax = warp_max_f(amax);
+    if (lane == 0) red_f[warp] = amax;
+    __syncthreads();
+    amax = 0.0f;
+    for (int w = 0; w < wpr; w++) amax = fmaxf(amax, red_f[m * wpr + w < DC_WARPS ? m * wpr + w : 0]);
+    const bool ok = amax < 0x1p32f;
+    const int ea = exp_bound(amax);
+    long long s1 = 0;
+    if (active)
+        for (int i = i0 + lane; i < i0 + chunk; i += 32) s1 += fx_scale(row[i], 52 - ea);
+    s1 = warp_sum_ll(s1);
+    __syncthreads();
+    if (lane == 0) red_l[warp] = s1;
+    __syncthreads();
+    s1 = 0;
+    for (int w = 0; w < wpr; w++) s1 += red_l[m * wpr + w < DC_WARPS ? m * wpr + w : 0];
+    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    float bmax = 0.0f;
+    if (active)
+        for (int i = i0 + lane; i < i0 + chunk; i += 32) bmax = fmaxf(bmax, fabsf(__fsub_rn(row[i], mu)));
+    bmax = warp_max_f(bmax);
+    __syncthreads();
+    if (lane == 0) red_f[warp] = bmax;
+    __syncthreads();
+    bmax = 0.0f;
+    for (int w = 0; w < wpr; w++) bmax = fmaxf(bmax, red_f[m * wpr + w < DC_WARPS ? m * wpr + w : 0]);
+    const int eb = exp_bound(bmax);
+    long long s2 = 0;
+    if (active)
+        for (int i = i0 + lane; i < i0 + chunk; i += 32) {
+            float c = __fsub_rn(row[i], mu);
+            s2 += fx_scale(__fmul_rn(c, c), 52 - 2 * eb);
         }
-        if (!warp_layernorm16(x, d, g, b, y, lane)) {
-            if (lane == 0) set_status(status, MNMT_EOVERFLOW);
-        }
-#pragma unroll
-        for (int u = 0; u < 16; u++) {
-            int i = u * 32 + lane;
-            if (i < d) {
-                a[(size_t)warp * d + i] = q8(y[u], inv);
-                if (write_back) r[(size_t)warp * d + i] = y[u];
-            }
+    s2 = warp_sum_ll(s2);
+    __syncthreads();
+    if (lane == 0) red_l[warp] = s2;
+    __syncthreads();
+    s2 = 0;
+    for (int w = 0; w < wpr; w++) s2 += red_l[m * wpr + w < DC_WARPS ? m * wpr + w : 0];
+    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+    if (active) {
+        if (!ok && wi == 0 && lane == 0) set_status(status, MNMT_EOVERFLOW);
+        for (int i = i0 + lane; i < i0 + chunk; i += 32) {
+            float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(row[i], mu), rstd), g[i]), b[i]);
+            a[(size_t)m * d + i] = q8(y, inv);
+            if (write_back) row[i] = y;
         }
     }
+    __syncthreads();
 }
 
-MNMT_DEV void dc_quant_rows(const float *r, int R, int d, float inv, int8_t *a) {
-    for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a[i] = q8(r[i], inv);
-}
-
-// attention of every (row, head) of the step, redundantly in each CTA.
-// self: keys 0..t-1 from the layer's cache, key t from the step's k/v rows;
-// cross: keys j < src_len of the row's sentence from the cross cache.
+// Attention of every (row, head) of the step, redundantly in each CTA.  The
+// 8 warps split the keys of an item (row, head) into ranges: scores and the
+// partial maximum per range, then the weights, partial Z and partial context
+// sums per range; the partials are exact integers, so they combine in any
+// order.  self: keys 0..t-1 from the layer's cache, key t from the step's own
+// k/v rows; cross: keys j < src_len of the row's sentence.
 template <int DH>
-MNMT_DEV void dc_attention(const DcParams &P, const DcLayer &Y, bool cross, const int8_t *q, int q_ld,
-                           const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx, int *att) {
+__device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, int cross, const int8_t *q,
+                                          int q_ld, const int8_t *knew, const int8_t *vnew, int kv_ld, int t,
+                                          int8_t *ctx, int *att, float *red_f, long long *pz,
+                                          long long *pn) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int H = P.H, T = P.T, S = P.S;
-    float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
-    int *sc = att + warp * P.att_cap;
+    const int H = P.H, T = P.T, S = P.S, R = P.R;
+    const float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
+    const int items = R * H;
+    const int ip = items >= DC_WARPS ? DC_WARPS : (items > 4 ? 8 : (items > 2 ? 4 : (items > 1 ? 2 : 1)));
+    const int wpi = DC_WARPS / ip;  // warps per item in a round of ip items
     constexpr int QC = DH / 16;
     constexpr int C = DH / 16, G = 32 / C;
-    for (int item = warp; item < P.R * H; item += DC_WARPS) {
-        const int m = item / H, h = item - m * H;
+    for (int base = 0; base < items; base += ip) {
+        const int it = base + warp / wpi, part = warp % wpi;
+        const bool live = it < items;
+        const int m = live ? it / H : 0, h = live ? it - m * H : 0;
         int n;
         const int8_t *kb, *vb;
-        int kstride;
         if (cross) {
             n = P.src_len[m];
             n = n < 1 ? 1 : (n > S ? S : n);
@@ -215,52 +227,62 @@ MNMT_DEV void dc_attention(const DcParams &P, const DcLayer &Y, bool cross, cons
             kb = Y.self_k + ((size_t)m * H + h) * T * DH;
             vb = Y.self_v + ((size_t)m * H + h) * T * DH;
         }
-        kstride = DH;
-        int4 qv[QC];
-#pragma unroll
-        for (int c = 0; c < QC; c++) qv[c] = reinterpret_cast<const int4 *>(q + (size_t)m * q_ld + h * DH)[c];
+        const int per = (n + wpi - 1) / wpi;
+        const int j0 = part * per, j1 = min(n, j0 + per);
+        int *sc = att + (warp / wpi) * P.att_cap;
+        // scores of this warp's key range and their maximum
         float mx = -INFINITY;
-        for (int j = lane; j < n; j += 32) {
-            const int4 *kr = (!cross && j == t)
-                                 ? reinterpret_cast<const int4 *>(knew + (size_t)m * kv_ld + h * DH)
-                                 : reinterpret_cast<const int4 *>(kb + (size_t)j * kstride);
-            int acc = 0;
+        if (live) {
+            int4 qv[QC];
 #pragma unroll
-            for (int c = 0; c < QC; c++) acc = dot16(qv[c], kr[c], acc);
-            float s = __fmul_rn(__int2float_rn(acc), sigma);
-            sc[j] = __float_as_int(s);
-            mx = fmaxf(mx, s);
+            for (int c = 0; c < QC; c++) qv[c] = reinterpret_cast<const int4 *>(q + (size_t)m * q_ld + h * DH)[c];
+            for (int j = j0 + lane; j < j1; j += 32) {
+                const int4 *kr = (!cross && j == t)
+                                     ? reinterpret_cast<const int4 *>(knew + (size_t)m * kv_ld + h * DH)
+                                     : reinterpret_cast<const int4 *>(kb + (size_t)j * DH);
+                int acc = 0;
+#pragma unroll
+                for (int c = 0; c < QC; c++) acc = dot16(qv[c], kr[c], acc);
+                float sv = __fmul_rn(__int2float_rn(acc), sigma);
+                sc[j] = __float_as_int(sv);
+                mx = fmaxf(mx, sv);
+            }
         }
         mx = warp_max_f(mx);
+        if (lane == 0) red_f[warp] = mx;
+        __syncthreads();
+        mx = -INFINITY;
+        for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp / wpi) * wpi + w]);
+        // weights, partial Z and partial context sums of this warp's keys
+        long long z = 0;
+        if (live)
+            for (int j = j0 + lane; j < j1; j += 32) {
+                int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
+                sc[j] = E;
+                z += E;
+            }
+        z = warp_sum_ll(z);
         __syncwarp();
-        long long Z = 0;
-        for (int j = lane; j < n; j += 32) {
-            int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
-            sc[j] = E;
-            Z += E;
-        }
-        Z = warp_sum_ll(Z);
-        __syncwarp();
-        // context: lane = (key group g, 16-value chunk c)
         const int g = lane / C, c = lane - g * C;
         int hi[16], lo[16];
 #pragma unroll
         for (int u = 0; u < 16; u++) hi[u] = lo[u] = 0;
-        for (int j = g; j < n; j += G) {
-            const int E = sc[j];
-            const int Eh = E >> 12, El = E & 4095;
-            const int4 v = (!cross && j == t) ? reinterpret_cast<const int4 *>(vnew + (size_t)m * kv_ld + h * DH)[c]
-                                              : reinterpret_cast<const int4 *>(vb + (size_t)j * kstride)[c];
-            const int w4[4] = {v.x, v.y, v.z, v.w};
+        if (live)
+            for (int j = j0 + g; j < j1; j += G) {
+                const int E = sc[j];
+                const int Eh = E >> 12, El = E & 4095;
+                const int4 v = (!cross && j == t) ? reinterpret_cast<const int4 *>(vnew + (size_t)m * kv_ld + h * DH)[c]
+                                                  : reinterpret_cast<const int4 *>(vb + (size_t)j * DH)[c];
+                const int w4[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int q4 = 0; q4 < 4; q4++) {
-                int b0 = sb0(w4[q4]), b1 = sb1(w4[q4]), b2 = sb2(w4[q4]), b3 = sb3(w4[q4]);
-                hi[q4 * 4 + 0] += Eh * b0; lo[q4 * 4 + 0] += El * b0;
-                hi[q4 * 4 + 1] += Eh * b1; lo[q4 * 4 + 1] += El * b1;
-                hi[q4 * 4 + 2] += Eh * b2; lo[q4 * 4 + 2] += El * b2;
-                hi[q4 * 4 + 3] += Eh * b3; lo[q4 * 4 + 3] += El * b3;
+                for (int q4 = 0; q4 < 4; q4++) {
+                    const int b0 = sb0(w4[q4]), b1 = sb1(w4[q4]), b2 = sb2(w4[q4]), b3 = sb3(w4[q4]);
+                    hi[q4 * 4 + 0] += Eh * b0; lo[q4 * 4 + 0] += El * b0;
+                    hi[q4 * 4 + 1] += Eh * b1; lo[q4 * 4 + 1] += El * b1;
+                    hi[q4 * 4 + 2] += Eh * b2; lo[q4 * 4 + 2] += El * b2;
+                    hi[q4 * 4 + 3] += Eh * b3; lo[q4 * 4 + 3] += El * b3;
+                }
             }
-        }
 #pragma unroll
         for (int o = C; o < 32; o <<= 1) {
 #pragma unroll
@@ -269,26 +291,48 @@ MNMT_DEV void dc_attention(const DcParams &P, const DcLayer &Y, bool cross, cons
                 lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
             }
         }
+        // partials of this warp: pn[warp][e] (exact int64), pz[warp]
         if (g == 0) {
-            const double dz = __ll2double_rn(Z);
-            int8_t *out = ctx + (size_t)m * P.d + h * DH + c * 16;
 #pragma unroll
-            for (int u = 0; u < 16; u++) {
-                long long N = (long long)hi[u] * 4096 + lo[u];
-                out[u] = q8(__double2float_rn(__ddiv_rn(__ll2double_rn(N), dz)), rho);
+            for (int u = 0; u < 16; u++) pn[warp * DH + c * 16 + u] = (long long)hi[u] * 4096 + lo[u];
+        }
+        if (lane == 0) pz[warp] = z;
+        __syncthreads();
+        // combine the ranges of each item and requantise
+        for (int x = threadIdx.x; x < ip * DH; x += DC_THREADS) {
+            const int ii = x / DH, e = x - ii * DH;
+            const int it2 = base + ii;
+            if (it2 < items) {
+                long long N = 0, Z = 0;
+                for (int w = 0; w < wpi; w++) {
+                    N += pn[(ii * wpi + w) * DH + e];
+                    Z += pz[ii * wpi + w];
+                }
+                const int m2 = it2 / H, h2 = it2 - m2 * H;
+                ctx[(size_t)m2 * P.d + h2 * DH + e] = q8(rn32_div(N, Z), rho);
             }
         }
-        __syncwarp();
+        __syncthreads();
     }
 }
 
 // ---------------------------------------------------------------------------
-// the step kernel
+// the step kernel: one generic phase body run 1 + 6 * n_dec times
 // ---------------------------------------------------------------------------
+enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
+
 template <int DH>
 __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcParams *__restrict__ Pp) {
-    const DcParams &P = *Pp;
-    if (*P.done) return;  // uniform for the whole cluster
+    if (*Pp->done) return;  // uniform for the whole cluster
+    extern __shared__ __align__(16) uint8_t smem[];
+    {
+        // the parameter block lives in shared memory for the whole step
+        const int n16 = (int)(sizeof(DcParams) / 16);
+        for (int i = threadIdx.x; i < n16; i += DC_THREADS)
+            reinterpret_cast<int4 *>(smem)[i] = reinterpret_cast<const int4 *>(Pp)[i];
+        __syncthreads();
+    }
+    const DcParams &P = *reinterpret_cast<const DcParams *>(smem);
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
     const int nc = P.nc;
@@ -296,7 +340,6 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     const int t = *P.t_ptr;
     const int nsd = d / nc, ns3 = 3 * d / nc, nsf = F / nc;
 
-    extern __shared__ __align__(16) uint8_t smem[];
     float *r_full = reinterpret_cast<float *>(smem + P.off_r);
     int8_t *a_full = reinterpret_cast<int8_t *>(smem + P.off_a);
     int8_t *qkv_full = reinterpret_cast<int8_t *>(smem + P.off_qkv);
@@ -306,170 +349,179 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     uint8_t *stage = smem + P.off_stage;
     int *att = reinterpret_cast<int *>(smem + P.off_att);
     uint8_t *ring = smem + P.off_ring;
+    float *lnp = reinterpret_cast<float *>(smem + P.off_ln);  // [n_dec][6][d] + final [2][d]
+    float *red_f = reinterpret_cast<float *>(smem + P.off_red);          // [8]
+    long long *red_l = reinterpret_cast<long long *>(smem + P.off_red + 64);  // [8]
+    long long *pn = reinterpret_cast<long long *>(smem + P.off_red + 128);    // [8][DH]
+    int *tok_s = reinterpret_cast<int *>(smem + P.off_red + 128 + 8 * DH * 8);  // [R]
     const int nphase = 1 + 6 * P.n_dec;
 
-    for (int ph = 0; ph < DC_NB - 1; ph++) dc_prefetch(P, ph, c, ring, P.slot_bytes, nphase);
-    int ph = 0;
-    auto begin_phase = [&]() -> const uint8_t * {
-        dc_wait_ring();
-        __syncthreads();
-        dc_prefetch(P, ph + DC_NB - 1, c, ring, P.slot_bytes, nphase);
-        return ring + (size_t)(ph % DC_NB) * P.slot_bytes;
-    };
-
-    // ---- embedding slice -> r_full (all CTAs) ----
+    // LayerNorm gains / biases of every layer (and the final LN), in the first
+    // cp.async group together with the first weight slice
     {
-        const uint8_t *slot = begin_phase();
-        float *st = reinterpret_cast<float *>(stage);
-        const int8_t *W = reinterpret_cast<const int8_t *>(slot);
-        const float *sw = reinterpret_cast<const float *>(slot + nsd * P.E);
-        const float *bb = sw + nsd;
-        for (int i = threadIdx.x; i < R * nsd; i += DC_THREADS) {
-            const int m = i / nsd, nl = i - m * nsd, n = c * nsd + nl;
-            int id = P.tok[m];
+        const int cpa = d / 4;  // 16-byte chunks per d-vector of fp32
+        const int nvec = 6 * P.n_dec + 2;
+        for (int i = threadIdx.x; i < nvec * cpa; i += DC_THREADS) {
+            const int v = i / cpa, k = i - v * cpa;
+            const float *src;
+            if (v < 6 * P.n_dec) {
+                const DcLayer &Y = P.layer[v / 6];
+                const int w = v % 6;
+                src = w == 0 ? Y.ln1_g : w == 1 ? Y.ln1_b : w == 2 ? Y.ln2_g : w == 3 ? Y.ln2_b : w == 4 ? Y.ln3_g : Y.ln3_b;
+            } else {
+                src = v == 6 * P.n_dec ? P.fin_g : P.fin_b;
+            }
+            if (src) dc_cp16(lnp + (size_t)v * d + k * 4, src + k * 4);
+        }
+        if (threadIdx.x < R) {
+            int id = P.tok[threadIdx.x];
             if (id < 0 || id >= P.V) {
                 set_status(P.status, MNMT_EINVAL);
                 id = 0;
             }
-            const float es = P.emb_s[id];
-            float x;
-            if (!P.factorised) {
-                float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], es), P.emb_scale);
-                x = __fadd_rn(v, P.pe[(size_t)t * d + n]);
+            tok_s[threadIdx.x] = id;
+        }
+    }
+    for (int ph = 0; ph < DC_NB - 1; ph++) dc_prefetch(P, ph, c, ring, P.slot_bytes, nphase);
+
+    for (int ph = 0; ph < nphase; ph++) {
+        const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
+        const int l = ph == 0 ? 0 : (ph - 1) / 6;
+        const DcLayer &Y = P.layer[l];
+        dc_wait_ring();
+        __syncthreads();
+        dc_prefetch(P, ph + DC_NB - 1, c, ring, P.slot_bytes, nphase);
+        const uint8_t *slot = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
+        const float *lnl = lnp + (size_t)6 * l * d;
+
+        // ---- the phase's input vector ----
+        const int8_t *A = a_full;
+        int K = d;
+        if (kind == K_EMB) {
+            if (P.factorised)
+                for (int i = threadIdx.x; i < R * P.E; i += DC_THREADS)
+                    a_full[i] = P.emb_q[(size_t)tok_s[i / P.E] * P.E + (i % P.E)];
+            K = P.E;
+            __syncthreads();
+        } else if (kind == K_QKV || kind == K_Q2 || kind == K_W1) {
+            // pre-LN: LN of this sublayer; post-LN: LN of the previous sublayer's
+            // residual (written back), or plain quantisation for the first one
+            const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
+            const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
+            if (P.pre_ln) {
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status,
+                             red_f, red_l);
+            } else if (kind == K_QKV) {
+                for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
+                __syncthreads();
             } else {
-                const int4 *qr = reinterpret_cast<const int4 *>(P.emb_q + (size_t)id * P.E);
-                const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * P.E);
-                int acc = 0;
-                for (int k = 0; k < P.E / 16; k++) acc = dot16(qr[k], wr[k], acc);
-                float y = dequant_bias(acc, es, sw[nl], bb[nl]);
-                x = __fadd_rn(__fmul_rn(y, P.emb_scale), P.pe[(size_t)t * d + n]);
+                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1,
+                             P.status, red_f, red_l);
             }
-            st[m * nsd + nl] = x;
+        } else if (kind == K_O || kind == K_O2) {
+            const int cross = kind == K_O2;
+            dc_attention<DH>(P, Y, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
+                             qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn);
+            A = ctx_full;
+        } else {  // K_W2
+            A = h_full;
+            K = F;
+        }
+
+        // ---- the phase's slice of outputs ----
+        int rows, n0, out_f32;
+        float sx, gam;
+        switch (kind) {
+            case K_EMB: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = 0.0f; gam = 0.0f; break;
+            case K_QKV: rows = ns3; n0 = c * ns3; out_f32 = 0; sx = Y.s_in1; gam = 0.0f; break;
+            case K_O: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_ctx1; gam = Y.gamma1; break;
+            case K_Q2: rows = nsd; n0 = c * nsd; out_f32 = 0; sx = Y.s_in2; gam = 0.0f; break;
+            case K_O2: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_ctx2; gam = Y.gamma2; break;
+            case K_W1: rows = nsf; n0 = c * nsf; out_f32 = 0; sx = Y.s_in3; gam = 0.0f; break;
+            default: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_h; gam = Y.gamma3; break;
+        }
+        float *stf = reinterpret_cast<float *>(stage);
+        int8_t *sti = reinterpret_cast<int8_t *>(stage);
+        if (kind == K_EMB && !P.factorised) {
+            for (int i = threadIdx.x; i < R * nsd; i += DC_THREADS) {
+                const int m = i / nsd, nl = i - m * nsd, n = n0 + nl, id = tok_s[m];
+                float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
+                stf[i] = __fadd_rn(v, P.pe[(size_t)t * d + n]);
+            }
+        } else {
+            const int8_t *W = reinterpret_cast<const int8_t *>(slot);
+            const float *sw = reinterpret_cast<const float *>(slot + rows * K);
+            const float *bb = sw + rows;
+            const float *iv = bb + rows;
+            const int kc = K / 16;
+            const int lpc = kc >= 32 ? 32 : kc;
+            const int gpw = 32 / lpc;
+            const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+            const int grp = lane / lpc, sl = lane % lpc;
+            for (int r0 = warp * gpw; r0 < rows; r0 += DC_WARPS * gpw) {
+                const int nl = r0 + grp;
+                int acc[DC_RMAX] = {0, 0, 0, 0};
+                if (nl < rows) {
+                    const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * K);
+                    for (int k = sl; k < kc; k += lpc) {
+                        const int4 w = wr[k];
+#pragma unroll
+                        for (int m = 0; m < DC_RMAX; m++)
+                            if (m < R) acc[m] = dot16(reinterpret_cast<const int4 *>(A + (size_t)m * K)[k], w, acc[m]);
+                    }
+                }
+#pragma unroll
+                for (int m = 0; m < DC_RMAX; m++)
+                    for (int o = lpc / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
+                if (sl == 0 && nl < rows) {
+                    const int n = n0 + nl;
+#pragma unroll
+                    for (int m = 0; m < DC_RMAX; m++) {
+                        if (m >= R) break;
+                        float y;
+                        if (kind == K_EMB) {
+                            y = dequant_bias(acc[m], P.emb_s[tok_s[m]], sw[nl], bb[nl]);
+                            stf[m * rows + nl] = __fadd_rn(__fmul_rn(y, P.emb_scale), P.pe[(size_t)t * d + n]);
+                            continue;
+                        }
+                        y = dequant_bias(acc[m], sx, sw[nl], bb[nl]);
+                        if (out_f32) {
+                            stf[m * rows + nl] = __fadd_rn(__fmul_rn(gam, r_full[(size_t)m * d + n]), y);
+                        } else {
+                            const int8_t v = q8(kind == K_W1 && !(y > 0.0f) ? 0.0f : y, iv[nl]);
+                            sti[m * rows + nl] = v;
+                            if (kind == K_QKV && n >= d) {  // K / V of position t into the layer's cache
+                                const int seg = n >= 2 * d;
+                                const int cc = n - (seg ? 2 * d : d);
+                                const int hh = cc / DH, ii = cc - hh * DH;
+                                (seg ? Y.self_v : Y.self_k)[(((size_t)m * P.H + hh) * P.T + t) * DH + ii] = v;
+                            }
+                        }
+                    }
+                }
+            }
         }
         __syncthreads();
-        dc_bcast(cl, stage, R, nsd * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, c * nsd * 4, nc);
+        // ---- publish the slice to every CTA ----
+        if (out_f32) {
+            dc_bcast(cl, stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
+        } else {
+            int8_t *full = kind == K_QKV ? qkv_full : (kind == K_Q2 ? q2_full : h_full);
+            const int width = kind == K_QKV ? 3 * d : (kind == K_Q2 ? d : F);
+            dc_bcast(cl, stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc);
+        }
         cl.sync();
-        ph++;
-    }
-
-    for (int l = 0; l < P.n_dec; l++) {
-        const DcLayer &Y = P.layer[l];
-        // ---- self-attention: q/k/v slice ----
-        {
-            if (P.pre_ln) dc_layernorm(r_full, R, d, Y.ln1_g, Y.ln1_b, 1.0f / Y.s_in1, a_full, false, P.status);
-            else dc_quant_rows(r_full, R, d, 1.0f / Y.s_in1, a_full);
-            const uint8_t *slot = begin_phase();
-            int8_t *st = reinterpret_cast<int8_t *>(stage);
-            const int n0 = c * ns3;
-            dc_gemv(slot, ns3, d, a_full, d, R, [&](int m, int nl, int acc, float sw, float bias) {
-                const int n = n0 + nl;
-                int8_t v = q8(dequant_bias(acc, Y.s_in1, sw, bias), Y.inv_qkv[n]);
-                st[m * ns3 + nl] = v;
-                if (n >= d) {  // K / V of position t into the layer's cache
-                    const int seg = n >= 2 * d;
-                    const int cc = n - (seg ? 2 * d : d);
-                    const int h = cc / DH, i = cc - h * DH;
-                    int8_t *dst = seg ? Y.self_v : Y.self_k;
-                    dst[(((size_t)m * P.H + h) * P.T + t) * DH + i] = v;
-                }
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, ns3, reinterpret_cast<uint8_t *>(qkv_full), 3 * d, n0, nc);
-            cl.sync();
-            ph++;
-        }
-        // ---- attention (all heads) + W_o slice + gamma-residual ----
-        {
-            dc_attention<DH>(P, Y, false, qkv_full, 3 * d, qkv_full + d, qkv_full + 2 * d, 3 * d, t, ctx_full, att);
-            const uint8_t *slot = begin_phase();  // includes the barrier that publishes ctx_full
-            float *st = reinterpret_cast<float *>(stage);
-            const int n0 = c * nsd;
-            dc_gemv(slot, nsd, d, ctx_full, d, R, [&](int m, int nl, int acc, float sw, float bias) {
-                float y = dequant_bias(acc, Y.s_ctx1, sw, bias);
-                st[m * nsd + nl] = __fadd_rn(__fmul_rn(Y.gamma1, r_full[(size_t)m * d + n0 + nl]), y);
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, nsd * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
-            cl.sync();
-            ph++;
-        }
-        // ---- cross-attention: q slice ----
-        {
-            if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, Y.ln2_g, Y.ln2_b, 1.0f / Y.s_in2, a_full, false, P.status);
-            } else {
-                dc_layernorm(r_full, R, d, Y.ln1_g, Y.ln1_b, 1.0f / Y.s_in2, a_full, true, P.status);
-            }
-            const uint8_t *slot = begin_phase();
-            int8_t *st = reinterpret_cast<int8_t *>(stage);
-            const int n0 = c * nsd;
-            dc_gemv(slot, nsd, d, a_full, d, R, [&](int m, int nl, int acc, float sw, float bias) {
-                st[m * nsd + nl] = q8(dequant_bias(acc, Y.s_in2, sw, bias), Y.inv_q2[n0 + nl]);
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, nsd, reinterpret_cast<uint8_t *>(q2_full), d, n0, nc);
-            cl.sync();
-            ph++;
-        }
-        // ---- cross-attention (all heads) + W_o slice + gamma-residual ----
-        {
-            dc_attention<DH>(P, Y, true, q2_full, d, nullptr, nullptr, 0, t, ctx_full, att);
-            const uint8_t *slot = begin_phase();
-            float *st = reinterpret_cast<float *>(stage);
-            const int n0 = c * nsd;
-            dc_gemv(slot, nsd, d, ctx_full, d, R, [&](int m, int nl, int acc, float sw, float bias) {
-                float y = dequant_bias(acc, Y.s_ctx2, sw, bias);
-                st[m * nsd + nl] = __fadd_rn(__fmul_rn(Y.gamma2, r_full[(size_t)m * d + n0 + nl]), y);
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, nsd * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
-            cl.sync();
-            ph++;
-        }
-        // ---- FFN1 slice (ReLU + q8) ----
-        {
-            if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, Y.ln3_g, Y.ln3_b, 1.0f / Y.s_in3, a_full, false, P.status);
-            } else {
-                dc_layernorm(r_full, R, d, Y.ln2_g, Y.ln2_b, 1.0f / Y.s_in3, a_full, true, P.status);
-            }
-            const uint8_t *slot = begin_phase();
-            int8_t *st = reinterpret_cast<int8_t *>(stage);
-            const int n0 = c * nsf;
-            dc_gemv(slot, nsf, d, a_full, d, R, [&](int m, int nl, int acc, float sw, float bias) {
-                float y = dequant_bias(acc, Y.s_in3, sw, bias);
-                st[m * nsf + nl] = q8(y > 0.0f ? y : 0.0f, Y.inv_h[n0 + nl]);
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, nsf, reinterpret_cast<uint8_t *>(h_full), F, n0, nc);
-            cl.sync();
-            ph++;
-        }
-        // ---- FFN2 slice + gamma-residual ----
-        {
-            const uint8_t *slot = begin_phase();
-            float *st = reinterpret_cast<float *>(stage);
-            const int n0 = c * nsd;
-            dc_gemv(slot, nsd, F, h_full, F, R, [&](int m, int nl, int acc, float sw, float bias) {
-                float y = dequant_bias(acc, Y.s_h, sw, bias);
-                st[m * nsd + nl] = __fadd_rn(__fmul_rn(Y.gamma3, r_full[(size_t)m * d + n0 + nl]), y);
-            });
-            __syncthreads();
-            dc_bcast(cl, stage, R, nsd * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
-            cl.sync();
-            ph++;
-        }
-        if (!P.pre_ln) {
-            // post-LN: the FFN's LayerNorm normalises the stream in place; the
-            // next sublayer input is quantised from it
+        if (kind == K_W2 && !P.pre_ln) {
+            // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
-            float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
-            dc_layernorm(r_full, R, d, Y.ln3_g, Y.ln3_b, inv, a_full, true, P.status);
-            __syncthreads();
+            const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, red_f, red_l);
         }
     }
     // ---- final LayerNorm + quantisation -> vocabulary input ----
-    if (P.pre_ln) dc_layernorm(r_full, R, d, P.fin_g, P.fin_b, 1.0f / P.s_dout, a_full, false, P.status);
+    if (P.pre_ln)
+        dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
+                     1.0f / P.s_dout, a_full, 0, P.status, red_f, red_l);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -610,6 +662,8 @@ size_t dc_layout(DcParams &P) {
         return (int)at;
     };
     const int R = P.R, d = P.d, F = P.F, nc = P.nc;
+    take(sizeof(DcParams));  // the parameter block itself
+    P.off_ln = take((size_t)(6 * P.n_dec + 2) * d * 4);
     P.off_r = take((size_t)R * d * 4);
     P.off_a = take((size_t)R * d);
     P.off_qkv = take((size_t)R * 3 * d);
@@ -622,13 +676,15 @@ size_t dc_layout(DcParams &P) {
     P.off_stage = take(stage_bytes);
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
+    P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // red_f, red_l, pn[8][dh], tokens
     // largest weight slice of any phase (rows * K + 8 * rows)
     int slot = 0;
     auto upd = [&](int rows, int K) {
-        int b = rows * K + 8 * rows;
+        int b = rows * K + 12 * rows;
         if (b > slot) slot = b;
     };
     if (P.factorised) upd(d / nc, P.E);
+    if (P.factorised && R * P.E > R * d) return (size_t)-1;  // a_full holds the embedding rows
     upd(3 * d / nc, d);
     upd(d / nc, d);
     upd(F / nc, d);

@@ -174,7 +174,7 @@ struct DcLayer {
     int8_t *self_k, *self_v;          // [R][H][T][dh]
     const int8_t *cross_k, *cross_v;  // [B][H][S][dh]
 };
-struct DcParams {
+struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
     const int8_t *emb_q;
     const float *emb_s;
@@ -190,9 +190,11 @@ struct DcParams {
     float *resid_out;
     int *status;
     // shared-memory carve-up (bytes), filled by dc_layout
-    int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, slot_bytes, att_cap;
+    int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, off_ln, off_red, slot_bytes,
+        att_cap;
     DcLayer layer[DC_LMAX];
 };
+static_assert(sizeof(DcParams) % 16 == 0, "the parameter block is copied in 16-byte chunks");
 int dc_cluster_size(int d);
 size_t dc_layout(DcParams &P);
 cudaError_t decode_cluster_init();

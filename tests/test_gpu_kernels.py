@@ -139,7 +139,7 @@ def test_attention_decode_full_size_sampled():
     assert np.array_equal(got[rows], ref)
 
 
-LN_CASES = [(1, 128, 1.0), (7, 256, 30.0), (33, 512, 700.0), (5, 2048, 1e-3), (100, 384, 3.0), (1, 64, 1e6)]
+LN_CASES = [(1, 128, 1.0), (7, 256, 30.0), (33, 512, 700.0), (5, 2048, 1e-3), (100, 1024, 3.0), (1, 64, 1e6)]
 
 
 @pytest.mark.parametrize("M,d,scale", LN_CASES)

@@ -232,3 +232,27 @@ def test_attention_vs_float64_softmax(n, sigma):
 def test_sigma_definition():
     assert O.sigma(f32(0.03), f32(0.05), 64) == f32(0.03 * 0.05 / 8.0) or \
         abs(O.sigma(f32(0.03), f32(0.05), 64) - f32(0.03) * f32(0.05) / 8.0) <= ulp32(0.03 * 0.05 / 8)
+
+
+def _nearest_f32(fr):
+    """Nearest float32 to an exact Fraction, ties to even (brute force over neighbours)."""
+    from fractions import Fraction
+    x = np.float32(float(fr))
+    cands = [np.nextafter(x, np.float32(-np.inf)), x, np.nextafter(x, np.float32(np.inf))]
+    best = min(cands, key=lambda c: (abs(Fraction(float(c)) - fr), int(np.float32(c).view(np.uint32)) & 1))
+    return np.float32(best)
+
+
+@pytest.mark.parametrize("n,sigma", [(3, 0.0), (7, 0.001), (64, 0.0004), (500, 0.0001)])
+def test_attention_weights_are_nearest_float_of_exact_quotient(n, sigma):
+    """P_j = E_j / Z rounded once to fp32 (E_j = rne(exp(s_j - max) 2^24) from the pinned exp)."""
+    from fractions import Fraction
+    q, K, V = _att_inputs(n + 5, n)
+    sigma = f32(sigma)
+    s = [f32(float(np.dot(K[j].astype(np.int64), q.astype(np.int64))) * sigma) for j in range(n)]
+    m = max(s)
+    E = [int(np.rint(np.float32(O.exp_own(f32(sj - m))) * np.float32(16777216.0))) for sj in s]
+    Z = sum(E)
+    P = O.attention_probs(q, K, sigma)
+    for j in range(n):
+        assert P[j] == _nearest_f32(Fraction(E[j], Z)), j
