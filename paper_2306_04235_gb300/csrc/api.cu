@@ -939,7 +939,7 @@ int setup_cluster_step(mnmt_session *s) {
         Y.self_k = s->sk + l * s->sk_layer; Y.self_v = s->sv + l * s->sk_layer;
         Y.cross_k = s->ck + l * s->ck_layer; Y.cross_v = s->cv + l * s->ck_layer;
     }
-    size_t smem = dc_layout(P);
+    size_t smem = dc_layout(P, 227 * 1024);
     if (!decode_cluster_fits(dh, nc, smem)) return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame

@@ -266,37 +266,46 @@ MNMT_DEV float rn32_div(long long n, long long z) {
 // 1 / sqrt(var + 1e-5) in IEEE fp32; returns false if |x| >= 2^32.
 // warp LayerNorm over a row held as VPL values per lane (element u*32 + lane)
 // ---------------------------------------------------------------------------
+// exact warp sum of int64 values with |v| < 2^58 per lane: three 20-bit
+// pieces summed by single-instruction warp reductions
+MNMT_DEV long long warp_sum_exact(long long v) {
+    int p0 = (int)(v & 0xFFFFF), p1 = (int)((v >> 20) & 0xFFFFF), p2 = (int)(v >> 40);
+    p0 = __reduce_add_sync(0xFFFFFFFFu, p0);
+    p1 = __reduce_add_sync(0xFFFFFFFFu, p1);
+    p2 = __reduce_add_sync(0xFFFFFFFFu, p2);
+    return (long long)p0 + (long long)p1 * (1LL << 20) + (long long)p2 * (1LL << 40);
+}
+
 template <int VPL>
 MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restrict__ g,
                              const float *__restrict__ b, float (&out)[VPL], int lane) {
-    float amax = 0.0f;
+    unsigned amax_bits = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++)
-        if (u * 32 + lane < d) amax = fmaxf(amax, fabsf(x[u]));
-    amax = warp_max_f(amax);
+        if (u * 32 + lane < d) amax_bits = max(amax_bits, __float_as_uint(x[u]) & 0x7FFFFFFFu);
+    const float amax = __uint_as_float(__reduce_max_sync(0xFFFFFFFFu, amax_bits));
     if (!(amax < 0x1p32f)) return false;
     const int ea = exp_bound(amax);
+    const int log2d = 31 - __clz(d);  // d is a power of two
     long long s1 = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
-    s1 = warp_sum_ll(s1);
-    const int log2d = 31 - __clz(d);  // d is a power of two
+    s1 = warp_sum_exact(s1);
     const float mu = rn32_pow2(s1, ea - 52 - log2d);
     float c[VPL];
-    float bmax = 0.0f;
+    unsigned bmax_bits = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++) {
         c[u] = __fsub_rn(x[u], mu);
-        if (u * 32 + lane < d) bmax = fmaxf(bmax, fabsf(c[u]));
+        if (u * 32 + lane < d) bmax_bits = max(bmax_bits, __float_as_uint(c[u]) & 0x7FFFFFFFu);
     }
-    bmax = warp_max_f(bmax);
-    const int eb = exp_bound(bmax);
+    const int eb = exp_bound(__uint_as_float(__reduce_max_sync(0xFFFFFFFFu, bmax_bits)));
     long long s2 = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
-    s2 = warp_sum_ll(s2);
+    s2 = warp_sum_exact(s2);
     const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
     const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
 #pragma unroll

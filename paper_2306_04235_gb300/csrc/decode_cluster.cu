@@ -2,24 +2,26 @@
 // on a single thread-block cluster, then the vocabulary projection fused with
 // the greedy update.
 //
-// A batch-1 decode step is a chain of ~13 dependent matrix-vector products and
-// two attentions per decoder layer (App. A), each only 16-260 KB of weights:
-// the step is bound by latency, not bandwidth.  Instead of one kernel per
-// operation, one cluster of NC CTAs (8 or 16 SMs) runs the whole decoder:
+// A batch-1 decode step is a chain of dependent matrix-vector products and two
+// attentions per decoder layer (App. A), each only 16-260 KB of weights: the
+// step is bound by latency, not bandwidth.  Instead of one kernel per
+// operation, one cluster of NC CTAs (up to 16 SMs) runs the whole decoder:
 //   * every CTA holds the full activation vectors of the step in shared memory
 //     (residual stream fp32 [R][d], LN output, q/k/v, context, FFN hidden);
 //   * a linear layer is split by output columns: CTA c computes its column
 //     slice from its weight slice and writes the result into the shared
 //     memory of every CTA of the cluster (distributed shared memory), then a
 //     hardware cluster barrier publishes it;
-//   * LayerNorm and attention (all heads, the step's query rows) are computed
+//   * LayerNorm and attention (all heads of the step's rows) are computed
 //     redundantly by every CTA, which removes two barriers per attention;
-//   * each CTA streams its weight slices from L2/HBM into a 3-slot shared
-//     memory ring with cp.async, two phases ahead of use.
-// Per step: 1 + 6 * n_dec cluster barriers, no global synchronisation, no
-// spin loops.  The arithmetic is exactly that of the other kernels (Fig. 5
-// quantisation points, fixed-point LayerNorm and softmax), so the step is
-// bit-identical to the multi-kernel path.
+//   * weight slices stream from L2/HBM into a 3-slot shared-memory ring with
+//     cp.async, two phases ahead of use; the keys and values the step attends
+//     to are staged into shared memory at kernel start when they fit.
+// The step is one compact phase loop (the instruction cache holds it) with
+// 1 + 6 * n_dec cluster barriers, no global synchronisation and no spin loop.
+// The arithmetic is exactly that of the other kernels (Fig. 5 quantisation
+// points, fixed-point LayerNorm and softmax), so the step is bit-identical to
+// the multi-kernel path.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -33,9 +35,6 @@ constexpr int DC_THREADS = 256;
 constexpr int DC_WARPS = DC_THREADS / 32;
 constexpr int DC_NB = 3;  // weight ring slots
 
-// ---------------------------------------------------------------------------
-// helpers
-// ---------------------------------------------------------------------------
 MNMT_DEV uint32_t dc_smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
 MNMT_DEV void dc_cp16(void *dst_smem, const void *src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dc_smem_u32(dst_smem)), "l"(src));
@@ -49,58 +48,23 @@ MNMT_DEV int sb1(int x) { return (x << 16) >> 24; }
 MNMT_DEV int sb2(int x) { return (x << 8) >> 24; }
 MNMT_DEV int sb3(int x) { return x >> 24; }
 
-struct DcSlice {
-    const int8_t *w;
-    const float *s, *b, *inv;  // inv: per-column requantisation constants (or null)
-    int rows, K;
-};
-
-// weight slice of phase ph for CTA c: phase 0 is the factorised embedding
-// projection (empty when not factorised), then per layer qkv, o, q2, o2, w1, w2
-MNMT_DEV DcSlice dc_slice(const DcParams &P, int ph, int c) {
-    DcSlice s{nullptr, nullptr, nullptr, nullptr, 0, 0};
-    const int nsd = P.d / P.nc, ns3 = 3 * P.d / P.nc, nsf = P.F / P.nc;
-    const DcLin *L = nullptr;
-    int n0 = 0;
-    if (ph == 0) {
-        if (!P.factorised) return s;
-        L = &P.proj;
-        s.rows = nsd;
-        s.K = P.E;
-        n0 = c * nsd;
-    } else {
-        const int l = (ph - 1) / 6, k = (ph - 1) % 6;
-        const DcLayer &Y = P.layer[l];
-        switch (k) {
-            case 0: L = &Y.qkv; s.rows = ns3; s.K = P.d; n0 = c * ns3; s.inv = Y.inv_qkv + n0; break;
-            case 1: L = &Y.o; s.rows = nsd; s.K = P.d; n0 = c * nsd; break;
-            case 2: L = &Y.q2; s.rows = nsd; s.K = P.d; n0 = c * nsd; s.inv = Y.inv_q2 + n0; break;
-            case 3: L = &Y.o2; s.rows = nsd; s.K = P.d; n0 = c * nsd; break;
-            case 4: L = &Y.w1; s.rows = nsf; s.K = P.d; n0 = c * nsf; s.inv = Y.inv_h + n0; break;
-            default: L = &Y.w2; s.rows = nsd; s.K = P.F; n0 = c * nsd; break;
-        }
-    }
-    s.w = L->w + (size_t)n0 * s.K;
-    s.s = L->s + n0;
-    s.b = L->b + n0;
-    return s;
+// async copy of `bytes` (a multiple of 16) from global to shared memory
+MNMT_DEV void dc_copy(void *dst, const void *src, int bytes) {
+    for (int i = threadIdx.x; i < bytes / 16; i += DC_THREADS)
+        dc_cp16(static_cast<uint8_t *>(dst) + i * 16, static_cast<const uint8_t *>(src) + i * 16);
 }
 
 // ring slot layout: W rows (rows * K bytes), then s[rows], b[rows], inv[rows] (fp32)
-MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring, int slot_bytes, int nphase) {
-    if (ph < nphase) {
-        DcSlice s = dc_slice(P, ph, c);
-        uint8_t *dst = ring + (size_t)(ph % DC_NB) * slot_bytes;
-        const int wchunks = s.rows * s.K / 16, vchunks = s.rows * 4 / 16;
-        const int nv = s.inv ? 3 : 2;
-        for (int i = threadIdx.x; i < wchunks + nv * vchunks; i += DC_THREADS) {
-            if (i < wchunks) {
-                dc_cp16(dst + i * 16, s.w + (size_t)i * 16);
-            } else {
-                const int j = i - wchunks, v = j / vchunks, k = j - v * vchunks;
-                const float *src = v == 0 ? s.s : (v == 1 ? s.b : s.inv);
-                dc_cp16(dst + wchunks * 16 + j * 16, reinterpret_cast<const uint8_t *>(src) + k * 16);
-            }
+MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring) {
+    if (ph < 1 + 6 * P.n_dec) {
+        const DcPhase &f = P.phase[ph];
+        if (f.rows) {
+            uint8_t *dst = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
+            const int wb = f.rows * f.K, vb = f.rows * 4;
+            dc_copy(dst, f.w + (size_t)c * wb, wb);
+            dc_copy(dst + wb, f.s + c * f.rows, vb);
+            dc_copy(dst + wb + vb, f.b + c * f.rows, vb);
+            if (f.inv) dc_copy(dst + wb + 2 * vb, f.inv + c * f.rows, vb);
         }
     }
     dc_commit();
@@ -120,89 +84,46 @@ MNMT_DEV void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int r
     }
 }
 
-// Block-wide LayerNorm of the R rows of r: 8/R' warps per row (R' = R rounded
-// up to a power of two), partial maxima and exact int64 sums combined through
-// shared memory.  q8(LN(r), inv) goes to a; with write_back the normalised row
-// also replaces r.  Same arithmetic as warp_layernorm.
+// LayerNorm of the R rows of r, warp m < R on row m; q8(LN(r), inv) into a,
+// and with write_back the normalised row also replaces r.  The caller
+// synchronises the block afterwards.
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
-                                          int8_t *a, int write_back, int *status, float *red_f,
-                                          long long *red_l) {
+                                          int8_t *a, int write_back, int *status) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int rp = R <= 1 ? 1 : (R <= 2 ? 2 : 4);
-    const int wpr = DC_WARPS / rp;          // warps per row
-    const int m = warp / wpr, wi = warp - m * wpr;
-    const bool active = m < R;
-    const int chunk = d / wpr;              // elements of the row this warp owns
-    const int i0 = wi * chunk;
-    const int log2d = 31 - __clz(d);
-    float *row = r + (size_t)m * d;
-    // max |x|
-    float amax = 0.0f;
-    if (active)
-        for (int i = i0 + lane; i < i0 + chunk; i += 32) amax = fmaxf(amax, fabsf(row[i]));
-    amax = warp_max_f(amax);
-    if (lane == 0) red_f[warp] = amax;
-    __syncthreads();
-    amax = 0.0f;
-    for (int w = 0; w < wpr; w++) amax = fmaxf(amax, red_f[m * wpr + w < DC_WARPS ? m * wpr + w : 0]);
-    const bool ok = amax < 0x1p32f;
-    const int ea = exp_bound(amax);
-    long long s1 = 0;
-    if (active)
-        for (int i = i0 + lane; i < i0 + chunk; i += 32) s1 += fx_scale(row[i], 52 - ea);
-    s1 = warp_sum_ll(s1);
-    __syncthreads();
-    if (lane == 0) red_l[warp] = s1;
-    __syncthreads();
-    s1 = 0;
-    for (int w = 0; w < wpr; w++) s1 += red_l[m * wpr + w < DC_WARPS ? m * wpr + w : 0];
-    const float mu = rn32_pow2(s1, ea - 52 - log2d);
-    float bmax = 0.0f;
-    if (active)
-        for (int i = i0 + lane; i < i0 + chunk; i += 32) bmax = fmaxf(bmax, fabsf(__fsub_rn(row[i], mu)));
-    bmax = warp_max_f(bmax);
-    __syncthreads();
-    if (lane == 0) red_f[warp] = bmax;
-    __syncthreads();
-    bmax = 0.0f;
-    for (int w = 0; w < wpr; w++) bmax = fmaxf(bmax, red_f[m * wpr + w < DC_WARPS ? m * wpr + w : 0]);
-    const int eb = exp_bound(bmax);
-    long long s2 = 0;
-    if (active)
-        for (int i = i0 + lane; i < i0 + chunk; i += 32) {
-            float c = __fsub_rn(row[i], mu);
-            s2 += fx_scale(__fmul_rn(c, c), 52 - 2 * eb);
-        }
-    s2 = warp_sum_ll(s2);
-    __syncthreads();
-    if (lane == 0) red_l[warp] = s2;
-    __syncthreads();
-    s2 = 0;
-    for (int w = 0; w < wpr; w++) s2 += red_l[m * wpr + w < DC_WARPS ? m * wpr + w : 0];
-    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
-    const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
-    if (active) {
-        if (!ok && wi == 0 && lane == 0) set_status(status, MNMT_EOVERFLOW);
-        for (int i = i0 + lane; i < i0 + chunk; i += 32) {
-            float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(row[i], mu), rstd), g[i]), b[i]);
-            a[(size_t)m * d + i] = q8(y, inv);
-            if (write_back) row[i] = y;
+    if (warp >= R) return;
+    float *row = r + (size_t)warp * d;
+    float x[16], y[16];
+#pragma unroll
+    for (int u = 0; u < 16; u++) {
+        const int i = u * 32 + lane;
+        x[u] = i < d ? row[i] : 0.0f;
+    }
+    if (!warp_layernorm<16>(x, d, g, b, y, lane)) {
+        if (lane == 0) set_status(status, MNMT_EOVERFLOW);
+        return;
+    }
+#pragma unroll
+    for (int u = 0; u < 16; u++) {
+        const int i = u * 32 + lane;
+        if (i < d) {
+            a[(size_t)warp * d + i] = q8(y[u], inv);
+            if (write_back) row[i] = y[u];
         }
     }
-    __syncthreads();
 }
 
-// Attention of every (row, head) of the step, redundantly in each CTA.  The
-// 8 warps split the keys of an item (row, head) into ranges: scores and the
-// partial maximum per range, then the weights, partial Z and partial context
-// sums per range; the partials are exact integers, so they combine in any
-// order.  self: keys 0..t-1 from the layer's cache, key t from the step's own
-// k/v rows; cross: keys j < src_len of the row's sentence.
+// Attention of every (row, head) of the step, redundantly in each CTA.  The 8
+// warps split the keys of an item (row, head) into ranges: scores and the
+// partial maximum per range, then weights, partial Z and partial context sums
+// per range; the partials are exact integers, so they combine in any order.
+// self: keys 0..t-1 from the layer's cache (staged or global), key t from the
+// step's own k/v rows; cross: keys j < src_len of the row's sentence.
 template <int DH>
-__device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, int cross, const int8_t *q,
-                                          int q_ld, const int8_t *knew, const int8_t *vnew, int kv_ld, int t,
-                                          int8_t *ctx, int *att, float *red_f, long long *pz,
-                                          long long *pn) {
+__device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
+                                          const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx,
+                                          int *att, float *red_f, long long *pz, long long *pn,
+                                          const uint8_t *smem) {
+    const DcLayer &Y = P.layer[l];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int H = P.H, T = P.T, S = P.S, R = P.R;
     const float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
@@ -220,17 +141,28 @@ __device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, i
         if (cross) {
             n = P.src_len[m];
             n = n < 1 ? 1 : (n > S ? S : n);
-            kb = Y.cross_k + ((size_t)m * H + h) * S * DH;
-            vb = Y.cross_v + ((size_t)m * H + h) * S * DH;
+            if (P.kv_staged) {
+                const int8_t *cb = reinterpret_cast<const int8_t *>(smem + P.off_kvc);
+                kb = cb + (((size_t)(l * 2 + 0) * R + m) * H + h) * S * DH;
+                vb = cb + (((size_t)(l * 2 + 1) * R + m) * H + h) * S * DH;
+            } else {
+                kb = Y.cross_k + ((size_t)m * H + h) * S * DH;
+                vb = Y.cross_v + ((size_t)m * H + h) * S * DH;
+            }
         } else {
             n = t + 1;
-            kb = Y.self_k + ((size_t)m * H + h) * T * DH;
-            vb = Y.self_v + ((size_t)m * H + h) * T * DH;
+            if (P.kv_staged) {
+                const int8_t *sbp = reinterpret_cast<const int8_t *>(smem + P.off_kvs);
+                kb = sbp + (((size_t)(l * 2 + 0) * R + m) * H + h) * T * DH;
+                vb = sbp + (((size_t)(l * 2 + 1) * R + m) * H + h) * T * DH;
+            } else {
+                kb = Y.self_k + ((size_t)m * H + h) * T * DH;
+                vb = Y.self_v + ((size_t)m * H + h) * T * DH;
+            }
         }
         const int per = (n + wpi - 1) / wpi;
         const int j0 = part * per, j1 = min(n, j0 + per);
         int *sc = att + (warp / wpi) * P.att_cap;
-        // scores of this warp's key range and their maximum
         float mx = -INFINITY;
         if (live) {
             int4 qv[QC];
@@ -243,7 +175,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, i
                 int acc = 0;
 #pragma unroll
                 for (int c = 0; c < QC; c++) acc = dot16(qv[c], kr[c], acc);
-                float sv = __fmul_rn(__int2float_rn(acc), sigma);
+                const float sv = __fmul_rn(__int2float_rn(acc), sigma);
                 sc[j] = __float_as_int(sv);
                 mx = fmaxf(mx, sv);
             }
@@ -253,11 +185,10 @@ __device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, i
         __syncthreads();
         mx = -INFINITY;
         for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp / wpi) * wpi + w]);
-        // weights, partial Z and partial context sums of this warp's keys
         long long z = 0;
         if (live)
             for (int j = j0 + lane; j < j1; j += 32) {
-                int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
+                const int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
                 sc[j] = E;
                 z += E;
             }
@@ -291,14 +222,12 @@ __device__ __noinline__ void dc_attention(const DcParams &P, const DcLayer &Y, i
                 lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
             }
         }
-        // partials of this warp: pn[warp][e] (exact int64), pz[warp]
         if (g == 0) {
 #pragma unroll
             for (int u = 0; u < 16; u++) pn[warp * DH + c * 16 + u] = (long long)hi[u] * 4096 + lo[u];
         }
         if (lane == 0) pz[warp] = z;
         __syncthreads();
-        // combine the ranges of each item and requantise
         for (int x = threadIdx.x; x < ip * DH; x += DC_THREADS) {
             const int ii = x / DH, e = x - ii * DH;
             const int it2 = base + ii;
@@ -336,9 +265,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
     const int nc = P.nc;
-    const int R = P.R, d = P.d, F = P.F;
+    const int R = P.R, d = P.d, F = P.F, H = P.H;
     const int t = *P.t_ptr;
-    const int nsd = d / nc, ns3 = 3 * d / nc, nsf = F / nc;
 
     float *r_full = reinterpret_cast<float *>(smem + P.off_r);
     int8_t *a_full = reinterpret_cast<int8_t *>(smem + P.off_a);
@@ -349,40 +277,52 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     uint8_t *stage = smem + P.off_stage;
     int *att = reinterpret_cast<int *>(smem + P.off_att);
     uint8_t *ring = smem + P.off_ring;
-    float *lnp = reinterpret_cast<float *>(smem + P.off_ln);  // [n_dec][6][d] + final [2][d]
-    float *red_f = reinterpret_cast<float *>(smem + P.off_red);          // [8]
+    float *lnp = reinterpret_cast<float *>(smem + P.off_ln);                  // [n_dec][6][d] + final [2][d]
+    float *red_f = reinterpret_cast<float *>(smem + P.off_red);               // [8]
     long long *red_l = reinterpret_cast<long long *>(smem + P.off_red + 64);  // [8]
     long long *pn = reinterpret_cast<long long *>(smem + P.off_red + 128);    // [8][DH]
     int *tok_s = reinterpret_cast<int *>(smem + P.off_red + 128 + 8 * DH * 8);  // [R]
     const int nphase = 1 + 6 * P.n_dec;
 
-    // LayerNorm gains / biases of every layer (and the final LN), in the first
-    // cp.async group together with the first weight slice
-    {
-        const int cpa = d / 4;  // 16-byte chunks per d-vector of fp32
-        const int nvec = 6 * P.n_dec + 2;
-        for (int i = threadIdx.x; i < nvec * cpa; i += DC_THREADS) {
-            const int v = i / cpa, k = i - v * cpa;
-            const float *src;
-            if (v < 6 * P.n_dec) {
-                const DcLayer &Y = P.layer[v / 6];
-                const int w = v % 6;
-                src = w == 0 ? Y.ln1_g : w == 1 ? Y.ln1_b : w == 2 ? Y.ln2_g : w == 3 ? Y.ln2_b : w == 4 ? Y.ln3_g : Y.ln3_b;
-            } else {
-                src = v == 6 * P.n_dec ? P.fin_g : P.fin_b;
-            }
-            if (src) dc_cp16(lnp + (size_t)v * d + k * 4, src + k * 4);
+    // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
+    for (int v = 0; v < 6 * P.n_dec + 2; v++) {
+        const float *src;
+        if (v < 6 * P.n_dec) {
+            const DcLayer &Y = P.layer[v / 6];
+            const int w = v % 6;
+            src = w == 0 ? Y.ln1_g : w == 1 ? Y.ln1_b : w == 2 ? Y.ln2_g : w == 3 ? Y.ln2_b : w == 4 ? Y.ln3_g : Y.ln3_b;
+        } else {
+            src = v == 6 * P.n_dec ? P.fin_g : P.fin_b;
         }
-        if (threadIdx.x < R) {
-            int id = P.tok[threadIdx.x];
-            if (id < 0 || id >= P.V) {
-                set_status(P.status, MNMT_EINVAL);
-                id = 0;
+        if (src) dc_copy(lnp + (size_t)v * d, src, d * 4);
+    }
+    if (threadIdx.x < R) {
+        int id = P.tok[threadIdx.x];
+        if (id < 0 || id >= P.V) {
+            set_status(P.status, MNMT_EINVAL);
+            id = 0;
+        }
+        tok_s[threadIdx.x] = id;
+    }
+    dc_prefetch(P, 0, c, ring);
+    // group 1: the second weight slice and the keys / values the step attends to
+    if (P.kv_staged) {
+        for (int l = 0; l < P.n_dec; l++) {
+            const DcLayer &Y = P.layer[l];
+            const int cb = R * P.S * d;  // one layer's cross K (or V): [R][H][S][dh]
+            dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 0) * cb, Y.cross_k, cb);
+            dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 1) * cb, Y.cross_v, cb);
+            if (t > 0) {
+                const int seg = t * DH;  // positions 0..t-1 of one (row, head)
+                for (int x = 0; x < 2 * R * H; x++) {
+                    const int kv = x / (R * H), mh = x - kv * R * H;
+                    const size_t off = ((size_t)(l * 2 + kv) * R * H + mh) * P.T * DH;
+                    dc_copy(smem + P.off_kvs + off, (kv ? Y.self_v : Y.self_k) + (size_t)mh * P.T * DH, seg);
+                }
             }
-            tok_s[threadIdx.x] = id;
         }
     }
-    for (int ph = 0; ph < DC_NB - 1; ph++) dc_prefetch(P, ph, c, ring, P.slot_bytes, nphase);
+    dc_prefetch(P, 1, c, ring);
 
     for (int ph = 0; ph < nphase; ph++) {
         const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
@@ -390,7 +330,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const DcLayer &Y = P.layer[l];
         dc_wait_ring();
         __syncthreads();
-        dc_prefetch(P, ph + DC_NB - 1, c, ring, P.slot_bytes, nphase);
+        dc_prefetch(P, ph + DC_NB - 1, c, ring);
         const uint8_t *slot = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
         const float *lnl = lnp + (size_t)6 * l * d;
 
@@ -402,50 +342,49 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 for (int i = threadIdx.x; i < R * P.E; i += DC_THREADS)
                     a_full[i] = P.emb_q[(size_t)tok_s[i / P.E] * P.E + (i % P.E)];
             K = P.E;
-            __syncthreads();
         } else if (kind == K_QKV || kind == K_Q2 || kind == K_W1) {
             // pre-LN: LN of this sublayer; post-LN: LN of the previous sublayer's
             // residual (written back), or plain quantisation for the first one
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status,
-                             red_f, red_l);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
-                __syncthreads();
             } else {
-                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1,
-                             P.status, red_f, red_l);
+                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
-            dc_attention<DH>(P, Y, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
-                             qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn);
+            dc_attention<DH>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
+                             qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn, smem);
             A = ctx_full;
         } else {  // K_W2
             A = h_full;
             K = F;
         }
+        __syncthreads();
 
         // ---- the phase's slice of outputs ----
-        int rows, n0, out_f32;
+        const int rows = ph == 0 ? d / nc : P.phase[ph].rows;
+        const int n0 = c * rows;
+        int out_f32;
         float sx, gam;
         switch (kind) {
-            case K_EMB: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = 0.0f; gam = 0.0f; break;
-            case K_QKV: rows = ns3; n0 = c * ns3; out_f32 = 0; sx = Y.s_in1; gam = 0.0f; break;
-            case K_O: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_ctx1; gam = Y.gamma1; break;
-            case K_Q2: rows = nsd; n0 = c * nsd; out_f32 = 0; sx = Y.s_in2; gam = 0.0f; break;
-            case K_O2: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_ctx2; gam = Y.gamma2; break;
-            case K_W1: rows = nsf; n0 = c * nsf; out_f32 = 0; sx = Y.s_in3; gam = 0.0f; break;
-            default: rows = nsd; n0 = c * nsd; out_f32 = 1; sx = Y.s_h; gam = Y.gamma3; break;
+            case K_EMB: out_f32 = 1; sx = 0.0f; gam = 0.0f; break;
+            case K_QKV: out_f32 = 0; sx = Y.s_in1; gam = 0.0f; break;
+            case K_O: out_f32 = 1; sx = Y.s_ctx1; gam = Y.gamma1; break;
+            case K_Q2: out_f32 = 0; sx = Y.s_in2; gam = 0.0f; break;
+            case K_O2: out_f32 = 1; sx = Y.s_ctx2; gam = Y.gamma2; break;
+            case K_W1: out_f32 = 0; sx = Y.s_in3; gam = 0.0f; break;
+            default: out_f32 = 1; sx = Y.s_h; gam = Y.gamma3; break;
         }
         float *stf = reinterpret_cast<float *>(stage);
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
         if (kind == K_EMB && !P.factorised) {
-            for (int i = threadIdx.x; i < R * nsd; i += DC_THREADS) {
-                const int m = i / nsd, nl = i - m * nsd, n = n0 + nl, id = tok_s[m];
-                float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
+            for (int i = threadIdx.x; i < R * rows; i += DC_THREADS) {
+                const int m = i / rows, nl = i - m * rows, n = n0 + nl, id = tok_s[m];
+                const float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
                 stf[i] = __fadd_rn(v, P.pe[(size_t)t * d + n]);
             }
         } else {
@@ -453,17 +392,19 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const float *sw = reinterpret_cast<const float *>(slot + rows * K);
             const float *bb = sw + rows;
             const float *iv = bb + rows;
-            const int kc = K / 16;
-            const int lpc = kc >= 32 ? 32 : kc;
-            const int gpw = 32 / lpc;
+            const int kc = K / 16;                 // 16-byte chunks per row
+            const int lpr = kc >= 4 ? kc / 4 : 1;  // lanes per row: each lane takes kc / lpr chunks
+            const int cpl = kc / lpr;
+            const int rpw = 32 / lpr;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-            const int grp = lane / lpc, sl = lane % lpc;
-            for (int r0 = warp * gpw; r0 < rows; r0 += DC_WARPS * gpw) {
-                const int nl = r0 + grp;
+            const int sub = lane % lpr;
+            for (int r0 = warp * rpw; r0 < rows; r0 += DC_WARPS * rpw) {
+                const int nl = r0 + lane / lpr;
                 int acc[DC_RMAX] = {0, 0, 0, 0};
                 if (nl < rows) {
                     const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * K);
-                    for (int k = sl; k < kc; k += lpc) {
+                    for (int q = 0; q < cpl; q++) {
+                        const int k = q * lpr + sub;  // consecutive lanes read consecutive chunks
                         const int4 w = wr[k];
 #pragma unroll
                         for (int m = 0; m < DC_RMAX; m++)
@@ -472,19 +413,19 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 }
 #pragma unroll
                 for (int m = 0; m < DC_RMAX; m++)
-                    for (int o = lpc / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
-                if (sl == 0 && nl < rows) {
+                    if (m < R)
+                        for (int o = lpr / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
+                if (sub == 0 && nl < rows) {
                     const int n = n0 + nl;
 #pragma unroll
                     for (int m = 0; m < DC_RMAX; m++) {
                         if (m >= R) break;
-                        float y;
                         if (kind == K_EMB) {
-                            y = dequant_bias(acc[m], P.emb_s[tok_s[m]], sw[nl], bb[nl]);
+                            const float y = dequant_bias(acc[m], P.emb_s[tok_s[m]], sw[nl], bb[nl]);
                             stf[m * rows + nl] = __fadd_rn(__fmul_rn(y, P.emb_scale), P.pe[(size_t)t * d + n]);
                             continue;
                         }
-                        y = dequant_bias(acc[m], sx, sw[nl], bb[nl]);
+                        const float y = dequant_bias(acc[m], sx, sw[nl], bb[nl]);
                         if (out_f32) {
                             stf[m * rows + nl] = __fadd_rn(__fmul_rn(gam, r_full[(size_t)m * d + n]), y);
                         } else {
@@ -494,7 +435,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                                 const int seg = n >= 2 * d;
                                 const int cc = n - (seg ? 2 * d : d);
                                 const int hh = cc / DH, ii = cc - hh * DH;
-                                (seg ? Y.self_v : Y.self_k)[(((size_t)m * P.H + hh) * P.T + t) * DH + ii] = v;
+                                (seg ? Y.self_v : Y.self_k)[(((size_t)m * H + hh) * P.T + t) * DH + ii] = v;
                             }
                         }
                     }
@@ -515,13 +456,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, red_f, red_l);
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status);
+            __syncthreads();
         }
     }
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     1.0f / P.s_dout, a_full, 0, P.status, red_f, red_l);
+                     1.0f / P.s_dout, a_full, 0, P.status);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -653,7 +595,25 @@ int dc_cluster_size(int d) {
     return nc >= 2 ? nc : 0;
 }
 
-size_t dc_layout(DcParams &P) {
+// Fills the phase table and the shared-memory carve-up; returns the bytes of
+// shared memory one CTA needs (staging the keys / values when they fit in
+// max_smem).
+size_t dc_layout(DcParams &P, size_t max_smem) {
+    const int R = P.R, d = P.d, F = P.F, nc = P.nc;
+    // phase table: slices of CTA c are rows [c * rows, (c + 1) * rows)
+    DcPhase z = {nullptr, nullptr, nullptr, nullptr, 0, 0};
+    P.phase[0] = z;
+    if (P.factorised) P.phase[0] = DcPhase{P.proj.w, P.proj.s, P.proj.b, nullptr, d / nc, P.E};
+    for (int l = 0; l < P.n_dec; l++) {
+        const DcLayer &Y = P.layer[l];
+        DcPhase *f = &P.phase[1 + 6 * l];
+        f[0] = DcPhase{Y.qkv.w, Y.qkv.s, Y.qkv.b, Y.inv_qkv, 3 * d / nc, d};
+        f[1] = DcPhase{Y.o.w, Y.o.s, Y.o.b, nullptr, d / nc, d};
+        f[2] = DcPhase{Y.q2.w, Y.q2.s, Y.q2.b, Y.inv_q2, d / nc, d};
+        f[3] = DcPhase{Y.o2.w, Y.o2.s, Y.o2.b, nullptr, d / nc, d};
+        f[4] = DcPhase{Y.w1.w, Y.w1.s, Y.w1.b, Y.inv_h, F / nc, d};
+        f[5] = DcPhase{Y.w2.w, Y.w2.s, Y.w2.b, nullptr, d / nc, F};
+    }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -661,7 +621,6 @@ size_t dc_layout(DcParams &P) {
         off += (bytes + 15) & ~(size_t)15;
         return (int)at;
     };
-    const int R = P.R, d = P.d, F = P.F, nc = P.nc;
     take(sizeof(DcParams));  // the parameter block itself
     P.off_ln = take((size_t)(6 * P.n_dec + 2) * d * 4);
     P.off_r = take((size_t)R * d * 4);
@@ -676,21 +635,23 @@ size_t dc_layout(DcParams &P) {
     P.off_stage = take(stage_bytes);
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
-    P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // red_f, red_l, pn[8][dh], tokens
-    // largest weight slice of any phase (rows * K + 8 * rows)
+    P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
     int slot = 0;
-    auto upd = [&](int rows, int K) {
-        int b = rows * K + 12 * rows;
+    for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
+        const DcPhase &f = P.phase[ph];
+        int b = f.rows * f.K + 12 * f.rows;
         if (b > slot) slot = b;
-    };
-    if (P.factorised) upd(d / nc, P.E);
-    if (P.factorised && R * P.E > R * d) return (size_t)-1;  // a_full holds the embedding rows
-    upd(3 * d / nc, d);
-    upd(d / nc, d);
-    upd(F / nc, d);
-    upd(d / nc, F);
+    }
     P.slot_bytes = (slot + 15) & ~15;
     P.off_ring = take((size_t)DC_NB * P.slot_bytes);
+    // keys / values of every decoder layer: cross [L][2][R][H][S][dh], self [L][2][R][H][T][dh]
+    const size_t kvc = (size_t)P.n_dec * 2 * R * P.S * d, kvs = (size_t)P.n_dec * 2 * R * P.T * d;
+    P.kv_staged = 0;
+    if (off + kvc + kvs + 32 <= max_smem) {
+        P.kv_staged = 1;
+        P.off_kvc = take(kvc);
+        P.off_kvs = take(kvs);
+    }
     return off;
 }
 

@@ -174,6 +174,14 @@ struct DcLayer {
     int8_t *self_k, *self_v;          // [R][H][T][dh]
     const int8_t *cross_k, *cross_v;  // [B][H][S][dh]
 };
+// weight slice table of the step's phases (phase 0: factorised embedding
+// projection, then per layer qkv, o, q2, o2, w1, w2); CTA c's slice is rows
+// [c * rows, (c + 1) * rows) of the [N][K] matrix
+struct DcPhase {
+    const int8_t *w;
+    const float *s, *b, *inv;  // inv: per-column requantisation constants (or null)
+    int rows, K;
+};
 struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
     const int8_t *emb_q;
@@ -192,11 +200,13 @@ struct alignas(16) DcParams {
     // shared-memory carve-up (bytes), filled by dc_layout
     int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, off_ln, off_red, slot_bytes,
         att_cap;
+    int kv_staged, off_kvs, off_kvc;  // self / cross keys and values staged in shared memory
     DcLayer layer[DC_LMAX];
+    DcPhase phase[1 + 6 * DC_LMAX];
 };
 static_assert(sizeof(DcParams) % 16 == 0, "the parameter block is copied in 16-byte chunks");
 int dc_cluster_size(int d);
-size_t dc_layout(DcParams &P);
+size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
 bool decode_cluster_fits(int dh, int nc, size_t smem);
 cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, cudaStream_t st);
