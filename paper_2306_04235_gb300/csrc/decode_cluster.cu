@@ -84,32 +84,123 @@ MNMT_DEV void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int r
     }
 }
 
-// LayerNorm of the R rows of r, warp m < R on row m; q8(LN(r), inv) into a,
-// and with write_back the normalised row also replaces r.  The caller
-// synchronises the block afterwards.
+// Block-wide LayerNorm of the R rows of r (same arithmetic as
+// warp_layernorm): element e of the flattened [R][d] array belongs to thread
+// e % 256; each warp's 32 elements lie in one row, so per-row maxima and exact
+// int64 sums are warp reductions (redux.sync) whose partials meet in shared
+// memory, d/32 partials per row.  q8(LN(r), inv) goes to a; with write_back
+// the normalised row also replaces r.  Ends with a block barrier.
+constexpr int DC_LN_EPT = 8;  // elements per thread: R * d <= 2048
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
-                                          int8_t *a, int write_back, int *status) {
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (warp >= R) return;
-    float *row = r + (size_t)warp * d;
-    float x[16], y[16];
+                                          int8_t *a, int write_back, int *status, unsigned *part_u,
+                                          long long *part_l) {
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int n = R * d, spr = d / 32;  // slots (warp partials) per row
+    const int log2d = 31 - __clz(d);
+    float x[DC_LN_EPT], cc[DC_LN_EPT];
+    int ea[DC_LN_EPT], eb[DC_LN_EPT];
+    float mu[DC_LN_EPT];
 #pragma unroll
-    for (int u = 0; u < 16; u++) {
-        const int i = u * 32 + lane;
-        x[u] = i < d ? row[i] : 0.0f;
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e = tid + DC_THREADS * u;
+        x[u] = e < n ? r[e] : 0.0f;
     }
-    if (!warp_layernorm<16>(x, d, g, b, y, lane)) {
-        if (lane == 0) set_status(status, MNMT_EOVERFLOW);
-        return;
-    }
+    // max |x| per row
 #pragma unroll
-    for (int u = 0; u < 16; u++) {
-        const int i = u * 32 + lane;
-        if (i < d) {
-            a[(size_t)warp * d + i] = q8(y[u], inv);
-            if (write_back) row[i] = y[u];
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e0 = tid - lane + DC_THREADS * u;  // warp-uniform
+        if (e0 < n) {
+            const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(x[u]) & 0x7FFFFFFFu);
+            if (lane == 0) part_u[e0 / 32] = m;
         }
     }
+    __syncthreads();
+    bool ok = true;
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e = tid + DC_THREADS * u;
+        ea[u] = 0;
+        if (e < n) {
+            const int s0 = (e / d) * spr;
+            unsigned m = 0;
+            for (int k = 0; k < spr; k++) m = max(m, part_u[s0 + k]);
+            const float amax = __uint_as_float(m);
+            ok = ok && amax < 0x1p32f;
+            ea[u] = exp_bound(amax);
+        }
+    }
+    // exact sum of x on the row's grid -> mean
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e0 = tid - lane + DC_THREADS * u;
+        if (e0 < n) {
+            const long long s = warp_sum_exact(fx_scale(x[u], 52 - ea[u]));
+            if (lane == 0) part_l[e0 / 32] = s;
+        }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e = tid + DC_THREADS * u;
+        mu[u] = 0.0f;
+        cc[u] = 0.0f;
+        if (e < n) {
+            const int s0 = (e / d) * spr;
+            long long s1 = 0;
+            for (int k = 0; k < spr; k++) s1 += part_l[s0 + k];
+            mu[u] = rn32_pow2(s1, ea[u] - 52 - log2d);
+            cc[u] = __fsub_rn(x[u], mu[u]);
+        }
+    }
+    __syncthreads();  // part_u / part_l are reused below
+    // max |x - mean| per row
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e0 = tid - lane + DC_THREADS * u;
+        if (e0 < n) {
+            const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(cc[u]) & 0x7FFFFFFFu);
+            if (lane == 0) part_u[e0 / 32] = m;
+        }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e = tid + DC_THREADS * u;
+        eb[u] = 0;
+        if (e < n) {
+            const int s0 = (e / d) * spr;
+            unsigned m = 0;
+            for (int k = 0; k < spr; k++) m = max(m, part_u[s0 + k]);
+            eb[u] = exp_bound(__uint_as_float(m));
+        }
+    }
+    // exact sum of squares on the row's grid -> biased variance
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e0 = tid - lane + DC_THREADS * u;
+        if (e0 < n) {
+            const long long s = warp_sum_exact(fx_scale(__fmul_rn(cc[u], cc[u]), 52 - 2 * eb[u]));
+            if (lane == 0) part_l[e0 / 32] = s;
+        }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int u = 0; u < DC_LN_EPT; u++) {
+        const int e = tid + DC_THREADS * u;
+        if (e < n) {
+            const int row = e / d, i = e - row * d;
+            const int s0 = row * spr;
+            long long s2 = 0;
+            for (int k = 0; k < spr; k++) s2 += part_l[s0 + k];
+            const float var = rn32_pow2(s2, 2 * eb[u] - 52 - log2d);
+            const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+            const float y = __fadd_rn(__fmul_rn(__fmul_rn(cc[u], rstd), g[i]), b[i]);
+            a[e] = q8(y, inv);
+            if (write_back) r[e] = y;
+        }
+    }
+    if (!ok) set_status(status, MNMT_EOVERFLOW);
+    __syncthreads();
 }
 
 // Attention of every (row, head) of the step, redundantly in each CTA.  The 8
@@ -131,7 +222,6 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
     const int ip = items >= DC_WARPS ? DC_WARPS : (items > 4 ? 8 : (items > 2 ? 4 : (items > 1 ? 2 : 1)));
     const int wpi = DC_WARPS / ip;  // warps per item in a round of ip items
     constexpr int QC = DH / 16;
-    constexpr int C = DH / 16, G = 32 / C;
     for (int base = 0; base < items; base += ip) {
         const int it = base + warp / wpi, part = warp % wpi;
         const bool live = it < items;
@@ -185,47 +275,50 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
         __syncthreads();
         mx = -INFINITY;
         for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp / wpi) * wpi + w]);
-        long long z = 0;
+        int zl = 0;
         if (live)
             for (int j = j0 + lane; j < j1; j += 32) {
                 const int E = softmax_weight(__fadd_rn(__int_as_float(sc[j]), -mx));
                 sc[j] = E;
-                z += E;
+                zl += E;  // at most 32 keys per lane: < 2^30
             }
-        z = warp_sum_ll(z);
+        const long long z = warp_sum_exact(zl);
         __syncwarp();
-        const int g = lane / C, c = lane - g * C;
-        int hi[16], lo[16];
+        // context: lane l owns elements [l * EPL, (l + 1) * EPL) of the head and
+        // walks the warp's keys (consecutive lanes read consecutive bytes)
+        constexpr int EPL = DH / 32;
+        int hi[EPL], lo[EPL];
 #pragma unroll
-        for (int u = 0; u < 16; u++) hi[u] = lo[u] = 0;
-        if (live)
-            for (int j = j0 + g; j < j1; j += G) {
+        for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
+        if (live) {
+#pragma unroll 4
+            for (int j = j0; j < j1; j++) {
                 const int E = sc[j];
                 const int Eh = E >> 12, El = E & 4095;
-                const int4 v = (!cross && j == t) ? reinterpret_cast<const int4 *>(vnew + (size_t)m * kv_ld + h * DH)[c]
-                                                  : reinterpret_cast<const int4 *>(vb + (size_t)j * DH)[c];
-                const int w4[4] = {v.x, v.y, v.z, v.w};
+                const int8_t *vr = (!cross && j == t) ? vnew + (size_t)m * kv_ld + h * DH : vb + (size_t)j * DH;
+                int v[EPL];
+                if constexpr (EPL == 1) {
+                    v[0] = vr[lane];
+                } else if constexpr (EPL == 2) {
+                    const char2 x2 = reinterpret_cast<const char2 *>(vr)[lane];
+                    v[0] = x2.x;
+                    v[1] = x2.y;
+                } else {
+                    const char4 x4 = reinterpret_cast<const char4 *>(vr)[lane];
+                    v[0] = x4.x;
+                    v[1] = x4.y;
+                    v[2] = x4.z;
+                    v[3] = x4.w;
+                }
 #pragma unroll
-                for (int q4 = 0; q4 < 4; q4++) {
-                    const int b0 = sb0(w4[q4]), b1 = sb1(w4[q4]), b2 = sb2(w4[q4]), b3 = sb3(w4[q4]);
-                    hi[q4 * 4 + 0] += Eh * b0; lo[q4 * 4 + 0] += El * b0;
-                    hi[q4 * 4 + 1] += Eh * b1; lo[q4 * 4 + 1] += El * b1;
-                    hi[q4 * 4 + 2] += Eh * b2; lo[q4 * 4 + 2] += El * b2;
-                    hi[q4 * 4 + 3] += Eh * b3; lo[q4 * 4 + 3] += El * b3;
+                for (int u = 0; u < EPL; u++) {
+                    hi[u] += Eh * v[u];
+                    lo[u] += El * v[u];
                 }
             }
-#pragma unroll
-        for (int o = C; o < 32; o <<= 1) {
-#pragma unroll
-            for (int u = 0; u < 16; u++) {
-                hi[u] += __shfl_xor_sync(0xFFFFFFFFu, hi[u], o);
-                lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
-            }
         }
-        if (g == 0) {
 #pragma unroll
-            for (int u = 0; u < 16; u++) pn[warp * DH + c * 16 + u] = (long long)hi[u] * 4096 + lo[u];
-        }
+        for (int u = 0; u < EPL; u++) pn[warp * DH + lane * EPL + u] = (long long)hi[u] * 4096 + lo[u];
         if (lane == 0) pz[warp] = z;
         __syncthreads();
         for (int x = threadIdx.x; x < ip * DH; x += DC_THREADS) {
@@ -282,6 +375,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     long long *red_l = reinterpret_cast<long long *>(smem + P.off_red + 64);  // [8]
     long long *pn = reinterpret_cast<long long *>(smem + P.off_red + 128);    // [8][DH]
     int *tok_s = reinterpret_cast<int *>(smem + P.off_red + 128 + 8 * DH * 8);  // [R]
+    unsigned *part_u = reinterpret_cast<unsigned *>(smem + P.off_part);           // [64] LN partials
+    long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 256);    // [64]
     const int nphase = 1 + 6 * P.n_dec;
 
     // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
@@ -348,11 +443,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, part_u, part_l);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
             } else {
-                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status);
+                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status, part_u,
+                             part_l);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
@@ -456,14 +552,13 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status);
-            __syncthreads();
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, part_u, part_l);
         }
     }
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     1.0f / P.s_dout, a_full, 0, P.status);
+                     1.0f / P.s_dout, a_full, 0, P.status, part_u, part_l);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -636,6 +731,8 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
+    P.off_part = take(256 + 512);                                   // LayerNorm partials (64 rows of 32)
+    if (R * d > 256 * 8) return (size_t)-1;                        // block LayerNorm covers R * d <= 2048
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const DcPhase &f = P.phase[ph];
