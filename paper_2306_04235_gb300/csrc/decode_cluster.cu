@@ -42,6 +42,10 @@ MNMT_DEV void dc_cp16(void *dst_smem, const void *src) {
 MNMT_DEV void dc_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 MNMT_DEV void dc_wait_ring() { asm volatile("cp.async.wait_group %0;\n" ::"n"(DC_NB - 2)); }
 
+// out-of-line copies of the exact roundings (one copy of the code each)
+__device__ __noinline__ float dc_rn32_div(long long n, long long z) { return rn32_div(n, z); }
+__device__ __noinline__ float dc_rn32_pow2(long long s, int e) { return rn32_pow2(s, e); }
+
 // signed bytes of a 32-bit word
 MNMT_DEV int sb0(int x) { return (x << 24) >> 24; }
 MNMT_DEV int sb1(int x) { return (x << 16) >> 24; }
@@ -55,7 +59,7 @@ MNMT_DEV void dc_copy(void *dst, const void *src, int bytes) {
 }
 
 // ring slot layout: W rows (rows * K bytes), then s[rows], b[rows], inv[rows] (fp32)
-MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring) {
+__device__ __noinline__ void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring) {
     if (ph < 1 + 6 * P.n_dec) {
         const DcPhase &f = P.phase[ph];
         if (f.rows) {
@@ -71,7 +75,7 @@ MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring) {
 }
 
 // copy stage [R][row_bytes] into every CTA's full buffer at column offset
-MNMT_DEV void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int row_bytes, uint8_t *full,
+__device__ __noinline__ void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int row_bytes, uint8_t *full,
                        int full_row_bytes, int col_off, int nc) {
     const int cpr = row_bytes / 16;
     const int total = nc * R * cpr;
@@ -88,118 +92,76 @@ MNMT_DEV void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int r
 // warp_layernorm): element e of the flattened [R][d] array belongs to thread
 // e % 256; each warp's 32 elements lie in one row, so per-row maxima and exact
 // int64 sums are warp reductions (redux.sync) whose partials meet in shared
-// memory, d/32 partials per row.  q8(LN(r), inv) goes to a; with write_back
-// the normalised row also replaces r.  Ends with a block barrier.
-constexpr int DC_LN_EPT = 8;  // elements per thread: R * d <= 2048
+// memory, d/32 partials per row.  The passes keep no per-element registers
+// (r - mean goes through shared memory) and are not unrolled, so the code
+// stays small.  q8(LN(r), inv) goes to a; with write_back the normalised row
+// also replaces r.  Ends with a block barrier.
+MNMT_DEV unsigned dc_row_max(const unsigned *part, int row, int spr) {
+    unsigned m = 0;
+    for (int k = 0; k < spr; k++) m = max(m, part[row * spr + k]);
+    return m;
+}
+MNMT_DEV long long dc_row_sum(const long long *part, int row, int spr) {
+    long long s = 0;
+    for (int k = 0; k < spr; k++) s += part[row * spr + k];
+    return s;
+}
+
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
                                           int8_t *a, int write_back, int *status, unsigned *part_u,
-                                          long long *part_l) {
+                                          long long *part_l, float *cbuf) {
     const int tid = threadIdx.x, lane = tid & 31;
-    const int n = R * d, spr = d / 32;  // slots (warp partials) per row
+    const int n = R * d, spr = d / 32;  // partial slots (warps) per row
     const int log2d = 31 - __clz(d);
-    float x[DC_LN_EPT], cc[DC_LN_EPT];
-    int ea[DC_LN_EPT], eb[DC_LN_EPT];
-    float mu[DC_LN_EPT];
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e = tid + DC_THREADS * u;
-        x[u] = e < n ? r[e] : 0.0f;
-    }
-    // max |x| per row
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e0 = tid - lane + DC_THREADS * u;  // warp-uniform
-        if (e0 < n) {
-            const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(x[u]) & 0x7FFFFFFFu);
-            if (lane == 0) part_u[e0 / 32] = m;
-        }
+    // pass 1: max |x| per warp chunk
+#pragma unroll 1
+    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+        const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(r[e0 + lane]) & 0x7FFFFFFFu);
+        if (lane == 0) part_u[e0 / 32] = m;
     }
     __syncthreads();
-    bool ok = true;
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e = tid + DC_THREADS * u;
-        ea[u] = 0;
-        if (e < n) {
-            const int s0 = (e / d) * spr;
-            unsigned m = 0;
-            for (int k = 0; k < spr; k++) m = max(m, part_u[s0 + k]);
-            const float amax = __uint_as_float(m);
-            ok = ok && amax < 0x1p32f;
-            ea[u] = exp_bound(amax);
-        }
-    }
-    // exact sum of x on the row's grid -> mean
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e0 = tid - lane + DC_THREADS * u;
-        if (e0 < n) {
-            const long long s = warp_sum_exact(fx_scale(x[u], 52 - ea[u]));
-            if (lane == 0) part_l[e0 / 32] = s;
-        }
+    // pass 2: exact sum of x on the row's grid
+#pragma unroll 1
+    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+        const unsigned am = dc_row_max(part_u, e0 / d, spr);
+        if (!(__uint_as_float(am) < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
+        const int ea = exp_bound(__uint_as_float(am));
+        const long long s = warp_sum_exact(fx_scale(r[e0 + lane], 52 - ea));
+        if (lane == 0) part_l[e0 / 32] = s;
     }
     __syncthreads();
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e = tid + DC_THREADS * u;
-        mu[u] = 0.0f;
-        cc[u] = 0.0f;
-        if (e < n) {
-            const int s0 = (e / d) * spr;
-            long long s1 = 0;
-            for (int k = 0; k < spr; k++) s1 += part_l[s0 + k];
-            mu[u] = rn32_pow2(s1, ea[u] - 52 - log2d);
-            cc[u] = __fsub_rn(x[u], mu[u]);
-        }
-    }
-    __syncthreads();  // part_u / part_l are reused below
-    // max |x - mean| per row
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e0 = tid - lane + DC_THREADS * u;
-        if (e0 < n) {
-            const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(cc[u]) & 0x7FFFFFFFu);
-            if (lane == 0) part_u[e0 / 32] = m;
-        }
+    // pass 3: c = x - mean (kept in cbuf), max |c| per warp chunk
+#pragma unroll 1
+    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+        const int row = e0 / d;
+        const int ea = exp_bound(__uint_as_float(dc_row_max(part_u, row, spr)));
+        const float mu = dc_rn32_pow2(dc_row_sum(part_l, row, spr), ea - 52 - log2d);
+        const float cv = __fsub_rn(r[e0 + lane], mu);
+        cbuf[e0 + lane] = cv;
+        const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(cv) & 0x7FFFFFFFu);
+        if (lane == 0) part_u[64 + e0 / 32] = m;
     }
     __syncthreads();
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e = tid + DC_THREADS * u;
-        eb[u] = 0;
-        if (e < n) {
-            const int s0 = (e / d) * spr;
-            unsigned m = 0;
-            for (int k = 0; k < spr; k++) m = max(m, part_u[s0 + k]);
-            eb[u] = exp_bound(__uint_as_float(m));
-        }
-    }
-    // exact sum of squares on the row's grid -> biased variance
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e0 = tid - lane + DC_THREADS * u;
-        if (e0 < n) {
-            const long long s = warp_sum_exact(fx_scale(__fmul_rn(cc[u], cc[u]), 52 - 2 * eb[u]));
-            if (lane == 0) part_l[e0 / 32] = s;
-        }
+    // pass 4: exact sum of c^2 on the row's grid
+#pragma unroll 1
+    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+        const int eb = exp_bound(__uint_as_float(dc_row_max(part_u + 64, e0 / d, spr)));
+        const float cv = cbuf[e0 + lane];
+        const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
+        if (lane == 0) part_l[64 + e0 / 32] = s;
     }
     __syncthreads();
-#pragma unroll
-    for (int u = 0; u < DC_LN_EPT; u++) {
-        const int e = tid + DC_THREADS * u;
-        if (e < n) {
-            const int row = e / d, i = e - row * d;
-            const int s0 = row * spr;
-            long long s2 = 0;
-            for (int k = 0; k < spr; k++) s2 += part_l[s0 + k];
-            const float var = rn32_pow2(s2, 2 * eb[u] - 52 - log2d);
-            const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
-            const float y = __fadd_rn(__fmul_rn(__fmul_rn(cc[u], rstd), g[i]), b[i]);
-            a[e] = q8(y, inv);
-            if (write_back) r[e] = y;
-        }
+    // pass 5: normalise, scale, shift, quantise
+#pragma unroll 1
+    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+        const int row = e0 / d, e = e0 + lane, i = e - row * d;
+        const int eb = exp_bound(__uint_as_float(dc_row_max(part_u + 64, row, spr)));
+        const float var = dc_rn32_pow2(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52 - log2d);
+        const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+        const float y = __fadd_rn(__fmul_rn(__fmul_rn(cbuf[e], rstd), g[i]), b[i]);
+        a[e] = q8(y, inv);
+        if (write_back) r[e] = y;
     }
-    if (!ok) set_status(status, MNMT_EOVERFLOW);
     __syncthreads();
 }
 
@@ -291,7 +253,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
 #pragma unroll
         for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
         if (live) {
-#pragma unroll 4
+#pragma unroll 2
             for (int j = j0; j < j1; j++) {
                 const int E = sc[j];
                 const int Eh = E >> 12, El = E & 4095;
@@ -331,7 +293,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                     Z += pz[ii * wpi + w];
                 }
                 const int m2 = it2 / H, h2 = it2 - m2 * H;
-                ctx[(size_t)m2 * P.d + h2 * DH + e] = q8(rn32_div(N, Z), rho);
+                ctx[(size_t)m2 * P.d + h2 * DH + e] = q8(dc_rn32_div(N, Z), rho);
             }
         }
         __syncthreads();
@@ -375,8 +337,9 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     long long *red_l = reinterpret_cast<long long *>(smem + P.off_red + 64);  // [8]
     long long *pn = reinterpret_cast<long long *>(smem + P.off_red + 128);    // [8][DH]
     int *tok_s = reinterpret_cast<int *>(smem + P.off_red + 128 + 8 * DH * 8);  // [R]
-    unsigned *part_u = reinterpret_cast<unsigned *>(smem + P.off_part);           // [64] LN partials
-    long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 256);    // [64]
+    unsigned *part_u = reinterpret_cast<unsigned *>(smem + P.off_part);           // [2][64] LN partials
+    long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 512);    // [2][64]
+    float *cbuf = reinterpret_cast<float *>(smem + P.off_cbuf);                   // [R][d]
     const int nphase = 1 + 6 * P.n_dec;
 
     // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
@@ -443,12 +406,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, part_u, part_l);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, part_u, part_l, cbuf);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
             } else {
                 dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status, part_u,
-                             part_l);
+                             part_l, cbuf);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
@@ -552,13 +515,13 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, part_u, part_l);
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, part_u, part_l, cbuf);
         }
     }
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     1.0f / P.s_dout, a_full, 0, P.status, part_u, part_l);
+                     1.0f / P.s_dout, a_full, 0, P.status, part_u, part_l, cbuf);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -731,8 +694,9 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
-    P.off_part = take(256 + 512);                                   // LayerNorm partials (64 rows of 32)
-    if (R * d > 256 * 8) return (size_t)-1;                        // block LayerNorm covers R * d <= 2048
+    P.off_part = take(512 + 1024);                                  // LayerNorm partials (2 x 64 warp chunks)
+    P.off_cbuf = take((size_t)R * d * 4);                           // LayerNorm x - mean
+    if (R * d > 64 * 32) return (size_t)-1;                         // 64 warp chunks of partials
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const DcPhase &f = P.phase[ph];
