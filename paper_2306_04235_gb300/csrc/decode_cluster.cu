@@ -24,6 +24,8 @@
 // the multi-kernel path.
 #include <cooperative_groups.h>
 
+#include <cstdlib>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -646,10 +648,15 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
-// CTAs per cluster: one 16-column slice of d per CTA, at most 16 CTAs
+// CTAs per cluster: a slice of at least 16 columns of d per CTA, at most
+// MNMT_DC_MAX_CTAS (default 16, the largest cluster; measured fastest) CTAs
 int dc_cluster_size(int d) {
+    int cap = 16;
+    if (const char *e = getenv("MNMT_DC_MAX_CTAS")) cap = atoi(e);
+    if (cap < 2) cap = 2;
+    if (cap > 16) cap = 16;
     int nc = d / 16;
-    if (nc > 16) nc = 16;
+    if (nc > cap) nc = cap;
     return nc >= 2 ? nc : 0;
 }
 
