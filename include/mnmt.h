@@ -200,6 +200,28 @@ int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, const float 
                 const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
                 int8_t *out_q, float *out_f, void *cuda_stream);
 
+/* Tensor-core form of mnmt_linear for layers where the batch makes the linear
+ * a dense contraction: the same results bit for bit, computed on the
+ * fifth-generation tensor cores (tcgen05) from fp16 copies of the int8 codes.
+ * A16 [M][K] and W16 [N][K] hold fp16 bit patterns of integers in [-128, 127]
+ * (mnmt_codes_to_f16 makes them); products of such integers and sums of 1024
+ * of them are exact in fp32, so the kernel accumulates K in chunks of 1024 and
+ * the result equals the int32 accumulator of mnmt_linear.  K a multiple of 8 in
+ * [8, 2048]; A16 and W16 16-byte aligned.  mode is one of mnmt_linear's, or
+ * MNMT_EPI_ARGMAX: keys[m] = max(keys[m], max over n of pack(y[m][n], n)) as in
+ * mnmt_linear_argmax (keys must be initialised by the caller).  *status
+ * (device int32, may be NULL) receives MNMT_ETIMEOUT if one of the kernel's
+ * pipeline waits runs out (one second); the affected tiles are then not
+ * written. */
+enum { MNMT_EPI_ARGMAX = 4 };
+int mnmt_linear_tc(const uint16_t *A16, const uint16_t *W16, const float *s_w, const float *bias, float s_x,
+                   const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
+                   int8_t *out_q, float *out_f, uint64_t *keys, int32_t *status, void *cuda_stream);
+
+/* dst[i] = the fp16 value of the int8 code src[i] (exact), i < n.  Device
+ * pointers, src and dst 16-byte aligned. */
+int mnmt_codes_to_f16(const int8_t *src, uint16_t *dst, size_t n, void *cuda_stream);
+
 /* Output-vocabulary projection fused with greedy selection (App. D): for each
  * row m, keys[m] = max over n of pack(y[m][n], n) with y as in mnmt_linear and
  * pack(y, n) = (ord(y) << 32) | (0xFFFFFFFF - n), where ord maps fp32 to uint32

@@ -60,6 +60,7 @@ static int lib_init() {
         if (g_init_err == cudaSuccess) g_init_err = attention_init();
         if (g_init_err == cudaSuccess) g_init_err = rows_init();
         if (g_init_err == cudaSuccess) g_init_err = decode_cluster_init();
+        if (g_init_err == cudaSuccess) g_init_err = linear_tc_init();
     });
     if (g_init_err != cudaSuccess)
         return fail(MNMT_ECUDA, "kernel set-up failed: %s", cudaGetErrorString(g_init_err));
@@ -246,6 +247,7 @@ struct mnmt_model {
     cudaStream_t stream;
     bool own_stream;
     uint8_t *d_blob;
+    __half *d_blob16;  // fp16 copy of every blob byte read as an int8 code (tensor-core operands)
     float *d_aux;
     size_t bytes;
     const int8_t *emb_q;
@@ -411,6 +413,18 @@ extern "C" int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stre
     m->out.b = reinterpret_cast<const float *>(m->d_blob + L.out_b);
     m->out.n = c.vocab;
     m->out.k = d;
+    // the tensor-core linears read the weight codes as fp16: convert the whole
+    // blob once (the fp32 regions become unused garbage); offsets stay 16-byte
+    // aligned, so W16 = d_blob16 + (W - d_blob) is 32-byte aligned
+    if (cudaMalloc(&m->d_blob16, bytes * 2) != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ENOMEM, "cudaMalloc of %zu fp16 weight bytes failed", bytes * 2);
+    }
+    if (launch_codes_to_f16_flat(reinterpret_cast<const int8_t *>(m->d_blob), m->d_blob16, bytes, m->stream) !=
+        cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ECUDA, "fp16 weight conversion failed");
+    }
     if (cudaMalloc(&m->d_aux, aux.size() * 4) != cudaSuccess) {
         mnmt_model_free(m);
         return fail(MNMT_ENOMEM, "cudaMalloc of derived constants failed");
@@ -429,6 +443,7 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
     if (!m) return;
     if (m->stream) cudaStreamSynchronize(m->stream);
     if (m->d_blob) cudaFree(m->d_blob);
+    if (m->d_blob16) cudaFree(m->d_blob16);
     if (m->d_aux) cudaFree(m->d_aux);
     if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);
     delete m;
@@ -438,6 +453,8 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
 // session
 // ---------------------------------------------------------------------------
 enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_STATUS = 5, ST_N = 8 };
+// layers of at least this many rows run on the tensor cores (one full M tile)
+constexpr size_t TC_MIN_ROWS = 128;
 
 struct mnmt_session {
     mnmt_model *m;
@@ -449,6 +466,8 @@ struct mnmt_session {
     size_t arena_bytes = 0;
     float *resid, *cum, *logits;
     int8_t *act, *qkv, *ctx, *hid, *qbuf, *enc_q, *ck, *cv, *sk, *sv;
+    __half *a16;        // fp16 copy of a tensor-core linear's input rows
+    bool use_tc = true;  // tensor-core linears for layers of >= TC_MIN_ROWS rows
     int32_t *src_ids, *src_lens, *tok, *fin, *hist, *parents, *anc, *out_ids, *out_lens;
     float *out_scores;
     unsigned long long *keys, *cand;
@@ -508,6 +527,8 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
            o_logits = piece(beam > 1 ? R * V * 4 : 256), o_outids = piece((size_t)max_batch * max_len * 4),
            o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
            o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams));
+    const size_t kmax = std::max(d, std::max(F, (size_t)c.d_embed));
+    size_t o_a16 = piece(rows >= TC_MIN_ROWS ? rows * kmax * 2 : 256);
     s->arena_bytes = off;
     if (cudaMalloc(&s->arena, off) != cudaSuccess) {
         delete s;
@@ -546,6 +567,11 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
     s->out_scores = reinterpret_cast<float *>(a + o_outsc);
     s->state = reinterpret_cast<int *>(a + o_state);
     s->d_dc = reinterpret_cast<DcParams *>(a + o_dc);
+    s->a16 = reinterpret_cast<__half *>(a + o_a16);
+    {
+        const char *v = std::getenv("MNMT_TC");
+        s->use_tc = !(v && v[0] == '0') && rows >= TC_MIN_ROWS;
+    }
     if (cudaMemsetAsync(s->arena, 0, off, m->stream) != cudaSuccess ||
         cudaStreamSynchronize(m->stream) != cudaSuccess) {
         mnmt_session_free(s);
@@ -577,6 +603,29 @@ Epi base_epi(int mode, float s_x, const Lin &l) {
     e.s_w = l.s;
     e.bias = l.b;
     return e;
+}
+
+// fp16 copy of the codes of weight w (tensor-core operand)
+const __half *w16_of(const mnmt_model *m, const int8_t *w) {
+    return m->d_blob16 + (w - reinterpret_cast<const int8_t *>(m->d_blob));
+}
+
+// The quantised linear of rows A [M][lda] (Eq. 3 + epilogue e): on the
+// tensor cores when the layer is a dense contraction (M >= TC_MIN_ROWS),
+// after an exact int8 -> fp16 copy of A; else on the IMMA / GEMV kernels.
+cudaError_t run_linear(mnmt_session *s, const int8_t *A, int lda, const Lin &l, int M, const Epi &e,
+                       cudaStream_t st) {
+    const mnmt_model *m = s->m;
+    if (s->use_tc && M >= TC_MIN_ROWS && l.k % 16 == 0) {
+        const __half *w16 = w16_of(m, l.w);
+        if (linear_tc_shape_ok(M, l.n, l.k, l.k, l.k, s->a16, w16)) {
+            cudaError_t err = launch_codes_to_f16(A, lda, s->a16, l.k, M, l.k, st);
+            if (err == cudaSuccess)
+                err = launch_linear_tc(s->a16, l.k, w16, l.k, M, l.n, l.k, e, s->state + ST_STATUS, st);
+            return err;
+        }
+    }
+    return launch_linear(A, lda, l.w, M, l.n, l.k, e, st);
 }
 
 #define LK(call)                                                                                   \
@@ -652,7 +701,7 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e.inv_out = A.inv_qkv;
         e.out = s->qkv;
         e.ldo = 3 * d;
-        LK(launch_linear(s->act, d, A.qkv.w, M, 3 * d, d, e, st));
+        LK(run_linear(s, s->act, d, A.qkv, M, e, st));  // N = 3 * d, K = d
         AttnEncArgs at;
         at.qkv = s->qkv;
         at.ctx = s->ctx;
@@ -669,19 +718,19 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e.f32 = s->resid;
         e.ldf = d;
         e.gamma = A.gamma;
-        LK(launch_linear(s->ctx, d, A.o.w, M, d, d, e, st));
+        LK(run_linear(s, s->ctx, d, A.o, M, e, st));  // N = d, K = d
         int rc = ln_after_residual(s, M, Fb.ln, A.ln, Fb.s_in, s->act, nullptr);
         if (rc) return rc;
         e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
         e.inv_out = Fb.inv_h;
         e.out = s->hid;
         e.ldo = F;
-        LK(launch_linear(s->act, d, Fb.w1.w, M, F, d, e, st));
+        LK(run_linear(s, s->act, d, Fb.w1, M, e, st));  // N = F, K = d
         e = base_epi(EPI_RESID, Fb.s_h, Fb.w2);
         e.f32 = s->resid;
         e.ldf = d;
         e.gamma = Fb.gamma;
-        LK(launch_linear(s->hid, F, Fb.w2.w, M, d, F, e, st));
+        LK(run_linear(s, s->hid, F, Fb.w2, M, e, st));  // N = d, K = F
         if (l + 1 < c.n_enc) {
             const SelfBlk &An = m->enc_self[l + 1];
             rc = ln_after_residual(s, M, An.ln, Fb.ln, An.s_in, s->act, nullptr);
@@ -700,7 +749,7 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e.H = H;
         e.dh = dh;
         e.S = S;
-        LK(launch_linear(s->enc_q, d, X.kv.w, M, 2 * d, d, e, st));
+        LK(run_linear(s, s->enc_q, d, X.kv, M, e, st));  // N = 2 * d, K = d
     }
     return MNMT_OK;
 }
@@ -778,7 +827,7 @@ int issue_decode_step(mnmt_session *s) {
         e.dh = dh;
         e.T = s->Tcap;
         e.skip = done;
-        LK(launch_linear(s->act, d, A.qkv.w, R, 3 * d, d, e, st));
+        LK(run_linear(s, s->act, d, A.qkv, R, e, st));  // N = 3 * d, K = d
         AttnDecArgs at;
         std::memset(&at, 0, sizeof(at));
         at.q = s->qbuf;
@@ -802,7 +851,7 @@ int issue_decode_step(mnmt_session *s) {
         e.ldf = d;
         e.gamma = A.gamma;
         e.skip = done;
-        LK(launch_linear(s->ctx, d, A.o.w, R, d, d, e, st));
+        LK(run_linear(s, s->ctx, d, A.o, R, e, st));  // N = d, K = d
         int rc = ln_after_residual(s, R, X.ln, A.ln, X.s_in, s->act, done);
         if (rc) return rc;
         e = base_epi(EPI_Q8, X.s_in, X.q);
@@ -810,7 +859,7 @@ int issue_decode_step(mnmt_session *s) {
         e.out = s->qbuf;
         e.ldo = d;
         e.skip = done;
-        LK(launch_linear(s->act, d, X.q.w, R, d, d, e, st));
+        LK(run_linear(s, s->act, d, X.q, R, e, st));  // N = d, K = d
         at.kc = s->ck + l * s->ck_layer;
         at.vc = s->cv + l * s->ck_layer;
         at.T = s->S;
@@ -825,7 +874,7 @@ int issue_decode_step(mnmt_session *s) {
         e.ldf = d;
         e.gamma = X.gamma;
         e.skip = done;
-        LK(launch_linear(s->ctx, d, X.o.w, R, d, d, e, st));
+        LK(run_linear(s, s->ctx, d, X.o, R, e, st));  // N = d, K = d
         rc = ln_after_residual(s, R, Fb.ln, X.ln, Fb.s_in, s->act, done);
         if (rc) return rc;
         e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
@@ -833,13 +882,13 @@ int issue_decode_step(mnmt_session *s) {
         e.out = s->hid;
         e.ldo = F;
         e.skip = done;
-        LK(launch_linear(s->act, d, Fb.w1.w, R, F, d, e, st));
+        LK(run_linear(s, s->act, d, Fb.w1, R, e, st));  // N = F, K = d
         e = base_epi(EPI_RESID, Fb.s_h, Fb.w2);
         e.f32 = s->resid;
         e.ldf = d;
         e.gamma = Fb.gamma;
         e.skip = done;
-        LK(launch_linear(s->hid, F, Fb.w2.w, R, d, F, e, st));
+        LK(run_linear(s, s->hid, F, Fb.w2, R, e, st));  // N = d, K = F
         if (l + 1 < c.n_dec) {
             const SelfBlk &An = m->dec_self[l + 1];
             rc = ln_after_residual(s, R, An.ln, Fb.ln, An.s_in, s->act, done);
@@ -852,7 +901,7 @@ int issue_decode_step(mnmt_session *s) {
         Epi e = base_epi(EPI_ARGMAX, m->s_dout, m->out);
         e.keys = s->keys;
         e.skip = done;
-        LK(launch_linear(s->act, d, m->out.w, R, c.vocab, d, e, st));
+        LK(run_linear(s, s->act, d, m->out, R, e, st));  // N = c.vocab, K = d
         GreedyArgs g;
         g.keys = s->keys;
         g.tok = s->tok;
@@ -871,7 +920,7 @@ int issue_decode_step(mnmt_session *s) {
         e.f32 = s->logits;
         e.ldf = c.vocab;
         e.skip = done;
-        LK(launch_linear(s->act, d, m->out.w, R, c.vocab, d, e, st));
+        LK(run_linear(s, s->act, d, m->out, R, e, st));  // N = c.vocab, K = d
         BeamArgs b;
         b.logits = s->logits;
         b.tok = s->tok;
@@ -1229,6 +1278,61 @@ extern "C" int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, c
     }
     cudaError_t err = launch_linear(A, K, W, M, N, K, e, static_cast<cudaStream_t>(cuda_stream));
     if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_linear_tc(const uint16_t *A16, const uint16_t *W16, const float *s_w, const float *bias,
+                              float s_x, const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K,
+                              int32_t mode, int8_t *out_q, float *out_f, uint64_t *keys, int32_t *status,
+                              void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!A16 || !W16 || !s_w || !bias || M < 1 || N < 1 || !linear_tc_shape_ok(M, N, K, K, K, A16, W16))
+        return fail(MNMT_EINVAL, "linear_tc: bad shape or alignment M=%d N=%d K=%d", M, N, K);
+    Epi e;
+    std::memset(&e, 0, sizeof(e));
+    e.s_x = s_x;
+    e.s_w = s_w;
+    e.bias = bias;
+    switch (mode) {
+        case MNMT_EPI_Q8:
+        case MNMT_EPI_RELU_Q8:
+            if (!out_q || !inv_out) return fail(MNMT_EINVAL, "linear_tc: int8 output needs out_q and inv_out");
+            e.mode = mode == MNMT_EPI_Q8 ? EPI_Q8 : EPI_RELU_Q8;
+            e.out = out_q;
+            e.ldo = N;
+            e.inv_out = inv_out;
+            break;
+        case MNMT_EPI_RESID:
+        case MNMT_EPI_F32:
+            if (!out_f) return fail(MNMT_EINVAL, "linear_tc: fp32 output needs out_f");
+            e.mode = mode == MNMT_EPI_RESID ? EPI_RESID : EPI_F32;
+            e.f32 = out_f;
+            e.ldf = N;
+            e.gamma = gamma;
+            break;
+        case MNMT_EPI_ARGMAX:
+            if (!keys) return fail(MNMT_EINVAL, "linear_tc: argmax needs keys");
+            e.mode = EPI_ARGMAX;
+            e.keys = reinterpret_cast<unsigned long long *>(keys);
+            break;
+        default:
+            return fail(MNMT_EINVAL, "linear_tc: unknown mode %d", mode);
+    }
+    cudaError_t err = launch_linear_tc(reinterpret_cast<const __half *>(A16), K, reinterpret_cast<const __half *>(W16),
+                                       K, M, N, K, e, status, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear_tc launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_codes_to_f16(const int8_t *src, uint16_t *dst, size_t n, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!src || !dst || ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst)) & 15))
+        return fail(MNMT_EINVAL, "codes_to_f16: null or unaligned pointer");
+    cudaError_t err = launch_codes_to_f16_flat(src, reinterpret_cast<__half *>(dst), n,
+                                               static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "codes_to_f16 launch: %s", cudaGetErrorString(err));
     return MNMT_OK;
 }
 

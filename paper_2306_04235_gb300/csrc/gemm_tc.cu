@@ -1,0 +1,467 @@
+// gemm_tc.cu -- the quantised linear of Sec. 3.3 / Eq. 3 on the fifth-generation
+// tensor cores (tcgen05), for layers where batch x beam (or batch x source
+// length) makes the layer a dense contraction.
+//
+// Exactness.  The int8 codes are carried as fp16 (every integer of magnitude
+// <= 2048 is an fp16 value), so each product a*w (|a*w| <= 2^14) is exact in
+// the fp32 accumulator.  A sum of at most 1024 such products has magnitude
+// <= 1024 * 128 * 128 = 2^24, so every partial sum is an integer that fp32
+// represents exactly and the accumulation is exact whatever order the tensor
+// core adds in.  K is therefore cut into chunks of 1024 (16 k-blocks of 64),
+// each accumulated into its own TMEM columns; with two chunks the epilogue adds
+// them with one fp32 addition, which returns fl(acc) -- the correctly rounded
+// exact sum, the same value as (float)acc of the int32 accumulator.
+//
+// Pipeline (one 128 x BN output tile per CTA, 192 threads):
+//   warp 0 lane 0   TMA producer: 128-byte-swizzled 128x64 (A) and BNx64 (W)
+//                   fp16 tiles into a STAGES-deep shared-memory ring;
+//   warp 1          allocates the TMEM accumulator; lane 0 issues
+//                   tcgen05.mma (M=128, N=BN, K=16 each) and releases ring
+//                   slots with tcgen05.commit;
+//   warps 2..5      stage the per-column constants, then drain TMEM with
+//                   tcgen05.ld (warp w reads lanes 32*(w%4)..+31 = tile rows)
+//                   and apply the fused epilogue of the linear.
+// Every mbarrier wait is bounded (one second of %globaltimer); a wait that
+// runs out records MNMT_ETIMEOUT in *status, the CTA stops issuing work, waits
+// (bounded) for its own copies and MMAs in flight, frees its TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_fp16.h>
+
+#include "common.cuh"
+#include "epilogue.cuh"
+#include "internal.h"
+#include "mnmt.h"
+
+namespace mnmt {
+namespace {
+
+constexpr int TC_BM = 128;
+constexpr int TC_BK = 64;             // fp16 per k-block: one 128-byte swizzle row
+constexpr int TC_KB_PER_CHUNK = 16;   // 16 x 64 = 1024 products per exact fp32 chunk
+constexpr int TC_THREADS = 192;
+constexpr unsigned long long TC_WAIT_NS = 1000000000ull;
+
+__device__ __forceinline__ uint32_t s_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// wait for the completion of the phase with the given parity; false if it has
+// not completed within TC_WAIT_NS
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    if (mbar_try(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try(bar, parity)) {
+        if (global_ns() - t0 > TC_WAIT_NS) return false;
+    }
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm, int x, int y, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], "
+        "[%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// shared-memory matrix descriptor of a K-major operand tile laid out by TMA with
+// 128-byte swizzling: rows of 128 bytes, 8-row (1024-byte) atoms stacked along
+// M/N (stride byte offset 1024); leading byte offset unused for this layout
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    return (uint64_t)((saddr >> 4) & 0x3FFFu) | ((uint64_t)1 << 16) | ((uint64_t)(1024 >> 4) << 32) |
+           ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// instruction descriptor of kind::f16: D fp32, A and B fp16, both K-major
+__host__ __device__ constexpr uint32_t idesc_f16(int m, int n) {
+    return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_f16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+        "%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+template <int NCOLS>
+__device__ __forceinline__ void tmem_alloc(uint32_t slot) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot), "r"(NCOLS)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+template <int NCOLS>
+__device__ __forceinline__ void tmem_free(uint32_t taddr) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(NCOLS) : "memory");
+}
+
+__host__ __device__ constexpr int pow2_cols(int c) { return c <= 32 ? 32 : c <= 64 ? 64 : c <= 128 ? 128 : c <= 256 ? 256 : 512; }
+
+template <int BN, int STAGES>
+struct TcLayout {
+    static constexpr uint32_t A_BYTES = TC_BM * TC_BK * 2;
+    static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
+    static constexpr uint32_t OFF_B = STAGES * A_BYTES;
+    static constexpr uint32_t OFF_COLS = OFF_B + STAGES * B_BYTES;
+    static constexpr uint32_t OFF_BARS = OFF_COLS + 3 * BN * 4;
+    static constexpr uint32_t OFF_MISC = OFF_BARS + (2 * STAGES + 1) * 8;
+    static constexpr uint32_t BYTES = OFF_MISC + 16;
+    static constexpr size_t SMEM = 1024 + BYTES;  // slack to align the ring to 1024 bytes
+};
+
+// 16 accumulators of one row -> int8 codes packed little-endian into 4 words:
+// q8(y, inv) = clamp(rne(fl(y * inv)), -127, 127), with the clamp taken first
+// (the same value: rne is monotone and +-127 are integers) and rne done by
+// adding 1.5 * 2^23, whose low byte is then the two's-complement code
+template <bool RELU>
+__device__ __forceinline__ void q8_pack16(const float (&a)[16], const float *sc, const float *bs, const float *inv,
+                                          uint32_t (&w)[4]) {
+#pragma unroll
+    for (int g = 0; g < 4; g++) {
+        uint32_t b[4];
+#pragma unroll
+        for (int i = 0; i < 4; i++) {
+            const int c = 4 * g + i;
+            float y = __fadd_rn(__fmul_rn(a[c], sc[c]), bs[c]);
+            if (RELU) y = y > 0.0f ? y : 0.0f;
+            float z = __fmul_rn(y, inv[c]);
+            z = fminf(fmaxf(z, -127.0f), 127.0f);
+            b[i] = __float_as_uint(__fadd_rn(z, 12582912.0f));
+        }
+        w[g] = __byte_perm(__byte_perm(b[0], b[1], 0x0040), __byte_perm(b[2], b[3], 0x0040), 0x5410);
+    }
+}
+
+template <int BN, int NCH, int STAGES>
+__global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ CUtensorMap tmA,
+                                                        const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
+                                                        Epi e, int *status) {
+    using L = TcLayout<BN, STAGES>;
+    constexpr int NCOLS = pow2_cols(NCH * BN);
+    constexpr uint32_t IDESC = idesc_f16(TC_BM, BN);
+    if (e.skip && *e.skip) return;
+
+    extern __shared__ uint8_t tc_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_raw) + 1023) & ~(uintptr_t)1023);
+    float *c_sc = reinterpret_cast<float *>(sm + L::OFF_COLS);
+    float *c_b = c_sc + BN;
+    float *c_inv = c_b + BN;
+    const uint32_t bars = s_addr(sm + L::OFF_BARS);  // full[STAGES], empty[STAGES], acc
+    auto full_bar = [&](int s) { return bars + 8u * s; };
+    auto empty_bar = [&](int s) { return bars + 8u * (STAGES + s); };
+    const uint32_t acc_bar = bars + 8u * (2 * STAGES);
+    uint32_t *misc = reinterpret_cast<uint32_t *>(sm + L::OFF_MISC);  // [0] tmem base, [1] abort, [2] consumed
+    volatile uint32_t *abort_flag = misc + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * BN;
+    const int nkb = (K + TC_BK - 1) / TC_BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; s++) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        mbar_init(acc_bar, 1);
+        misc[1] = 0;
+        misc[2] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        tmem_alloc<NCOLS>(s_addr(misc));
+        tc_fence_before();
+    }
+    if (warp >= 2) {
+        for (int i = threadIdx.x - 64; i < BN; i += TC_THREADS - 64) {
+            const int n = n0 + i;
+            const bool ok = n < N;
+            c_sc[i] = ok ? __fmul_rn(e.s_x, e.s_w[n]) : 0.0f;
+            c_b[i] = ok ? e.bias[n] : 0.0f;
+            c_inv[i] = ok && e.inv_out ? e.inv_out[n] : 0.0f;
+        }
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = misc[0];
+
+    int issued = 0;
+    if (warp == 0 && lane == 0) {
+        // ---- TMA producer ----
+        for (int kb = 0; kb < nkb; kb++) {
+            const int s = kb % STAGES;
+            if (kb >= STAGES && !mbar_wait(empty_bar(s), (uint32_t)((kb / STAGES - 1) & 1))) {
+                *abort_flag = 1;
+                set_status(status, MNMT_ETIMEOUT);
+                break;
+            }
+            if (*abort_flag) break;
+            mbar_expect_tx(full_bar(s), L::A_BYTES + L::B_BYTES);
+            tma_load_2d(s_addr(sm + s * L::A_BYTES), &tmA, kb * TC_BK, m0, full_bar(s));
+            tma_load_2d(s_addr(sm + L::OFF_B + s * L::B_BYTES), &tmB, kb * TC_BK, n0, full_bar(s));
+            issued = kb + 1;
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer ----
+        int consumed = 0;
+        for (int kb = 0; kb < nkb; kb++) {
+            const int s = kb % STAGES;
+            if (!mbar_wait(full_bar(s), (uint32_t)((kb / STAGES) & 1))) {
+                *abort_flag = 1;
+                set_status(status, MNMT_ETIMEOUT);
+                break;
+            }
+            consumed = kb + 1;
+            if (*abort_flag) break;
+            tc_fence_after();
+            const uint32_t d = tbase + (uint32_t)((kb / TC_KB_PER_CHUNK) * BN);
+            const uint64_t ad = sw128_desc(s_addr(sm + s * L::A_BYTES));
+            const uint64_t bd = sw128_desc(s_addr(sm + L::OFF_B + s * L::B_BYTES));
+#pragma unroll
+            for (int k = 0; k < TC_BK / 16; k++)
+                mma_f16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC,
+                        (uint32_t)((kb % TC_KB_PER_CHUNK) | k));
+            mma_commit(empty_bar(s));
+        }
+        misc[2] = (uint32_t)consumed;
+        mma_commit(acc_bar);  // arrives once every MMA issued above has completed
+    } else if (warp >= 2) {
+        // ---- epilogue: TMEM -> registers -> fused epilogue -> global ----
+        const int q = warp & 3;
+        const int row = m0 + 32 * q + lane;
+        bool ok = mbar_wait(acc_bar, 0);
+        if (!ok) {
+            *abort_flag = 1;
+            set_status(status, MNMT_ETIMEOUT);
+        }
+        tc_fence_after();
+        ok = __all_sync(0xFFFFFFFFu, ok && *abort_flag == 0);
+        if (ok) {
+            const int t = e.t_ptr ? *e.t_ptr : 0;
+            const uint32_t taddr = tbase + ((uint32_t)(32 * q) << 16);
+            const bool vec_q8 = (e.mode == EPI_Q8 || e.mode == EPI_RELU_Q8) && (e.ldo % 16) == 0 &&
+                                (reinterpret_cast<uintptr_t>(e.out) & 15) == 0;
+            unsigned long long best = 0ull;
+#pragma unroll 1
+            for (int j = 0; j < BN / 16; j++) {
+                uint32_t r0[16], r1[16];
+                tmem_ld16(taddr + 16 * j, r0);
+                if (NCH == 2) tmem_ld16(taddr + BN + 16 * j, r1);
+                tmem_wait_ld();
+                float a[16];
+#pragma unroll
+                for (int i = 0; i < 16; i++)
+                    a[i] = NCH == 2 ? __fadd_rn(__uint_as_float(r0[i]), __uint_as_float(r1[i]))
+                                    : __uint_as_float(r0[i]);
+                const int col0 = n0 + 16 * j;
+                if (col0 >= N) break;
+                const float *sc = c_sc + 16 * j, *bs = c_b + 16 * j, *inv = c_inv + 16 * j;
+                if (e.mode == EPI_ARGMAX) {
+#pragma unroll
+                    for (int i = 0; i < 16; i++) {
+                        if (col0 + i < N) {
+                            const float y = __fadd_rn(__fmul_rn(a[i], sc[i]), bs[i]);
+                            const unsigned long long kk = pack_key(y, (uint32_t)(col0 + i));
+                            best = kk > best ? kk : best;
+                        }
+                    }
+                } else if (vec_q8 && col0 + 16 <= N) {
+                    uint32_t w[4];
+                    if (e.mode == EPI_RELU_Q8)
+                        q8_pack16<true>(a, sc, bs, inv, w);
+                    else
+                        q8_pack16<false>(a, sc, bs, inv, w);
+                    if (row < M)
+                        *reinterpret_cast<uint4 *>(e.out + (size_t)row * e.ldo + col0) =
+                            make_uint4(w[0], w[1], w[2], w[3]);
+                } else if (row < M) {
+#pragma unroll
+                    for (int i = 0; i < 16; i++)
+                        if (col0 + i < N) epi_store_f(e, row, col0 + i, a[i], t);
+                }
+            }
+            if (e.mode == EPI_ARGMAX && row < M) atomicMax(e.keys + row, best);
+        }
+    }
+
+    // ---- teardown ----
+    __syncthreads();
+    if (warp == 0 && lane == 0 && *abort_flag) {
+        // copies the MMA issuer never consumed are still landing in this CTA's ring
+        for (int kb = (int)misc[2]; kb < issued; kb++) mbar_wait(full_bar(kb % STAGES), (uint32_t)((kb / STAGES) & 1));
+    }
+    if (warp == 1) {
+        if (lane == 0 && *abort_flag) mbar_wait(acc_bar, 0);
+        __syncwarp();
+        tc_fence_after();
+        tmem_free<NCOLS>(tbase);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// int8 codes -> fp16 (exact); 16 codes per thread and step
+// ---------------------------------------------------------------------------
+__global__ void codes_to_f16_kernel(const int8_t *__restrict__ src, int ld_src, __half *__restrict__ dst, int ld_dst,
+                                    int rows, int cols) {
+    const int per_row = cols >> 4;
+    const long total = (long)rows * per_row;
+    for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
+        const int r = (int)(i / per_row), c = (int)(i - (long)r * per_row) << 4;
+        const int4 v = *reinterpret_cast<const int4 *>(src + (size_t)r * ld_src + c);
+        const int8_t *b = reinterpret_cast<const int8_t *>(&v);
+        __align__(16) __half h[16];
+#pragma unroll
+        for (int k = 0; k < 16; k++) h[k] = __short2half_rn((short)b[k]);
+        int4 *o = reinterpret_cast<int4 *>(dst + (size_t)r * ld_dst + c);
+        o[0] = *reinterpret_cast<const int4 *>(h);
+        o[1] = *reinterpret_cast<const int4 *>(h + 8);
+    }
+}
+
+__global__ void codes_to_f16_tail(const int8_t *src, __half *dst, size_t from, size_t n) {
+    size_t i = from + blockIdx.x * (size_t)blockDim.x + threadIdx.x;
+    if (i < n) dst[i] = __short2half_rn((short)src[i]);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+bool make_map(CUtensorMap *tm, const __half *p, int cols, int rows, int ld, int box_rows) {
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)TC_BK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = g_encode(tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(p), dims, strides, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int BN, int NCH, int STAGES>
+cudaError_t tc_attr() {
+    return cudaFuncSetAttribute(linear_tc<BN, NCH, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)TcLayout<BN, STAGES>::SMEM);
+}
+
+template <int BN, int NCH, int STAGES>
+cudaError_t tc_launch(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, const Epi &e, int *status,
+                      cudaStream_t st) {
+    dim3 grid((M + TC_BM - 1) / TC_BM, (N + BN - 1) / BN);
+    linear_tc<BN, NCH, STAGES><<<grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st>>>(ta, tb, M, N, K, e, status);
+    return cudaGetLastError();
+}
+
+constexpr int TC_STAGES = 4;
+
+}  // namespace
+
+cudaError_t linear_tc_init() {
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    cudaError_t err = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (err != cudaSuccess) return err;
+    if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    err = tc_attr<128, 1, TC_STAGES>();
+    if (err == cudaSuccess) err = tc_attr<128, 2, TC_STAGES>();
+    return err;
+}
+
+bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16) {
+    return g_encode && M >= 1 && N >= 1 && K >= 8 && K <= 2 * TC_KB_PER_CHUNK * TC_BK && K % 8 == 0 && lda >= K &&
+           ldw >= K && lda % 8 == 0 && ldw % 8 == 0 && ((reinterpret_cast<uintptr_t>(A16) | reinterpret_cast<uintptr_t>(W16)) & 15) == 0;
+}
+
+cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int ldw, int M, int N, int K,
+                             const Epi &e, int *status, cudaStream_t st) {
+    if (M <= 0 || N <= 0) return cudaSuccess;
+    if (!linear_tc_shape_ok(M, N, K, lda, ldw, A16, W16)) return cudaErrorInvalidValue;
+    CUtensorMap ta, tb;
+    if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, 128)) return cudaErrorInvalidValue;
+    if (K > TC_KB_PER_CHUNK * TC_BK) return tc_launch<128, 2, TC_STAGES>(ta, tb, M, N, K, e, status, st);
+    return tc_launch<128, 1, TC_STAGES>(ta, tb, M, N, K, e, status, st);
+}
+
+cudaError_t launch_codes_to_f16(const int8_t *src, int ld_src, __half *dst, int ld_dst, int rows, int cols,
+                                cudaStream_t st) {
+    if (rows <= 0 || cols <= 0) return cudaSuccess;
+    if (cols % 16 || ld_src % 16 || ld_dst % 8 || (reinterpret_cast<uintptr_t>(src) & 15) ||
+        (reinterpret_cast<uintptr_t>(dst) & 15))
+        return cudaErrorInvalidValue;
+    const long units = (long)rows * (cols / 16);
+    long blocks = (units + 255) / 256;
+    if (blocks > 152 * 8) blocks = 152 * 8;
+    codes_to_f16_kernel<<<(int)blocks, 256, 0, st>>>(src, ld_src, dst, ld_dst, rows, cols);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_codes_to_f16_flat(const int8_t *src, __half *dst, size_t n, cudaStream_t st) {
+    const size_t body = n & ~(size_t)15;
+    cudaError_t err = cudaSuccess;
+    // the body as rows of 2^20 codes (the row count stays an int)
+    const size_t row = (size_t)1 << 20;
+    size_t done = 0;
+    if (body >= row) {
+        err = launch_codes_to_f16(src, (int)row, dst, (int)row, (int)(body / row), (int)row, st);
+        done = body / row * row;
+    }
+    if (err == cudaSuccess && body > done)
+        err = launch_codes_to_f16(src + done, (int)(body - done), dst + done, (int)(body - done), 1,
+                                  (int)(body - done), st);
+    if (err == cudaSuccess && n > body) {
+        codes_to_f16_tail<<<1, 32, 0, st>>>(src, dst, body, n);
+        err = cudaGetLastError();
+    }
+    return err;
+}
+
+}  // namespace mnmt

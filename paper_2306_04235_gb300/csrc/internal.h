@@ -2,6 +2,7 @@
 // libmnmt (host code + sm_103a kernels).
 #pragma once
 
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -51,6 +52,18 @@ cudaError_t rows_init();
 // ---- launchers (stream-ordered, no synchronisation) ----
 cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int N, int K, const Epi &e,
                           cudaStream_t st);
+
+// tensor-core (tcgen05) linear over fp16 copies of the int8 codes: A16 [M][lda],
+// W16 [N][ldw]; K <= 2048 and a multiple of 8; *status (device, may be null)
+// receives MNMT_ETIMEOUT if a pipeline wait runs out
+cudaError_t linear_tc_init();
+bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16);
+cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int ldw, int M, int N, int K,
+                             const Epi &e, int *status, cudaStream_t st);
+// int8 codes -> fp16 (exact): rows x cols (cols, ld_src multiples of 16), or flat
+cudaError_t launch_codes_to_f16(const int8_t *src, int ld_src, __half *dst, int ld_dst, int rows, int cols,
+                                cudaStream_t st);
+cudaError_t launch_codes_to_f16_flat(const int8_t *src, __half *dst, size_t n, cudaStream_t st);
 
 struct LnArgs {
     const float *r;   // [M][d] input rows (row stride d)

@@ -16,57 +16,10 @@
 //                  shared memory and ldmatrix fragment loads.  sm_103a has no
 //                  int8 form of tcgen05.mma, so this is the exact int8 tensor path.
 #include "common.cuh"
+#include "epilogue.cuh"
 #include "internal.h"
 
 namespace mnmt {
-
-// ---------------------------------------------------------------------------
-// epilogue of one output element
-// ---------------------------------------------------------------------------
-MNMT_DEV void epi_store(const Epi &e, int m, int n, int32_t acc, int t) {
-    float y = dequant_bias(acc, e.s_x, e.s_w[n], e.bias[n]);
-    switch (e.mode) {
-        case EPI_Q8:
-            e.out[(size_t)m * e.ldo + n] = q8(y, e.inv_out[n]);
-            break;
-        case EPI_RELU_Q8:
-            e.out[(size_t)m * e.ldo + n] = q8(y > 0.0f ? y : 0.0f, e.inv_out[n]);
-            break;
-        case EPI_RESID: {
-            float *p = e.f32 + (size_t)m * e.ldf + n;
-            *p = __fadd_rn(__fmul_rn(e.gamma, *p), y);
-            break;
-        }
-        case EPI_F32:
-            e.f32[(size_t)m * e.ldf + n] = y;
-            break;
-        case EPI_QKV_DEC: {
-            int8_t v = q8(y, e.inv_out[n]);
-            if (n < e.d) {
-                e.out[(size_t)m * e.ldo + n] = v;
-            } else {
-                int seg = n >= 2 * e.d;
-                int c = n - (seg ? 2 * e.d : e.d);
-                int h = c / e.dh, i = c - h * e.dh;
-                int8_t *dst = seg ? e.vc : e.kc;
-                dst[(((size_t)m * e.H + h) * e.T + t) * e.dh + i] = v;
-            }
-            break;
-        }
-        case EPI_KV_CROSS: {
-            int8_t v = q8(y, e.inv_out[n]);
-            int b = m / e.S, s = m - b * e.S;
-            int seg = n >= e.d;
-            int c = n - (seg ? e.d : 0);
-            int h = c / e.dh, i = c - h * e.dh;
-            int8_t *dst = seg ? e.vc : e.kc;
-            dst[(((size_t)b * e.H + h) * e.S + s) * e.dh + i] = v;
-            break;
-        }
-        default:
-            break;
-    }
-}
 
 // ---------------------------------------------------------------------------
 // small-M path

@@ -18,7 +18,7 @@ from . import build as _build
 
 OK, EINVAL, ENOMEM, ECUDA, ETIMEOUT, EFORMAT, EOVERFLOW = 0, -1, -2, -3, -4, -5, -6
 DEVICE_PTRS = 1
-EPI_Q8, EPI_RELU_Q8, EPI_RESID, EPI_F32 = 0, 1, 2, 3
+EPI_Q8, EPI_RELU_Q8, EPI_RESID, EPI_F32, EPI_ARGMAX = 0, 1, 2, 3, 4
 (TAP_ENC_OUT, TAP_CROSS_K, TAP_CROSS_V, TAP_SELF_K, TAP_SELF_V, TAP_DEC_OUT, TAP_LOGITS, TAP_RESID,
  TAP_HISTORY, TAP_PARENTS, TAP_ANCESTRY) = range(1, 12)
 
@@ -75,8 +75,11 @@ def _declare(L):
     L.mnmt_linear_argmax_ids_noalloc.restype = C.c_int
     L.mnmt_attention_decode.argtypes = [p, p, p, p, i32, i32, i32, i32, f, f, p, p]
     L.mnmt_layernorm.argtypes = [p, p, p, i32, i32, f, p, p, p, p]
+    L.mnmt_linear_tc.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p, p]
+    L.mnmt_codes_to_f16.argtypes = [p, p, sz, p]
     for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
-              "mnmt_decode_step", "mnmt_translate", "mnmt_linear", "mnmt_linear_argmax", "mnmt_attention_decode", "mnmt_layernorm"]:
+              "mnmt_decode_step", "mnmt_translate", "mnmt_linear", "mnmt_linear_argmax", "mnmt_attention_decode", "mnmt_layernorm",
+              "mnmt_linear_tc", "mnmt_codes_to_f16"]:
         getattr(L, n).restype = C.c_int
 
 
@@ -191,6 +194,19 @@ def mnmt_linear_argmax_ids_noalloc(A, W, s_w, bias, s_x, M, N, K, ids, stream=No
     """Greedy vocabulary argmax into int32 ids with library-owned scratch (no allocation)."""
     _chk(lib().mnmt_linear_argmax_ids_noalloc(_ptr(A), _ptr(W), _ptr(s_w), _ptr(bias), float(s_x), M, N, K,
                                               _ptr(ids), _stream_handle(stream)))
+
+
+def mnmt_linear_tc(A16, W16, s_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_q=None, out_f=None, keys=None,
+                   status=None, stream=None):
+    """Tensor-core quantised linear over fp16 copies of the int8 codes (see mnmt_codes_to_f16)."""
+    _chk(lib().mnmt_linear_tc(_ptr(A16), _ptr(W16), _ptr(s_w), _ptr(bias), float(s_x), _ptr(inv_out), float(gamma),
+                              M, N, K, mode, _ptr(out_q), _ptr(out_f), _ptr(keys), _ptr(status),
+                              _stream_handle(stream)))
+
+
+def mnmt_codes_to_f16(src, dst, n, stream=None):
+    """dst[i] = fp16(src[i]) for n int8 codes (device buffers)."""
+    _chk(lib().mnmt_codes_to_f16(_ptr(src), _ptr(dst), n, _stream_handle(stream)))
 
 
 def argmax_from_keys(keys: np.ndarray) -> np.ndarray:
