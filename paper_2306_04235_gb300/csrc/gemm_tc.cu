@@ -12,15 +12,17 @@
 // them with one fp32 addition, which returns fl(acc) -- the correctly rounded
 // exact sum, the same value as (float)acc of the int32 accumulator.
 //
-// Pipeline (one 128 x BN output tile per CTA, 192 threads):
+// Pipeline (persistent CTAs, 128 x BN output tiles, 320 threads):
 //   warp 0 lane 0   TMA producer: 128-byte-swizzled 128x64 (A) and BNx64 (W)
 //                   fp16 tiles into a STAGES-deep shared-memory ring;
-//   warp 1          allocates the TMEM accumulator; lane 0 issues
-//                   tcgen05.mma (M=128, N=BN, K=16 each) and releases ring
-//                   slots with tcgen05.commit;
-//   warps 2..5      stage the per-column constants, then drain TMEM with
-//                   tcgen05.ld (warp w reads lanes 32*(w%4)..+31 = tile rows)
-//                   and apply the fused epilogue of the linear.
+//   warp 1          allocates two TMEM accumulator buffers; lane 0 issues
+//                   tcgen05.mma (M=128, N=BN, K=16 each), releases ring slots
+//                   with tcgen05.commit and signals each finished tile;
+//   warps 2..9      stage the per-column constants of a tile, then drain its
+//                   TMEM buffer with tcgen05.ld (warp w reads lanes
+//                   32*(w%4)..+31 = tile rows, half of the columns) and apply
+//                   the fused epilogue of the linear while the MMAs of the
+//                   next tile fill the other buffer.
 // Every mbarrier wait is bounded (one second of %globaltimer); a wait that
 // runs out records MNMT_ETIMEOUT in *status, the CTA stops issuing work, waits
 // (bounded) for its own copies and MMAs in flight, frees its TMEM and returns.
@@ -39,7 +41,8 @@ namespace {
 constexpr int TC_BM = 128;
 constexpr int TC_BK = 64;             // fp16 per k-block: one 128-byte swizzle row
 constexpr int TC_KB_PER_CHUNK = 16;   // 16 x 64 = 1024 products per exact fp32 chunk
-constexpr int TC_THREADS = 192;
+constexpr int TC_EPI_WARPS = 8;                  // two warps per TMEM lane quarter
+constexpr int TC_THREADS = 64 + TC_EPI_WARPS * 32;  // producer warp, MMA warp, epilogue warps
 constexpr unsigned long long TC_WAIT_NS = 1000000000ull;
 
 __device__ __forceinline__ uint32_t s_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -149,12 +152,20 @@ struct TcLayout {
     static constexpr uint32_t A_BYTES = TC_BM * TC_BK * 2;
     static constexpr uint32_t B_BYTES = BN * TC_BK * 2;
     static constexpr uint32_t OFF_B = STAGES * A_BYTES;
-    static constexpr uint32_t OFF_COLS = OFF_B + STAGES * B_BYTES;
-    static constexpr uint32_t OFF_BARS = OFF_COLS + 3 * BN * 4;
-    static constexpr uint32_t OFF_MISC = OFF_BARS + (2 * STAGES + 1) * 8;
+    static constexpr uint32_t OFF_COLS = OFF_B + STAGES * B_BYTES;      // [2][3][BN] fp32
+    static constexpr uint32_t OFF_BARS = OFF_COLS + 2 * 3 * BN * 4;
+    static constexpr int NBARS = 2 * STAGES + 5;  // full[S], empty[S], acc_full[2], acc_empty[2], done
+    static constexpr uint32_t OFF_MISC = OFF_BARS + NBARS * 8;
     static constexpr uint32_t BYTES = OFF_MISC + 16;
     static constexpr size_t SMEM = 1024 + BYTES;  // slack to align the ring to 1024 bytes
 };
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+// named barrier over the epilogue warps only
+__device__ __forceinline__ void epi_bar_sync() { asm volatile("bar.sync 1, %0;" ::"n"(TC_EPI_WARPS * 32) : "memory"); }
 
 // 16 accumulators of one row -> int8 codes packed little-endian into 4 words:
 // q8(y, inv) = clamp(rne(fl(y * inv)), -127, 127), with the clamp taken first
@@ -179,29 +190,109 @@ __device__ __forceinline__ void q8_pack16(const float (&a)[16], const float *sc,
     }
 }
 
+// the 16-column epilogue below applies (every destination row segment of 16
+// outputs is contiguous and 16-byte aligned)
+__device__ __forceinline__ bool epi_vec_ok(const Epi &e) {
+    const auto al = [](const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+    switch (e.mode) {
+        case EPI_Q8:
+        case EPI_RELU_Q8:
+            return e.ldo % 16 == 0 && al(e.out);
+        case EPI_RESID:
+        case EPI_F32:
+            return e.ldf % 4 == 0 && al(e.f32);
+        case EPI_QKV_DEC:
+            return e.ldo % 16 == 0 && al(e.out) && al(e.kc) && al(e.vc) && e.dh % 16 == 0 && e.d % 16 == 0;
+        case EPI_KV_CROSS:
+            return al(e.kc) && al(e.vc) && e.dh % 16 == 0 && e.d % 16 == 0;
+        default:
+            return false;
+    }
+}
+
+// The epilogue of outputs (row, col0 .. col0+15) of one row, col0 a multiple
+// of 16, all columns < N: the same arithmetic as epi_store_f, with one 16-byte
+// access per 16 int8 codes or 4 fp32 values.
+__device__ __forceinline__ void epi_store16(const Epi &e, int row, int col0, const float (&a)[16], const float *sc,
+                                            const float *bs, const float *inv, int t) {
+    if (e.mode == EPI_RESID || e.mode == EPI_F32) {
+        float4 *p = reinterpret_cast<float4 *>(e.f32 + (size_t)row * e.ldf + col0);
+        float4 r[4];
+        if (e.mode == EPI_RESID) {
+#pragma unroll
+            for (int g = 0; g < 4; g++) r[g] = p[g];
+        }
+#pragma unroll
+        for (int g = 0; g < 4; g++) {
+            float y[4];
+#pragma unroll
+            for (int i = 0; i < 4; i++) y[i] = __fadd_rn(__fmul_rn(a[4 * g + i], sc[4 * g + i]), bs[4 * g + i]);
+            if (e.mode == EPI_RESID) {
+                y[0] = __fadd_rn(__fmul_rn(e.gamma, r[g].x), y[0]);
+                y[1] = __fadd_rn(__fmul_rn(e.gamma, r[g].y), y[1]);
+                y[2] = __fadd_rn(__fmul_rn(e.gamma, r[g].z), y[2]);
+                y[3] = __fadd_rn(__fmul_rn(e.gamma, r[g].w), y[3]);
+            }
+            p[g] = make_float4(y[0], y[1], y[2], y[3]);
+        }
+        return;
+    }
+    uint32_t w[4];
+    if (e.mode == EPI_RELU_Q8)
+        q8_pack16<true>(a, sc, bs, inv, w);
+    else
+        q8_pack16<false>(a, sc, bs, inv, w);
+    int8_t *dst;
+    if (e.mode == EPI_QKV_DEC) {
+        if (col0 < e.d) {
+            dst = e.out + (size_t)row * e.ldo + col0;
+        } else {
+            const int seg = col0 >= 2 * e.d;
+            const int c = col0 - (seg ? 2 * e.d : e.d);
+            const int h = c / e.dh, i = c - h * e.dh;
+            dst = (seg ? e.vc : e.kc) + (((size_t)row * e.H + h) * e.T + t) * e.dh + i;
+        }
+    } else if (e.mode == EPI_KV_CROSS) {
+        const int b = row / e.S, sp = row - b * e.S;
+        const int seg = col0 >= e.d;
+        const int c = col0 - (seg ? e.d : 0);
+        const int h = c / e.dh, i = c - h * e.dh;
+        dst = (seg ? e.vc : e.kc) + (((size_t)b * e.H + h) * e.S + sp) * e.dh + i;
+    } else {
+        dst = e.out + (size_t)row * e.ldo + col0;
+    }
+    *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Persistent kernel: CTA c takes output tiles c, c + gridDim.x, ... (M-tile
+// index fastest, so the CTAs of one wave share weight tiles in L2).  The TMA
+// ring runs continuously across tiles; the accumulator is double-buffered in
+// TMEM so the epilogue of one tile overlaps the MMAs of the next.
 template <int BN, int NCH, int STAGES>
-__global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ CUtensorMap tmA,
-                                                        const __grid_constant__ CUtensorMap tmB, int M, int N, int K,
-                                                        Epi e, int *status) {
+__global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant__ CUtensorMap tmA,
+                                                           const __grid_constant__ CUtensorMap tmB, int M, int N,
+                                                           int K, Epi e, int *status) {
     using L = TcLayout<BN, STAGES>;
-    constexpr int NCOLS = pow2_cols(NCH * BN);
+    constexpr int ACC_COLS = NCH * BN;  // one accumulator buffer
+    constexpr int NCOLS = pow2_cols(2 * ACC_COLS);
     constexpr uint32_t IDESC = idesc_f16(TC_BM, BN);
     if (e.skip && *e.skip) return;
 
     extern __shared__ uint8_t tc_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_raw) + 1023) & ~(uintptr_t)1023);
-    float *c_sc = reinterpret_cast<float *>(sm + L::OFF_COLS);
-    float *c_b = c_sc + BN;
-    float *c_inv = c_b + BN;
-    const uint32_t bars = s_addr(sm + L::OFF_BARS);  // full[STAGES], empty[STAGES], acc
+    float *cols = reinterpret_cast<float *>(sm + L::OFF_COLS);
+    const uint32_t bars = s_addr(sm + L::OFF_BARS);
     auto full_bar = [&](int s) { return bars + 8u * s; };
     auto empty_bar = [&](int s) { return bars + 8u * (STAGES + s); };
-    const uint32_t acc_bar = bars + 8u * (2 * STAGES);
+    auto accf_bar = [&](int b) { return bars + 8u * (2 * STAGES + b); };
+    auto acce_bar = [&](int b) { return bars + 8u * (2 * STAGES + 2 + b); };
+    const uint32_t done_bar = bars + 8u * (2 * STAGES + 4);
     uint32_t *misc = reinterpret_cast<uint32_t *>(sm + L::OFF_MISC);  // [0] tmem base, [1] abort, [2] consumed
     volatile uint32_t *abort_flag = misc + 1;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int m0 = blockIdx.x * TC_BM, n0 = blockIdx.y * BN;
+    const int mt = (M + TC_BM - 1) / TC_BM;
+    const int tiles = mt * ((N + BN - 1) / BN);
     const int nkb = (K + TC_BK - 1) / TC_BK;
 
     if (threadIdx.x == 0) {
@@ -209,7 +300,11 @@ __global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ 
             mbar_init(full_bar(s), 1);
             mbar_init(empty_bar(s), 1);
         }
-        mbar_init(acc_bar, 1);
+        for (int b = 0; b < 2; b++) {
+            mbar_init(accf_bar(b), 1);
+            mbar_init(acce_bar(b), TC_EPI_WARPS);
+        }
+        mbar_init(done_bar, 1);
         misc[1] = 0;
         misc[2] = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -219,78 +314,98 @@ __global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ 
         tmem_alloc<NCOLS>(s_addr(misc));
         tc_fence_before();
     }
-    if (warp >= 2) {
-        for (int i = threadIdx.x - 64; i < BN; i += TC_THREADS - 64) {
-            const int n = n0 + i;
-            const bool ok = n < N;
-            c_sc[i] = ok ? __fmul_rn(e.s_x, e.s_w[n]) : 0.0f;
-            c_b[i] = ok ? e.bias[n] : 0.0f;
-            c_inv[i] = ok && e.inv_out ? e.inv_out[n] : 0.0f;
-        }
-    }
     __syncthreads();
     tc_fence_after();
     const uint32_t tbase = misc[0];
 
-    int issued = 0;
+    uint32_t issued = 0;
     if (warp == 0 && lane == 0) {
-        // ---- TMA producer ----
-        for (int kb = 0; kb < nkb; kb++) {
-            const int s = kb % STAGES;
-            if (kb >= STAGES && !mbar_wait(empty_bar(s), (uint32_t)((kb / STAGES - 1) & 1))) {
-                *abort_flag = 1;
-                set_status(status, MNMT_ETIMEOUT);
-                break;
+        // ---- TMA producer: k-blocks of all this CTA's tiles through the ring ----
+        uint32_t it = 0;
+        for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+            const int m0 = (tile % mt) * TC_BM, n0 = (tile / mt) * BN;
+            for (int kb = 0; kb < nkb; kb++, it++) {
+                const int s = (int)(it % STAGES);
+                if (it >= STAGES && !mbar_wait(empty_bar(s), (it / STAGES - 1) & 1)) {
+                    *abort_flag = 1;
+                    set_status(status, MNMT_ETIMEOUT);
+                }
+                if (*abort_flag) break;
+                mbar_expect_tx(full_bar(s), L::A_BYTES + L::B_BYTES);
+                tma_load_2d(s_addr(sm + s * L::A_BYTES), &tmA, kb * TC_BK, m0, full_bar(s));
+                tma_load_2d(s_addr(sm + L::OFF_B + s * L::B_BYTES), &tmB, kb * TC_BK, n0, full_bar(s));
+                issued = it + 1;
             }
-            if (*abort_flag) break;
-            mbar_expect_tx(full_bar(s), L::A_BYTES + L::B_BYTES);
-            tma_load_2d(s_addr(sm + s * L::A_BYTES), &tmA, kb * TC_BK, m0, full_bar(s));
-            tma_load_2d(s_addr(sm + L::OFF_B + s * L::B_BYTES), &tmB, kb * TC_BK, n0, full_bar(s));
-            issued = kb + 1;
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer ----
-        int consumed = 0;
-        for (int kb = 0; kb < nkb; kb++) {
-            const int s = kb % STAGES;
-            if (!mbar_wait(full_bar(s), (uint32_t)((kb / STAGES) & 1))) {
+        uint32_t it = 0, lt = 0;
+        for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x, lt++) {
+            const int buf = (int)(lt & 1);
+            if (lt >= 2 && !mbar_wait(acce_bar(buf), ((lt >> 1) - 1) & 1)) {
                 *abort_flag = 1;
                 set_status(status, MNMT_ETIMEOUT);
                 break;
             }
-            consumed = kb + 1;
-            if (*abort_flag) break;
             tc_fence_after();
-            const uint32_t d = tbase + (uint32_t)((kb / TC_KB_PER_CHUNK) * BN);
-            const uint64_t ad = sw128_desc(s_addr(sm + s * L::A_BYTES));
-            const uint64_t bd = sw128_desc(s_addr(sm + L::OFF_B + s * L::B_BYTES));
+            const uint32_t dbase = tbase + (uint32_t)(buf * ACC_COLS);
+            for (int kb = 0; kb < nkb; kb++, it++) {
+                const int s = (int)(it % STAGES);
+                if (!mbar_wait(full_bar(s), (it / STAGES) & 1)) {
+                    *abort_flag = 1;
+                    set_status(status, MNMT_ETIMEOUT);
+                }
+                if (*abort_flag) break;
+                misc[2] = it + 1;
+                tc_fence_after();
+                const uint32_t d = dbase + (uint32_t)((kb / TC_KB_PER_CHUNK) * BN);
+                const uint64_t ad = sw128_desc(s_addr(sm + s * L::A_BYTES));
+                const uint64_t bd = sw128_desc(s_addr(sm + L::OFF_B + s * L::B_BYTES));
 #pragma unroll
-            for (int k = 0; k < TC_BK / 16; k++)
-                mma_f16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC,
-                        (uint32_t)((kb % TC_KB_PER_CHUNK) | k));
-            mma_commit(empty_bar(s));
+                for (int k = 0; k < TC_BK / 16; k++)
+                    mma_f16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC,
+                            (uint32_t)((kb % TC_KB_PER_CHUNK) | k));
+                mma_commit(empty_bar(s));
+            }
+            if (*abort_flag) break;
+            mma_commit(accf_bar(buf));
         }
-        misc[2] = (uint32_t)consumed;
-        mma_commit(acc_bar);  // arrives once every MMA issued above has completed
+        mma_commit(done_bar);  // arrives once every MMA issued above has completed
     } else if (warp >= 2) {
         // ---- epilogue: TMEM -> registers -> fused epilogue -> global ----
-        const int q = warp & 3;
-        const int row = m0 + 32 * q + lane;
-        bool ok = mbar_wait(acc_bar, 0);
-        if (!ok) {
-            *abort_flag = 1;
-            set_status(status, MNMT_ETIMEOUT);
-        }
-        tc_fence_after();
-        ok = __all_sync(0xFFFFFFFFu, ok && *abort_flag == 0);
-        if (ok) {
-            const int t = e.t_ptr ? *e.t_ptr : 0;
-            const uint32_t taddr = tbase + ((uint32_t)(32 * q) << 16);
-            const bool vec_q8 = (e.mode == EPI_Q8 || e.mode == EPI_RELU_Q8) && (e.ldo % 16) == 0 &&
-                                (reinterpret_cast<uintptr_t>(e.out) & 15) == 0;
+        const int ew = warp - 2;                       // 0 .. TC_EPI_WARPS-1
+        const int q = warp & 3;                        // TMEM lane quarter of this warp
+        const int half = ew >> 2;                      // which half of the tile's columns
+        const int t = e.t_ptr ? *e.t_ptr : 0;
+        const bool vec = epi_vec_ok(e);
+        uint32_t lt = 0;
+        for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, lt++) {
+            const int buf = (int)(lt & 1);
+            const int m0 = (tile % mt) * TC_BM, n0 = (tile / mt) * BN;
+            // per-column constants of this tile, double-buffered by tile parity
+            float *c_sc = cols + buf * 3 * BN, *c_b = c_sc + BN, *c_inv = c_b + BN;
+            for (int i = ew * 32 + lane; i < BN; i += TC_EPI_WARPS * 32) {
+                const int n = n0 + i;
+                const bool ok = n < N;
+                c_sc[i] = ok ? __fmul_rn(e.s_x, e.s_w[n]) : 0.0f;
+                c_b[i] = ok ? e.bias[n] : 0.0f;
+                c_inv[i] = ok && e.inv_out ? e.inv_out[n] : 0.0f;
+            }
+            epi_bar_sync();
+            // every epilogue warp runs every tile of the loop (the named barrier
+            // above needs all of them); after an abort the tiles are skipped
+            bool ok = *abort_flag == 0 && mbar_wait(accf_bar(buf), (lt >> 1) & 1);
+            if (!ok && *abort_flag == 0) {
+                *abort_flag = 1;
+                set_status(status, MNMT_ETIMEOUT);
+            }
+            tc_fence_after();
+            ok = __all_sync(0xFFFFFFFFu, ok && *abort_flag == 0);
+            const int row = m0 + 32 * q + lane;
+            const uint32_t taddr = tbase + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * ACC_COLS);
             unsigned long long best = 0ull;
 #pragma unroll 1
-            for (int j = 0; j < BN / 16; j++) {
+            for (int j = half * (BN / 32); ok && j < (half + 1) * (BN / 32); j++) {
                 uint32_t r0[16], r1[16];
                 tmem_ld16(taddr + 16 * j, r0);
                 if (NCH == 2) tmem_ld16(taddr + BN + 16 * j, r1);
@@ -301,7 +416,7 @@ __global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ 
                     a[i] = NCH == 2 ? __fadd_rn(__uint_as_float(r0[i]), __uint_as_float(r1[i]))
                                     : __uint_as_float(r0[i]);
                 const int col0 = n0 + 16 * j;
-                if (col0 >= N) break;
+                if (col0 >= N) continue;
                 const float *sc = c_sc + 16 * j, *bs = c_b + 16 * j, *inv = c_inv + 16 * j;
                 if (e.mode == EPI_ARGMAX) {
 #pragma unroll
@@ -312,22 +427,19 @@ __global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ 
                             best = kk > best ? kk : best;
                         }
                     }
-                } else if (vec_q8 && col0 + 16 <= N) {
-                    uint32_t w[4];
-                    if (e.mode == EPI_RELU_Q8)
-                        q8_pack16<true>(a, sc, bs, inv, w);
-                    else
-                        q8_pack16<false>(a, sc, bs, inv, w);
-                    if (row < M)
-                        *reinterpret_cast<uint4 *>(e.out + (size_t)row * e.ldo + col0) =
-                            make_uint4(w[0], w[1], w[2], w[3]);
+                } else if (vec && col0 + 16 <= N) {
+                    if (row < M) epi_store16(e, row, col0, a, sc, bs, inv, t);
                 } else if (row < M) {
 #pragma unroll
                     for (int i = 0; i < 16; i++)
                         if (col0 + i < N) epi_store_f(e, row, col0 + i, a[i], t);
                 }
             }
-            if (e.mode == EPI_ARGMAX && row < M) atomicMax(e.keys + row, best);
+            // this warp is done with the accumulator buffer
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acce_bar(buf));
+            if (e.mode == EPI_ARGMAX && row < M && best) atomicMax(e.keys + row, best);
         }
     }
 
@@ -335,10 +447,10 @@ __global__ void __launch_bounds__(TC_THREADS) linear_tc(const __grid_constant__ 
     __syncthreads();
     if (warp == 0 && lane == 0 && *abort_flag) {
         // copies the MMA issuer never consumed are still landing in this CTA's ring
-        for (int kb = (int)misc[2]; kb < issued; kb++) mbar_wait(full_bar(kb % STAGES), (uint32_t)((kb / STAGES) & 1));
+        for (uint32_t it = misc[2]; it < issued; it++) mbar_wait(full_bar((int)(it % STAGES)), (it / STAGES) & 1);
     }
     if (warp == 1) {
-        if (lane == 0 && *abort_flag) mbar_wait(acc_bar, 0);
+        if (lane == 0) mbar_wait(done_bar, 0);
         __syncwarp();
         tc_fence_after();
         tmem_free<NCOLS>(tbase);
@@ -374,6 +486,7 @@ __global__ void codes_to_f16_tail(const int8_t *src, __half *dst, size_t from, s
 // host side
 // ---------------------------------------------------------------------------
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+int g_num_sms = 148;
 
 bool make_map(CUtensorMap *tm, const __half *p, int cols, int rows, int ld, int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
@@ -395,12 +508,13 @@ cudaError_t tc_attr() {
 template <int BN, int NCH, int STAGES>
 cudaError_t tc_launch(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, const Epi &e, int *status,
                       cudaStream_t st) {
-    dim3 grid((M + TC_BM - 1) / TC_BM, (N + BN - 1) / BN);
+    const long tiles = (long)((M + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
+    const int grid = (int)(tiles < g_num_sms ? tiles : g_num_sms);
     linear_tc<BN, NCH, STAGES><<<grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st>>>(ta, tb, M, N, K, e, status);
     return cudaGetLastError();
 }
 
-constexpr int TC_STAGES = 4;
+constexpr int TC_STAGES = 6;
 
 }  // namespace
 
@@ -411,6 +525,9 @@ cudaError_t linear_tc_init() {
     if (err != cudaSuccess) return err;
     if (q != cudaDriverEntryPointSuccess || !fn) return cudaErrorSymbolNotFound;
     g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    int dev = 0;
+    if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
+    if ((err = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return err;
     err = tc_attr<128, 1, TC_STAGES>();
     if (err == cudaSuccess) err = tc_attr<128, 2, TC_STAGES>();
     return err;

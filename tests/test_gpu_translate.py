@@ -275,3 +275,45 @@ def test_bench_workload_uses_cluster_step(stream):
         assert mnmt.mnmt_session_decode_path(tr.session) == 1
     finally:
         tr.close()
+
+
+def _with_tc(on: bool):
+    import os
+    if on:
+        os.environ.pop("MNMT_TC", None)
+    else:
+        os.environ["MNMT_TC"] = "0"
+
+
+@pytest.mark.parametrize("kind", list(MINI))
+@pytest.mark.parametrize("beam", [1, 4])
+def test_tensor_core_rows_match_oracle(kind, beam, stream):
+    """Batches of >= 128 decoder rows (and encoder rows) run their linears on
+    the tcgen05 kernel: tokens, lengths and scores still equal the oracle's."""
+    cfg = MINI[kind]
+    blob = synth.build_blob(cfg, 41, gamma_range=(0.5, 1.5))
+    B = 160 // beam
+    ids, lens = synth.source_batch(cfg.vocab, B, 1, 40, 42)
+    T = 20
+    _with_tc(True)
+    g_ids, g_len, g_sc = _gpu(blob, ids, lens, beam, T, stream)
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, beam, T, n_threads=8)
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_len, o_len)
+    assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
+
+
+def test_tensor_core_and_imma_paths_bit_identical(stream):
+    """The same batched beam workload through the tcgen05 linears and through
+    the IMMA linears (MNMT_TC=0): identical outputs."""
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs("small-b32-s10to80-beam4-t128")
+    outs = []
+    for on in (True, False):
+        _with_tc(on)
+        try:
+            outs.append(_gpu(blob, ids, lens, beam, T, stream))
+        finally:
+            _with_tc(True)
+    for a, b in zip(*outs):
+        assert np.array_equal(a.view(np.uint32) if a.dtype == np.float32 else a,
+                              b.view(np.uint32) if b.dtype == np.float32 else b)
