@@ -13,9 +13,12 @@ tokens.  Metric: decoded tokens per second (whole job over all GPUs).
   e2e       the same metric through the C ABI with pinned HOST buffers: the
             host->device copy of the source ids and the device->host copy of
             the output ids are inside the timed region
-  roofline  the dominant kernel (the fused vocabulary projection + argmax,
-            M=1 x N=32000 x K=256) timed with CUDA events on its stream over
-            as many launches as the timed region ran, L2 flushed before each
+  roofline  the decode step, the unit that dominates the translation time (at
+            batch 1 one graph launch of the thread-block-cluster step kernel
+            plus the fused vocabulary projection + argmax kernel), timed with
+            CUDA events on the library's stream one step at a time with L2
+            flushed before each; algorithmic bytes = the weights, scales and
+            biases every step must read plus its K/V cache reads
   cpu_baseline  the CPU oracle on a bounded sample of the same workload
 
 --impl reference runs the CPU oracle (the reference of this path) on the host
@@ -111,14 +114,42 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def kernels_per_translation(cfg, beam, steps):
-    """Kernels the library launches for one translation: encoder (embedding,
-    7 per layer, cross K/V per decoder layer), search init, decoder steps
-    (embedding, 11 per layer, vocabulary projection, 1 greedy / 2 beam search
-    kernels), final backtrack."""
-    enc = 1 + 7 * cfg.n_enc + cfg.n_dec
-    step = 1 + 11 * cfg.n_dec + 1 + (1 if beam == 1 else 2)
-    return enc + 1 + step * steps + 1
+def kernels_per_translation(cfg, B, S, beam, steps_launched, cluster):
+    """Kernels the library launches for one translation.  Encoder: embedding,
+    7 per layer, cross K/V per decoder layer, plus one int8 -> fp16 operand
+    copy before each linear of >= 128 rows (4 per layer and the cross K/V).
+    Search init and final backtrack.  Per decode step: the cluster step (step
+    kernel + vocabulary kernel), or embedding, 11 per layer, vocabulary
+    projection, 1 greedy / 2 beam kernels (+ 6 per layer and 1 operand copies
+    at >= 128 rows)."""
+    tc_enc = B * S >= 128
+    enc = 1 + 7 * cfg.n_enc + cfg.n_dec + (4 * cfg.n_enc + cfg.n_dec if tc_enc else 0)
+    if cluster:
+        step = 2
+    else:
+        tc_dec = B * beam >= 128
+        step = 1 + 11 * cfg.n_dec + 1 + (1 if beam == 1 else 2) + (6 * cfg.n_dec + 1 if tc_dec else 0)
+    return enc + 1 + step * steps_launched + 1
+
+
+def decode_step_bytes(cfg, R, B, S, t):
+    """Algorithmic bytes one decode step must move for R hypotheses of B
+    sentences (padded source length S) at step t: every decoder weight (int8),
+    its per-output-channel scale and bias (fp32) and the requantisation
+    constants of its int8 outputs, the LayerNorm vectors, the factorised
+    projection, the vocabulary matrix with its scales and biases, the embedding
+    rows and the positional row, and the K/V caches read (self [t+1] positions
+    per hypothesis, cross [S] per sentence)."""
+    d, F, V, E, L = cfg.d_model, cfg.d_ffn, cfg.vocab, cfg.d_embed, cfg.n_dec
+    w = L * (6 * d * d + 2 * F * d)
+    rows = L * (6 * d + F)
+    inv = L * (4 * d + F)
+    ln = (3 * L + (1 if cfg.pre_ln else 0)) * 2 * d * 4
+    proj = (E * d + 8 * d) if E != d else 0
+    vocab = V * d + 8 * V
+    emb = R * (E + 4) + d * 4
+    kv = 2 * L * R * (t + 1) * d + 2 * L * B * S * d
+    return w + 8 * rows + 4 * inv + ln + proj + vocab + emb + kv
 
 
 def cpu_sample(workload, n_sent, threads):
@@ -277,8 +308,9 @@ def run_gpu(args):
     e2e_value = e2e_tok * world * len(e2e_times) / sum(e2e_times)
     assert torch.equal(h_out, o_ids.cpu()), "host and device paths disagree"
 
-    # dominant kernel: fused vocabulary projection + argmax (M=1)
-    roof = measure_vocab_kernel(args, cfg, mnmt, torch, stream, flush, n_launch=min(args.steps * steps_run, 640))
+    # the decode step, one at a time (cold L2) and back to back (warm)
+    cluster = mnmt.mnmt_session_decode_path(sess) == 1
+    roof = measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster)
 
     if rank == 0:
         cpu = None
@@ -290,7 +322,8 @@ def run_gpu(args):
                    "kind": "oracle",
                    "sample": f"{n_sent} translation(s) of {wl.batch} sentence(s) drawn like the workload, "
                              f"one per thread ({cdt:.1f} s)"}
-        launches = kernels_per_translation(cfg, wl.beam, steps_run) * args.steps
+        launched = min(T, -(-steps_run // 16) * 16)  # the host checks for completion every 16 steps
+        launches = kernels_per_translation(cfg, B, S, wl.beam, launched, cluster) * args.steps
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
@@ -315,38 +348,44 @@ def run_gpu(args):
     return 0
 
 
-def measure_vocab_kernel(args, cfg, mnmt, torch, stream, flush, n_launch):
-    """The fused vocabulary projection + argmax at batch 1 (the largest weight
-    stream of a decode step), timed with CUDA events on its stream, L2 flushed
-    before each launch.  Algorithmic bytes: the [V][d] int8 weights, the fp32
-    scales and biases, the int8 input row and the 8-byte key."""
-    V, d = cfg.vocab, cfg.d_model
-    W = torch.from_numpy(synth.uniform_int8(3, "W", (V, d))).cuda()
-    s_w = torch.from_numpy(synth.uniform_f32(3, "s", (V,), 1e-4, 2e-4)).cuda()
-    b = torch.from_numpy(synth.uniform_f32(3, "b", (V,), -0.1, 0.1)).cuda()
-    A = torch.from_numpy(synth.uniform_int8(3, "A", (1, d))).cuda()
-    keys = torch.zeros(1, dtype=torch.int64, device="cuda")
-    algo_bytes = V * d + V * 8 + d + 8
-    ms = []
-    for i in range(n_launch + 3):
+def measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster):
+    """Decode steps of one encoded batch timed with CUDA events on the
+    library's stream: one step per event pair with L2 flushed before each
+    (cold: the weights come from HBM, as the roofline assumes), then the same
+    number of steps back to back (warm: the weights stay in the 129 MB L2)."""
+    R = B * wl.beam
+    n = max(1, min(steps_run, wl.max_len))
+    mnmt.mnmt_encode(sess, d_ids, d_lens, B, S, mnmt.DEVICE_PTRS)
+    cold = []
+    for t in range(n):
         with torch.cuda.stream(stream):
-            flush.fill_(i & 0xFF)
-            keys.zero_()
+            flush.fill_(t & 0xFF)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
-        mnmt.mnmt_linear_argmax(A, W, s_w, b, 0.01, 1, V, d, keys, stream)
+        mnmt.mnmt_decode_steps(sess, 1)
         with torch.cuda.stream(stream):
             e1.record(stream)
-        if i >= 3:
-            ms.append((e0, e1))
+        cold.append((e0, e1))
+    mnmt.mnmt_encode(sess, d_ids, d_lens, B, S, mnmt.DEVICE_PTRS)
+    with torch.cuda.stream(stream):
+        w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        w0.record(stream)
+    mnmt.mnmt_decode_steps(sess, n)
+    with torch.cuda.stream(stream):
+        w1.record(stream)
     stream.synchronize()
-    avg_ms = sum(a.elapsed_time(b2) for a, b2 in ms) / len(ms)
+    cold_us = [a.elapsed_time(b) * 1e3 for a, b in cold]
+    avg_us = sum(cold_us) / len(cold_us)
+    warm_us = w0.elapsed_time(w1) * 1e3 / n
+    algo = sum(decode_step_bytes(cfg, R, B, S, t) for t in range(n)) / n
     peak, kind = _peaks()
-    achieved = algo_bytes / (avg_ms * 1e-3) / 1e9
-    return {"kernel": "linear_smallm<1,16,2> (vocab projection + argmax, M=1 N=%d K=%d)" % (V, d),
-            "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-            "peak_kind": f"{kind} hbm_gbs (burst, kernel timed alone)", "traffic": None,
-            "algorithmic_bytes": algo_bytes, "avg_us": avg_ms * 1e3, "launches": len(ms)}
+    achieved = algo / (avg_us * 1e-6) / 1e9
+    unit = ("decode_cluster_kernel + vocab_greedy_kernel (one graph launch)" if cluster
+            else "multi-kernel decode step (one graph launch)")
+    return {"kernel": f"decode step: {unit}, R={R} rows, S={S}", "bound": "hbm", "achieved": achieved, "peak": peak,
+            "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{kind} hbm_gbs (burst)",
+            "traffic": None, "algorithmic_bytes": int(algo), "avg_us": avg_us, "warm_avg_us": warm_us,
+            "launches": len(cold_us)}
 
 
 def main():

@@ -116,6 +116,14 @@ void mnmt_session_free(mnmt_session *s);
 int mnmt_encode(mnmt_session *s, const int32_t *src_ids, const int32_t *src_lens, int32_t B,
                 int32_t S_pad, int32_t flags);
 
+/* Queues n incremental decoder steps (at most the steps left before max_len)
+ * on the model's stream and returns without waiting: the steps run back to
+ * back with no host round trip between them, and steps after every sentence
+ * has finished do nothing.  Read the outcome with mnmt_debug_tap
+ * (MNMT_TAP_HISTORY / MNMT_TAP_PARENTS) or a later mnmt_decode_step.  Returns
+ * the number of steps queued, or a negative error code. */
+int mnmt_decode_steps(mnmt_session *s, int32_t n);
+
 /* One incremental decoder step for every hypothesis (greedy or beam), then
  * synchronises.  Host outputs, each NULL to skip: tokens [B*beam] (token
  * chosen at this step per hypothesis), parents [B*beam] (beam index within the

@@ -16,6 +16,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstddef>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -479,6 +480,7 @@ struct mnmt_session {
     // cluster decode step (small greedy batches)
     DcParams *d_dc = nullptr;
     bool use_cluster = false;
+    int dc_S = 0;  // host source of the parameter block's S when it is updated
     int dc_nc = 0;
     size_t dc_smem = 0;
 };
@@ -988,7 +990,11 @@ int setup_cluster_step(mnmt_session *s) {
         Y.self_k = s->sk + l * s->sk_layer; Y.self_v = s->sv + l * s->sk_layer;
         Y.cross_k = s->ck + l * s->ck_layer; Y.cross_v = s->cv + l * s->ck_layer;
     }
+    // lay shared memory out for the session's longest source, so that the
+    // captured step serves every padded length (only P.S changes per batch)
+    P.S = s->Smax;
     size_t smem = dc_layout(P, 227 * 1024);
+    P.S = s->S;
     if (!decode_cluster_fits(dh, nc, smem)) return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
@@ -1000,6 +1006,15 @@ int setup_cluster_step(mnmt_session *s) {
 
 int ensure_graph(mnmt_session *s) {
     if (s->gexec && s->graph_B == s->B && s->graph_S == s->S) return MNMT_OK;
+    if (s->gexec && s->graph_B == s->B && s->use_cluster) {
+        // the cluster step reads the padded source length from its parameter
+        // block: update it in stream order and keep the captured graph
+        s->dc_S = s->S;
+        CK(cudaMemcpyAsync(reinterpret_cast<uint8_t *>(s->d_dc) + offsetof(DcParams, S), &s->dc_S, sizeof(int),
+                           cudaMemcpyHostToDevice, s->m->stream));
+        s->graph_S = s->S;
+        return MNMT_OK;
+    }
     if (s->gexec) {
         cudaGraphExecDestroy(s->gexec);
         s->gexec = nullptr;
@@ -1089,6 +1104,22 @@ extern "C" int mnmt_encode(mnmt_session *s, const int32_t *src_ids, const int32_
     CK(cudaMemcpyAsync(s->state + ST_TMAX, s->h_state + ST_TMAX, 4, cudaMemcpyHostToDevice, st));
     s->steps = 0;
     return MNMT_OK;
+}
+
+extern "C" int mnmt_decode_steps(mnmt_session *s, int32_t n) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    if (s->poisoned) return fail(s->poisoned, "session poisoned by an earlier failure");
+    if (s->B < 1) return fail(MNMT_EINVAL, "decode_steps before encode");
+    if (n < 0) return fail(MNMT_EINVAL, "negative step count");
+    const int left = s->max_len - s->steps;
+    if (n > left) n = left;
+    if (n == 0) return 0;
+    int rc = ensure_graph(s);
+    if (rc) return poison(s, rc);
+    cudaStream_t st = s->m->stream;
+    for (int i = 0; i < n; i++) CK(cudaGraphLaunch(s->gexec, st));
+    s->steps += n;
+    return n;
 }
 
 extern "C" int mnmt_decode_step(mnmt_session *s, int32_t *tokens, int32_t *parents, float *scores,

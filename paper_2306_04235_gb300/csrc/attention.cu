@@ -15,7 +15,7 @@
 //                ancestry table when hypotheses were reordered) or over the
 //                cross-attention keys of the row's sentence.  Bound by the
 //                cache bytes it streams.
-//   attn_encoder one block per (sentence, head, 32-query chunk): K and V of
+//   attn_encoder one block per (sentence, head, chunk of 4..32 queries): K and V of
 //                the head staged in shared memory, keys masked past the
 //                source length.
 #include "common.cuh"
@@ -145,7 +145,7 @@ constexpr int ENC_MAX_KEYS = 512;
 constexpr int ENC_QCHUNK = 32;
 
 template <int DH>
-__global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a) {
+__global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, int qchunk) {
     extern __shared__ __align__(16) uint8_t esm[];
     constexpr int KS = DH + 16;  // padded key row: conflict-free 16-byte lane reads
     const int bh = blockIdx.x;
@@ -170,8 +170,8 @@ __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a) {
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int *sc = wsm + warp * S;
-    const int q0 = blockIdx.y * ENC_QCHUNK;
-    const int q1 = min(q0 + ENC_QCHUNK, S);
+    const int q0 = blockIdx.y * qchunk;
+    const int q1 = min(q0 + qchunk, S);
     constexpr int EPL = DH / 32;
     for (int qi = q0 + warp; qi < q1; qi += ENC_WARPS) {
         int4 qv[CH];
@@ -225,8 +225,12 @@ template <int DH>
 static cudaError_t launch_enc(const AttnEncArgs &a, cudaStream_t st) {
     size_t smem = (size_t)a.S * (DH + 16) + (size_t)a.S * DH + (size_t)ENC_WARPS * a.S * sizeof(int);
     auto k = attn_encoder<DH>;
-    dim3 grid(a.B * a.H, (a.S + ENC_QCHUNK - 1) / ENC_QCHUNK);
-    k<<<grid, 32 * ENC_WARPS, smem, st>>>(a);
+    // queries per block: the most (up to 32) that still gives every SM two
+    // blocks; small batches get one query per warp so the GPU fills up
+    int qc = ENC_QCHUNK;
+    while (qc > ENC_WARPS && (long)a.B * a.H * ((a.S + qc - 1) / qc) < 2 * 152) qc >>= 1;
+    dim3 grid(a.B * a.H, (a.S + qc - 1) / qc);
+    k<<<grid, 32 * ENC_WARPS, smem, st>>>(a, qc);
     return cudaGetLastError();
 }
 

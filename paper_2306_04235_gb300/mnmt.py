@@ -65,6 +65,7 @@ def _declare(L):
     L.mnmt_session_free.argtypes = [p]; L.mnmt_session_free.restype = None
     L.mnmt_encode.argtypes = [p, p, p, i32, i32, i32]
     L.mnmt_decode_step.argtypes = [p, p, p, p, p]
+    L.mnmt_decode_steps.argtypes = [p, i32]; L.mnmt_decode_steps.restype = C.c_int
     L.mnmt_translate.argtypes = [p, p, p, i32, i32, i32, i32, p, p, p]
     L.mnmt_debug_tap.argtypes = [p, i32, i32, p, sz]; L.mnmt_debug_tap.restype = C.c_int64
     L.mnmt_session_decode_path.argtypes = [p]; L.mnmt_session_decode_path.restype = C.c_int
@@ -147,6 +148,14 @@ def mnmt_session_free(session: int):
 
 def mnmt_encode(session: int, src_ids, src_lens, B: int, S_pad: int, flags: int = 0):
     _chk(lib().mnmt_encode(session, _ptr(src_ids), _ptr(src_lens), B, S_pad, flags))
+
+
+def mnmt_decode_steps(session: int, n: int) -> int:
+    """Queue n decode steps without waiting; returns the number queued."""
+    r = lib().mnmt_decode_steps(session, n)
+    if r < 0:
+        raise MnmtError(r, last_error())
+    return r
 
 
 def mnmt_decode_step(session: int, R: int):

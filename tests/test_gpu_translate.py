@@ -169,6 +169,48 @@ def test_decode_step_api_matches_translate(beam, stream):
         assert seq[:n] == list(o_ids[b, :n])
 
 
+@pytest.mark.parametrize("beam", [1, 3])
+def test_queued_decode_steps_match_stepwise_decode(beam, stream):
+    """mnmt_decode_steps queues steps without host round trips: the token and
+    parent history equals the one of step-by-step decoding, and steps past the
+    length limit are not queued."""
+    cfg = MINI["fact"]
+    blob = synth.build_blob(cfg, 8)
+    ids, lens = synth.source_batch(cfg.vocab, 2, 3, 20, 9)
+    T, R = 12, 2 * beam
+    tr = mnmt.Translator(blob, 2, ids.shape[1], beam, T, stream)
+    try:
+        mnmt.mnmt_encode(tr.session, ids, lens, 2, ids.shape[1])
+        steps = [mnmt.mnmt_decode_step(tr.session, R) for _ in range(T)]
+        mnmt.mnmt_encode(tr.session, ids, lens, 2, ids.shape[1])
+        assert mnmt.mnmt_decode_steps(tr.session, 5) == 5
+        assert mnmt.mnmt_decode_steps(tr.session, 100) == T - 5
+        assert mnmt.mnmt_decode_steps(tr.session, 1) == 0
+        hist = mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_HISTORY, 0, np.int32, (T, R))
+        par = mnmt.mnmt_debug_tap(tr.session, mnmt.TAP_PARENTS, 0, np.int32, (T, R))
+    finally:
+        tr.close()
+    assert np.array_equal(hist, np.stack([s[0] for s in steps]))
+    if beam > 1:
+        assert np.array_equal(par, np.stack([s[1] for s in steps]))
+
+
+def test_cluster_step_graph_serves_changing_source_lengths(stream):
+    """One session translating sentences of different padded lengths in turn
+    (the cluster step keeps its captured graph and only updates the length)."""
+    cfg, blob, _, _, beam, T = synth.workload_inputs("small-b1-s10to50-greedy64")
+    tr = mnmt.Translator(blob, 1, 50, 1, T, stream)
+    try:
+        for i, S in enumerate([37, 12, 50, 12, 29]):
+            ids, lens = synth.source_batch(cfg.vocab, 1, S, S, 70 + i)
+            g_ids, g_len, _ = tr.translate(ids, lens, T)
+            assert mnmt.mnmt_session_decode_path(tr.session) == 1
+            o_ids, o_len, _ = O.translate(blob, ids, lens, 1, T, n_threads=1)
+            assert np.array_equal(g_ids, o_ids) and np.array_equal(g_len, o_len), S
+    finally:
+        tr.close()
+
+
 def test_device_pointer_path_equals_host_path(stream):
     cfg = MINI["pre"]
     blob = synth.build_blob(cfg, 5)
