@@ -5,12 +5,13 @@
 // greedy argmax).
 //
 // Two kernels:
-//   linear_smallm  M <= 16 rows (batch-1 and small-batch decode): every weight
+//   linear_smallm  M <= 64 rows, in chunks of <= 16 rows per grid row
+//                  (batch-1 encoder, batch-1 and small-batch decode): every weight
 //                  row is streamed once with 16-byte coalesced loads, the M
 //                  activation rows sit in shared memory, products use dp4a and
 //                  a lane group's partial sums meet by warp shuffles.  Bound by
 //                  weight bytes (HBM or L2).
-//   linear_mma     M > 16: CTA tiles of the int8 GEMM on the warp-level s8
+//   linear_mma     M > 64: CTA tiles of the int8 GEMM on the warp-level s8
 //                  tensor-core instruction (mma.sync m16n8k32, exact int32
 //                  accumulate), cp.async multi-stage pipeline with XOR-swizzled
 //                  shared memory and ldmatrix fragment loads.  sm_103a has no
@@ -25,6 +26,7 @@ namespace mnmt {
 // small-M path
 // ---------------------------------------------------------------------------
 constexpr int SM_THREADS = 256;
+constexpr int SMALL_CHUNKED_MAX_M = 64;
 
 // MT: rows held (>= M); LPC: lanes per weight row (K/16 chunks spread over
 // LPC lanes); U: weight rows in flight per lane group.
@@ -35,6 +37,10 @@ __global__ void __launch_bounds__(SM_THREADS) linear_smallm(const int8_t *__rest
     if (e.skip && *e.skip) return;
     extern __shared__ int4 smA[];  // [MT][K/16]
     const int kc = K >> 4;
+    // blockIdx.y selects the chunk of MT rows this block computes
+    const int m0 = blockIdx.y * MT;
+    A += (size_t)m0 * lda;
+    M -= m0;
     for (int i = threadIdx.x; i < MT * kc; i += SM_THREADS) {
         int m = i / kc, c = i - m * kc;
         smA[i] = (m < M) ? reinterpret_cast<const int4 *>(A + (size_t)m * lda)[c] : make_int4(0, 0, 0, 0);
@@ -93,10 +99,21 @@ __global__ void __launch_bounds__(SM_THREADS) linear_smallm(const int8_t *__rest
                             best[m] = k > best[m] ? k : best[m];
                         }
                     }
+                } else if (e.mode == EPI_RESID) {
+                    // every residual load first: the stores may alias them
+                    float r[MT];
+#pragma unroll
+                    for (int m = 0; m < MT; m++) r[m] = m < M ? e.f32[(size_t)(m0 + m) * e.ldf + n] : 0.0f;
+#pragma unroll
+                    for (int m = 0; m < MT; m++)
+                        if (m < M)
+                            e.f32[(size_t)(m0 + m) * e.ldf + n] =
+                                __fadd_rn(__fmul_rn(e.gamma, r[m]),
+                                          dequant_bias(acc[u][m], e.s_x, e.s_w[n], e.bias[n]));
                 } else {
 #pragma unroll
                     for (int m = 0; m < MT; m++)
-                        if (m < M) epi_store(e, m, n, acc[u][m], t);
+                        if (m < M) epi_store(e, m0 + m, n, acc[u][m], t);
                 }
             }
         }
@@ -112,7 +129,7 @@ __global__ void __launch_bounds__(SM_THREADS) linear_smallm(const int8_t *__rest
         if (threadIdx.x < MT && (int)threadIdx.x < M) {
             unsigned long long v = 0;
             for (int w = 0; w < SM_THREADS / 32; w++) v = red[w][threadIdx.x] > v ? red[w][threadIdx.x] : v;
-            atomicMax(e.keys + threadIdx.x, v);
+            atomicMax(e.keys + m0 + threadIdx.x, v);
         }
     }
 }
@@ -267,6 +284,34 @@ __global__ void __launch_bounds__(WARPS_M *WARPS_N * 32)
         }
         return;
     }
+    if (e.mode == EPI_RESID) {
+        // every residual load first: the stores may alias them
+        float r[MI][NI][4];
+#pragma unroll
+        for (int mi = 0; mi < MI; mi++)
+#pragma unroll
+            for (int ni = 0; ni < NI; ni++)
+#pragma unroll
+                for (int q = 0; q < 4; q++) {
+                    int row = bm + wm * WTM + mi * 16 + (lane >> 2) + (q >> 1) * 8;
+                    int col = bn + wn * WTN + ni * 8 + (lane & 3) * 2 + (q & 1);
+                    r[mi][ni][q] = (row < M && col < N) ? e.f32[(size_t)row * e.ldf + col] : 0.0f;
+                }
+#pragma unroll
+        for (int mi = 0; mi < MI; mi++)
+#pragma unroll
+            for (int ni = 0; ni < NI; ni++)
+#pragma unroll
+                for (int q = 0; q < 4; q++) {
+                    int row = bm + wm * WTM + mi * 16 + (lane >> 2) + (q >> 1) * 8;
+                    int col = bn + wn * WTN + ni * 8 + (lane & 3) * 2 + (q & 1);
+                    if (row < M && col < N)
+                        e.f32[(size_t)row * e.ldf + col] =
+                            __fadd_rn(__fmul_rn(e.gamma, r[mi][ni][q]),
+                                      dequant_bias(acc[mi][ni][q], e.s_x, e.s_w[col], e.bias[col]));
+                }
+        return;
+    }
 #pragma unroll
     for (int mi = 0; mi < MI; mi++)
 #pragma unroll
@@ -300,6 +345,7 @@ template <int MT>
 static cudaError_t launch_small(const int8_t *A, int lda, const int8_t *W, int M, int N, int K, const Epi &e,
                                 cudaStream_t st) {
     const int kc = K / 16;
+    const int chunks = (M + MT - 1) / MT;  // row chunks of MT, one per grid row
     size_t smem = (size_t)MT * kc * 16;
     int lpc = kc >= 32 ? 32 : (kc >= 16 ? 16 : 8);
     constexpr int U = 2;
@@ -307,12 +353,13 @@ static cudaError_t launch_small(const int8_t *A, int lda, const int8_t *W, int M
     int blocks = (N + cpb - 1) / cpb;
     if (blocks > 4 * 152) blocks = 4 * 152;
     if (smem > 48 * 1024) return cudaErrorInvalidValue;  // K <= 3072 at M <= 16
+    const dim3 grid(blocks, chunks);
     if (lpc == 32) {
-        linear_smallm<MT, 32, U><<<blocks, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        linear_smallm<MT, 32, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
     } else if (lpc == 16) {
-        linear_smallm<MT, 16, U><<<blocks, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        linear_smallm<MT, 16, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
     } else {
-        linear_smallm<MT, 8, U><<<blocks, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        linear_smallm<MT, 8, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
     }
     return cudaGetLastError();
 }
@@ -337,6 +384,9 @@ cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int 
         if (M <= 8) return launch_small<8>(A, lda, W, M, N, K, e, st);
         return launch_small<16>(A, lda, W, M, N, K, e, st);
     }
+    // up to 64 rows: chunks of 16 rows over the grid's y dimension (the
+    // weights are re-read per chunk from L2; more blocks than IMMA tiles)
+    if (M <= SMALL_CHUNKED_MAX_M && K <= 2048) return launch_small<16>(A, lda, W, M, N, K, e, st);
     long tiles_big = (long)((M + 127) / 128) * ((N + 127) / 128);
     if (tiles_big >= 152) return launch_mma<128, 128, 2, 4, 4>(A, lda, W, M, N, K, e, st);
     return launch_mma<64, 64, 2, 2, 4>(A, lda, W, M, N, K, e, st);
