@@ -5,13 +5,14 @@
 // greedy argmax).
 //
 // Two kernels:
-//   linear_smallm  M <= 64 rows, in chunks of <= 16 rows per grid row
-//                  (batch-1 encoder, batch-1 and small-batch decode): every weight
+//   linear_smallm  M <= 16 rows, or up to 64 rows of a narrow layer, in chunks
+//                  of <= 16 rows per grid row (batch-1 encoder, batch-1 and
+//                  small-batch decode): every weight
 //                  row is streamed once with 16-byte coalesced loads, the M
 //                  activation rows sit in shared memory, products use dp4a and
 //                  a lane group's partial sums meet by warp shuffles.  Bound by
 //                  weight bytes (HBM or L2).
-//   linear_mma     M > 64: CTA tiles of the int8 GEMM on the warp-level s8
+//   linear_mma     other M > 16: CTA tiles of the int8 GEMM on the warp-level s8
 //                  tensor-core instruction (mma.sync m16n8k32, exact int32
 //                  accumulate), cp.async multi-stage pipeline with XOR-swizzled
 //                  shared memory and ldmatrix fragment loads.  sm_103a has no
@@ -384,9 +385,11 @@ cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int 
         if (M <= 8) return launch_small<8>(A, lda, W, M, N, K, e, st);
         return launch_small<16>(A, lda, W, M, N, K, e, st);
     }
-    // up to 64 rows: chunks of 16 rows over the grid's y dimension (the
-    // weights are re-read per chunk from L2; more blocks than IMMA tiles)
-    if (M <= SMALL_CHUNKED_MAX_M && K <= 2048) return launch_small<16>(A, lda, W, M, N, K, e, st);
+    // up to 64 rows over few output tiles (narrow N): chunks of 16 rows over
+    // the grid's y dimension spread the work over more blocks than the IMMA
+    // tiling would (the weights are re-read per chunk, from L2)
+    const long tiles64 = (long)((M + 63) / 64) * ((N + 63) / 64);
+    if (M <= SMALL_CHUNKED_MAX_M && K <= 2048 && tiles64 < 8) return launch_small<16>(A, lda, W, M, N, K, e, st);
     long tiles_big = (long)((M + 127) / 128) * ((N + 127) / 128);
     if (tiles_big >= 152) return launch_mma<128, 128, 2, 4, 4>(A, lda, W, M, N, K, e, st);
     return launch_mma<64, 64, 2, 2, 4>(A, lda, W, M, N, K, e, st);
