@@ -348,6 +348,12 @@ def run_gpu(args):
     return 0
 
 
+# DRAM bytes of one decode step (dram__bytes_read.sum + dram__bytes_write.sum
+# of its kernels, one ncu capture of this bench's command); only for the step
+# kernels they were taken on -- refresh whenever those kernels change
+STEP_TRAFFIC = {("small-b1-s10to50-greedy64", True): 10_560_256}
+
+
 def measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster):
     """Decode steps of one encoded batch timed with CUDA events on the
     library's stream: one step per event pair with L2 flushed before each
@@ -384,7 +390,7 @@ def measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens
             else "multi-kernel decode step (one graph launch)")
     return {"kernel": f"decode step: {unit}, R={R} rows, S={S}", "bound": "hbm", "achieved": achieved, "peak": peak,
             "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{kind} hbm_gbs (burst)",
-            "traffic": None, "algorithmic_bytes": int(algo), "avg_us": avg_us, "warm_avg_us": warm_us,
+            "traffic": STEP_TRAFFIC.get((wl.name, cluster)), "algorithmic_bytes": int(algo), "avg_us": avg_us, "warm_avg_us": warm_us,
             "launches": len(cold_us)}
 
 

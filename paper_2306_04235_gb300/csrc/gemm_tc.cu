@@ -33,6 +33,7 @@
 #include "common.cuh"
 #include "epilogue.cuh"
 #include "internal.h"
+#include "mbarrier.cuh"
 #include "mnmt.h"
 
 namespace mnmt {
@@ -43,46 +44,8 @@ constexpr int TC_BK = 64;             // fp16 per k-block: one 128-byte swizzle 
 constexpr int TC_KB_PER_CHUNK = 16;   // 16 x 64 = 1024 products per exact fp32 chunk
 constexpr int TC_EPI_WARPS = 8;                  // two warps per TMEM lane quarter
 constexpr int TC_THREADS = 64 + TC_EPI_WARPS * 32;  // producer warp, MMA warp, epilogue warps
-constexpr unsigned long long TC_WAIT_NS = 1000000000ull;
 
 __device__ __forceinline__ uint32_t s_addr(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ unsigned long long global_ns() {
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// wait for the completion of the phase with the given parity; false if it has
-// not completed within TC_WAIT_NS
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    if (mbar_try(bar, parity)) return true;
-    const unsigned long long t0 = global_ns();
-    while (!mbar_try(bar, parity)) {
-        if (global_ns() - t0 > TC_WAIT_NS) return false;
-    }
-    return true;
-}
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm, int x, int y, uint32_t bar) {
     asm volatile(
@@ -159,10 +122,6 @@ struct TcLayout {
     static constexpr uint32_t BYTES = OFF_MISC + 16;
     static constexpr size_t SMEM = 1024 + BYTES;  // slack to align the ring to 1024 bytes
 };
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 
 // named barrier over the epilogue warps only
 __device__ __forceinline__ void epi_bar_sync() { asm volatile("bar.sync 1, %0;" ::"n"(TC_EPI_WARPS * 32) : "memory"); }
