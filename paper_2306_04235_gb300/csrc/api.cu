@@ -456,6 +456,8 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
 enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_STATUS = 5, ST_N = 8 };
 // layers of at least this many rows run on the tensor cores (one full M tile)
 constexpr size_t TC_MIN_ROWS = 128;
+// steps per multi-step decode graph (and per completion check of translate)
+constexpr int GRAPH_STEPS = 16;
 
 struct mnmt_session {
     mnmt_model *m;
@@ -476,6 +478,7 @@ struct mnmt_session {
     int *h_state = nullptr;  // pinned mirror of state
     size_t ck_layer, sk_layer;  // per-layer strides of the caches (elements)
     cudaGraphExec_t gexec = nullptr;
+    cudaGraphExec_t gexec_n = nullptr;  // GRAPH_STEPS consecutive steps (cluster path)
     int graph_B = -1, graph_S = -1;
     // cluster decode step (small greedy batches)
     DcParams *d_dc = nullptr;
@@ -587,6 +590,7 @@ extern "C" void mnmt_session_free(mnmt_session *s) {
     if (!s) return;
     if (s->m && s->m->stream) cudaStreamSynchronize(s->m->stream);
     if (s->gexec) cudaGraphExecDestroy(s->gexec);
+    if (s->gexec_n) cudaGraphExecDestroy(s->gexec_n);
     if (s->arena) cudaFree(s->arena);
     if (s->h_state) cudaFreeHost(s->h_state);
     delete s;
@@ -1004,41 +1008,68 @@ int setup_cluster_step(mnmt_session *s) {
     return MNMT_OK;
 }
 
-int ensure_graph(mnmt_session *s) {
-    if (s->gexec && s->graph_B == s->B && s->graph_S == s->S) return MNMT_OK;
-    if (s->gexec && s->graph_B == s->B && s->use_cluster) {
-        // the cluster step reads the padded source length from its parameter
-        // block: update it in stream order and keep the captured graph
-        s->dc_S = s->S;
-        CK(cudaMemcpyAsync(reinterpret_cast<uint8_t *>(s->d_dc) + offsetof(DcParams, S), &s->dc_S, sizeof(int),
-                           cudaMemcpyHostToDevice, s->m->stream));
-        s->graph_S = s->S;
-        return MNMT_OK;
-    }
-    if (s->gexec) {
-        cudaGraphExecDestroy(s->gexec);
-        s->gexec = nullptr;
-    }
+// capture `steps` consecutive decode steps into one executable graph
+int capture_steps(mnmt_session *s, int steps, cudaGraphExec_t *out) {
     cudaStream_t st = s->m->stream;
-    int rc0 = setup_cluster_step(s);
-    if (rc0) return rc0;
     cudaGraph_t g = nullptr;
     CK(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
-    int rc = issue_decode_step(s);
+    int rc = MNMT_OK;
+    for (int i = 0; i < steps && !rc; i++) rc = issue_decode_step(s);
     cudaError_t ce = cudaStreamEndCapture(st, &g);
     if (rc) {
         if (g) cudaGraphDestroy(g);
         return rc;
     }
     if (ce != cudaSuccess) return fail(MNMT_ECUDA, "graph capture failed: %s", cudaGetErrorString(ce));
-    ce = cudaGraphInstantiate(&s->gexec, g, 0);
+    ce = cudaGraphInstantiate(out, g, 0);
     cudaGraphDestroy(g);
     if (ce != cudaSuccess) {
-        s->gexec = nullptr;
+        *out = nullptr;
         return fail(MNMT_ECUDA, "graph instantiation failed: %s", cudaGetErrorString(ce));
     }
+    return MNMT_OK;
+}
+
+int ensure_graph(mnmt_session *s) {
+    if (s->gexec && s->graph_B == s->B && s->graph_S == s->S) return MNMT_OK;
+    if (s->gexec && s->graph_B == s->B && s->use_cluster) {
+        // the cluster step reads the padded source length from its parameter
+        // block: update it in stream order and keep the captured graphs
+        s->dc_S = s->S;
+        CK(cudaMemcpyAsync(reinterpret_cast<uint8_t *>(s->d_dc) + offsetof(DcParams, S), &s->dc_S, sizeof(int),
+                           cudaMemcpyHostToDevice, s->m->stream));
+        s->graph_S = s->S;
+        return MNMT_OK;
+    }
+    for (cudaGraphExec_t *ge : {&s->gexec, &s->gexec_n})
+        if (*ge) {
+            cudaGraphExecDestroy(*ge);
+            *ge = nullptr;
+        }
+    int rc = setup_cluster_step(s);
+    if (rc) return rc;
+    if ((rc = capture_steps(s, 1, &s->gexec))) return rc;
+    // the cluster step also gets a graph of GRAPH_STEPS steps, inside which
+    // each step's kernel starts while the previous step's vocabulary kernel
+    // runs (programmatic dependent launch)
+    if (s->use_cluster && (rc = capture_steps(s, GRAPH_STEPS, &s->gexec_n))) return rc;
     s->graph_B = s->B;
     s->graph_S = s->S;
+    return MNMT_OK;
+}
+
+// queue n decode steps (graph launches, no synchronisation)
+int launch_steps(mnmt_session *s, int n) {
+    cudaStream_t st = s->m->stream;
+    while (n > 0) {
+        if (s->gexec_n && n >= GRAPH_STEPS) {
+            CK(cudaGraphLaunch(s->gexec_n, st));
+            n -= GRAPH_STEPS;
+        } else {
+            CK(cudaGraphLaunch(s->gexec, st));
+            n--;
+        }
+    }
     return MNMT_OK;
 }
 
@@ -1116,8 +1147,7 @@ extern "C" int mnmt_decode_steps(mnmt_session *s, int32_t n) {
     if (n == 0) return 0;
     int rc = ensure_graph(s);
     if (rc) return poison(s, rc);
-    cudaStream_t st = s->m->stream;
-    for (int i = 0; i < n; i++) CK(cudaGraphLaunch(s->gexec, st));
+    if ((rc = launch_steps(s, n))) return poison(s, rc);
     s->steps += n;
     return n;
 }
@@ -1157,11 +1187,11 @@ extern "C" int mnmt_translate(mnmt_session *s, const int32_t *src_ids, const int
     s->h_state[ST_TMAX] = max_len;
     CK(cudaMemcpyAsync(s->state + ST_TMAX, s->h_state + ST_TMAX, 4, cudaMemcpyHostToDevice, st));
     if ((rc = ensure_graph(s))) return poison(s, rc);
-    const int CHECK = 16;
+    const int CHECK = GRAPH_STEPS;
     int steps = 0;
     while (steps < max_len) {
         int n = max_len - steps < CHECK ? max_len - steps : CHECK;
-        for (int i = 0; i < n; i++) CK(cudaGraphLaunch(s->gexec, st));
+        if ((rc = launch_steps(s, n))) return poison(s, rc);
         steps += n;
         if (steps < max_len) {
             if ((rc = sync_state(s))) return rc;

@@ -44,6 +44,11 @@ MNMT_DEV void dc_cp16(void *dst_smem, const void *src) {
 MNMT_DEV void dc_commit() { asm volatile("cp.async.commit_group;\n" ::); }
 MNMT_DEV void dc_wait_ring() { asm volatile("cp.async.wait_group %0;\n" ::"n"(DC_NB - 2)); }
 
+// programmatic dependent launch: wait for the preceding kernel of the stream
+// (and the memory it wrote); allow the following kernel to launch
+MNMT_DEV void dc_grid_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+MNMT_DEV void dc_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+
 // out-of-line copies of the exact roundings (one copy of the code each)
 __device__ __noinline__ float dc_rn32_div(long long n, long long z) { return rn32_div(n, z); }
 __device__ __noinline__ float dc_rn32_pow2(long long s, int e) { return rn32_pow2(s, e); }
@@ -92,75 +97,75 @@ __device__ __noinline__ void dc_bcast(cg::cluster_group &cl, const uint8_t *stag
 
 // Block-wide LayerNorm of the R rows of r (same arithmetic as
 // warp_layernorm): element e of the flattened [R][d] array belongs to thread
-// e % 256; each warp's 32 elements lie in one row, so per-row maxima and exact
-// int64 sums are warp reductions (redux.sync) whose partials meet in shared
-// memory, d/32 partials per row.  The passes keep no per-element registers
-// (r - mean goes through shared memory) and are not unrolled, so the code
-// stays small.  q8(LN(r), inv) goes to a; with write_back the normalised row
-// also replaces r.  Ends with a block barrier.
-MNMT_DEV unsigned dc_row_max(const unsigned *part, int row, int spr) {
-    unsigned m = 0;
-    for (int k = 0; k < spr; k++) m = max(m, part[row * spr + k]);
-    return m;
-}
+// e % 256; each warp's 32 elements lie in one row, so the exact int64 sums are
+// warp reductions (redux.sync) whose partials meet in shared memory, d/32
+// partials per row.  The row's largest and smallest values arrive with the
+// residual itself (mm [R][nc] ordered-bit pairs, one per CTA slice, written
+// by the epilogue that produced r), which gives both grids without a pass of
+// their own: max|r| = max(|max r|, |min r|) and, fl(x - mu) being monotone in
+// x, max|fl(r - mu)| = max(|fl(max r - mu)|, |fl(min r - mu)|).  Three passes:
+// exact sum of r, exact sum of (r - mu)^2, normalise.  q8(LN(r), inv) goes to
+// a; with write_back the normalised row also replaces r.  Ends with a block
+// barrier.
 MNMT_DEV long long dc_row_sum(const long long *part, int row, int spr) {
     long long s = 0;
     for (int k = 0; k < spr; k++) s += part[row * spr + k];
     return s;
 }
 
+// the row's max and min from the nc slice records (one warp, all lanes)
+MNMT_DEV void dc_row_extremes(const unsigned *mm, int row, int nc, float &hi, float &lo) {
+    const int lane = threadIdx.x & 31;
+    const unsigned kh = lane < nc ? mm[(row * nc + lane) * 2 + 0] : 0u;
+    const unsigned kl = lane < nc ? mm[(row * nc + lane) * 2 + 1] : 0xFFFFFFFFu;
+    hi = from_ordered_bits(__reduce_max_sync(0xFFFFFFFFu, kh));
+    lo = from_ordered_bits(__reduce_min_sync(0xFFFFFFFFu, kl));
+}
+
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
-                                          int8_t *a, int write_back, int *status, unsigned *part_u,
-                                          long long *part_l, float *cbuf) {
+                                          int8_t *a, int write_back, int *status, const unsigned *mm, int nc,
+                                          long long *part_l) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int n = R * d, spr = d / 32;  // partial slots (warps) per row
     const int log2d = 31 - __clz(d);
-    // pass 1: max |x| per warp chunk
+    // pass 1: exact sum of x on the grid of max |x|
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
-        const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(r[e0 + lane]) & 0x7FFFFFFFu);
-        if (lane == 0) part_u[e0 / 32] = m;
-    }
-    __syncthreads();
-    // pass 2: exact sum of x on the row's grid
-#pragma unroll 1
-    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
-        const unsigned am = dc_row_max(part_u, e0 / d, spr);
-        if (!(__uint_as_float(am) < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
-        const int ea = exp_bound(__uint_as_float(am));
-        const long long s = warp_sum_exact(fx_scale(r[e0 + lane], 52 - ea));
+        float hi, lo;
+        dc_row_extremes(mm, e0 / d, nc, hi, lo);
+        const float am = fmaxf(fabsf(hi), fabsf(lo));
+        if (!(am < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
+        const long long s = warp_sum_exact(fx_scale(r[e0 + lane], 52 - exp_bound(am)));
         if (lane == 0) part_l[e0 / 32] = s;
     }
     __syncthreads();
-    // pass 3: c = x - mean (kept in cbuf), max |c| per warp chunk
+    // pass 2: exact sum of c^2 = fl(x - mean)^2 on the grid of max |c|
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
         const int row = e0 / d;
-        const int ea = exp_bound(__uint_as_float(dc_row_max(part_u, row, spr)));
+        float hi, lo;
+        dc_row_extremes(mm, row, nc, hi, lo);
+        const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
         const float mu = dc_rn32_pow2(dc_row_sum(part_l, row, spr), ea - 52 - log2d);
+        const int eb = exp_bound(fmaxf(fabsf(__fsub_rn(hi, mu)), fabsf(__fsub_rn(lo, mu))));
         const float cv = __fsub_rn(r[e0 + lane], mu);
-        cbuf[e0 + lane] = cv;
-        const unsigned m = __reduce_max_sync(0xFFFFFFFFu, __float_as_uint(cv) & 0x7FFFFFFFu);
-        if (lane == 0) part_u[64 + e0 / 32] = m;
-    }
-    __syncthreads();
-    // pass 4: exact sum of c^2 on the row's grid
-#pragma unroll 1
-    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
-        const int eb = exp_bound(__uint_as_float(dc_row_max(part_u + 64, e0 / d, spr)));
-        const float cv = cbuf[e0 + lane];
         const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
         if (lane == 0) part_l[64 + e0 / 32] = s;
+        if (lane == 0 && (e0 % d) == 0) {
+            reinterpret_cast<float *>(part_l + 128)[2 * row] = mu;  // per row: mu, 2^eb grid
+            reinterpret_cast<int *>(part_l + 128)[2 * row + 1] = eb;
+        }
     }
     __syncthreads();
-    // pass 5: normalise, scale, shift, quantise
+    // pass 3: normalise, scale, shift, quantise
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
         const int row = e0 / d, e = e0 + lane, i = e - row * d;
-        const int eb = exp_bound(__uint_as_float(dc_row_max(part_u + 64, row, spr)));
+        const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
+        const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
         const float var = dc_rn32_pow2(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52 - log2d);
         const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
-        const float y = __fadd_rn(__fmul_rn(__fmul_rn(cbuf[e], rstd), g[i]), b[i]);
+        const float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(r[e], mu), rstd), g[i]), b[i]);
         a[e] = q8(y, inv);
         if (write_back) r[e] = y;
     }
@@ -309,6 +314,11 @@ enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
 
 template <int DH>
 __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcParams *__restrict__ Pp) {
+    // Launched as a programmatic dependent of the previous step's vocabulary
+    // kernel: everything up to dc_grid_wait() reads only data that no kernel
+    // of the decode loop writes (parameters, weights, LayerNorm vectors, the
+    // encoder's cross keys / values), so it overlaps the previous kernel.
+    // `done` only turns 0 -> 1 within a translation: seen set, it is final.
     if (*Pp->done) return;  // uniform for the whole cluster
     extern __shared__ __align__(16) uint8_t smem[];
     {
@@ -323,7 +333,6 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     const int c = (int)cl.block_rank();
     const int nc = P.nc;
     const int R = P.R, d = P.d, F = P.F, H = P.H;
-    const int t = *P.t_ptr;
 
     float *r_full = reinterpret_cast<float *>(smem + P.off_r);
     int8_t *a_full = reinterpret_cast<int8_t *>(smem + P.off_a);
@@ -339,9 +348,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     long long *red_l = reinterpret_cast<long long *>(smem + P.off_red + 64);  // [8]
     long long *pn = reinterpret_cast<long long *>(smem + P.off_red + 128);    // [8][DH]
     int *tok_s = reinterpret_cast<int *>(smem + P.off_red + 128 + 8 * DH * 8);  // [R]
-    unsigned *part_u = reinterpret_cast<unsigned *>(smem + P.off_part);           // [2][64] LN partials
-    long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 512);    // [2][64]
-    float *cbuf = reinterpret_cast<float *>(smem + P.off_cbuf);                   // [R][d]
+    unsigned *mm = reinterpret_cast<unsigned *>(smem + P.off_part);               // [R][nc][2] slice max / min of r
+    long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 512);    // [2][64] LN partials, [R] (mu, eb)
     const int nphase = 1 + 6 * P.n_dec;
 
     // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
@@ -356,14 +364,6 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
         if (src) dc_copy(lnp + (size_t)v * d, src, d * 4);
     }
-    if (threadIdx.x < R) {
-        int id = P.tok[threadIdx.x];
-        if (id < 0 || id >= P.V) {
-            set_status(P.status, MNMT_EINVAL);
-            id = 0;
-        }
-        tok_s[threadIdx.x] = id;
-    }
     dc_prefetch(P, 0, c, ring);
     // group 1: the second weight slice and the keys / values the step attends to
     if (P.kv_staged) {
@@ -372,6 +372,26 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int cb = R * P.S * d;  // one layer's cross K (or V): [R][H][S][dh]
             dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 0) * cb, Y.cross_k, cb);
             dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 1) * cb, Y.cross_v, cb);
+        }
+    }
+    // ---- the previous step's results: token, position, self keys / values ----
+    dc_grid_wait();
+    if (*P.done) {  // uniform for the whole cluster; no copy may outlive the CTA
+        asm volatile("cp.async.wait_all;\n" ::);
+        return;
+    }
+    const int t = *P.t_ptr;
+    if (threadIdx.x < R) {
+        int id = P.tok[threadIdx.x];
+        if (id < 0 || id >= P.V) {
+            set_status(P.status, MNMT_EINVAL);
+            id = 0;
+        }
+        tok_s[threadIdx.x] = id;
+    }
+    if (P.kv_staged) {
+        for (int l = 0; l < P.n_dec; l++) {
+            const DcLayer &Y = P.layer[l];
             if (t > 0) {
                 const int seg = t * DH;  // positions 0..t-1 of one (row, head)
                 for (int x = 0; x < 2 * R * H; x++) {
@@ -408,12 +428,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, part_u, part_l, cbuf);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, mm, nc, part_l);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
             } else {
-                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status, part_u,
-                             part_l, cbuf);
+                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status, mm, nc,
+                             part_l);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
@@ -506,6 +526,19 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         __syncthreads();
         // ---- publish the slice to every CTA ----
         if (out_f32) {
+            // the slice's largest and smallest residual value per row (rows <= 32),
+            // for the next LayerNorm's grids
+            if (threadIdx.x < 32 * R) {
+                const int m = threadIdx.x >> 5, ln = threadIdx.x & 31;
+                const unsigned k = ln < rows ? ordered_bits(stf[m * rows + ln]) : 0u;
+                const unsigned kh = __reduce_max_sync(0xFFFFFFFFu, k);
+                const unsigned kl = __reduce_min_sync(0xFFFFFFFFu, ln < rows ? k : 0xFFFFFFFFu);
+                if (ln < nc) {
+                    unsigned *dst = cl.map_shared_rank(mm + (m * nc + c) * 2, ln);
+                    dst[0] = kh;
+                    dst[1] = kl;
+                }
+            }
             dc_bcast(cl, stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
         } else {
             int8_t *full = kind == K_QKV ? qkv_full : (kind == K_Q2 ? q2_full : h_full);
@@ -517,13 +550,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, part_u, part_l, cbuf);
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l);
         }
     }
+    dc_launch_dependents();  // the vocabulary kernel may start its prologue
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     1.0f / P.s_dout, a_full, 0, P.status, part_u, part_l, cbuf);
+                     1.0f / P.s_dout, a_full, 0, P.status, mm, nc, part_l);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -544,6 +578,10 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
                                                            const float *__restrict__ bias, float s_x, int M, int N,
                                                            int K, unsigned long long *keys, int *ticket,
                                                            GreedyArgs g) {
+    // launched as a programmatic dependent of the step kernel: let the next
+    // step's kernel start its own prologue, then wait for this step's input
+    dc_launch_dependents();
+    dc_grid_wait();
     if (*g.done) return;
     extern __shared__ int4 vsm[];  // [MT][K/16]
     const int kc = K >> 4;
@@ -701,8 +739,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
-    P.off_part = take(512 + 1024);                                  // LayerNorm partials (2 x 64 warp chunks)
-    P.off_cbuf = take((size_t)R * d * 4);                           // LayerNorm x - mean
+    P.off_part = take(512 + 1024 + 64);  // slice extremes [R][nc][2], LN partials [2][64], per-row (mu, eb)
     if (R * d > 64 * 32) return (size_t)-1;                         // 64 warp chunks of partials
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
@@ -745,13 +782,15 @@ bool decode_cluster_fits(int dh, int nc, size_t smem) {
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
     cfg.dynamicSmemBytes = smem;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = nc;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     int clusters = 0;
     if (cudaOccupancyMaxActiveClusters(&clusters, k, &cfg) != cudaSuccess) {
         cudaGetLastError();
@@ -789,13 +828,22 @@ cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s
     const int cpb = 8 * (32 / lpc) * 4;
     int blocks = (N + cpb - 1) / cpb;
     if (blocks > 2 * 152) blocks = 2 * 152;
-    size_t smem;
-    switch (M) {
-        case 1: smem = (size_t)1 * kc * 16; vocab_greedy_kernel<1><<<blocks, 256, smem, st>>>(A, W, s_w, bias, s_x, M, N, K, keys, ticket, g); break;
-        case 2: smem = (size_t)2 * kc * 16; vocab_greedy_kernel<2><<<blocks, 256, smem, st>>>(A, W, s_w, bias, s_x, M, N, K, keys, ticket, g); break;
-        default: smem = (size_t)4 * kc * 16; vocab_greedy_kernel<4><<<blocks, 256, smem, st>>>(A, W, s_w, bias, s_x, M, N, K, keys, ticket, g); break;
+    const int mt = M == 1 ? 1 : (M == 2 ? 2 : 4);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(blocks);
+    cfg.blockDim = dim3(256);
+    cfg.dynamicSmemBytes = (size_t)mt * kc * 16;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    switch (mt) {
+        case 1: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<1>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
+        case 2: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<2>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
+        default: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<4>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
     }
-    return cudaGetLastError();
 }
 
 }  // namespace mnmt
