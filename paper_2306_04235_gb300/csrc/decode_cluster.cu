@@ -408,6 +408,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
         const int l = ph == 0 ? 0 : (ph - 1) / 6;
         const DcLayer &Y = P.layer[l];
+        // from the last phase on, the vocabulary kernel may launch and fetch its weights
+        if (ph == nphase - 1) dc_launch_dependents();
         dc_wait_ring();
         __syncthreads();
         dc_prefetch(P, ph + DC_NB - 1, c, ring);
@@ -553,7 +555,6 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l);
         }
     }
-    dc_launch_dependents();  // the vocabulary kernel may start its prologue
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
@@ -570,72 +571,72 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
 }
 
 // ---------------------------------------------------------------------------
-// vocabulary projection + greedy argmax + greedy update (last block)
+// vocabulary projection + greedy argmax + greedy update (last block).  Each
+// block owns a contiguous range of output rows, held in shared memory.
 // ---------------------------------------------------------------------------
 template <int MT>
 __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restrict__ A, const int8_t *__restrict__ W,
                                                            const float *__restrict__ s_w,
                                                            const float *__restrict__ bias, float s_x, int M, int N,
-                                                           int K, unsigned long long *keys, int *ticket,
-                                                           GreedyArgs g) {
-    // launched as a programmatic dependent of the step kernel: let the next
-    // step's kernel start its own prologue, then wait for this step's input
+                                                           int K, int rows_per_block, unsigned long long *keys,
+                                                           int *ticket, GreedyArgs g) {
+    // Launched as a programmatic dependent of the step kernel: the block's
+    // weight rows, scales and biases (static) are fetched into shared memory
+    // while the step kernel finishes; only the input row waits for it.
     dc_launch_dependents();
-    dc_grid_wait();
-    if (*g.done) return;
-    extern __shared__ int4 vsm[];  // [MT][K/16]
+    extern __shared__ __align__(16) int4 vsm[];  // [rows][K/16] weights, [MT][K/16] input, [rows] scale, [rows] bias
     const int kc = K >> 4;
-    for (int i = threadIdx.x; i < MT * kc; i += 256) {
-        int m = i / kc, c = i - m * kc;
-        vsm[i] = m < M ? reinterpret_cast<const int4 *>(A + (size_t)m * K)[c] : make_int4(0, 0, 0, 0);
+    const int n0 = blockIdx.x * rows_per_block;
+    const int nr = min(rows_per_block, N - n0);
+    int4 *ws = vsm;
+    int4 *as = vsm + (size_t)rows_per_block * kc;
+    float *scs = reinterpret_cast<float *>(as + MT * kc);
+    float *bss = scs + rows_per_block;
+    for (int i = threadIdx.x; i < nr * kc; i += 256) dc_cp16(ws + i, reinterpret_cast<const int4 *>(W + (size_t)n0 * K) + i);
+    dc_commit();
+    for (int i = threadIdx.x; i < nr; i += 256) {
+        scs[i] = __fmul_rn(s_x, s_w[n0 + i]);
+        bss[i] = bias[n0 + i];
     }
+    dc_grid_wait();
+    if (*g.done) {  // no copy may outlive the block
+        asm volatile("cp.async.wait_all;\n" ::);
+        return;
+    }
+    for (int i = threadIdx.x; i < MT * kc; i += 256) {
+        const int m = i / kc, c = i - m * kc;
+        as[i] = m < M ? reinterpret_cast<const int4 *>(A + (size_t)m * K)[c] : make_int4(0, 0, 0, 0);
+    }
+    asm volatile("cp.async.wait_all;\n" ::);
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int lpc = kc >= 32 ? 32 : kc;
-    const int gpw = 32 / lpc;
-    const int grp = lane / lpc, sl = lane % lpc;
-    constexpr int U = 4;
-    const int cpb = 8 * gpw * U;
+    const int lpr = kc >= 32 ? 32 : kc;  // lanes per weight row (kc is a power of two)
+    const int rpw = 32 / lpr;            // rows per warp and pass
+    const int grp = lane / lpr, sl = lane % lpr;
     unsigned long long best[MT];
 #pragma unroll
     for (int m = 0; m < MT; m++) best[m] = 0ull;
-    for (int base = blockIdx.x * cpb; base < N; base += gridDim.x * cpb) {
-        int acc[U][MT];
+    for (int r0 = warp * rpw; r0 < nr; r0 += 8 * rpw) {
+        const int row = r0 + grp;
+        int acc[MT];
 #pragma unroll
-        for (int u = 0; u < U; u++)
+        for (int m = 0; m < MT; m++) acc[m] = 0;
+        if (row < nr)
+            for (int cc = sl; cc < kc; cc += lpr) {
+                const int4 w = ws[(size_t)row * kc + cc];
 #pragma unroll
-            for (int m = 0; m < MT; m++) acc[u][m] = 0;
-        for (int c0 = 0; c0 < kc; c0 += lpc) {
-            const int c = c0 + sl;
-            int4 w[U];
-#pragma unroll
-            for (int u = 0; u < U; u++) {
-                int n = base + (u * 8 + warp) * gpw + grp;
-                w[u] = (n < N && c < kc) ? __ldg(reinterpret_cast<const int4 *>(W + (size_t)n * K) + c)
-                                         : make_int4(0, 0, 0, 0);
+                for (int m = 0; m < MT; m++) acc[m] = dot16(as[m * kc + cc], w, acc[m]);
             }
-            if (c < kc) {
 #pragma unroll
-                for (int m = 0; m < MT; m++) {
-                    int4 a = vsm[m * kc + c];
+        for (int m = 0; m < MT; m++)
+            for (int o = lpr / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
+        if (sl == 0 && row < nr) {
 #pragma unroll
-                    for (int u = 0; u < U; u++) acc[u][m] = dot16(a, w[u], acc[u][m]);
-                }
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < U; u++) {
-#pragma unroll
-            for (int m = 0; m < MT; m++)
-                for (int o = lpc / 2; o > 0; o >>= 1) acc[u][m] += __shfl_xor_sync(0xFFFFFFFFu, acc[u][m], o);
-            const int n = base + (u * 8 + warp) * gpw + grp;
-            if (sl == 0 && n < N) {
-#pragma unroll
-                for (int m = 0; m < MT; m++) {
-                    if (m < M) {
-                        unsigned long long k = pack_key(dequant_bias(acc[u][m], s_x, s_w[n], bias[n]), (uint32_t)n);
-                        best[m] = k > best[m] ? k : best[m];
-                    }
+            for (int m = 0; m < MT; m++) {
+                if (m < M) {
+                    const float y = __fadd_rn(__fmul_rn(__int2float_rn(acc[m]), scs[row]), bss[row]);
+                    const unsigned long long k = pack_key(y, (uint32_t)(n0 + row));
+                    best[m] = k > best[m] ? k : best[m];
                 }
             }
         }
@@ -770,6 +771,16 @@ cudaError_t decode_cluster_init() {
     setk((const void *)decode_cluster_kernel<32>);
     setk((const void *)decode_cluster_kernel<64>);
     setk((const void *)decode_cluster_kernel<128>);
+    // the vocabulary kernel keeps its SMs in the largest shared-memory
+    // configuration, so the next step's cluster (about 200 KB per CTA) can
+    // become resident beside it as soon as it is allowed to launch
+    for (const void *k : {(const void *)vocab_greedy_kernel<1>, (const void *)vocab_greedy_kernel<2>,
+                          (const void *)vocab_greedy_kernel<4>})
+        if (err == cudaSuccess)
+            err = cudaFuncSetAttribute(k, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    for (const void *k : {(const void *)vocab_greedy_kernel<1>, (const void *)vocab_greedy_kernel<2>,
+                          (const void *)vocab_greedy_kernel<4>})
+        if (err == cudaSuccess) err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, 100 * 1024);
     return err;
 }
 
@@ -824,15 +835,17 @@ cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
                                 cudaStream_t st) {
     const int kc = K / 16;
-    const int lpc = kc >= 32 ? 32 : kc;
-    const int cpb = 8 * (32 / lpc) * 4;
-    int blocks = (N + cpb - 1) / cpb;
-    if (blocks > 2 * 152) blocks = 2 * 152;
+    if (M < 1 || M > 4 || K % 16 || (kc & (kc - 1))) return cudaErrorInvalidValue;
+    // two blocks per SM, each holding its contiguous rows in shared memory
+    int blocks = 2 * 152;
+    int rows = (N + blocks - 1) / blocks;
+    if ((size_t)rows * K > 96 * 1024) rows = (96 * 1024) / K;
+    blocks = (N + rows - 1) / rows;
     const int mt = M == 1 ? 1 : (M == 2 ? 2 : 4);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(blocks);
     cfg.blockDim = dim3(256);
-    cfg.dynamicSmemBytes = (size_t)mt * kc * 16;
+    cfg.dynamicSmemBytes = (size_t)rows * K + (size_t)mt * K + 8 * (size_t)rows;
     cfg.stream = st;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -840,9 +853,9 @@ cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     switch (mt) {
-        case 1: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<1>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
-        case 2: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<2>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
-        default: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<4>, A, W, s_w, bias, s_x, M, N, K, keys, ticket, g);
+        case 1: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<1>, A, W, s_w, bias, s_x, M, N, K, rows, keys, ticket, g);
+        case 2: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<2>, A, W, s_w, bias, s_x, M, N, K, rows, keys, ticket, g);
+        default: return cudaLaunchKernelEx(&cfg, vocab_greedy_kernel<4>, A, W, s_w, bias, s_x, M, N, K, rows, keys, ticket, g);
     }
 }
 
