@@ -482,6 +482,7 @@ struct mnmt_session {
     int graph_B = -1, graph_S = -1;
     // cluster decode step (small greedy batches)
     DcParams *d_dc = nullptr;
+    float *dc_ln = nullptr;  // the cluster step's LayerNorm vectors, contiguous
     bool use_cluster = false;
     int dc_S = 0;  // host source of the parameter block's S when it is updated
     int dc_nc = 0;
@@ -531,7 +532,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
            o_anc = piece(R * max_len * 4), o_keys = piece(R * 8), o_cand = piece(R * beam * 8),
            o_logits = piece(beam > 1 ? R * V * 4 : 256), o_outids = piece((size_t)max_batch * max_len * 4),
            o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
-           o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams));
+           o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams)), o_dcln = piece((6 * L + 2) * d * 4);
     const size_t kmax = std::max(d, std::max(F, (size_t)c.d_embed));
     size_t o_a16 = piece(rows >= TC_MIN_ROWS ? rows * kmax * 2 : 256);
     s->arena_bytes = off;
@@ -572,6 +573,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
     s->out_scores = reinterpret_cast<float *>(a + o_outsc);
     s->state = reinterpret_cast<int *>(a + o_state);
     s->d_dc = reinterpret_cast<DcParams *>(a + o_dc);
+    s->dc_ln = reinterpret_cast<float *>(a + o_dcln);
     s->a16 = reinterpret_cast<__half *>(a + o_a16);
     {
         const char *v = std::getenv("MNMT_TC");
@@ -993,6 +995,23 @@ int setup_cluster_step(mnmt_session *s) {
         Y.inv_qkv = A.inv_qkv; Y.inv_q2 = X.inv_q; Y.inv_h = Fb.inv_h;
         Y.self_k = s->sk + l * s->sk_layer; Y.self_v = s->sv + l * s->sk_layer;
         Y.cross_k = s->ck + l * s->ck_layer; Y.cross_v = s->cv + l * s->ck_layer;
+    }
+    // the LayerNorm vectors in one contiguous array (one copy per step)
+    {
+        const size_t vb = (size_t)d * 4;
+        CK(cudaMemsetAsync(s->dc_ln, 0, (6 * c.n_dec + 2) * vb, m->stream));
+        for (int l = 0; l < c.n_dec; l++) {
+            const DcLayer &Y = P.layer[l];
+            const float *src[6] = {Y.ln1_g, Y.ln1_b, Y.ln2_g, Y.ln2_b, Y.ln3_g, Y.ln3_b};
+            for (int w = 0; w < 6; w++)
+                if (src[w])
+                    CK(cudaMemcpyAsync(s->dc_ln + (size_t)(6 * l + w) * d, src[w], vb, cudaMemcpyDeviceToDevice,
+                                       m->stream));
+        }
+        if (P.fin_g) CK(cudaMemcpyAsync(s->dc_ln + (size_t)6 * c.n_dec * d, P.fin_g, vb, cudaMemcpyDeviceToDevice, m->stream));
+        if (P.fin_b)
+            CK(cudaMemcpyAsync(s->dc_ln + (size_t)(6 * c.n_dec + 1) * d, P.fin_b, vb, cudaMemcpyDeviceToDevice, m->stream));
+        P.ln_all = s->dc_ln;
     }
     // lay shared memory out for the session's longest source, so that the
     // captured step serves every padded length (only P.S changes per batch)

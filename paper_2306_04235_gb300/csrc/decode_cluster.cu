@@ -353,25 +353,17 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     const int nphase = 1 + 6 * P.n_dec;
 
     // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
-    for (int v = 0; v < 6 * P.n_dec + 2; v++) {
-        const float *src;
-        if (v < 6 * P.n_dec) {
-            const DcLayer &Y = P.layer[v / 6];
-            const int w = v % 6;
-            src = w == 0 ? Y.ln1_g : w == 1 ? Y.ln1_b : w == 2 ? Y.ln2_g : w == 3 ? Y.ln2_b : w == 4 ? Y.ln3_g : Y.ln3_b;
-        } else {
-            src = v == 6 * P.n_dec ? P.fin_g : P.fin_b;
-        }
-        if (src) dc_copy(lnp + (size_t)v * d, src, d * 4);
-    }
+    dc_copy(lnp, P.ln_all, (6 * P.n_dec + 2) * d * 4);
     dc_prefetch(P, 0, c, ring);
     // group 1: the second weight slice and the keys / values the step attends to
     if (P.kv_staged) {
-        for (int l = 0; l < P.n_dec; l++) {
-            const DcLayer &Y = P.layer[l];
-            const int cb = R * P.S * d;  // one layer's cross K (or V): [R][H][S][dh]
-            dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 0) * cb, Y.cross_k, cb);
-            dc_copy(smem + P.off_kvc + (size_t)(l * 2 + 1) * cb, Y.cross_v, cb);
+        // one layer's cross K (or V) is one contiguous [R][H][S][dh] block: the
+        // 2 * n_dec blocks go in one flat loop of 16-byte chunks
+        const int cpb = R * P.S * d / 16;
+        for (int i = threadIdx.x; i < 2 * P.n_dec * cpb; i += DC_THREADS) {
+            const int blk = i / cpb, ch = i - blk * cpb;
+            const DcLayer &Y = P.layer[blk >> 1];
+            dc_cp16(smem + P.off_kvc + (size_t)i * 16, (blk & 1 ? Y.cross_v : Y.cross_k) + (size_t)ch * 16);
         }
     }
     // ---- the previous step's results: token, position, self keys / values ----
@@ -389,17 +381,17 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
         tok_s[threadIdx.x] = id;
     }
-    if (P.kv_staged) {
-        for (int l = 0; l < P.n_dec; l++) {
-            const DcLayer &Y = P.layer[l];
-            if (t > 0) {
-                const int seg = t * DH;  // positions 0..t-1 of one (row, head)
-                for (int x = 0; x < 2 * R * H; x++) {
-                    const int kv = x / (R * H), mh = x - kv * R * H;
-                    const size_t off = ((size_t)(l * 2 + kv) * R * H + mh) * P.T * DH;
-                    dc_copy(smem + P.off_kvs + off, (kv ? Y.self_v : Y.self_k) + (size_t)mh * P.T * DH, seg);
-                }
-            }
+    if (P.kv_staged && t > 0) {
+        // positions 0..t-1 of every (layer, K/V, row, head): segments of t * dh
+        // bytes, [T][dh] apart in the cache, in one flat loop of 16-byte chunks
+        const int cps = t * (d / H) / 16, nseg = 2 * P.n_dec * R * H;
+        for (int i = threadIdx.x; i < nseg * cps; i += DC_THREADS) {
+            const int sg = i / cps, ch = i - sg * cps;
+            const int lkv = sg / (R * H), mh = sg - lkv * R * H;
+            const DcLayer &Y = P.layer[lkv >> 1];
+            const size_t off = ((size_t)lkv * R * H + mh) * P.T * (d / H);
+            dc_cp16(smem + P.off_kvs + off + (size_t)ch * 16,
+                    (lkv & 1 ? Y.self_v : Y.self_k) + (size_t)mh * P.T * (d / H) + (size_t)ch * 16);
         }
     }
     dc_prefetch(P, 1, c, ring);

@@ -203,6 +203,7 @@ struct alignas(16) DcParams {
     float emb_scale;
     const float *pe;
     const float *fin_g, *fin_b;
+    const float *ln_all;  // every LayerNorm vector of the step, contiguous: [n_dec][6][d] then final [2][d]
     float s_dout;
     const int32_t *tok;
     const int *t_ptr, *done;
