@@ -227,13 +227,14 @@ __device__ __forceinline__ void epi_store16(const Epi &e, int row, int col0, con
 // index fastest, so the CTAs of one wave share weight tiles in L2).  The TMA
 // ring runs continuously across tiles; the accumulator is double-buffered in
 // TMEM so the epilogue of one tile overlaps the MMAs of the next.
-template <int BN, int NCH, int STAGES>
+template <int BN, int NCH, int STAGES, int NBUF>
 __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant__ CUtensorMap tmA,
                                                            const __grid_constant__ CUtensorMap tmB, int M, int N,
                                                            int K, Epi e, int *status) {
     using L = TcLayout<BN, STAGES>;
-    constexpr int ACC_COLS = NCH * BN;  // one accumulator buffer
-    constexpr int NCOLS = pow2_cols(2 * ACC_COLS);
+    constexpr int ACC_COLS = NCH * BN;  // one accumulator buffer (NBUF of them)
+    constexpr int NCOLS = pow2_cols(NBUF * ACC_COLS);
+    static_assert(NBUF * ACC_COLS <= 512, "TMEM holds 512 columns");
     constexpr uint32_t IDESC = idesc_f16(TC_BM, BN);
     if (e.skip && *e.skip) return;
 
@@ -300,8 +301,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
         // ---- MMA issuer ----
         uint32_t it = 0, lt = 0;
         for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x, lt++) {
-            const int buf = (int)(lt & 1);
-            if (lt >= 2 && !mbar_wait(acce_bar(buf), ((lt >> 1) - 1) & 1)) {
+            const int buf = (int)(lt % NBUF);
+            if (lt >= NBUF && !mbar_wait(acce_bar(buf), ((lt / NBUF) - 1) & 1)) {
                 *abort_flag = 1;
                 set_status(status, MNMT_ETIMEOUT);
                 break;
@@ -339,10 +340,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
         const bool vec = epi_vec_ok(e);
         uint32_t lt = 0;
         for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x, lt++) {
-            const int buf = (int)(lt & 1);
+            const int buf = (int)(lt % NBUF);
             const int m0 = (tile % mt) * TC_BM, n0 = (tile / mt) * BN;
             // per-column constants of this tile, double-buffered by tile parity
-            float *c_sc = cols + buf * 3 * BN, *c_b = c_sc + BN, *c_inv = c_b + BN;
+            float *c_sc = cols + (lt & 1) * 3 * BN, *c_b = c_sc + BN, *c_inv = c_b + BN;
             for (int i = ew * 32 + lane; i < BN; i += TC_EPI_WARPS * 32) {
                 const int n = n0 + i;
                 const bool ok = n < N;
@@ -353,7 +354,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
             epi_bar_sync();
             // every epilogue warp runs every tile of the loop (the named barrier
             // above needs all of them); after an abort the tiles are skipped
-            bool ok = *abort_flag == 0 && mbar_wait(accf_bar(buf), (lt >> 1) & 1);
+            bool ok = *abort_flag == 0 && mbar_wait(accf_bar(buf), (lt / NBUF) & 1);
             if (!ok && *abort_flag == 0) {
                 *abort_flag = 1;
                 set_status(status, MNMT_ETIMEOUT);
@@ -458,22 +459,26 @@ bool make_map(CUtensorMap *tm, const __half *p, int cols, int rows, int ld, int 
     return r == CUDA_SUCCESS;
 }
 
-template <int BN, int NCH, int STAGES>
+template <int BN, int NCH, int STAGES, int NBUF>
 cudaError_t tc_attr() {
-    return cudaFuncSetAttribute(linear_tc<BN, NCH, STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    return cudaFuncSetAttribute(linear_tc<BN, NCH, STAGES, NBUF>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 (int)TcLayout<BN, STAGES>::SMEM);
 }
 
-template <int BN, int NCH, int STAGES>
+template <int BN, int NCH, int STAGES, int NBUF>
 cudaError_t tc_launch(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, const Epi &e, int *status,
                       cudaStream_t st) {
     const long tiles = (long)((M + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
     const int grid = (int)(tiles < g_num_sms ? tiles : g_num_sms);
-    linear_tc<BN, NCH, STAGES><<<grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st>>>(ta, tb, M, N, K, e, status);
+    linear_tc<BN, NCH, STAGES, NBUF><<<grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st>>>(ta, tb, M, N, K, e, status);
     return cudaGetLastError();
 }
 
 constexpr int TC_STAGES = 6;
+// 128 x 256 tiles: half the A-tile bytes per FLOP, for grids with enough
+// tiles; with two K chunks the 512-column accumulator fills TMEM, so that
+// variant keeps one accumulator buffer (its epilogue does not overlap)
+constexpr int TC_STAGES_WIDE = 4;
 
 }  // namespace
 
@@ -487,8 +492,10 @@ cudaError_t linear_tc_init() {
     int dev = 0;
     if ((err = cudaGetDevice(&dev)) != cudaSuccess) return err;
     if ((err = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return err;
-    err = tc_attr<128, 1, TC_STAGES>();
-    if (err == cudaSuccess) err = tc_attr<128, 2, TC_STAGES>();
+    err = tc_attr<128, 1, TC_STAGES, 2>();
+    if (err == cudaSuccess) err = tc_attr<128, 2, TC_STAGES, 2>();
+    if (err == cudaSuccess) err = tc_attr<256, 1, TC_STAGES_WIDE, 2>();
+    if (err == cudaSuccess) err = tc_attr<256, 2, TC_STAGES_WIDE, 1>();
     return err;
 }
 
@@ -501,10 +508,16 @@ cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int 
                              const Epi &e, int *status, cudaStream_t st) {
     if (M <= 0 || N <= 0) return cudaSuccess;
     if (!linear_tc_shape_ok(M, N, K, lda, ldw, A16, W16)) return cudaErrorInvalidValue;
+    const bool two_chunks = K > TC_KB_PER_CHUNK * TC_BK;
+    const long tiles_wide = (long)((M + TC_BM - 1) / TC_BM) * ((N + 255) / 256);
+    const bool wide = N >= 256 && tiles_wide >= g_num_sms;
     CUtensorMap ta, tb;
-    if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, 128)) return cudaErrorInvalidValue;
-    if (K > TC_KB_PER_CHUNK * TC_BK) return tc_launch<128, 2, TC_STAGES>(ta, tb, M, N, K, e, status, st);
-    return tc_launch<128, 1, TC_STAGES>(ta, tb, M, N, K, e, status, st);
+    if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, wide ? 256 : 128))
+        return cudaErrorInvalidValue;
+    if (wide && two_chunks) return tc_launch<256, 2, TC_STAGES_WIDE, 1>(ta, tb, M, N, K, e, status, st);
+    if (wide) return tc_launch<256, 1, TC_STAGES_WIDE, 2>(ta, tb, M, N, K, e, status, st);
+    if (two_chunks) return tc_launch<128, 2, TC_STAGES, 2>(ta, tb, M, N, K, e, status, st);
+    return tc_launch<128, 1, TC_STAGES, 2>(ta, tb, M, N, K, e, status, st);
 }
 
 cudaError_t launch_codes_to_f16(const int8_t *src, int ld_src, __half *dst, int ld_dst, int rows, int cols,

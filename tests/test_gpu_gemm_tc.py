@@ -156,3 +156,17 @@ def test_linear_tc_rejects_bad_shapes():
             mnmt.mnmt_linear_tc(A16, W16, s, s, 1.0, s, 1.0, 256, 64, K, mnmt.EPI_F32, None, out)
     with pytest.raises(mnmt.MnmtError):
         mnmt.mnmt_linear_tc(A16, W16, s, s, 1.0, s, 1.0, 256, 64, 24, mnmt.EPI_Q8, None, out)
+
+
+@pytest.mark.parametrize("M,N,K", [(4864, 1024, 1040), (4864, 1000, 520), (19456, 512, 2048)])
+@pytest.mark.parametrize("mode", [mnmt.EPI_Q8, mnmt.EPI_RESID])
+def test_linear_tc_wide_tiles_sampled(M, N, K, mode):
+    """Grids large enough for the 128 x 256 tiles (with one and with two exact
+    K chunks, ragged N and K), checked on sampled rows."""
+    A, W, s_w, b, inv, s_x = _inputs(M + N + K + 3, M, N, K)
+    resid = synth.uniform_f32(9, "r", (M, N), -3, 3) if mode == mnmt.EPI_RESID else None
+    got = _tc(A, W, s_w, b, inv, s_x, mode, 0.875, resid)
+    rows = sorted({0, 127, 128, 129, 255, 256, M // 3, M - 129, M - 1})
+    ref = O.linear(A[rows], W, s_w, b, s_x, mode, inv_out=inv, gamma=np.float32(0.875),
+                   resid=None if resid is None else resid[rows])
+    assert _same(got[rows], ref)
