@@ -62,6 +62,7 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
     for (int c = 0; c < QC; c++) qv[c] = qp[c];
 
     float mx = -INFINITY;
+#pragma unroll 4
     for (int j = lane; j < n; j += 32) {
         const int4 *kr = reinterpret_cast<const int4 *>(a.kc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH);
         int acc = 0;
@@ -85,30 +86,35 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
     int hi[EPL], lo[EPL];
 #pragma unroll
     for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
-    for (int j = 0; j < n; j++) {
-        int E = sc[j];
-        int Eh = E >> 12, El = E & 4095;
+    // the lane's EPL value bytes of key j (little-endian in the low bytes)
+    auto vload = [&](int j) -> uint32_t {
         const int8_t *vr = a.vc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH + lane * EPL;
-        int v[EPL];
-        if constexpr (EPL == 1) {
-            v[0] = vr[0];
-        } else if constexpr (EPL == 2) {
-            char2 x = *reinterpret_cast<const char2 *>(vr);
-            v[0] = x.x;
-            v[1] = x.y;
-        } else {
-            char4 x = *reinterpret_cast<const char4 *>(vr);
-            v[0] = x.x;
-            v[1] = x.y;
-            v[2] = x.z;
-            v[3] = x.w;
-        }
+        if constexpr (EPL == 1) return (uint32_t)(uint8_t)vr[0];
+        else if constexpr (EPL == 2) return (uint32_t)*reinterpret_cast<const uint16_t *>(vr);
+        else return *reinterpret_cast<const uint32_t *>(vr);
+    };
+    auto vacc = [&](int j, uint32_t raw) {
+        const int E = sc[j];
+        const int Eh = E >> 12, El = E & 4095;
 #pragma unroll
         for (int u = 0; u < EPL; u++) {
-            hi[u] += Eh * v[u];
-            lo[u] += El * v[u];
+            const int v = (int)(int8_t)(raw >> (8 * u));
+            hi[u] += Eh * v;
+            lo[u] += El * v;
         }
+    };
+    // keys in groups of 8: the 8 value loads are issued before any is used,
+    // so their latencies overlap
+    constexpr int UJ = 8;
+    int j = 0;
+    for (; j + UJ <= n; j += UJ) {
+        uint32_t raw[UJ];
+#pragma unroll
+        for (int u = 0; u < UJ; u++) raw[u] = vload(j + u);
+#pragma unroll
+        for (int u = 0; u < UJ; u++) vacc(j + u, raw[u]);
     }
+    for (; j < n; j++) vacc(j, vload(j));
     int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + lane * EPL;
 #pragma unroll
     for (int u = 0; u < EPL; u++) {
