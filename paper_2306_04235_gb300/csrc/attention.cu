@@ -18,12 +18,19 @@
 //   attn_encoder one block per (sentence, head, chunk of 4..32 queries): K and V of
 //                the head staged in shared memory, keys masked past the
 //                source length.
+#include <type_traits>
+
 #include "common.cuh"
 #include "internal.h"
 
 namespace mnmt {
 
 constexpr int DEC_MAX_KEYS = 1024;
+
+// 32-bit word k of a 4-, 8- or 16-byte vector held in registers
+MNMT_DEV uint32_t vec_word(uint32_t v, int) { return v; }
+MNMT_DEV uint32_t vec_word(const uint2 &v, int k) { return k ? v.y : v.x; }
+MNMT_DEV uint32_t vec_word(const uint4 &v, int k) { return k == 0 ? v.x : k == 1 ? v.y : k == 2 ? v.z : v.w; }
 
 template <int DH>
 __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
@@ -82,44 +89,59 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
     Z = warp_sum_ll(Z);
     __syncwarp();
 
-    constexpr int EPL = DH / 32;  // context elements per lane
-    int hi[EPL], lo[EPL];
+    // context: the warp takes CG keys at a time, one per group of 8 lanes;
+    // lane gl of a group holds EPG consecutive elements of the head, read as
+    // one EPG-byte load per key.  N_e = sum_j E_j v_j[e] is split into 12-bit
+    // halves of E_j so that every partial stays an exact int32.
+    constexpr int CG = 4, LPG = 32 / CG, EPG = DH / LPG;
+    using VecT = typename std::conditional<EPG == 4, uint32_t, typename std::conditional<EPG == 8, uint2, uint4>::type>::type;
+    const int grp = lane / LPG, gl = lane % LPG;
+    int hi[EPG], lo[EPG];
 #pragma unroll
-    for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
-    // the lane's EPL value bytes of key j (little-endian in the low bytes)
-    auto vload = [&](int j) -> uint32_t {
-        const int8_t *vr = a.vc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH + lane * EPL;
-        if constexpr (EPL == 1) return (uint32_t)(uint8_t)vr[0];
-        else if constexpr (EPL == 2) return (uint32_t)*reinterpret_cast<const uint16_t *>(vr);
-        else return *reinterpret_cast<const uint32_t *>(vr);
+    for (int u = 0; u < EPG; u++) hi[u] = lo[u] = 0;
+    auto vload = [&](int j) -> VecT {
+        return *reinterpret_cast<const VecT *>(a.vc + (((size_t)prow[j] * a.H + h) * a.T + j) * DH + gl * EPG);
     };
-    auto vacc = [&](int j, uint32_t raw) {
+    auto vacc = [&](int j, const VecT &raw) {
         const int E = sc[j];
         const int Eh = E >> 12, El = E & 4095;
 #pragma unroll
-        for (int u = 0; u < EPL; u++) {
-            const int v = (int)(int8_t)(raw >> (8 * u));
+        for (int u = 0; u < EPG; u++) {
+            const int v = (int)(int8_t)(vec_word(raw, u >> 2) >> (8 * (u & 3)));
             hi[u] += Eh * v;
             lo[u] += El * v;
         }
     };
-    // keys in groups of 8: the 8 value loads are issued before any is used,
-    // so their latencies overlap
-    constexpr int UJ = 8;
-    int j = 0;
-    for (; j + UJ <= n; j += UJ) {
-        uint32_t raw[UJ];
+    // groups of UJ rounds: every value load of the batch is issued before any
+    // is used, so their latencies overlap
+    constexpr int UJ = DH == 128 ? 2 : 4;
+    int j0 = 0;
+    for (; j0 + CG * UJ <= n; j0 += CG * UJ) {
+        VecT raw[UJ];
 #pragma unroll
-        for (int u = 0; u < UJ; u++) raw[u] = vload(j + u);
+        for (int u = 0; u < UJ; u++) raw[u] = vload(j0 + u * CG + grp);
 #pragma unroll
-        for (int u = 0; u < UJ; u++) vacc(j + u, raw[u]);
+        for (int u = 0; u < UJ; u++) vacc(j0 + u * CG + grp, raw[u]);
     }
-    for (; j < n; j++) vacc(j, vload(j));
-    int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + lane * EPL;
+    for (int j = j0 + grp; j < n; j += CG) vacc(j, vload(j));
+    // sum over the CG groups (lanes gl, gl+8, gl+16, gl+24): every lane gets the totals
 #pragma unroll
-    for (int u = 0; u < EPL; u++) {
-        long long N = (long long)hi[u] * 4096 + lo[u];
-        out[u] = q8(rn32_div(N, Z), a.rho);
+    for (int u = 0; u < EPG; u++) {
+#pragma unroll
+        for (int o = LPG; o < 32; o <<= 1) {
+            hi[u] += __shfl_xor_sync(0xFFFFFFFFu, hi[u], o);
+            lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
+        }
+    }
+    // lane (grp, gl) writes elements gl * EPG + grp * EPG / CG + [0, EPG / CG)
+    constexpr int OPL = EPG / CG;
+    int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + gl * EPG + grp * OPL;
+#pragma unroll
+    for (int u = 0; u < EPG; u++) {
+        if (u / OPL == grp) {
+            long long N = (long long)hi[u] * 4096 + lo[u];
+            out[u - grp * OPL] = q8(rn32_div(N, Z), a.rho);
+        }
     }
 }
 
