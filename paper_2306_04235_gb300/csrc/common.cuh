@@ -36,6 +36,10 @@ MNMT_DEV float dequant_bias(int32_t acc, float s_x, float s_w, float b) {
 MNMT_DEV long long fx_scale(float v, int shift) {
     uint32_t bits = __float_as_uint(v);
     uint32_t ex = (bits >> 23) & 0xFFu;
+    // fast path: v normal and v 2^shift a normal float below 2^62 -- the
+    // scaling is then exact and the conversion rounds half to even
+    if (ex != 0 && (int)ex + shift >= 1 && (int)ex + shift <= 127 + 61)
+        return __float2ll_rn(__uint_as_float(bits + ((uint32_t)shift << 23)));
     uint32_t man = bits & 0x7FFFFFu;
     int e;
     if (ex == 0) {
@@ -183,6 +187,14 @@ MNMT_DEV int dot16(int4 a, int4 b, int acc) {
 // nearest float (ties to even) to S * 2^e, subnormals included
 MNMT_DEV float rn32_pow2(long long S, int e) {
     if (S == 0) return 0.0f;
+    {
+        // fast path: the integer rounds to float once (half to even); scaling
+        // by 2^e is exact while the result stays a normal float
+        const float f = __ll2float_rn(S);
+        const uint32_t fb = __float_as_uint(f);
+        const int fe = (int)((fb >> 23) & 0xFFu) + e;
+        if (fe >= 1 && fe <= 254) return __uint_as_float(fb + ((uint32_t)e << 23));
+    }
     const unsigned long long a = S < 0 ? 0ull - (unsigned long long)S : (unsigned long long)S;
     const int nb = 64 - __clzll(a);  // significant bits of a
     const int E = nb - 1 + e;        // floor(log2 |value|)

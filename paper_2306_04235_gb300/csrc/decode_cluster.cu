@@ -109,7 +109,9 @@ __device__ __noinline__ void dc_bcast(cg::cluster_group &cl, const uint8_t *stag
 // barrier.
 MNMT_DEV long long dc_row_sum(const long long *part, int row, int spr) {
     long long s = 0;
-    for (int k = 0; k < spr; k++) s += part[row * spr + k];
+#pragma unroll
+    for (int k = 0; k < 16; k++)  // spr = d / 32 <= 16: every load issued at once
+        if (k < spr) s += part[row * spr + k];
     return s;
 }
 
