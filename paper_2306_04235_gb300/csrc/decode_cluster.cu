@@ -51,7 +51,17 @@ MNMT_DEV void dc_launch_dependents() { asm volatile("griddepcontrol.launch_depen
 
 // out-of-line copies of the exact roundings (one copy of the code each)
 __device__ __noinline__ float dc_rn32_div(long long n, long long z) { return rn32_div(n, z); }
-__device__ __noinline__ float dc_rn32_pow2(long long s, int e) { return rn32_pow2(s, e); }
+__device__ __noinline__ float dc_rn32_pow2_full(long long s, int e) { return rn32_pow2(s, e); }
+// the common case inline (one conversion, exact while the result is a normal
+// float), the rest out of line
+MNMT_DEV float dc_rn32_pow2(long long s, int e) {
+    if (s != 0) {
+        const uint32_t fb = __float_as_uint(__ll2float_rn(s));
+        const int fe = (int)((fb >> 23) & 0xFFu) + e;
+        if (fe >= 1 && fe <= 254) return __uint_as_float(fb + ((uint32_t)e << 23));
+    }
+    return dc_rn32_pow2_full(s, e);
+}
 
 // signed bytes of a 32-bit word
 MNMT_DEV int sb0(int x) { return (x << 24) >> 24; }
