@@ -140,7 +140,7 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
     for (int u = 0; u < EPG; u++) {
         if (u / OPL == grp) {
             long long N = (long long)hi[u] * 4096 + lo[u];
-            out[u - grp * OPL] = q8(rn32_div(N, Z), a.rho);
+            out[u - grp * OPL] = q8_quotient(N, Z, a.rho, rn32_div);
         }
     }
 }
@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, in
 #pragma unroll
         for (int u = 0; u < EPL; u++) {
             long long N = (long long)hi[u] * 4096 + lo[u];
-            out[u] = q8(rn32_div(N, Z), a.rho);
+            out[u] = q8_quotient(N, Z, a.rho, rn32_div);
         }
         __syncwarp();
     }

@@ -269,6 +269,25 @@ MNMT_DEV float rn32_div(long long n, long long z) {
     return n < 0 ? -q : q;
 }
 
+// q8(nearest float to n / z, rho): the quantised attention context of Eq. 2.
+// The approximate quotient fl(fl(n) / fl(z)) is within 2^-22 (relative) of
+// the exact rounded one -- three roundings of 2^-24 each, plus the exact
+// quotient's own -- which is at most 4 ulp, 8 across a binade boundary;
+// fl(x * rho), the rounding and the clamp are monotone in x, so when both ends
+// of the +-8-ulp bracket give the same code, so does the exact quotient.  Only
+// a bracket that straddles a rounding boundary needs the exact quotient.
+template <typename ExactDiv>
+MNMT_DEV int8_t q8_quotient(long long n, long long z, float rho, ExactDiv exact) {
+    if (n == 0) return q8(0.0f, rho);
+    const unsigned long long a = n < 0 ? 0ull - (unsigned long long)n : (unsigned long long)n;
+    const uint32_t qb = __float_as_uint(__fdiv_rn(__ull2float_rn(a), __ll2float_rn(z)));
+    const float sgn = n < 0 ? -1.0f : 1.0f;
+    const int8_t lo = q8(__fmul_rn(sgn, __uint_as_float(qb - 8u)), rho);
+    const int8_t hi = q8(__fmul_rn(sgn, __uint_as_float(qb + 8u)), rho);
+    if (lo == hi) return lo;
+    return q8(exact(n, z), rho);
+}
+
 // ---------------------------------------------------------------------------
 // LayerNorm (App. A / App. D) of one row by one warp.  Mean and biased
 // variance are exact fixed-point sums: the row's largest magnitude (an

@@ -312,7 +312,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                     Z += pz[ii * wpi + w];
                 }
                 const int m2 = it2 / H, h2 = it2 - m2 * H;
-                ctx[(size_t)m2 * P.d + h2 * DH + e] = q8(dc_rn32_div(N, Z), rho);
+                ctx[(size_t)m2 * P.d + h2 * DH + e] = q8_quotient(N, Z, rho, dc_rn32_div);
             }
         }
         __syncthreads();

@@ -169,3 +169,22 @@ def test_layernorm_constant_row_and_overflow_status():
     mnmt.mnmt_layernorm(dev(r), dev(g), dev(b), 2, d, 1.0, of, None, status)
     assert np.array_equal(host(of)[0], b)
     assert host(status)[0] == mnmt.EOVERFLOW
+
+
+@pytest.mark.parametrize("rho", [0.5, 1.0, 0.25])
+def test_attention_context_on_rounding_ties(rho):
+    """Equal scores make the context an exact mean of the values; with these
+    rho the scaled context lands exactly on (or next to) .5 rounding ties, so
+    the kernel's approximate-quotient shortcut must defer to the exact
+    quotient.  Both must agree with the oracle."""
+    R, H, dh, T = 6, 4, 64, 8
+    q = np.zeros((R, H, dh), np.int8)                         # all scores 0 -> equal weights
+    Kc = synth.uniform_int8(31, "k", (R, H, T, dh))
+    Vc = synth.uniform_int8(31, "v", (R, H, T, dh), -9, 9)
+    Vc[:, :, 1::2] = Vc[:, :, 0::2] + 1                        # pair sums odd: means at .5 / .25 steps
+    n_keys = np.array([2, 4, 8, 6, 1, 3], np.int32)
+    sigma = np.float32(1e-3)
+    ctx = torch.zeros((R, H, dh), dtype=torch.int8, device="cuda")
+    mnmt.mnmt_attention_decode(dev(q), dev(Kc), dev(Vc), dev(n_keys), R, H, dh, T, sigma, np.float32(rho), ctx)
+    ref = O.attention_decode(q, Kc, Vc, n_keys, sigma, np.float32(rho))
+    assert np.array_equal(host(ctx), ref)
