@@ -34,6 +34,8 @@ MNMT_DEV uint32_t vec_word(const uint4 &v, int k) { return k == 0 ? v.x : k == 1
 
 template <int DH>
 __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (a.skip && *a.skip) return;
     extern __shared__ int dsm[];
     const int r = blockIdx.x;
@@ -151,13 +153,13 @@ cudaError_t launch_attention_decode(const AttnDecArgs &a, cudaStream_t st) {
     dim3 block(32 * a.H);
     switch (a.dh) {
         case 32:
-            attn_decode<32><<<a.R, block, smem, st>>>(a);
+            launch_pdl(attn_decode<32>, a.R, block, smem, st, a);
             break;
         case 64:
-            attn_decode<64><<<a.R, block, smem, st>>>(a);
+            launch_pdl(attn_decode<64>, a.R, block, smem, st, a);
             break;
         case 128:
-            attn_decode<128><<<a.R, block, smem, st>>>(a);
+            launch_pdl(attn_decode<128>, a.R, block, smem, st, a);
             break;
         default:
             return cudaErrorInvalidValue;
@@ -174,6 +176,8 @@ constexpr int ENC_QCHUNK = 32;
 
 template <int DH>
 __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, int qchunk) {
+    pdl_allow_next();
+    pdl_grid_wait();
     extern __shared__ __align__(16) uint8_t esm[];
     constexpr int KS = DH + 16;  // padded key row: conflict-free 16-byte lane reads
     const int bh = blockIdx.x;
@@ -258,7 +262,7 @@ static cudaError_t launch_enc(const AttnEncArgs &a, cudaStream_t st) {
     int qc = ENC_QCHUNK;
     while (qc > ENC_WARPS && (long)a.B * a.H * ((a.S + qc - 1) / qc) < 2 * 152) qc >>= 1;
     dim3 grid(a.B * a.H, (a.S + qc - 1) / qc);
-    k<<<grid, 32 * ENC_WARPS, smem, st>>>(a, qc);
+    launch_pdl(k, grid, 32 * ENC_WARPS, smem, st, a, qc);
     return cudaGetLastError();
 }
 

@@ -15,6 +15,16 @@
 #define MNMT_DEV __device__ __forceinline__
 
 // ---------------------------------------------------------------------------
+// programmatic dependent launch: every kernel of the library is launched
+// allowed to start before its predecessor in the stream has finished; it lets
+// its own successor launch at once, then waits for the predecessor (and the
+// memory it wrote) before it reads anything.  Every kernel waits, so waiting
+// for the predecessor also covers everything before it.
+// ---------------------------------------------------------------------------
+MNMT_DEV void pdl_allow_next() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+MNMT_DEV void pdl_grid_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+
+// ---------------------------------------------------------------------------
 // quantiser: q8(x, inv) = clamp(round_half_even(fl(x * inv)), -127, 127)
 // ---------------------------------------------------------------------------
 MNMT_DEV int8_t q8(float x, float inv) {

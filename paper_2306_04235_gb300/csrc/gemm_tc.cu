@@ -231,6 +231,8 @@ template <int BN, int NCH, int STAGES, int NBUF>
 __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant__ CUtensorMap tmA,
                                                            const __grid_constant__ CUtensorMap tmB, int M, int N,
                                                            int K, Epi e, int *status) {
+    pdl_allow_next();
+    pdl_grid_wait();
     using L = TcLayout<BN, STAGES>;
     constexpr int ACC_COLS = NCH * BN;  // one accumulator buffer (NBUF of them)
     constexpr int NCOLS = pow2_cols(NBUF * ACC_COLS);
@@ -422,6 +424,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
 // ---------------------------------------------------------------------------
 __global__ void codes_to_f16_kernel(const int8_t *__restrict__ src, int ld_src, __half *__restrict__ dst, int ld_dst,
                                     int rows, int cols) {
+    pdl_allow_next();
+    pdl_grid_wait();
     const int per_row = cols >> 4;
     const long total = (long)rows * per_row;
     for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < total; i += (long)gridDim.x * blockDim.x) {
@@ -438,6 +442,8 @@ __global__ void codes_to_f16_kernel(const int8_t *__restrict__ src, int ld_src, 
 }
 
 __global__ void codes_to_f16_tail(const int8_t *src, __half *dst, size_t from, size_t n) {
+    pdl_allow_next();
+    pdl_grid_wait();
     size_t i = from + blockIdx.x * (size_t)blockDim.x + threadIdx.x;
     if (i < n) dst[i] = __short2half_rn((short)src[i]);
 }
@@ -470,7 +476,7 @@ cudaError_t tc_launch(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N
                       cudaStream_t st) {
     const long tiles = (long)((M + TC_BM - 1) / TC_BM) * ((N + BN - 1) / BN);
     const int grid = (int)(tiles < g_num_sms ? tiles : g_num_sms);
-    linear_tc<BN, NCH, STAGES, NBUF><<<grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st>>>(ta, tb, M, N, K, e, status);
+    launch_pdl(linear_tc<BN, NCH, STAGES, NBUF>, grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st, ta, tb, M, N, K, e, status);
     return cudaGetLastError();
 }
 
@@ -529,7 +535,7 @@ cudaError_t launch_codes_to_f16(const int8_t *src, int ld_src, __half *dst, int 
     const long units = (long)rows * (cols / 16);
     long blocks = (units + 255) / 256;
     if (blocks > 152 * 8) blocks = 152 * 8;
-    codes_to_f16_kernel<<<(int)blocks, 256, 0, st>>>(src, ld_src, dst, ld_dst, rows, cols);
+    launch_pdl(codes_to_f16_kernel, (int)blocks, 256, 0, st, src, ld_src, dst, ld_dst, rows, cols);
     return cudaGetLastError();
 }
 
@@ -547,7 +553,7 @@ cudaError_t launch_codes_to_f16_flat(const int8_t *src, __half *dst, size_t n, c
         err = launch_codes_to_f16(src + done, (int)(body - done), dst + done, (int)(body - done), 1,
                                   (int)(body - done), st);
     if (err == cudaSuccess && n > body) {
-        codes_to_f16_tail<<<1, 32, 0, st>>>(src, dst, body, n);
+        launch_pdl(codes_to_f16_tail, 1, 32, 0, st, src, dst, body, n);
         err = cudaGetLastError();
     }
     return err;

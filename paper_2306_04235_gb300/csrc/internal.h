@@ -10,6 +10,29 @@
 
 namespace mnmt {
 
+// Launch with programmatic stream serialisation (see pdl_grid_wait in
+// common.cuh): the kernel may start while its predecessor finishes.  Inside a
+// stream capture the launch is a plain one: a graph already launches its
+// kernel nodes back to back, and the measured decode-step graphs ran slower
+// with programmatic edges between the multi-kernel step's nodes.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) cs = cudaStreamCaptureStatusNone;
+    cfg.attrs = attr;
+    cfg.numAttrs = cs == cudaStreamCaptureStatusActive ? 0 : 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // Epilogue of a quantised linear (Sec. 3.3, Fig. 5).  y = fl(fl(acc *
 // fl(s_x * s_w[n])) + bias[n]) then, per mode:
 enum EpiMode {

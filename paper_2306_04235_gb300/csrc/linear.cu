@@ -35,6 +35,8 @@ template <int MT, int LPC, int U>
 __global__ void __launch_bounds__(SM_THREADS) linear_smallm(const int8_t *__restrict__ A, int lda,
                                                            const int8_t *__restrict__ W, int M, int N,
                                                            int K, Epi e) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (e.skip && *e.skip) return;
     extern __shared__ int4 smA[];  // [MT][K/16]
     const int kc = K >> 4;
@@ -174,6 +176,8 @@ __global__ void __launch_bounds__(WARPS_M *WARPS_N * 32)
     constexpr int WTM = BM / WARPS_M, WTN = BN / WARPS_N;
     constexpr int MI = WTM / 16, NI = WTN / 8;
     static_assert(NI % 2 == 0, "B fragments are loaded two n8 tiles at a time");
+    pdl_allow_next();
+    pdl_grid_wait();
     if (e.skip && *e.skip) return;
     extern __shared__ __align__(128) uint8_t smem[];
     uint8_t *sA = smem;
@@ -356,11 +360,11 @@ static cudaError_t launch_small(const int8_t *A, int lda, const int8_t *W, int M
     if (smem > 48 * 1024) return cudaErrorInvalidValue;  // K <= 3072 at M <= 16
     const dim3 grid(blocks, chunks);
     if (lpc == 32) {
-        linear_smallm<MT, 32, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        launch_pdl(linear_smallm<MT, 32, U>, grid, SM_THREADS, smem, st, A, lda, W, M, N, K, e);
     } else if (lpc == 16) {
-        linear_smallm<MT, 16, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        launch_pdl(linear_smallm<MT, 16, U>, grid, SM_THREADS, smem, st, A, lda, W, M, N, K, e);
     } else {
-        linear_smallm<MT, 8, U><<<grid, SM_THREADS, smem, st>>>(A, lda, W, M, N, K, e);
+        launch_pdl(linear_smallm<MT, 8, U>, grid, SM_THREADS, smem, st, A, lda, W, M, N, K, e);
     }
     return cudaGetLastError();
 }
@@ -371,7 +375,7 @@ static cudaError_t launch_mma(const int8_t *A, int lda, const int8_t *W, int M, 
     auto k = linear_mma<BM, BN, WM, WN, STAGES>;
     size_t smem = (size_t)STAGES * (BM + BN) * 64;
     dim3 grid((N + BN - 1) / BN, (M + BM - 1) / BM);
-    k<<<grid, WM * WN * 32, smem, st>>>(A, lda, W, M, N, K, e);
+    launch_pdl(k, grid, WM * WN * 32, smem, st, A, lda, W, M, N, K, e);
     return cudaGetLastError();
 }
 

@@ -18,6 +18,8 @@ namespace mnmt {
 // ---------------------------------------------------------------------------
 template <int VPL>
 __global__ void __launch_bounds__(256) layernorm_kernel(LnArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (a.skip && *a.skip) return;
     const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -47,11 +49,11 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
     if (a.M <= 0) return cudaSuccess;
     dim3 grid((a.M + 7) / 8), block(256);
     int vpl = (a.d + 31) / 32;
-    if (vpl <= 4) layernorm_kernel<4><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 8) layernorm_kernel<8><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 16) layernorm_kernel<16><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 32) layernorm_kernel<32><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 64) layernorm_kernel<64><<<grid, block, 0, st>>>(a);
+    if (vpl <= 4) launch_pdl(layernorm_kernel<4>, grid, block, 0, st, a);
+    else if (vpl <= 8) launch_pdl(layernorm_kernel<8>, grid, block, 0, st, a);
+    else if (vpl <= 16) launch_pdl(layernorm_kernel<16>, grid, block, 0, st, a);
+    else if (vpl <= 32) launch_pdl(layernorm_kernel<32>, grid, block, 0, st, a);
+    else if (vpl <= 64) launch_pdl(layernorm_kernel<64>, grid, block, 0, st, a);
     else return cudaErrorInvalidValue;
     return cudaGetLastError();
 }
@@ -64,6 +66,8 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
 // ---------------------------------------------------------------------------
 template <int VPL>
 __global__ void __launch_bounds__(256) embed_kernel(EmbedArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (a.skip && *a.skip) return;
     const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -126,11 +130,11 @@ cudaError_t launch_embed(const EmbedArgs &a, cudaStream_t st) {
     if (a.M <= 0) return cudaSuccess;
     dim3 grid((a.M + 7) / 8), block(256);
     int vpl = (a.d + 31) / 32;
-    if (vpl <= 4) embed_kernel<4><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 8) embed_kernel<8><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 16) embed_kernel<16><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 32) embed_kernel<32><<<grid, block, 0, st>>>(a);
-    else if (vpl <= 64) embed_kernel<64><<<grid, block, 0, st>>>(a);
+    if (vpl <= 4) launch_pdl(embed_kernel<4>, grid, block, 0, st, a);
+    else if (vpl <= 8) launch_pdl(embed_kernel<8>, grid, block, 0, st, a);
+    else if (vpl <= 16) launch_pdl(embed_kernel<16>, grid, block, 0, st, a);
+    else if (vpl <= 32) launch_pdl(embed_kernel<32>, grid, block, 0, st, a);
+    else if (vpl <= 64) launch_pdl(embed_kernel<64>, grid, block, 0, st, a);
     else return cudaErrorInvalidValue;
     return cudaGetLastError();
 }
@@ -139,6 +143,8 @@ cudaError_t launch_embed(const EmbedArgs &a, cudaStream_t st) {
 // search state
 // ---------------------------------------------------------------------------
 __global__ void search_init_kernel(InitArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < a.R) {
         a.tok[i] = a.bos;
@@ -164,12 +170,14 @@ cudaError_t launch_search_init(const InitArgs &a, cudaStream_t st) {
     int blocks = (n + 255) / 256;
     if (blocks < 1) blocks = 1;
     if (blocks > 1024) blocks = 1024;
-    search_init_kernel<<<blocks, 256, 0, st>>>(a);
+    launch_pdl(search_init_kernel, blocks, 256, 0, st, a);
     return cudaGetLastError();
 }
 
 // greedy: argmax key -> token; after EOS a sentence emits PAD
 __global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (*a.done) return;
     const int t = *a.t_ptr;
     int fin_all = 1;
@@ -194,7 +202,7 @@ __global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
 
 cudaError_t launch_greedy_update(const GreedyArgs &a, cudaStream_t st) {
     int threads = a.R < 1024 ? ((a.R + 31) / 32) * 32 : 1024;
-    greedy_update_kernel<<<1, threads, 0, st>>>(a);
+    launch_pdl(greedy_update_kernel, 1, threads, 0, st, a);
     return cudaGetLastError();
 }
 
@@ -220,6 +228,8 @@ MNMT_DEV void topk_insert(unsigned long long (&lst)[KM], int k, unsigned long lo
 
 template <int KM>
 __global__ void __launch_bounds__(BR_THREADS) beam_rows_kernel(BeamArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (*a.done) return;
     const int r = blockIdx.x;
     const int k = a.k;
@@ -293,6 +303,8 @@ __global__ void __launch_bounds__(BR_THREADS) beam_rows_kernel(BeamArgs a) {
 
 // per sentence: best k of the k*k row candidates; reorder state
 __global__ void __launch_bounds__(256) beam_select_kernel(BeamArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     if (*a.done) return;
     const int b = blockIdx.x;
     const int k = a.k, V = a.V, T = a.T;
@@ -374,13 +386,13 @@ __global__ void __launch_bounds__(256) beam_select_kernel(BeamArgs a) {
 cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
     if (a.k < 1 || a.k > BEAM_MAX) return cudaErrorInvalidValue;
     int R = a.B * a.k;
-    if (a.k <= 4) beam_rows_kernel<4><<<R, BR_THREADS, 0, st>>>(a);
-    else if (a.k <= 8) beam_rows_kernel<8><<<R, BR_THREADS, 0, st>>>(a);
-    else beam_rows_kernel<16><<<R, BR_THREADS, 0, st>>>(a);
+    if (a.k <= 4) launch_pdl(beam_rows_kernel<4>, R, BR_THREADS, 0, st, a);
+    else if (a.k <= 8) launch_pdl(beam_rows_kernel<8>, R, BR_THREADS, 0, st, a);
+    else launch_pdl(beam_rows_kernel<16>, R, BR_THREADS, 0, st, a);
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     size_t smem = (size_t)a.k * a.T * sizeof(int);
-    beam_select_kernel<<<a.B, 256, smem, st>>>(a);
+    launch_pdl(beam_select_kernel, a.B, 256, smem, st, a);
     return cudaGetLastError();
 }
 
@@ -389,6 +401,8 @@ cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
 // backtracked through the parent pointers
 // ---------------------------------------------------------------------------
 __global__ void finalize_kernel(FinalArgs a) {
+    pdl_allow_next();
+    pdl_grid_wait();
     const int b = blockIdx.x;
     if (threadIdx.x != 0) return;
     const int steps = *a.t_ptr;
@@ -418,7 +432,7 @@ cudaError_t rows_init() {
 }
 
 cudaError_t launch_finalize(const FinalArgs &a, cudaStream_t st) {
-    finalize_kernel<<<a.B, 32, 0, st>>>(a);
+    launch_pdl(finalize_kernel, a.B, 32, 0, st, a);
     return cudaGetLastError();
 }
 
