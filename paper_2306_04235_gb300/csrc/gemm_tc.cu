@@ -485,6 +485,9 @@ constexpr int TC_STAGES = 6;
 // tiles; with two K chunks the 512-column accumulator fills TMEM, so that
 // variant keeps one accumulator buffer (its epilogue does not overlap)
 constexpr int TC_STAGES_WIDE = 4;
+// 128 x 64 tiles for grids that would leave SMs idle (a few hundred rows):
+// twice the CTAs, and each streams a third fewer bytes per k-block
+constexpr int TC_STAGES_NARROW = 8;
 
 }  // namespace
 
@@ -502,6 +505,8 @@ cudaError_t linear_tc_init() {
     if (err == cudaSuccess) err = tc_attr<128, 2, TC_STAGES, 2>();
     if (err == cudaSuccess) err = tc_attr<256, 1, TC_STAGES_WIDE, 2>();
     if (err == cudaSuccess) err = tc_attr<256, 2, TC_STAGES_WIDE, 1>();
+    if (err == cudaSuccess) err = tc_attr<64, 1, TC_STAGES_NARROW, 2>();
+    if (err == cudaSuccess) err = tc_attr<64, 2, TC_STAGES_NARROW, 2>();
     return err;
 }
 
@@ -517,9 +522,13 @@ cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int 
     const bool two_chunks = K > TC_KB_PER_CHUNK * TC_BK;
     const long tiles_wide = (long)((M + TC_BM - 1) / TC_BM) * ((N + 255) / 256);
     const bool wide = N >= 256 && tiles_wide >= g_num_sms;
+    const long tiles_128 = (long)((M + TC_BM - 1) / TC_BM) * ((N + 127) / 128);
+    const bool narrow = !wide && tiles_128 < g_num_sms;
     CUtensorMap ta, tb;
-    if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, wide ? 256 : 128))
+    if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, wide ? 256 : (narrow ? 64 : 128)))
         return cudaErrorInvalidValue;
+    if (narrow && two_chunks) return tc_launch<64, 2, TC_STAGES_NARROW, 2>(ta, tb, M, N, K, e, status, st);
+    if (narrow) return tc_launch<64, 1, TC_STAGES_NARROW, 2>(ta, tb, M, N, K, e, status, st);
     if (wide && two_chunks) return tc_launch<256, 2, TC_STAGES_WIDE, 1>(ta, tb, M, N, K, e, status, st);
     if (wide) return tc_launch<256, 1, TC_STAGES_WIDE, 2>(ta, tb, M, N, K, e, status, st);
     if (two_chunks) return tc_launch<128, 2, TC_STAGES, 2>(ta, tb, M, N, K, e, status, st);
