@@ -469,7 +469,10 @@ struct mnmt_session {
     size_t arena_bytes = 0;
     float *resid, *cum, *logits;
     int8_t *act, *qkv, *ctx, *hid, *qbuf, *enc_q, *ck, *cv, *sk, *sv;
-    __half *a16;        // fp16 copy of a tensor-core linear's input rows
+    __half *a16;        // fp16 copy of a tensor-core linear's input rows (other buffers)
+    // fp16 mirrors of the int8 activation buffers, written by their producers
+    // when the consumer is a tensor-core linear
+    __half *act16 = nullptr, *ctx16 = nullptr, *hid16 = nullptr, *encq16 = nullptr;
     bool use_tc = true;  // tensor-core linears for layers of >= TC_MIN_ROWS rows
     int32_t *src_ids, *src_lens, *tok, *fin, *hist, *parents, *anc, *out_ids, *out_lens;
     float *out_scores;
@@ -534,7 +537,10 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
            o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
            o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams)), o_dcln = piece((6 * L + 2) * d * 4);
     const size_t kmax = std::max(d, std::max(F, (size_t)c.d_embed));
-    size_t o_a16 = piece(rows >= TC_MIN_ROWS ? rows * kmax * 2 : 256);
+    const bool tc_any = rows >= TC_MIN_ROWS;
+    size_t o_a16 = piece(tc_any ? rows * kmax * 2 : 256);
+    size_t o_act16 = piece(tc_any ? rows * kmax * 2 : 256), o_ctx16 = piece(tc_any ? rows * d * 2 : 256),
+           o_hid16 = piece(tc_any ? rows * F * 2 : 256), o_encq16 = piece(tc_any ? ME * d * 2 : 256);
     s->arena_bytes = off;
     if (cudaMalloc(&s->arena, off) != cudaSuccess) {
         delete s;
@@ -575,6 +581,10 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
     s->d_dc = reinterpret_cast<DcParams *>(a + o_dc);
     s->dc_ln = reinterpret_cast<float *>(a + o_dcln);
     s->a16 = reinterpret_cast<__half *>(a + o_a16);
+    s->act16 = reinterpret_cast<__half *>(a + o_act16);
+    s->ctx16 = reinterpret_cast<__half *>(a + o_ctx16);
+    s->hid16 = reinterpret_cast<__half *>(a + o_hid16);
+    s->encq16 = reinterpret_cast<__half *>(a + o_encq16);
     {
         const char *v = std::getenv("MNMT_TC");
         s->use_tc = !(v && v[0] == '0') && rows >= TC_MIN_ROWS;
@@ -618,18 +628,42 @@ const __half *w16_of(const mnmt_model *m, const int8_t *w) {
     return m->d_blob16 + (w - reinterpret_cast<const int8_t *>(m->d_blob));
 }
 
+// does a linear of M rows run on the tensor cores (then its input comes from
+// the fp16 mirror its producer wrote)
+bool tc_rows(const mnmt_session *s, int M) { return s->use_tc && (size_t)M >= TC_MIN_ROWS; }
+
+// fp16 mirror of one of the session's int8 activation buffers
+__half *mirror16(mnmt_session *s, const int8_t *buf) {
+    if (buf == s->act) return s->act16;
+    if (buf == s->ctx) return s->ctx16;
+    if (buf == s->hid) return s->hid16;
+    if (buf == s->enc_q) return s->encq16;
+    return nullptr;
+}
+
+// the fp16 copy a producer of buf (M rows) must also write, or null
+__half *out16_for(mnmt_session *s, const int8_t *buf, int M) { return tc_rows(s, M) ? mirror16(s, buf) : nullptr; }
+
 // The quantised linear of rows A [M][lda] (Eq. 3 + epilogue e): on the
 // tensor cores when the layer is a dense contraction (M >= TC_MIN_ROWS),
-// after an exact int8 -> fp16 copy of A; else on the IMMA / GEMV kernels.
+// reading the fp16 mirror of A that A's producer wrote; else on the IMMA /
+// GEMV kernels.
 cudaError_t run_linear(mnmt_session *s, const int8_t *A, int lda, const Lin &l, int M, const Epi &e,
                        cudaStream_t st) {
     const mnmt_model *m = s->m;
-    if (s->use_tc && M >= TC_MIN_ROWS && l.k % 16 == 0) {
+    if (tc_rows(s, M) && l.k % 16 == 0) {
         const __half *w16 = w16_of(m, l.w);
-        if (linear_tc_shape_ok(M, l.n, l.k, l.k, l.k, s->a16, w16)) {
-            cudaError_t err = launch_codes_to_f16(A, lda, s->a16, l.k, M, l.k, st);
+        const __half *a16 = mirror16(s, A);
+        int lda16 = lda;
+        if (!a16) {  // not a mirrored buffer: convert here
+            a16 = s->a16;
+            lda16 = l.k;
+        }
+        if (linear_tc_shape_ok(M, l.n, l.k, lda16, l.k, a16, w16)) {
+            cudaError_t err = cudaSuccess;
+            if (a16 == s->a16) err = launch_codes_to_f16(A, lda, s->a16, l.k, M, l.k, st);
             if (err == cudaSuccess)
-                err = launch_linear_tc(s->a16, l.k, w16, l.k, M, l.n, l.k, e, s->state + ST_STATUS, st);
+                err = launch_linear_tc(a16, lda16, w16, l.k, M, l.n, l.k, e, s->state + ST_STATUS, st);
             return err;
         }
     }
@@ -654,6 +688,7 @@ int ln_after_residual(mnmt_session *s, int M, const LnP &ln_pre_next, const LnP 
     a.d = m->c.d_model;
     a.inv = 1.0f / s_next;
     a.out_q = act_out;
+    a.out16 = out16_for(s, act_out, M);
     a.status = s->state + ST_STATUS;
     a.skip = skip;
     if (m->c.pre_ln) {
@@ -694,6 +729,7 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e.V = c.vocab;
         e.r = s->resid;
         e.out_q = s->act;
+        e.out16 = out16_for(s, s->act, M);
         if (c.pre_ln) {
             e.ln_g = m->enc_self[0].ln.g;
             e.ln_b = m->enc_self[0].ln.b;
@@ -711,8 +747,10 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e.ldo = 3 * d;
         LK(run_linear(s, s->act, d, A.qkv, M, e, st));  // N = 3 * d, K = d
         AttnEncArgs at;
+        std::memset(&at, 0, sizeof(at));
         at.qkv = s->qkv;
         at.ctx = s->ctx;
+        at.ctx16 = out16_for(s, s->ctx, M);
         at.len = s->src_lens;
         at.B = B;
         at.S = S;
@@ -732,6 +770,7 @@ int run_encoder(mnmt_session *s, int B, int S) {
         e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
         e.inv_out = Fb.inv_h;
         e.out = s->hid;
+        e.out16 = out16_for(s, s->hid, M);
         e.ldo = F;
         LK(run_linear(s, s->act, d, Fb.w1, M, e, st));  // N = F, K = d
         e = base_epi(EPI_RESID, Fb.s_h, Fb.w2);
@@ -810,6 +849,7 @@ int issue_decode_step(mnmt_session *s) {
         e.V = c.vocab;
         e.r = s->resid;
         e.out_q = s->act;
+        e.out16 = out16_for(s, s->act, R);
         if (c.pre_ln) {
             e.ln_g = m->dec_self[0].ln.g;
             e.ln_b = m->dec_self[0].ln.b;
@@ -842,6 +882,7 @@ int issue_decode_step(mnmt_session *s) {
         at.kc = s->sk + l * s->sk_layer;
         at.vc = s->sv + l * s->sk_layer;
         at.ctx = s->ctx;
+        at.ctx16 = out16_for(s, s->ctx, R);
         at.R = R;
         at.H = H;
         at.dh = dh;
@@ -888,6 +929,7 @@ int issue_decode_step(mnmt_session *s) {
         e = base_epi(EPI_RELU_Q8, Fb.s_in, Fb.w1);
         e.inv_out = Fb.inv_h;
         e.out = s->hid;
+        e.out16 = out16_for(s, s->hid, R);
         e.ldo = F;
         e.skip = done;
         LK(run_linear(s, s->act, d, Fb.w1, R, e, st));  // N = F, K = d

@@ -137,12 +137,14 @@ __global__ void __launch_bounds__(32 * 16) attn_decode(AttnDecArgs a) {
     }
     // lane (grp, gl) writes elements gl * EPG + grp * EPG / CG + [0, EPG / CG)
     constexpr int OPL = EPG / CG;
-    int8_t *out = a.ctx + (size_t)r * a.H * DH + h * DH + gl * EPG + grp * OPL;
+    const size_t o = (size_t)r * a.H * DH + h * DH + gl * EPG + grp * OPL;
 #pragma unroll
     for (int u = 0; u < EPG; u++) {
         if (u / OPL == grp) {
             long long N = (long long)hi[u] * 4096 + lo[u];
-            out[u - grp * OPL] = q8_quotient(N, Z, a.rho, rn32_div);
+            const int8_t v = q8_quotient(N, Z, a.rho, rn32_div);
+            a.ctx[o + u - grp * OPL] = v;
+            if (a.ctx16) a.ctx16[o + u - grp * OPL] = __short2half_rn(v);
         }
     }
 }
@@ -243,11 +245,13 @@ __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, in
                 lo[u] += El * v;
             }
         }
-        int8_t *out = a.ctx + ((size_t)b * S + qi) * a.d + h * DH + lane * EPL;
+        const size_t o = ((size_t)b * S + qi) * a.d + h * DH + lane * EPL;
 #pragma unroll
         for (int u = 0; u < EPL; u++) {
             long long N = (long long)hi[u] * 4096 + lo[u];
-            out[u] = q8_quotient(N, Z, a.rho, rn32_div);
+            const int8_t v = q8_quotient(N, Z, a.rho, rn32_div);
+            a.ctx[o + u] = v;
+            if (a.ctx16) a.ctx16[o + u] = __short2half_rn(v);
         }
         __syncwarp();
     }

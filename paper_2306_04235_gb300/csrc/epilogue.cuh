@@ -15,11 +15,12 @@ MNMT_DEV void epi_store_f(const Epi &e, int m, int n, float accf, int t) {
     float y = __fadd_rn(__fmul_rn(accf, __fmul_rn(e.s_x, e.s_w[n])), e.bias[n]);
     switch (e.mode) {
         case EPI_Q8:
-            e.out[(size_t)m * e.ldo + n] = q8(y, e.inv_out[n]);
+        case EPI_RELU_Q8: {
+            const int8_t v = q8(e.mode == EPI_RELU_Q8 && !(y > 0.0f) ? 0.0f : y, e.inv_out[n]);
+            e.out[(size_t)m * e.ldo + n] = v;
+            if (e.out16) e.out16[(size_t)m * e.ldo + n] = __short2half_rn(v);
             break;
-        case EPI_RELU_Q8:
-            e.out[(size_t)m * e.ldo + n] = q8(y > 0.0f ? y : 0.0f, e.inv_out[n]);
-            break;
+        }
         case EPI_RESID: {
             float *p = e.f32 + (size_t)m * e.ldf + n;
             *p = __fadd_rn(__fmul_rn(e.gamma, *p), y);

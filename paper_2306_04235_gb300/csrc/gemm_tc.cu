@@ -156,7 +156,7 @@ __device__ __forceinline__ bool epi_vec_ok(const Epi &e) {
     switch (e.mode) {
         case EPI_Q8:
         case EPI_RELU_Q8:
-            return e.ldo % 16 == 0 && al(e.out);
+            return e.ldo % 16 == 0 && al(e.out) && al(e.out16);
         case EPI_RESID:
         case EPI_F32:
             return e.ldf % 4 == 0 && al(e.f32);
@@ -219,6 +219,20 @@ __device__ __forceinline__ void epi_store16(const Epi &e, int row, int col0, con
         dst = (seg ? e.vc : e.kc) + (((size_t)b * e.H + h) * e.S + sp) * e.dh + i;
     } else {
         dst = e.out + (size_t)row * e.ldo + col0;
+        if (e.out16) {
+            // the fp16 copy of the 16 codes (exact), as two 16-byte stores
+            uint32_t h[8];
+#pragma unroll
+            for (int k = 0; k < 8; k++) {
+                const uint32_t word = w[k >> 1] >> (16 * (k & 1));
+                const __half lo = __short2half_rn((short)(int8_t)(word & 0xFFu));
+                const __half hi = __short2half_rn((short)(int8_t)((word >> 8) & 0xFFu));
+                h[k] = (uint32_t)__half_as_ushort(lo) | ((uint32_t)__half_as_ushort(hi) << 16);
+            }
+            uint4 *d16 = reinterpret_cast<uint4 *>(e.out16 + (size_t)row * e.ldo + col0);
+            d16[0] = make_uint4(h[0], h[1], h[2], h[3]);
+            d16[1] = make_uint4(h[4], h[5], h[6], h[7]);
+        }
     }
     *reinterpret_cast<uint4 *>(dst) = make_uint4(w[0], w[1], w[2], w[3]);
 }

@@ -52,6 +52,7 @@ struct Epi {
     const float *bias;
     const float *inv_out;
     int8_t *out;
+    __half *out16;  // EPI_Q8 / EPI_RELU_Q8: optional fp16 copy of out (same layout)
     int ldo;
     float *f32;
     int ldf;
@@ -92,6 +93,7 @@ struct LnArgs {
     const float *r;   // [M][d] input rows (row stride d)
     float *out_f;     // optional fp32 output (may alias r)
     int8_t *out_q;    // optional int8 output
+    __half *out16;    // optional fp16 copy of out_q (tensor-core operand)
     const float *g, *b;
     float inv;
     int M, d;
@@ -114,6 +116,7 @@ struct EmbedArgs {
     int M, d, E, V;
     float *r;              // fp32 [M][d] residual out
     int8_t *out_q;         // int8 sublayer input out
+    __half *out16;         // optional fp16 copy of out_q (tensor-core operand)
     const float *ln_g, *ln_b;  // if non-null: out_q = q8(LN(x), inv) else q8(x, inv)
     float inv;
     int *status;
@@ -125,6 +128,7 @@ struct AttnDecArgs {
     const int8_t *q;        // [R][d] (head h at h*dh)
     const int8_t *kc, *vc;  // self: [R][H][T][dh]; cross: [B][H][S][dh]
     int8_t *ctx;            // [R][d]
+    __half *ctx16;          // optional fp16 copy of ctx (tensor-core operand)
     int R, H, dh, T;        // T = cache capacity (self) or S_pad (cross)
     int cross;              // 0 = self (keys 0..t), 1 = cross (keys < src_len[r / beam])
     int beam;
@@ -140,6 +144,7 @@ cudaError_t launch_attention_decode(const AttnDecArgs &a, cudaStream_t st);
 struct AttnEncArgs {
     const int8_t *qkv;  // [B*S][3d]: q | k | v
     int8_t *ctx;        // [B*S][d]
+    __half *ctx16;      // optional fp16 copy of ctx (tensor-core operand)
     const int *len;     // [B]
     int B, S, H, dh, d;
     float sigma, rho;

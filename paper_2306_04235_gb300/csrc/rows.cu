@@ -40,7 +40,11 @@ __global__ void __launch_bounds__(256) layernorm_kernel(LnArgs a) {
         int i = u * 32 + lane;
         if (i < a.d) {
             if (a.out_f) a.out_f[(size_t)row * a.d + i] = y[u];
-            if (a.out_q) a.out_q[(size_t)row * a.d + i] = q8(y[u], a.inv);
+            if (a.out_q) {
+                const int8_t v = q8(y[u], a.inv);
+                a.out_q[(size_t)row * a.d + i] = v;
+                if (a.out16) a.out16[(size_t)row * a.d + i] = __short2half_rn(v);
+            }
         }
     }
 }
@@ -121,7 +125,9 @@ __global__ void __launch_bounds__(256) embed_kernel(EmbedArgs a) {
         int i = u * 32 + lane;
         if (i < a.d) {
             a.r[(size_t)row * a.d + i] = x[u];
-            a.out_q[(size_t)row * a.d + i] = q8(a.ln_g ? y[u] : x[u], a.inv);
+            const int8_t v = q8(a.ln_g ? y[u] : x[u], a.inv);
+            a.out_q[(size_t)row * a.d + i] = v;
+            if (a.out16) a.out16[(size_t)row * a.d + i] = __short2half_rn(v);
         }
     }
 }
