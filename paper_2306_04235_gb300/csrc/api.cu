@@ -454,8 +454,8 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
 // session
 // ---------------------------------------------------------------------------
 enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_STATUS = 5, ST_N = 8 };
-// layers of at least this many rows run on the tensor cores (one full M tile)
-constexpr size_t TC_MIN_ROWS = 128;
+// layers of more rows than the GEMV kernel takes (16) run on the tensor cores
+constexpr size_t TC_MIN_ROWS = 17;
 // steps per multi-step decode graph (and per completion check of translate)
 constexpr int GRAPH_STEPS = 16;
 
