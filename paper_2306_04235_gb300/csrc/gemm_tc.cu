@@ -172,14 +172,15 @@ __device__ __forceinline__ bool epi_vec_ok(const Epi &e) {
 // The epilogue of outputs (row, col0 .. col0+15) of one row, col0 a multiple
 // of 16, all columns < N: the same arithmetic as epi_store_f, with one 16-byte
 // access per 16 int8 codes or 4 fp32 values.
+// rpre, if given, holds the 16 residual values of a RESID store, loaded earlier.
 __device__ __forceinline__ void epi_store16(const Epi &e, int row, int col0, const float (&a)[16], const float *sc,
-                                            const float *bs, const float *inv, int t) {
+                                            const float *bs, const float *inv, int t, const float4 *rpre = nullptr) {
     if (e.mode == EPI_RESID || e.mode == EPI_F32) {
         float4 *p = reinterpret_cast<float4 *>(e.f32 + (size_t)row * e.ldf + col0);
         float4 r[4];
         if (e.mode == EPI_RESID) {
 #pragma unroll
-            for (int g = 0; g < 4; g++) r[g] = p[g];
+            for (int g = 0; g < 4; g++) r[g] = rpre ? rpre[g] : p[g];
         }
 #pragma unroll
         for (int g = 0; g < 4; g++) {
@@ -294,29 +295,37 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
     tc_fence_after();
     const uint32_t tbase = misc[0];
 
+    // The producer and the MMA issuer are single threads whose per-k-block
+    // cost (mbarrier tests, TMA and MMA issue) bounds small grids, so their
+    // loops test the shared abort flag once per tile, not per k-block.
     uint32_t issued = 0;
     if (warp == 0 && lane == 0) {
         // ---- TMA producer: k-blocks of all this CTA's tiles through the ring ----
         uint32_t it = 0;
-        for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+        bool failed = false;
+        const uint32_t a_ring = s_addr(sm), b_ring = s_addr(sm + L::OFF_B);
+        for (int tile = blockIdx.x; tile < tiles && !failed && !*abort_flag; tile += gridDim.x) {
             const int m0 = (tile % mt) * TC_BM, n0 = (tile / mt) * BN;
             for (int kb = 0; kb < nkb; kb++, it++) {
                 const int s = (int)(it % STAGES);
                 if (it >= STAGES && !mbar_wait(empty_bar(s), (it / STAGES - 1) & 1)) {
                     *abort_flag = 1;
                     set_status(status, MNMT_ETIMEOUT);
+                    failed = true;
+                    break;
                 }
-                if (*abort_flag) break;
                 mbar_expect_tx(full_bar(s), L::A_BYTES + L::B_BYTES);
-                tma_load_2d(s_addr(sm + s * L::A_BYTES), &tmA, kb * TC_BK, m0, full_bar(s));
-                tma_load_2d(s_addr(sm + L::OFF_B + s * L::B_BYTES), &tmB, kb * TC_BK, n0, full_bar(s));
+                tma_load_2d(a_ring + s * L::A_BYTES, &tmA, kb * TC_BK, m0, full_bar(s));
+                tma_load_2d(b_ring + s * L::B_BYTES, &tmB, kb * TC_BK, n0, full_bar(s));
                 issued = it + 1;
             }
         }
     } else if (warp == 1 && lane == 0) {
         // ---- MMA issuer ----
         uint32_t it = 0, lt = 0;
-        for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x, lt++) {
+        bool failed = false;
+        const uint64_t a_desc = sw128_desc(s_addr(sm)), b_desc = sw128_desc(s_addr(sm + L::OFF_B));
+        for (int tile = blockIdx.x; tile < tiles && !failed && !*abort_flag; tile += gridDim.x, lt++) {
             const int buf = (int)(lt % NBUF);
             if (lt >= NBUF && !mbar_wait(acce_bar(buf), ((lt / NBUF) - 1) & 1)) {
                 *abort_flag = 1;
@@ -330,28 +339,33 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
                 if (!mbar_wait(full_bar(s), (it / STAGES) & 1)) {
                     *abort_flag = 1;
                     set_status(status, MNMT_ETIMEOUT);
+                    failed = true;
+                    break;
                 }
-                if (*abort_flag) break;
-                misc[2] = it + 1;
                 tc_fence_after();
                 const uint32_t d = dbase + (uint32_t)((kb / TC_KB_PER_CHUNK) * BN);
-                const uint64_t ad = sw128_desc(s_addr(sm + s * L::A_BYTES));
-                const uint64_t bd = sw128_desc(s_addr(sm + L::OFF_B + s * L::B_BYTES));
+                // descriptor start addresses advance in 16-byte units
+                const uint64_t ad = a_desc + (uint64_t)((s * L::A_BYTES) >> 4);
+                const uint64_t bd = b_desc + (uint64_t)((s * L::B_BYTES) >> 4);
 #pragma unroll
                 for (int k = 0; k < TC_BK / 16; k++)
                     mma_f16(d, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC,
                             (uint32_t)((kb % TC_KB_PER_CHUNK) | k));
                 mma_commit(empty_bar(s));
             }
-            if (*abort_flag) break;
+            if (failed) break;
             mma_commit(accf_bar(buf));
         }
+        misc[2] = it;          // k-blocks whose copies this thread saw land
         mma_commit(done_bar);  // arrives once every MMA issued above has completed
     } else if (warp >= 2) {
         // ---- epilogue: TMEM -> registers -> fused epilogue -> global ----
         const int ew = warp - 2;                       // 0 .. TC_EPI_WARPS-1
         const int q = warp & 3;                        // TMEM lane quarter of this warp
         const int half = ew >> 2;                      // which half of the tile's columns
+        constexpr int JN = BN / 32;                    // 16-column chunks per thread and tile
+        constexpr int PRE_CH = BN == 64 ? JN : 0;      // residual chunks loaded ahead
+        constexpr int EPI_UNROLL = PRE_CH > 0 ? PRE_CH : 1;
         const int t = e.t_ptr ? *e.t_ptr : 0;
         const bool vec = epi_vec_ok(e);
         uint32_t lt = 0;
@@ -368,6 +382,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
                 c_inv[i] = ok && e.inv_out ? e.inv_out[n] : 0.0f;
             }
             epi_bar_sync();
+            const int row = m0 + 32 * q + lane;
+            // 128 x 64 tiles: a residual epilogue loads its 32 residual values
+            // while the tile's MMAs run (the store then waits on no load)
+            float4 rpre[4 * PRE_CH > 0 ? 4 * PRE_CH : 1];
+            const bool pre = PRE_CH > 0 && e.mode == EPI_RESID && vec && row < M;
+            if (pre) {
+#pragma unroll
+                for (int jj = 0; jj < PRE_CH; jj++) {
+                    const int col0 = n0 + 16 * (half * JN + jj);
+                    if (col0 + 16 <= N) {
+                        const float4 *p = reinterpret_cast<const float4 *>(e.f32 + (size_t)row * e.ldf + col0);
+#pragma unroll
+                        for (int g = 0; g < 4; g++) rpre[4 * jj + g] = p[g];
+                    }
+                }
+            }
             // every epilogue warp runs every tile of the loop (the named barrier
             // above needs all of them); after an abort the tiles are skipped
             bool ok = *abort_flag == 0 && mbar_wait(accf_bar(buf), (lt / NBUF) & 1);
@@ -377,11 +407,11 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
             }
             tc_fence_after();
             ok = __all_sync(0xFFFFFFFFu, ok && *abort_flag == 0);
-            const int row = m0 + 32 * q + lane;
             const uint32_t taddr = tbase + ((uint32_t)(32 * q) << 16) + (uint32_t)(buf * ACC_COLS);
             unsigned long long best = 0ull;
-#pragma unroll 1
-            for (int j = half * (BN / 32); ok && j < (half + 1) * (BN / 32); j++) {
+#pragma unroll EPI_UNROLL
+            for (int jj = 0; ok && jj < JN; jj++) {
+                const int j = half * JN + jj;
                 uint32_t r0[16], r1[16];
                 tmem_ld16(taddr + 16 * j, r0);
                 if (NCH == 2) tmem_ld16(taddr + BN + 16 * j, r1);
@@ -404,7 +434,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
                         }
                     }
                 } else if (vec && col0 + 16 <= N) {
-                    if (row < M) epi_store16(e, row, col0, a, sc, bs, inv, t);
+                    if (row < M) epi_store16(e, row, col0, a, sc, bs, inv, t, PRE_CH > 0 && pre ? rpre + 4 * jj : nullptr);
                 } else if (row < M) {
 #pragma unroll
                     for (int i = 0; i < 16; i++)

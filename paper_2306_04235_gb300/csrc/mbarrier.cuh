@@ -39,15 +39,33 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// wait for the completion of the phase with the given parity; false if it has
-// not completed within MNMT_WAIT_NS
-static __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
-    if (mbar_try(bar, parity)) return true;
+// non-blocking test of the phase with the given parity
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// the waiting part of mbar_wait, out of line
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity) {
     const unsigned long long t0 = global_ns();
     while (!mbar_try(bar, parity)) {
         if (global_ns() - t0 > MNMT_WAIT_NS) return false;
     }
     return true;
+}
+
+// wait for the completion of the phase with the given parity; false if it has
+// not completed within MNMT_WAIT_NS.  A phase that has already completed costs
+// one inline test (pipelines whose data is usually ready make no call).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+    return mbar_test(bar, parity) || mbar_wait_slow(bar, parity);
 }
 
 // 1-D bulk copy global -> this CTA's shared memory, completing on bar
