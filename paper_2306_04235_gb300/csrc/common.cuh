@@ -46,10 +46,18 @@ MNMT_DEV float dequant_bias(int32_t acc, float s_x, float s_w, float b) {
 MNMT_DEV long long fx_scale(float v, int shift) {
     uint32_t bits = __float_as_uint(v);
     uint32_t ex = (bits >> 23) & 0xFFu;
-    // fast path: v normal and v 2^shift a normal float below 2^62 -- the
-    // scaling is then exact and the conversion rounds half to even
-    if (ex != 0 && (int)ex + shift >= 1 && (int)ex + shift <= 127 + 61)
-        return __float2ll_rn(__uint_as_float(bits + ((uint32_t)shift << 23)));
+    // fast path: v normal and y = v 2^shift a normal float below 2^62 -- the
+    // scaling is then exact.  |y| >= 2^23 is an integer, its significand
+    // shifted left; |y| < 2^23 rounds half to even into 32 bits (the 64-bit
+    // float-to-integer conversion runs at a small fraction of this rate)
+    if (ex != 0 && (int)ex + shift >= 1 && (int)ex + shift <= 127 + 61) {
+        const int ey = (int)ex + shift;  // biased exponent of y
+        if (ey >= 127 + 23) {
+            const long long q = (long long)((bits & 0x7FFFFFu) | 0x800000u) << (ey - 150);
+            return (bits >> 31) ? -q : q;
+        }
+        return (long long)__float2int_rn(__uint_as_float(bits + ((uint32_t)shift << 23)));
+    }
     uint32_t man = bits & 0x7FFFFFu;
     int e;
     if (ex == 0) {
@@ -75,11 +83,14 @@ MNMT_DEV long long fx_scale(float v, int shift) {
     return (bits >> 31) ? -q : q;
 }
 
-// exponent e with |v| < 2^e (0 for v == 0), as frexpf
+// exponent e with 2^(e-1) <= |v| < 2^e (0 for v == 0), as frexpf, read from the
+// bits: normal v of biased exponent E gives E - 126; a subnormal with an
+// n-bit significand gives n - 149
 MNMT_DEV int exp_bound(float v) {
-    int e = 0;
-    if (v != 0.0f) frexpf(v, &e);
-    return e;
+    const uint32_t a = __float_as_uint(v) & 0x7FFFFFFFu;
+    const int E = (int)(a >> 23);
+    if (E != 0) return E - 126;
+    return a == 0 ? 0 : (32 - __clz((int)a)) - 149;
 }
 
 // ---------------------------------------------------------------------------
@@ -315,6 +326,45 @@ MNMT_DEV long long warp_sum_exact(long long v) {
     p1 = __reduce_add_sync(0xFFFFFFFFu, p1);
     p2 = __reduce_add_sync(0xFFFFFFFFu, p2);
     return (long long)p0 + (long long)p1 * (1LL << 20) + (long long)p2 * (1LL << 40);
+}
+
+// LayerNorm of one row held by a warp (x[u] = element u*32 + lane); gv / bv
+// are the matching gamma / beta values, loaded by the caller
+template <int VPL>
+MNMT_DEV bool warp_layernorm_v(const float (&x)[VPL], int d, const float (&gv)[VPL], const float (&bv)[VPL],
+                               float (&out)[VPL], int lane) {
+    unsigned amax_bits = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) amax_bits = max(amax_bits, __float_as_uint(x[u]) & 0x7FFFFFFFu);
+    const float amax = __uint_as_float(__reduce_max_sync(0xFFFFFFFFu, amax_bits));
+    if (!(amax < 0x1p32f)) return false;
+    const int ea = exp_bound(amax);
+    const int log2d = 31 - __clz(d);  // d is a power of two
+    long long s1 = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
+    s1 = warp_sum_exact(s1);
+    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    float c[VPL];
+    unsigned bmax_bits = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++) {
+        c[u] = __fsub_rn(x[u], mu);
+        if (u * 32 + lane < d) bmax_bits = max(bmax_bits, __float_as_uint(c[u]) & 0x7FFFFFFFu);
+    }
+    const int eb = exp_bound(__uint_as_float(__reduce_max_sync(0xFFFFFFFFu, bmax_bits)));
+    long long s2 = 0;
+#pragma unroll
+    for (int u = 0; u < VPL; u++)
+        if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
+    s2 = warp_sum_exact(s2);
+    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+#pragma unroll
+    for (int u = 0; u < VPL; u++) out[u] = __fadd_rn(__fmul_rn(__fmul_rn(c[u], rstd), gv[u]), bv[u]);
+    return true;
 }
 
 template <int VPL>

@@ -14,36 +14,98 @@
 namespace mnmt {
 
 // ---------------------------------------------------------------------------
-// LayerNorm kernel: one warp per row
+// LayerNorm kernel: one block of LN_T threads per row, thread t holding the
+// VPT contiguous elements t*VPT ..  The row is short (d <= 2048) and a decode
+// step has only a few hundred rows, so the work of a row is spread over four
+// warps to shorten each thread's dependent chain; the order-free maxima and
+// exact fixed-point sums combine across warps through shared memory.  The
+// row, gamma and beta are loaded together before the skip flag is tested.
 // ---------------------------------------------------------------------------
-template <int VPL>
-__global__ void __launch_bounds__(256) layernorm_kernel(LnArgs a) {
+constexpr int LN_T = 128;
+
+template <int VPT>
+__global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     pdl_allow_next();
     pdl_grid_wait();
-    if (a.skip && *a.skip) return;
-    const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
-    const int lane = threadIdx.x & 31;
-    if (row >= a.M) return;
-    const float *r = a.r + (size_t)row * a.d;
-    float x[VPL], y[VPL];
+    __shared__ unsigned s_amax[LN_T / 32], s_bmax[LN_T / 32];
+    __shared__ long long s_s1[LN_T / 32], s_s2[LN_T / 32];
+    const int row = blockIdx.x, d = a.d;
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int i0 = threadIdx.x * VPT;
+    const float *r = a.r + (size_t)row * d;
+    float x[VPT], gv[VPT], bv[VPT];
 #pragma unroll
-    for (int u = 0; u < VPL; u++) {
-        int i = u * 32 + lane;
-        x[u] = i < a.d ? r[i] : 0.0f;
+    for (int v = 0; v < VPT; v++) {
+        const bool in = i0 + v < d;
+        x[v] = in ? r[i0 + v] : 0.0f;
+        gv[v] = in ? a.g[i0 + v] : 0.0f;
+        bv[v] = in ? a.b[i0 + v] : 0.0f;
     }
-    if (!warp_layernorm<VPL>(x, a.d, a.g, a.b, y, lane)) {
-        if (lane == 0) set_status(a.status, MNMT_EOVERFLOW);
+    if (a.skip && *a.skip) return;
+    // row maximum magnitude -> the grid of the exact sum of the elements
+    unsigned am = 0;
+#pragma unroll
+    for (int v = 0; v < VPT; v++) am = max(am, __float_as_uint(x[v]) & 0x7FFFFFFFu);  // padding is 0
+    am = __reduce_max_sync(0xFFFFFFFFu, am);
+    if (lane == 0) s_amax[w] = am;
+    __syncthreads();
+    am = s_amax[0];
+#pragma unroll
+    for (int k = 1; k < LN_T / 32; k++) am = max(am, s_amax[k]);
+    const float amax = __uint_as_float(am);
+    if (!(amax < 0x1p32f)) {
+        if (threadIdx.x == 0) set_status(a.status, MNMT_EOVERFLOW);
         return;
     }
+    const int ea = exp_bound(amax);
+    const int log2d = 31 - __clz(d);  // d is a power of two
+    long long s1 = 0;
 #pragma unroll
-    for (int u = 0; u < VPL; u++) {
-        int i = u * 32 + lane;
-        if (i < a.d) {
-            if (a.out_f) a.out_f[(size_t)row * a.d + i] = y[u];
+    for (int v = 0; v < VPT; v++) s1 += fx_scale(x[v], 52 - ea);  // padding adds 0
+    s1 = warp_sum_exact(s1);
+    if (lane == 0) s_s1[w] = s1;
+    __syncthreads();
+    s1 = 0;
+#pragma unroll
+    for (int k = 0; k < LN_T / 32; k++) s1 += s_s1[k];
+    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    // centred values -> their maximum magnitude -> the grid of the variance sum
+    float c[VPT];
+    unsigned bm = 0;
+#pragma unroll
+    for (int v = 0; v < VPT; v++) {
+        c[v] = __fsub_rn(x[v], mu);
+        if (i0 + v < d) bm = max(bm, __float_as_uint(c[v]) & 0x7FFFFFFFu);
+    }
+    bm = __reduce_max_sync(0xFFFFFFFFu, bm);
+    if (lane == 0) s_bmax[w] = bm;
+    __syncthreads();
+    bm = s_bmax[0];
+#pragma unroll
+    for (int k = 1; k < LN_T / 32; k++) bm = max(bm, s_bmax[k]);
+    const int eb = exp_bound(__uint_as_float(bm));
+    long long s2 = 0;
+#pragma unroll
+    for (int v = 0; v < VPT; v++)
+        if (i0 + v < d) s2 += fx_scale(__fmul_rn(c[v], c[v]), 52 - 2 * eb);
+    s2 = warp_sum_exact(s2);
+    if (lane == 0) s_s2[w] = s2;
+    __syncthreads();
+    s2 = 0;
+#pragma unroll
+    for (int k = 0; k < LN_T / 32; k++) s2 += s_s2[k];
+    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+#pragma unroll
+    for (int v = 0; v < VPT; v++) {
+        const int i = i0 + v;
+        if (i < d) {
+            const float y = __fadd_rn(__fmul_rn(__fmul_rn(c[v], rstd), gv[v]), bv[v]);
+            if (a.out_f) a.out_f[(size_t)row * d + i] = y;
             if (a.out_q) {
-                const int8_t v = q8(y[u], a.inv);
-                a.out_q[(size_t)row * a.d + i] = v;
-                if (a.out16) a.out16[(size_t)row * a.d + i] = __short2half_rn(v);
+                const int8_t q = q8(y, a.inv);
+                a.out_q[(size_t)row * d + i] = q;
+                if (a.out16) a.out16[(size_t)row * d + i] = __short2half_rn(q);
             }
         }
     }
@@ -51,13 +113,12 @@ __global__ void __launch_bounds__(256) layernorm_kernel(LnArgs a) {
 
 cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
     if (a.M <= 0) return cudaSuccess;
-    dim3 grid((a.M + 7) / 8), block(256);
-    int vpl = (a.d + 31) / 32;
-    if (vpl <= 4) launch_pdl(layernorm_kernel<4>, grid, block, 0, st, a);
-    else if (vpl <= 8) launch_pdl(layernorm_kernel<8>, grid, block, 0, st, a);
-    else if (vpl <= 16) launch_pdl(layernorm_kernel<16>, grid, block, 0, st, a);
-    else if (vpl <= 32) launch_pdl(layernorm_kernel<32>, grid, block, 0, st, a);
-    else if (vpl <= 64) launch_pdl(layernorm_kernel<64>, grid, block, 0, st, a);
+    const int vpt = (a.d + LN_T - 1) / LN_T;
+    if (vpt <= 1) launch_pdl(layernorm_kernel<1>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 2) launch_pdl(layernorm_kernel<2>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 4) launch_pdl(layernorm_kernel<4>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 8) launch_pdl(layernorm_kernel<8>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 16) launch_pdl(layernorm_kernel<16>, a.M, LN_T, 0, st, a);
     else return cudaErrorInvalidValue;
     return cudaGetLastError();
 }

@@ -159,6 +159,35 @@ def test_layernorm_matches_oracle(M, d, scale):
     assert np.array_equal(host(oq), ref_q)
 
 
+def test_layernorm_wide_magnitude_rows():
+    """Rows whose terms land on every branch of the fixed-point conversion: one
+    large value sets the grid, the others scale to integers far above 2^23,
+    to values just below 2^23 with .5 fractions (rounded half to even), and to
+    values under 1/2 (rounded to zero)."""
+    M, d = 6, 512
+    st = synth.Stream(77, "w")
+    r = np.zeros((M, d), np.float32)
+    for m in range(M):
+        big = np.float32(2.0 ** (20 - 3 * m))
+        e = st.randint(-44 - 3 * m, -4 - 3 * m, d)                  # exponents around the 2^23 boundary of the grid
+        odd = (2 * st.randint(0, 1 << 22, d) + 1).astype(np.float64)  # odd significands: .5 fractions after scaling
+        sign = np.where(st.randint(0, 2, d) == 1, -1.0, 1.0)
+        r[m] = (sign * odd * np.exp2(e.astype(np.float64) - 23)).astype(np.float32)
+        r[m, 3] = big
+        r[m, 100] = -big / 2
+    g = synth.uniform_f32(5, "g", (d,), 0.5, 1.5)
+    b = synth.uniform_f32(5, "b", (d,), -0.2, 0.2)
+    inv = np.float32(127 / 4.0)
+    of = torch.zeros((M, d), dtype=torch.float32, device="cuda")
+    oq = torch.zeros((M, d), dtype=torch.int8, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    mnmt.mnmt_layernorm(dev(r), dev(g), dev(b), M, d, inv, of, oq, status)
+    ref_f, ref_q = O.layernorm(r, g, b, inv)
+    assert host(status)[0] == 0
+    assert np.array_equal(host(of).view(np.uint32), ref_f.view(np.uint32))
+    assert np.array_equal(host(oq), ref_q)
+
+
 def test_layernorm_constant_row_and_overflow_status():
     d = 256
     g = np.ones(d, np.float32); b = synth.uniform_f32(1, "b", (d,), -1, 1)
