@@ -100,7 +100,10 @@ MNMT_DEV int exp_bound(float v) {
 // ---------------------------------------------------------------------------
 MNMT_DEV float exp_own(float x) {
     if (x < -87.0f) return 0.0f;
-    float n = rintf(__fmul_rn(x, 0x1.715476p+0f));
+    // n = rne(x log2(e)) in [-126, 0] by adding 1.5 2^23 (ulp 1 there: the sum
+    // rounds the fraction half to even and its low bits hold n)
+    const float t = __fadd_rn(__fmul_rn(x, 0x1.715476p+0f), 12582912.0f);
+    const float n = __fsub_rn(t, 12582912.0f);
     float r = __fmaf_rn(-n, 0x1.62e4p-1f, x);
     r = __fmaf_rn(-n, 0x1.7f7d1cp-20f, r);
     float p = 0x1.a01a02p-13f;
@@ -111,7 +114,7 @@ MNMT_DEV float exp_own(float x) {
     p = __fmaf_rn(p, r, 0.5f);
     p = __fmaf_rn(p, r, 1.0f);
     p = __fmaf_rn(p, r, 1.0f);
-    int ni = __float2int_rz(n);
+    const int ni = (int)(__float_as_uint(t) - 0x4B400000u);
     float two_n = __uint_as_float((uint32_t)(ni + 127) << 23);
     return __fmul_rn(p, two_n);
 }

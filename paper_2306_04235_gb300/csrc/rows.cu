@@ -293,11 +293,74 @@ MNMT_DEV void topk_insert(unsigned long long (&lst)[KM], int k, unsigned long lo
     }
 }
 
-template <int KM>
-__global__ void __launch_bounds__(BR_THREADS) beam_rows_kernel(BeamArgs a) {
+// rne(exp_own(x) 2^24) for x <= 0, the weight of one softmax term.  Below 2^23
+// the rounding to an integer is done by adding 2^23 (whose ulp is 1) and
+// reading the low bits; the few weights in [2^23, 2^24] (x within ln 2 of
+// the maximum) are integers already.
+MNMT_DEV int32_t softmax_weight_fast(float x) {
+    const float w = __fmul_rn(exp_own(x), 16777216.0f);
+    if (w < 0x1p23f) return (int32_t)(__float_as_uint(__fadd_rn(w, 0x1p23f)) - 0x4B000000u);
+    return __float2int_rn(w);
+}
+
+// Block-wide selection of the n largest keys held in the threads' descending
+// lists lst[0..KL): n rounds of a maximum over the list heads.  The keys land
+// in sel[0..n) (0 where fewer exist); every thread must call it.
+template <int KL, int NT>
+__device__ void block_select(const unsigned long long (&lst)[KL], int n, unsigned long long *sel,
+                             unsigned long long *s_key) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    int head = 0;
+    for (int i = 0; i < n; i++) {
+        unsigned long long mine = 0ull;
+#pragma unroll
+        for (int h = 0; h < KL; h++)
+            if (h == head) mine = lst[h];
+        const unsigned long long w = warp_max_u64(mine);
+        if (lane == 0) s_key[warp] = w;
+        __syncthreads();
+        unsigned long long best = s_key[0];
+        for (int j = 1; j < NT / 32; j++) best = s_key[j] > best ? s_key[j] : best;
+        if (mine == best && best != 0ull) head++;  // keys are unique
+        if (threadIdx.x == 0) sel[i] = best;
+        __syncthreads();
+    }
+}
+
+// Insert key into a warp-distributed descending list (lane j < KC holds the
+// j-th best key, 0 where empty; keys are unique); returns the logit of the
+// list's last entry once the list is full (-inf before).
+template <int KC>
+MNMT_DEV float warp_list_insert(unsigned long long &wl, unsigned long long key, int lane, float thr) {
+    const unsigned long long last = __shfl_sync(0xFFFFFFFFu, wl, KC - 1);
+    if (key <= last) return thr;
+    const int pos = __popc(__ballot_sync(0xFFFFFFFFu, lane < KC && wl > key));  // entries ranked above key
+    const unsigned long long up = __shfl_up_sync(0xFFFFFFFFu, wl, 1);
+    if (lane < KC) wl = lane < pos ? wl : (lane == pos ? key : up);
+    const unsigned long long nl = __shfl_sync(0xFFFFFFFFu, wl, KC - 1);
+    return nl != 0ull ? key_value(nl) : thr;
+}
+
+// One block per hypothesis row: the log-softmax of Sec. 3 / App. D's beam
+// search (m = max, Z = sum of rne(e^(l - m) 2^24), lambda = ln Z - 24 ln 2,
+// score = cum + ((l - m) - lambda)) and the k best (score, flat index) keys.
+// The score is a non-decreasing function of the logit, so the k best lie
+// among the logits ranked best by (logit desc, id asc): the pass that sums Z
+// also keeps each warp's KC = KM + 4 best logits (a warp-wide threshold makes
+// updates rare), and the k best scores are taken from the row's KC best
+// logits.  That is exact unless the last of those candidates could still tie
+// the k-th score (rounding can merge scores); such a row is scanned again in
+// full.
+// CAND = false skips the candidates and always scans the scores (fewer,
+// simpler passes: better where a few rows leave the SMs short of warps).
+template <int KM, int NT, bool CAND>
+__global__ void __launch_bounds__(NT) beam_rows_kernel(BeamArgs a) {
     pdl_allow_next();
     pdl_grid_wait();
     if (*a.done) return;
+    constexpr int KC = KM + 4;
+    static_assert(KC <= 32, "a warp holds the candidate list");
+    constexpr int NW = NT / 32;
     const int r = blockIdx.x;
     const int k = a.k;
     const int V = a.V;
@@ -305,67 +368,162 @@ __global__ void __launch_bounds__(BR_THREADS) beam_rows_kernel(BeamArgs a) {
     unsigned long long *out = a.cand + (size_t)r * k;
     __shared__ float s_m;
     __shared__ float s_lam;
-    __shared__ long long s_z[BR_THREADS / 32];
-    __shared__ float s_mx[BR_THREADS / 32];
-    __shared__ unsigned long long s_key[BR_THREADS / 32];
+    __shared__ int s_full;
+    __shared__ long long s_z[NW];
+    __shared__ float s_mx[NW];
+    __shared__ unsigned long long s_key[NW];
+    __shared__ unsigned long long s_wl[NW][KC];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     if (a.fin[r]) {
         // a finished hypothesis offers itself once, unchanged, with token PAD
-        for (int i = threadIdx.x; i < k; i += BR_THREADS)
+        for (int i = threadIdx.x; i < k; i += NT)
             out[i] = i == 0 ? pack_key(a.cum[r], (uint32_t)(lb * V + a.pad)) : 0ull;
         return;
     }
     const float *l = a.logits + (size_t)r * V;
+    const bool v4 = (V & 3) == 0 && (reinterpret_cast<uintptr_t>(l) & 15) == 0;
+    const float4 *l4 = reinterpret_cast<const float4 *>(l);
     float mx = -INFINITY;
-    for (int n = threadIdx.x; n < V; n += BR_THREADS) mx = fmaxf(mx, l[n]);
+    if (v4) {
+        for (int n = threadIdx.x; n < V / 4; n += NT) {
+            const float4 v = l4[n];
+            mx = fmaxf(mx, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)));
+        }
+    } else {
+        for (int n = threadIdx.x; n < V; n += NT) mx = fmaxf(mx, l[n]);
+    }
     mx = warp_max_f(mx);
     if (lane == 0) s_mx[warp] = mx;
     __syncthreads();
     if (threadIdx.x == 0) {
         float m = s_mx[0];
-        for (int w = 1; w < BR_THREADS / 32; w++) m = fmaxf(m, s_mx[w]);
+        for (int w = 1; w < NW; w++) m = fmaxf(m, s_mx[w]);
         s_m = m;
     }
     __syncthreads();
     const float m = s_m;
+    // Z, and this warp's KC best (logit, id) keys
     long long z = 0;
-    for (int n = threadIdx.x; n < V; n += BR_THREADS) z += softmax_weight(__fsub_rn(l[n], m));
+    unsigned long long wl = 0ull;
+    float thr = -INFINITY;  // warp-uniform
+    // four logits per lane and step: their weights, then one warp vote on
+    // whether any of them can enter the warp's list
+    auto visit4 = [&](const float4 v, int n0) {
+        const int32_t w4 = softmax_weight_fast(__fsub_rn(v.x, m)) + softmax_weight_fast(__fsub_rn(v.y, m)) +
+                           softmax_weight_fast(__fsub_rn(v.z, m)) + softmax_weight_fast(__fsub_rn(v.w, m));
+        z += w4;  // each weight <= 2^24
+        unsigned msk = __ballot_sync(0xFFFFFFFFu, fmaxf(fmaxf(v.x, v.y), fmaxf(v.z, v.w)) >= thr);
+        while (msk) {
+            const int src = __ffs(msk) - 1;
+            msk &= msk - 1;
+            const int ns = __shfl_sync(0xFFFFFFFFu, n0, src);
+            const float xs[4] = {__shfl_sync(0xFFFFFFFFu, v.x, src), __shfl_sync(0xFFFFFFFFu, v.y, src),
+                                 __shfl_sync(0xFFFFFFFFu, v.z, src), __shfl_sync(0xFFFFFFFFu, v.w, src)};
+#pragma unroll
+            for (int e = 0; e < 4; e++)
+                if (xs[e] >= thr) thr = warp_list_insert<KC>(wl, pack_key(xs[e], (uint32_t)(ns + e)), lane, thr);
+        }
+    };
+    // every lane of a warp runs the same number of steps (the votes); logits
+    // past the row end read as -inf (weight 0, ranked below every logit)
+    const float NI = -INFINITY;
+    if (!CAND) {
+        if (v4) {
+            for (int n = threadIdx.x; n < V / 4; n += NT) {
+                const float4 v = l4[n];
+                z += softmax_weight_fast(__fsub_rn(v.x, m)) + softmax_weight_fast(__fsub_rn(v.y, m)) +
+                     softmax_weight_fast(__fsub_rn(v.z, m)) + softmax_weight_fast(__fsub_rn(v.w, m));
+            }
+        } else {
+            for (int n = threadIdx.x; n < V; n += NT) z += softmax_weight_fast(__fsub_rn(l[n], m));
+        }
+    } else if (v4) {
+        // four loads in flight per lane before the (branchy) visits
+        const int n4 = V / 4;
+        for (int base = warp * 32; base < n4; base += 4 * NT) {
+            float4 v[4];
+#pragma unroll
+            for (int u = 0; u < 4; u++) {
+                const int n = base + u * NT + lane;
+                v[u] = n < n4 ? l4[n] : make_float4(NI, NI, NI, NI);
+            }
+#pragma unroll
+            for (int u = 0; u < 4; u++) visit4(v[u], 4 * (base + u * NT + lane));
+        }
+    } else {
+        for (int base = warp * 128; base < V; base += 4 * NT) {
+            const int n = base + 4 * lane;
+            visit4(make_float4(n < V ? l[n] : NI, n + 1 < V ? l[n + 1] : NI, n + 2 < V ? l[n + 2] : NI,
+                               n + 3 < V ? l[n + 3] : NI),
+                   n);
+        }
+    }
     z = warp_sum_ll(z);
     if (lane == 0) s_z[warp] = z;
+    if (CAND && lane < KC) s_wl[warp][lane] = wl;
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (!CAND && threadIdx.x == 0) {
         long long Z = 0;
-        for (int w = 0; w < BR_THREADS / 32; w++) Z += s_z[w];
-        // lambda = ln Z - 24 ln 2 (log of the normaliser of the 2^-24 weights)
+        for (int w = 0; w < NW; w++) Z += s_z[w];
         s_lam = __double2float_rn(__dadd_rn(log_own(__ll2double_rn(Z)), -0x1.0a2b23f3bab73p+4));
+        s_full = 1;
+    }
+    if (CAND && warp == 0) {
+        long long Z = 0;
+        for (int w = 0; w < NW; w++) Z += s_z[w];
+        // lambda = ln Z - 24 ln 2 (log of the normaliser of the 2^-24 weights)
+        const float lam = __double2float_rn(__dadd_rn(log_own(__ll2double_rn(Z)), -0x1.0a2b23f3bab73p+4));
+        // the row's KC best candidates: KC rounds of a maximum over the heads
+        // of the warps' lists (lane w < NW walks list w)
+        int head = 0;
+        unsigned long long cand = 0ull;  // lane j ends with the j-th best
+        for (int j = 0; j < KC; j++) {
+            const unsigned long long mine = lane < NW && head < KC ? s_wl[lane][head] : 0ull;
+            const unsigned long long best = warp_max_u64(mine);
+            if (mine == best && best != 0ull) head++;
+            if (lane == j) cand = best;
+        }
+        const int nc = V < KC ? V : KC;
+        const float cum = a.cum[r];
+        // final keys; lane KC-1 holds the lowest-ranked candidate
+        float sc = 0.0f;
+        unsigned long long fk = 0ull;
+        if (lane < nc) {
+            sc = __fadd_rn(cum, __fsub_rn(__fsub_rn(key_value(cand), m), lam));
+            fk = pack_key(sc, (uint32_t)(lb * V) + key_index(cand));
+        }
+        const float sc_last = __shfl_sync(0xFFFFFFFFu, sc, nc - 1);
+        // the k best final keys, best first
+        unsigned long long kth = 0ull;
+        for (int i = 0; i < k; i++) {
+            const unsigned long long best = warp_max_u64(fk);
+            if (fk == best) fk = 0ull;
+            if (lane == i) kth = best;
+        }
+        // every other element scores <= sc_last; it cannot displace the k-th
+        // key unless it can tie its score
+        const unsigned long long kk = __shfl_sync(0xFFFFFFFFu, kth, k - 1);
+        const bool exact = CAND && (nc == V || sc_last < key_value(kk));
+        if (exact && lane < k) out[lane] = kth;
+        if (lane == 0) {
+            s_full = !exact;
+            s_lam = lam;
+        }
     }
     __syncthreads();
+    if (!s_full) return;
+    // full scan of the scores (rare: a tie at the candidate boundary)
     const float lam = s_lam;
     const float cum = a.cum[r];
-    unsigned long long lst[KM];
+    unsigned long long top[KM];
 #pragma unroll
-    for (int i = 0; i < KM; i++) lst[i] = 0ull;
-    for (int n = threadIdx.x; n < V; n += BR_THREADS) {
-        float lp = __fsub_rn(__fsub_rn(l[n], m), lam);
-        float sc = __fadd_rn(cum, lp);
-        topk_insert<KM>(lst, k, pack_key(sc, (uint32_t)(lb * V + n)));
+    for (int i = 0; i < KM; i++) top[i] = 0ull;
+    for (int n = threadIdx.x; n < V; n += NT) {
+        const float lp = __fsub_rn(__fsub_rn(l[n], m), lam);
+        const float sc = __fadd_rn(cum, lp);
+        topk_insert<KM>(top, k, pack_key(sc, (uint32_t)(lb * V + n)));
     }
-    // block-wide selection of the k best: k rounds of a max over list heads
-    int head = 0;
-    for (int i = 0; i < k; i++) {
-        unsigned long long mine = 0ull;
-#pragma unroll
-        for (int h = 0; h < KM; h++)
-            if (h == head && h < k) mine = lst[h];
-        unsigned long long w = warp_max_u64(mine);
-        if (lane == 0) s_key[warp] = w;
-        __syncthreads();
-        unsigned long long best = s_key[0];
-        for (int j = 1; j < BR_THREADS / 32; j++) best = s_key[j] > best ? s_key[j] : best;
-        if (mine == best && best != 0ull) head++;
-        if (threadIdx.x == 0) out[i] = best;
-        __syncthreads();
-    }
+    block_select<KM, NT>(top, k, out, s_key);
 }
 
 // per sentence: best k of the k*k row candidates; reorder state
@@ -453,9 +611,17 @@ __global__ void __launch_bounds__(256) beam_select_kernel(BeamArgs a) {
 cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
     if (a.k < 1 || a.k > BEAM_MAX) return cudaErrorInvalidValue;
     int R = a.B * a.k;
-    if (a.k <= 4) launch_pdl(beam_rows_kernel<4>, R, BR_THREADS, 0, st, a);
-    else if (a.k <= 8) launch_pdl(beam_rows_kernel<8>, R, BR_THREADS, 0, st, a);
-    else launch_pdl(beam_rows_kernel<16>, R, BR_THREADS, 0, st, a);
+    // up to one row per SM: the plain scan (its simple loops keep more loads
+    // in flight per warp); more rows: the candidate pass
+    if (R <= 152) {
+        if (a.k <= 4) launch_pdl(beam_rows_kernel<4, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
+        else if (a.k <= 8) launch_pdl(beam_rows_kernel<8, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
+        else launch_pdl(beam_rows_kernel<16, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
+    } else {
+        if (a.k <= 4) launch_pdl(beam_rows_kernel<4, BR_THREADS, true>, R, BR_THREADS, 0, st, a);
+        else if (a.k <= 8) launch_pdl(beam_rows_kernel<8, BR_THREADS, true>, R, BR_THREADS, 0, st, a);
+        else launch_pdl(beam_rows_kernel<16, BR_THREADS, true>, R, BR_THREADS, 0, st, a);
+    }
     cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess) return err;
     size_t smem = (size_t)a.k * a.T * sizeof(int);
