@@ -351,7 +351,7 @@ def run_gpu(args):
 # DRAM bytes of one decode step (dram__bytes_read.sum + dram__bytes_write.sum
 # of its kernels, one ncu capture of this bench's command); only for the step
 # kernels they were taken on -- refresh whenever those kernels change
-STEP_TRAFFIC = {("small-b1-s10to50-greedy64", True): 10_560_256}
+STEP_TRAFFIC = {("small-b1-s10to50-greedy64", True): 10_582_950}
 
 
 def measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster):
