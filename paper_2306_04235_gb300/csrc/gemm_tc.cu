@@ -493,10 +493,278 @@ __global__ void codes_to_f16_tail(const int8_t *src, __half *dst, size_t from, s
 }
 
 // ---------------------------------------------------------------------------
+// Split-K over a thread-block cluster, for grids with few 128 x 64 tiles
+// (the few-hundred-row linears of a batched decode step).  The S CTAs of a
+// cluster share one output tile and take consecutive ranges of its k-blocks;
+// each range holds at most 16 k-blocks (1024 products), so a CTA's fp32
+// accumulator is an exact integer.  The partials are converted to int32 and
+// reduce-scattered through distributed shared memory: CTA c owns columns
+// [c BN/S, (c+1) BN/S) of the tile, receives every CTA's partial of them in
+// its slot array, adds them in int32 (exact: |acc| <= 2048 * 2^14) and runs
+// the linear's epilogue on (float)acc -- the correctly rounded accumulator,
+// as in the unsplit kernel.  Every thread of every CTA reaches the one
+// cluster barrier (also after a timed-out wait), and no CTA touches another's
+// shared memory after it.
+// ---------------------------------------------------------------------------
+constexpr int SK_BN = 64;
+constexpr int SK_STAGES = 6;
+
+template <int S>
+struct SkLayout {
+    static constexpr uint32_t A_BYTES = TC_BM * TC_BK * 2;
+    static constexpr uint32_t B_BYTES = SK_BN * TC_BK * 2;
+    static constexpr uint32_t OFF_B = SK_STAGES * A_BYTES;
+    static constexpr uint32_t OFF_RECV = OFF_B + SK_STAGES * B_BYTES;  // [S][128][BN/S] int32
+    static constexpr uint32_t RECV_BYTES = S * TC_BM * (SK_BN / S) * 4;
+    static constexpr uint32_t OFF_COLS = OFF_RECV + RECV_BYTES;          // [3][BN/S] fp32
+    static constexpr uint32_t OFF_BARS = OFF_COLS + 3 * (SK_BN / S) * 4;
+    static constexpr int NBARS = 2 * SK_STAGES + 2;                     // full[S], empty[S], acc_full, done
+    static constexpr uint32_t OFF_MISC = OFF_BARS + NBARS * 8;
+    static constexpr uint32_t BYTES = OFF_MISC + 16;
+    static constexpr size_t SMEM = 1024 + BYTES;
+};
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// shared::cluster address of the same offset in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t map_rank(uint32_t saddr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, int a, int b, int c, int d) {
+    asm volatile("st.shared::cluster.v4.s32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
+                 : "memory");
+}
+
+__device__ __forceinline__ void cluster_barrier() {
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
+// the two halves of a cluster barrier phase: every thread arrives once the
+// CTA is set up and waits before its first access to another CTA's memory
+// (all CTAs of the cluster have then started)
+__device__ __forceinline__ void cluster_arrive_relaxed() { asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire;" ::: "memory"); }
+
+template <int S>
+__global__ void __launch_bounds__(TC_THREADS, 1) linear_tc_sk(const __grid_constant__ CUtensorMap tmA,
+                                                              const __grid_constant__ CUtensorMap tmB, int M, int N,
+                                                              int K, Epi e, int *status) {
+    pdl_allow_next();
+    pdl_grid_wait();
+    using L = SkLayout<S>;
+    constexpr int SW = SK_BN / S;  // columns this CTA finishes
+    constexpr uint32_t IDESC = idesc_f16(TC_BM, SK_BN);
+    if (e.skip && *e.skip) return;  // one flag for every CTA of the grid
+
+    extern __shared__ uint8_t tc_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(tc_raw) + 1023) & ~(uintptr_t)1023);
+    float *c_sc = reinterpret_cast<float *>(sm + L::OFF_COLS), *c_b = c_sc + SW, *c_inv = c_b + SW;
+    const uint32_t bars = s_addr(sm + L::OFF_BARS);
+    auto full_bar = [&](int s) { return bars + 8u * s; };
+    auto empty_bar = [&](int s) { return bars + 8u * (SK_STAGES + s); };
+    const uint32_t accf_bar = bars + 8u * (2 * SK_STAGES), done_bar = accf_bar + 8u;
+    uint32_t *misc = reinterpret_cast<uint32_t *>(sm + L::OFF_MISC);  // [0] tmem base, [1] abort, [2] consumed
+    volatile uint32_t *abort_flag = misc + 1;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_rank();
+    const int tile = blockIdx.x / S;
+    const int mt = (M + TC_BM - 1) / TC_BM;
+    const int m0 = (tile % mt) * TC_BM, n0 = (tile / mt) * SK_BN;
+    const int nkb = (K + TC_BK - 1) / TC_BK;
+    const int per = (nkb + S - 1) / S;
+    const int kb0 = min(nkb, (int)rank * per), kb1 = min(nkb, kb0 + per);
+    const bool has_k = kb1 > kb0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < SK_STAGES; s++) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        mbar_init(accf_bar, 1);
+        mbar_init(done_bar, 1);
+        misc[1] = 0;
+        misc[2] = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+    }
+    if (warp == 1) {
+        tmem_alloc<SK_BN>(s_addr(misc));
+        tc_fence_before();
+    }
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tbase = misc[0];
+    cluster_arrive_relaxed();
+
+    uint32_t issued = 0;
+    if (warp == 0 && lane == 0) {
+        // ---- TMA producer: this CTA's k-blocks of the tile ----
+        const uint32_t a_ring = s_addr(sm), b_ring = s_addr(sm + L::OFF_B);
+        uint32_t it = 0;
+        for (int kb = kb0; kb < kb1; kb++, it++) {
+            const int s = (int)(it % SK_STAGES);
+            if (it >= SK_STAGES && !mbar_wait(empty_bar(s), (it / SK_STAGES - 1) & 1)) {
+                *abort_flag = 1;
+                set_status(status, MNMT_ETIMEOUT);
+                break;
+            }
+            mbar_expect_tx(full_bar(s), L::A_BYTES + L::B_BYTES);
+            tma_load_2d(a_ring + s * L::A_BYTES, &tmA, kb * TC_BK, m0, full_bar(s));
+            tma_load_2d(b_ring + s * L::B_BYTES, &tmB, kb * TC_BK, n0, full_bar(s));
+            issued = it + 1;
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---- MMA issuer: one accumulation over the range (<= 1024 products) ----
+        const uint64_t a_desc = sw128_desc(s_addr(sm)), b_desc = sw128_desc(s_addr(sm + L::OFF_B));
+        uint32_t it = 0;
+        for (int kb = kb0; kb < kb1; kb++, it++) {
+            const int s = (int)(it % SK_STAGES);
+            if (!mbar_wait(full_bar(s), (it / SK_STAGES) & 1)) {
+                *abort_flag = 1;
+                set_status(status, MNMT_ETIMEOUT);
+                break;
+            }
+            tc_fence_after();
+            const uint64_t ad = a_desc + (uint64_t)((s * L::A_BYTES) >> 4);
+            const uint64_t bd = b_desc + (uint64_t)((s * L::B_BYTES) >> 4);
+#pragma unroll
+            for (int k = 0; k < TC_BK / 16; k++)
+                mma_f16(tbase, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC, (uint32_t)(it | k));
+            mma_commit(empty_bar(s));
+        }
+        misc[2] = it;
+        mma_commit(accf_bar);  // also after a timed-out wait: the epilogue reaches the cluster barrier
+        mma_commit(done_bar);
+    }
+
+    // ---- epilogue warps: send the partials, then finish the owned columns ----
+    const int ew = warp - 2, q = warp & 3, half = ew >> 2;
+    const int row = m0 + 32 * q + lane;
+    const int oc = 16 * half;                          // owned chunk of this thread (within SW)
+    const int col0 = n0 + (int)rank * SW + oc;
+    const bool vec = epi_vec_ok(e);
+    const int t = e.t_ptr ? *e.t_ptr : 0;
+    float4 rpre[4];
+    bool pre = false;
+    if (warp >= 2) {
+        for (int i = ew * 32 + lane; i < SW; i += TC_EPI_WARPS * 32) {
+            const int n = n0 + (int)rank * SW + i;
+            const bool in = n < N;
+            c_sc[i] = in ? __fmul_rn(e.s_x, e.s_w[n]) : 0.0f;
+            c_b[i] = in ? e.bias[n] : 0.0f;
+            c_inv[i] = in && e.inv_out ? e.inv_out[n] : 0.0f;
+        }
+        pre = e.mode == EPI_RESID && vec && oc < SW && row < M && col0 + 16 <= N;
+        if (pre) {
+            const float4 *p = reinterpret_cast<const float4 *>(e.f32 + (size_t)row * e.ldf + col0);
+#pragma unroll
+            for (int g = 0; g < 4; g++) rpre[g] = p[g];
+        }
+        bool ok = *abort_flag == 0 && mbar_wait(accf_bar, 0);
+        if (!ok && *abort_flag == 0) {
+            *abort_flag = 1;
+            set_status(status, MNMT_ETIMEOUT);
+        }
+        tc_fence_after();
+        ok = __all_sync(0xFFFFFFFFu, ok && *abort_flag == 0);
+        cluster_wait();  // every CTA of the cluster has started
+        if (ok) {
+            const uint32_t taddr = tbase + ((uint32_t)(32 * q) << 16);
+            const uint32_t recv = s_addr(sm + L::OFF_RECV);
+#pragma unroll
+            for (int jj = 0; jj < 2; jj++) {
+                const int j = 2 * half + jj;  // 16-column chunk of the tile
+                int v[16];
+                if (has_k) {
+                    uint32_t r0[16];
+                    tmem_ld16(taddr + 16 * j, r0);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 16; i++) v[i] = __float2int_rn(__uint_as_float(r0[i]));  // exact integers
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 16; i++) v[i] = 0;
+                }
+                const int owner = (16 * j) / SW, cin = 16 * j - owner * SW;
+                const uint32_t dst = map_rank(recv + (uint32_t)(((rank * TC_BM + 32 * q + lane) * SW + cin) * 4),
+                                              (uint32_t)owner);
+#pragma unroll
+                for (int g = 0; g < 4; g++) st_cluster_v4(dst + 16 * g, v[4 * g], v[4 * g + 1], v[4 * g + 2], v[4 * g + 3]);
+            }
+        }
+        tc_fence_before();
+    }
+    if (warp < 2) cluster_wait();
+    // every thread of every CTA: the partials have landed in their owners
+    cluster_barrier();
+    if (warp >= 2 && oc < SW && *abort_flag == 0 && row < M && col0 < N) {
+        const int *rv = reinterpret_cast<const int *>(sm + L::OFF_RECV);
+        int acc[16];
+#pragma unroll
+        for (int i = 0; i < 16; i++) acc[i] = 0;
+#pragma unroll
+        for (int src = 0; src < S; src++) {
+            const int4 *p = reinterpret_cast<const int4 *>(rv + ((size_t)src * TC_BM + 32 * q + lane) * SW + oc);
+#pragma unroll
+            for (int g = 0; g < 4; g++) {
+                const int4 w = p[g];
+                acc[4 * g] += w.x;
+                acc[4 * g + 1] += w.y;
+                acc[4 * g + 2] += w.z;
+                acc[4 * g + 3] += w.w;
+            }
+        }
+        float a[16];
+#pragma unroll
+        for (int i = 0; i < 16; i++) a[i] = __int2float_rn(acc[i]);  // fl(acc), as the unsplit kernel
+        const float *sc = c_sc + oc, *bs = c_b + oc, *inv = c_inv + oc;
+        if (e.mode == EPI_ARGMAX) {
+            unsigned long long best = 0ull;
+#pragma unroll
+            for (int i = 0; i < 16; i++) {
+                if (col0 + i < N) {
+                    const float y = __fadd_rn(__fmul_rn(a[i], sc[i]), bs[i]);
+                    const unsigned long long kk = pack_key(y, (uint32_t)(col0 + i));
+                    best = kk > best ? kk : best;
+                }
+            }
+            if (best) atomicMax(e.keys + row, best);
+        } else if (vec && col0 + 16 <= N) {
+            epi_store16(e, row, col0, a, sc, bs, inv, t, pre ? rpre : nullptr);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 16; i++)
+                if (col0 + i < N) epi_store_f(e, row, col0 + i, a[i], t);
+        }
+    }
+
+    // ---- teardown ----
+    __syncthreads();
+    if (warp == 0 && lane == 0 && *abort_flag) {
+        for (uint32_t it = misc[2]; it < issued; it++) mbar_wait(full_bar((int)(it % SK_STAGES)), (it / SK_STAGES) & 1);
+    }
+    if (warp == 1) {
+        if (lane == 0) mbar_wait(done_bar, 0);
+        __syncwarp();
+        tc_fence_after();
+        tmem_free<SK_BN>(tbase);
+    }
+}
+
+// ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 int g_num_sms = 148;
+int g_sk_clusters[5] = {0, 0, 0, 0, 0};  // clusters of S split-K CTAs that fit at once (S = 2, 4)
 
 bool make_map(CUtensorMap *tm, const __half *p, int cols, int rows, int ld, int box_rows) {
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
@@ -522,6 +790,50 @@ cudaError_t tc_launch(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N
     const int grid = (int)(tiles < g_num_sms ? tiles : g_num_sms);
     launch_pdl(linear_tc<BN, NCH, STAGES, NBUF>, grid, TC_THREADS, TcLayout<BN, STAGES>::SMEM, st, ta, tb, M, N, K, e, status);
     return cudaGetLastError();
+}
+
+// cluster attribute (S, 1, 1) and programmatic dependent launch outside
+// stream captures, as launch_pdl
+template <int S>
+cudaLaunchConfig_t sk_config(long tiles, cudaStream_t st, cudaLaunchAttribute (&attr)[2], bool pdl) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)(tiles * S));
+    cfg.blockDim = dim3(TC_THREADS);
+    cfg.dynamicSmemBytes = SkLayout<S>::SMEM;
+    cfg.stream = st;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl ? 2 : 1;
+    return cfg;
+}
+
+template <int S>
+cudaError_t tc_sk_init() {
+    cudaError_t err = cudaFuncSetAttribute(linear_tc_sk<S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)SkLayout<S>::SMEM);
+    if (err != cudaSuccess) return err;
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = sk_config<S>(64, nullptr, attr, false);
+    int n = 0;
+    err = cudaOccupancyMaxActiveClusters(&n, linear_tc_sk<S>, &cfg);
+    g_sk_clusters[S] = err == cudaSuccess ? n : 0;
+    return err;
+}
+
+template <int S>
+cudaError_t tc_launch_sk(const CUtensorMap &ta, const CUtensorMap &tb, int M, int N, int K, const Epi &e, int *status,
+                         cudaStream_t st) {
+    const long tiles = (long)((M + TC_BM - 1) / TC_BM) * ((N + SK_BN - 1) / SK_BN);
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) cs = cudaStreamCaptureStatusNone;
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = sk_config<S>(tiles, st, attr, cs != cudaStreamCaptureStatusActive);
+    return cudaLaunchKernelEx(&cfg, linear_tc_sk<S>, ta, tb, M, N, K, e, status);
 }
 
 constexpr int TC_STAGES = 6;
@@ -551,6 +863,8 @@ cudaError_t linear_tc_init() {
     if (err == cudaSuccess) err = tc_attr<256, 2, TC_STAGES_WIDE, 1>();
     if (err == cudaSuccess) err = tc_attr<64, 1, TC_STAGES_NARROW, 2>();
     if (err == cudaSuccess) err = tc_attr<64, 2, TC_STAGES_NARROW, 2>();
+    if (err == cudaSuccess) err = tc_sk_init<2>();
+    if (err == cudaSuccess) err = tc_sk_init<4>();
     return err;
 }
 
@@ -571,6 +885,17 @@ cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int 
     CUtensorMap ta, tb;
     if (!make_map(&ta, A16, K, M, lda, TC_BM) || !make_map(&tb, W16, K, N, ldw, wide ? 256 : (narrow ? 64 : 128)))
         return cudaErrorInvalidValue;
+    if (narrow) {
+        // split K over a cluster when the 128 x 64 tiles leave SMs idle: S CTAs
+        // per tile, each with at most 16 k-blocks (one exact chunk); K of at
+        // least 8 k-blocks (measured: splitting 4 k-blocks in two was slower)
+        const long tiles64 = (long)((M + TC_BM - 1) / TC_BM) * ((N + SK_BN - 1) / SK_BN);
+        const int nkb = (K + TC_BK - 1) / TC_BK;
+        if (nkb >= 8 && tiles64 * 4 <= g_num_sms && tiles64 <= g_sk_clusters[4])
+            return tc_launch_sk<4>(ta, tb, M, N, K, e, status, st);
+        if (nkb >= 8 && nkb <= 32 && tiles64 * 2 <= g_num_sms && tiles64 <= g_sk_clusters[2])
+            return tc_launch_sk<2>(ta, tb, M, N, K, e, status, st);
+    }
     if (narrow && two_chunks) return tc_launch<64, 2, TC_STAGES_NARROW, 2>(ta, tb, M, N, K, e, status, st);
     if (narrow) return tc_launch<64, 1, TC_STAGES_NARROW, 2>(ta, tb, M, N, K, e, status, st);
     if (wide && two_chunks) return tc_launch<256, 2, TC_STAGES_WIDE, 1>(ta, tb, M, N, K, e, status, st);
