@@ -49,6 +49,21 @@ def test_small_models_match_oracle(kind, beam, stream):
     assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
 
 
+@pytest.mark.parametrize("kind,beam", [("fact", 4), ("pre", 3)])
+def test_many_sentences_beam_search_matches_oracle(kind, beam, stream):
+    """80 sentences: enough that the cross attention serves all beams of a
+    sentence from one block (the batched-beam layout)."""
+    cfg = MINI[kind]
+    blob = synth.build_blob(cfg, 31, gamma_range=(0.5, 1.5))
+    ids, lens = synth.source_batch(cfg.vocab, 80, 1, 30, 32)
+    T = 12
+    g_ids, g_len, g_sc = _gpu(blob, ids, lens, beam, T, stream)
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, beam, T, n_threads=8)
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_len, o_len)
+    assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
+
+
 def test_tiny_workload_tokens_and_taps(stream):
     cfg, blob, ids, lens, beam, T = synth.workload_inputs("tiny-b1-s16-greedy16")
     d, H, L = cfg.d_model, cfg.n_heads, cfg.n_dec
