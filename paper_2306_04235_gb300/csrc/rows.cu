@@ -17,13 +17,11 @@ namespace mnmt {
 // LayerNorm kernel: one block of LN_T threads per row, thread t holding the
 // VPT contiguous elements t*VPT ..  The row is short (d <= 2048) and a decode
 // step has only a few hundred rows, so the work of a row is spread over four
-// warps to shorten each thread's dependent chain; the order-free maxima and
+// or eight warps to shorten each thread's dependent chain; the order-free maxima and
 // exact fixed-point sums combine across warps through shared memory.  The
 // row, gamma and beta are loaded together before the skip flag is tested.
 // ---------------------------------------------------------------------------
-constexpr int LN_T = 128;
-
-template <int VPT>
+template <int VPT, int LN_T>
 __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     pdl_allow_next();
     pdl_grid_wait();
@@ -111,16 +109,23 @@ __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     }
 }
 
-cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
-    if (a.M <= 0) return cudaSuccess;
+template <int LN_T>
+cudaError_t launch_layernorm_t(const LnArgs &a, cudaStream_t st) {
     const int vpt = (a.d + LN_T - 1) / LN_T;
-    if (vpt <= 1) launch_pdl(layernorm_kernel<1>, a.M, LN_T, 0, st, a);
-    else if (vpt <= 2) launch_pdl(layernorm_kernel<2>, a.M, LN_T, 0, st, a);
-    else if (vpt <= 4) launch_pdl(layernorm_kernel<4>, a.M, LN_T, 0, st, a);
-    else if (vpt <= 8) launch_pdl(layernorm_kernel<8>, a.M, LN_T, 0, st, a);
-    else if (vpt <= 16) launch_pdl(layernorm_kernel<16>, a.M, LN_T, 0, st, a);
+    if (vpt <= 1) launch_pdl(layernorm_kernel<1, LN_T>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 2) launch_pdl(layernorm_kernel<2, LN_T>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 4) launch_pdl(layernorm_kernel<4, LN_T>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 8) launch_pdl(layernorm_kernel<8, LN_T>, a.M, LN_T, 0, st, a);
+    else if (vpt <= 16) launch_pdl(layernorm_kernel<16, LN_T>, a.M, LN_T, 0, st, a);
     else return cudaErrorInvalidValue;
     return cudaGetLastError();
+}
+
+// a decode step's few hundred rows: 256 threads per row (shorter chains);
+// an encoder's thousands: 128 (measured on the 512-row and 16384-row cases)
+cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
+    if (a.M <= 0) return cudaSuccess;
+    return a.M <= 1024 ? launch_layernorm_t<256>(a, st) : launch_layernorm_t<128>(a, st);
 }
 
 // ---------------------------------------------------------------------------
