@@ -478,7 +478,8 @@ struct mnmt_session {
     float *out_scores;
     unsigned long long *keys, *cand;
     int *state;
-    int *h_state = nullptr;  // pinned mirror of state
+    int *h_state = nullptr;  // pinned mirror of state, then a second slot for the look-ahead copy
+    cudaEvent_t ev_look = nullptr;  // marks the look-ahead copy of translate's decode loop
     size_t ck_layer, sk_layer;  // per-layer strides of the caches (elements)
     cudaGraphExec_t gexec = nullptr;
     cudaGraphExec_t gexec_n = nullptr;  // GRAPH_STEPS consecutive steps (cluster path)
@@ -546,10 +547,16 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
         delete s;
         return fail(MNMT_ENOMEM, "cudaMalloc of %zu session bytes failed", off);
     }
-    if (cudaMallocHost(&s->h_state, ST_N * 4) != cudaSuccess) {
+    if (cudaMallocHost(&s->h_state, 2 * ST_N * 4) != cudaSuccess) {
         cudaFree(s->arena);
         delete s;
         return fail(MNMT_ENOMEM, "pinned host allocation failed");
+    }
+    if (cudaEventCreateWithFlags(&s->ev_look, cudaEventDisableTiming) != cudaSuccess) {
+        cudaFreeHost(s->h_state);
+        cudaFree(s->arena);
+        delete s;
+        return fail(MNMT_ECUDA, "event creation failed");
     }
     uint8_t *a = s->arena;
     s->resid = reinterpret_cast<float *>(a + o_resid);
@@ -605,6 +612,7 @@ extern "C" void mnmt_session_free(mnmt_session *s) {
     if (s->gexec_n) cudaGraphExecDestroy(s->gexec_n);
     if (s->arena) cudaFree(s->arena);
     if (s->h_state) cudaFreeHost(s->h_state);
+    if (s->ev_look) cudaEventDestroy(s->ev_look);
     delete s;
 }
 
@@ -1248,16 +1256,25 @@ extern "C" int mnmt_translate(mnmt_session *s, const int32_t *src_ids, const int
     s->h_state[ST_TMAX] = max_len;
     CK(cudaMemcpyAsync(s->state + ST_TMAX, s->h_state + ST_TMAX, 4, cudaMemcpyHostToDevice, st));
     if ((rc = ensure_graph(s))) return poison(s, rc);
+    // Chunks of GRAPH_STEPS steps with one chunk of look-ahead: a copy of the
+    // state after the chunks queued so far is taken, the next chunk is queued,
+    // and only then is the copy read, so the device never waits for the host.
+    // Steps queued after every hypothesis finished are no-ops (each step
+    // kernel tests the done flag).
     const int CHECK = GRAPH_STEPS;
-    int steps = 0;
+    int steps = max_len < CHECK ? max_len : CHECK;
+    if ((rc = launch_steps(s, steps))) return poison(s, rc);
+    int *look = s->h_state + ST_N;
     while (steps < max_len) {
-        int n = max_len - steps < CHECK ? max_len - steps : CHECK;
+        CK(cudaMemcpyAsync(look, s->state, ST_N * 4, cudaMemcpyDeviceToHost, st));
+        CK(cudaEventRecord(s->ev_look, st));
+        const int n = max_len - steps < CHECK ? max_len - steps : CHECK;
         if ((rc = launch_steps(s, n))) return poison(s, rc);
         steps += n;
-        if (steps < max_len) {
-            if ((rc = sync_state(s))) return rc;
-            if (s->h_state[ST_DONE]) break;
-        }
+        const cudaError_t e = cudaEventSynchronize(s->ev_look);
+        if (e != cudaSuccess) return poison(s, fail(MNMT_ECUDA, "device work failed: %s", cudaGetErrorString(e)));
+        if (look[ST_STATUS]) return poison(s, fail(look[ST_STATUS], "device reported status %d", look[ST_STATUS]));
+        if (look[ST_DONE]) break;
     }
     s->steps = steps;
     const bool dev = flags & MNMT_DEVICE_PTRS;
