@@ -160,9 +160,10 @@ __global__ void __launch_bounds__(XS ? 32 * 32 : 32 * 16) attn_decode(AttnDecArg
 cudaError_t launch_attention_decode(const AttnDecArgs &a, cudaStream_t st) {
     if (a.H > 16 || a.T < 1 || a.T > DEC_MAX_KEYS) return cudaErrorInvalidValue;
     // cross attention with beams: the beams of a sentence share a block, when
-    // there are sentences enough for half of the 152 SMs (measured: +3.8 us per
-    // step at 128 sentences, -1.7 us at 32, where the blocks were too few)
-    const bool xs = a.cross && a.beam > 1 && a.beam * a.H <= 32 && a.R % a.beam == 0 && a.R / a.beam >= 76;
+    // there are sentences enough for half of the SMs (measured on 152 SMs:
+    // 3.8 us per step faster at 128 sentences, 1.7 us slower at 32)
+    const bool xs = a.cross && a.beam > 1 && a.beam * a.H <= 32 && a.R % a.beam == 0 &&
+                    2 * (a.R / a.beam) >= device_sm_count();
     const size_t smem = (size_t)(xs ? a.beam * a.H : 1 + a.H) * a.T * sizeof(int);
     const dim3 block(32 * a.H * (xs ? a.beam : 1));
     const int grid = xs ? a.R / a.beam : a.R;

@@ -868,6 +868,8 @@ cudaError_t linear_tc_init() {
     return err;
 }
 
+int device_sm_count() { return g_num_sms; }
+
 bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16) {
     return g_encode && M >= 1 && N >= 1 && K >= 8 && K <= 2 * TC_KB_PER_CHUNK * TC_BK && K % 8 == 0 && lda >= K &&
            ldw >= K && lda % 8 == 0 && ldw % 8 == 0 && ((reinterpret_cast<uintptr_t>(A16) | reinterpret_cast<uintptr_t>(W16)) & 15) == 0;

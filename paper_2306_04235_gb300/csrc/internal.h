@@ -81,6 +81,7 @@ cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int 
 // W16 [N][ldw]; K <= 2048 and a multiple of 8; *status (device, may be null)
 // receives MNMT_ETIMEOUT if a pipeline wait runs out
 cudaError_t linear_tc_init();
+int device_sm_count();  // SMs of the current device (read by linear_tc_init)
 bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16);
 cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int ldw, int M, int N, int K,
                              const Epi &e, int *status, cudaStream_t st);

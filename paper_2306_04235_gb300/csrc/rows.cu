@@ -618,7 +618,7 @@ cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
     int R = a.B * a.k;
     // up to one row per SM: the plain scan (its simple loops keep more loads
     // in flight per warp); more rows: the candidate pass
-    if (R <= 152) {
+    if (R <= device_sm_count()) {
         if (a.k <= 4) launch_pdl(beam_rows_kernel<4, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
         else if (a.k <= 8) launch_pdl(beam_rows_kernel<8, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
         else launch_pdl(beam_rows_kernel<16, BR_THREADS, false>, R, BR_THREADS, 0, st, a);
