@@ -23,6 +23,9 @@
 //                   32*(w%4)..+31 = tile rows, half of the columns) and apply
 //                   the fused epilogue of the linear while the MMAs of the
 //                   next tile fill the other buffer.
+// Grids of few 128 x 64 tiles run linear_tc_sk instead: the same pipeline for
+// one tile per CTA, K split over a 2- or 4-CTA cluster, the partials reduced
+// exactly in int32 through distributed shared memory (see its header).
 // Every mbarrier wait is bounded (one second of %globaltimer); a wait that
 // runs out records MNMT_ETIMEOUT in *status, the CTA stops issuing work, waits
 // (bounded) for its own copies and MMAs in flight, frees its TMEM and returns.
