@@ -230,6 +230,14 @@ int mnmt_linear_tc(const uint16_t *A16, const uint16_t *W16, const float *s_w, c
  * pointers, src and dst 16-byte aligned. */
 int mnmt_codes_to_f16(const int8_t *src, uint16_t *dst, size_t n, void *cuda_stream);
 
+/* Diagnostic of the bounded waits of the tensor-core pipelines: one thread
+ * block waits on a shared-memory transaction barrier that nothing completes.
+ * The wait gives up after one second (the limit of every such wait in
+ * mnmt_linear_tc), the kernel records MNMT_ETIMEOUT in *status (device int32,
+ * required) and returns; no fault is raised and the context stays usable.
+ * Returns once the kernel is queued. */
+int mnmt_wait_timeout_selftest(int32_t *status, void *cuda_stream);
+
 /* Output-vocabulary projection fused with greedy selection (App. D): for each
  * row m, keys[m] = max over n of pack(y[m][n], n) with y as in mnmt_linear and
  * pack(y, n) = (ord(y) << 32) | (0xFFFFFFFF - n), where ord maps fp32 to uint32

@@ -1475,6 +1475,15 @@ extern "C" int mnmt_codes_to_f16(const int8_t *src, uint16_t *dst, size_t n, voi
     return MNMT_OK;
 }
 
+extern "C" int mnmt_wait_timeout_selftest(int32_t *status, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!status) return fail(MNMT_EINVAL, "wait_timeout_selftest: status is required");
+    cudaError_t err = launch_wait_timeout_selftest(status, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "wait_timeout_selftest launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
 extern "C" int mnmt_linear_argmax(const int8_t *A, const int8_t *W, const float *s_w, const float *bias,
                                   float s_x, int32_t M, int32_t N, int32_t K, uint64_t *keys, void *cuda_stream) {
     int rc = lib_init();

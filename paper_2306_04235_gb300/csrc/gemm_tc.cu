@@ -762,6 +762,19 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc_sk(const __grid_const
     }
 }
 
+// One thread waits (bounded) on a barrier phase that never completes: the
+// give-up path of every pipeline wait above, exercised without a fault.
+__global__ void wait_timeout_selftest_kernel(int *status) {
+    __shared__ __align__(8) unsigned long long bar;
+    const uint32_t b = s_addr(&bar);
+    if (threadIdx.x == 0) {
+        mbar_init(b, 1);  // one arrival expected; none comes
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait(b, 0)) set_status(status, MNMT_ETIMEOUT);
+}
+
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
@@ -872,6 +885,11 @@ cudaError_t linear_tc_init() {
 }
 
 int device_sm_count() { return g_num_sms; }
+
+cudaError_t launch_wait_timeout_selftest(int *status, cudaStream_t st) {
+    wait_timeout_selftest_kernel<<<1, 32, 0, st>>>(status);
+    return cudaGetLastError();
+}
 
 bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16) {
     return g_encode && M >= 1 && N >= 1 && K >= 8 && K <= 2 * TC_KB_PER_CHUNK * TC_BK && K % 8 == 0 && lda >= K &&

@@ -82,6 +82,7 @@ cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int 
 // receives MNMT_ETIMEOUT if a pipeline wait runs out
 cudaError_t linear_tc_init();
 int device_sm_count();  // SMs of the current device (read by linear_tc_init)
+cudaError_t launch_wait_timeout_selftest(int *status, cudaStream_t st);
 bool linear_tc_shape_ok(int M, int N, int K, int lda, int ldw, const void *A16, const void *W16);
 cudaError_t launch_linear_tc(const __half *A16, int lda, const __half *W16, int ldw, int M, int N, int K,
                              const Epi &e, int *status, cudaStream_t st);

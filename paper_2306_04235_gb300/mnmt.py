@@ -78,9 +78,10 @@ def _declare(L):
     L.mnmt_layernorm.argtypes = [p, p, p, i32, i32, f, p, p, p, p]
     L.mnmt_linear_tc.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p, p]
     L.mnmt_codes_to_f16.argtypes = [p, p, sz, p]
+    L.mnmt_wait_timeout_selftest.argtypes = [p, p]
     for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
               "mnmt_decode_step", "mnmt_translate", "mnmt_linear", "mnmt_linear_argmax", "mnmt_attention_decode", "mnmt_layernorm",
-              "mnmt_linear_tc", "mnmt_codes_to_f16"]:
+              "mnmt_linear_tc", "mnmt_codes_to_f16", "mnmt_wait_timeout_selftest"]:
         getattr(L, n).restype = C.c_int
 
 
@@ -216,6 +217,11 @@ def mnmt_linear_tc(A16, W16, s_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_
 def mnmt_codes_to_f16(src, dst, n, stream=None):
     """dst[i] = fp16(src[i]) for n int8 codes (device buffers)."""
     _chk(lib().mnmt_codes_to_f16(_ptr(src), _ptr(dst), n, _stream_handle(stream)))
+
+
+def mnmt_wait_timeout_selftest(status, stream=None):
+    """Queue one block whose barrier wait runs out (one second): *status -> ETIMEOUT."""
+    _chk(lib().mnmt_wait_timeout_selftest(_ptr(status), _stream_handle(stream)))
 
 
 def argmax_from_keys(keys: np.ndarray) -> np.ndarray:

@@ -3,6 +3,8 @@ through the C ABI (mnmt_codes_to_f16, mnmt_linear_tc).  The int8 codes travel
 as fp16 and the fp32 accumulation is exact per chunk of 1024 products, so every
 output must equal the oracle's int32-accumulator result bit for bit (Sec. 3.3,
 Eq. 3 and the Fig. 5 epilogues)."""
+import time
+
 import numpy as np
 import pytest
 
@@ -170,3 +172,18 @@ def test_linear_tc_wide_tiles_sampled(M, N, K, mode):
     ref = O.linear(A[rows], W, s_w, b, s_x, mode, inv_out=inv, gamma=np.float32(0.875),
                    resid=None if resid is None else resid[rows])
     assert _same(got[rows], ref)
+
+
+def test_bounded_wait_gives_up_with_status():
+    """The give-up path of the pipelines' barrier waits: a wait that nothing
+    completes returns after its one-second limit with MNMT_ETIMEOUT in the
+    status word (no fault), and the device keeps working: a linear launched
+    afterwards is still exact."""
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    t0 = time.perf_counter()
+    mnmt.mnmt_wait_timeout_selftest(status)
+    assert host(status)[0] == mnmt.ETIMEOUT
+    assert 0.5 < time.perf_counter() - t0 < 60
+    A, W, s_w, b, inv, s_x = _inputs(5, 200, 96, 512)
+    got = _tc(A, W, s_w, b, inv, s_x, mnmt.EPI_Q8)
+    assert _same(got, O.linear(A, W, s_w, b, s_x, mnmt.EPI_Q8, inv_out=inv))
