@@ -322,7 +322,9 @@ def run_gpu(args):
                    "kind": "oracle",
                    "sample": f"{n_sent} translation(s) of {wl.batch} sentence(s) drawn like the workload, "
                              f"one per thread ({cdt:.1f} s)"}
-        launched = min(T, -(-steps_run // 16) * 16)  # the host checks for completion every 16 steps
+        # translate queues steps in chunks of 16 with one chunk of look-ahead:
+        # a translation that finishes early has one more (no-op) chunk queued
+        launched = T if steps_run >= T else min(T, -(-steps_run // 16) * 16 + 16)
         launches = kernels_per_translation(cfg, B, S, wl.beam, launched, cluster) * args.steps
         line = {
             "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
