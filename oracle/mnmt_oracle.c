@@ -635,6 +635,21 @@ static int decode_step(const omodel *m, const oenc *enc, ocache *cache, int tok,
 /* search                                                                    */
 /* ------------------------------------------------------------------------ */
 
+/* Normaliser of the beam search's log-softmax over one logit row (App. D
+ * decodes with log-probabilities; their arithmetic is unstated): m = max_n l[n]
+ * (order-free), fixed-point weights E_n = rne(exp(fl(l[n] - m)) 2^24) summed
+ * exactly as Z = sum E_n, and lambda = fl32(ln Z - 24 ln 2), i.e. the natural
+ * log of the sum of exp(l[n] - m) on the 2^-24 grid.  Returns Z. */
+static int64_t log_softmax_norm(const float *l, int V, float *m_out, float *lam_out) {
+    float mx = l[0];
+    for (int n = 1; n < V; n++) if (l[n] > mx) mx = l[n];
+    int64_t Z = 0;
+    for (int n = 0; n < V; n++) Z += (int64_t)rintf(exp_own(l[n] - mx) * 16777216.0f);
+    *m_out = mx;
+    *lam_out = (float)(log_own((double)Z) - 0x1.0a2b23f3bab73p+4); /* 24 ln 2 */
+    return Z;
+}
+
 /* greedy: argmax, ties to the lowest id */
 static int argmax_f(const float *l, int V) {
     int best = 0;
@@ -754,12 +769,8 @@ static int beam_one(const omodel *m, const oenc *enc, int k, int max_len, int32_
                 continue;
             }
             if ((st = decode_step(m, enc, &cache[i], tok[i], t, &w, logits, NULL))) goto done_w;
-            /* log-softmax: m = max, Z = sum rne(exp(l - m) 2^24), lambda = ln Z - 24 ln 2 */
-            float mx = logits[0];
-            for (int n = 1; n < V; n++) if (logits[n] > mx) mx = logits[n];
-            int64_t Z = 0;
-            for (int n = 0; n < V; n++) Z += (int64_t)rintf(exp_own(logits[n] - mx) * 16777216.0f);
-            float lam = (float)(log_own((double)Z) - 0x1.0a2b23f3bab73p+4);
+            float mx, lam;
+            log_softmax_norm(logits, V, &mx, &lam);
             for (int n = 0; n < V; n++) {
                 float lp = (logits[n] - mx) - lam;
                 ocand cd = {cum[i] + lp, (int64_t)i * V + n};
@@ -1079,14 +1090,19 @@ int oracle_embed(const void *blob, size_t bytes, const int32_t *ids, const int32
     return st;
 }
 
-/* Beam-search log-probabilities of one logit row: lp[n] = fl(fl(l - m) - lambda). */
+/* Beam-search log-probabilities of one logit row: lp[n] = fl(fl(l - m) - lambda),
+ * with m and lambda from log_softmax_norm (the function beam_one uses). */
 int oracle_log_softmax(const float *l, int V, float *lp) {
-    float mx = l[0];
-    for (int n = 1; n < V; n++) if (l[n] > mx) mx = l[n];
-    int64_t Z = 0;
-    for (int n = 0; n < V; n++) Z += (int64_t)rintf(exp_own(l[n] - mx) * 16777216.0f);
-    float lam = (float)(log_own((double)Z) - 0x1.0a2b23f3bab73p+4);
+    float mx, lam;
+    log_softmax_norm(l, V, &mx, &lam);
     for (int n = 0; n < V; n++) lp[n] = (l[n] - mx) - lam;
+    return OR_OK;
+}
+
+/* The normaliser alone: *m = max_n l[n], *lam = lambda, *Z = the fixed-point sum. */
+int oracle_log_softmax_norm(const float *l, int V, float *m, float *lam, int64_t *Z) {
+    int64_t z = log_softmax_norm(l, V, m, lam);
+    if (Z) *Z = z;
     return OR_OK;
 }
 

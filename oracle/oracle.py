@@ -68,10 +68,12 @@ def _declare(L):
     L.oracle_decode_forced.argtypes = [_p, _sz, _p, _i, _i, _p, _i, _p]
     L.oracle_embed.argtypes = [_p, _sz, _p, _p, _i, _p]
     L.oracle_log_softmax.argtypes = [_p, _i, _p]
+    L.oracle_log_softmax_norm.argtypes = [_p, _i, _p, _p, _p]
     L.oracle_translate.argtypes = [_p, _sz, _p, _p, _i, _i, _i, _i, _i, _p, _p, _p]
     for name in ["oracle_check_blob", "oracle_linear", "oracle_layernorm", "oracle_attention_decode",
                  "oracle_attention_probs", "oracle_encode", "oracle_decode_trace",
-                 "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_translate"]:
+                 "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_log_softmax_norm",
+                 "oracle_translate"]:
         getattr(L, name).restype = _i
 
 
@@ -223,6 +225,14 @@ def log_softmax(l):
     lp = np.zeros_like(l)
     _chk(lib().oracle_log_softmax(_ptr(l), l.shape[0], _ptr(lp)))
     return lp
+
+
+def log_softmax_norm(l):
+    """(m, lambda, Z) of the beam search's log-softmax of one logit row."""
+    l = np.ascontiguousarray(l, np.float32)
+    m = np.zeros(1, np.float32); lam = np.zeros(1, np.float32); Z = np.zeros(1, np.int64)
+    _chk(lib().oracle_log_softmax_norm(_ptr(l), l.shape[0], _ptr(m), _ptr(lam), _ptr(Z)))
+    return float(m[0]), float(lam[0]), int(Z[0])
 
 
 def translate(blob, src, lens, beam, max_len, n_threads=1):

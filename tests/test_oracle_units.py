@@ -256,3 +256,85 @@ def test_attention_weights_are_nearest_float_of_exact_quotient(n, sigma):
     P = O.attention_probs(q, K, sigma)
     for j in range(n):
         assert P[j] == _nearest_f32(Fraction(E[j], Z)), j
+
+
+# ------------------------------------------------- beam log-softmax normaliser
+def _lse64(l):
+    l = l.astype(np.float64)
+    m = l.max()
+    return m + math.log(np.exp(l - m).sum())
+
+
+def _lp_tolerance(l, lp, Z):
+    """Bound of |lp - (l - logsumexp(l))| implied by the definition: the weights
+    E_n = rne(exp_own(x) 2^24) carry exp_own's 2-ulp relative error and at most
+    1/2 absolute rounding each, so ln Z is within (2^-21 Z + V/2) / Z of the
+    exact value; fl32(lambda) adds half an ulp of lambda; fl(l - m) and
+    fl(. - lambda) one half-ulp each."""
+    V = l.shape[0]
+    m = float(l.max())
+    dlnz = (2.0 ** -21 * Z + 0.5 * V) / Z + 1e-14
+    lam = math.log(Z) - 24 * math.log(2.0)
+    return dlnz + 2.0 ** -24 * (abs(lam) + np.abs(l.astype(np.float64) - m) + np.abs(lp.astype(np.float64)))
+
+
+@pytest.mark.parametrize("V,scale", [(8000, 0.1), (8000, 3.0), (32000, 0.1), (32000, 3.0), (32000, 30.0),
+                                     (4, 1.0), (300, 10.0)])
+def test_log_softmax_vs_float64(V, scale):
+    """lp[n] = fl(fl(l - m) - lambda) against float64 l - logsumexp(l); a wrong
+    constant (log2 for ln, a dropped 24 ln 2, a sign) is off by >= 0.3."""
+    for row in range(3):
+        l = (synth.Stream(V + row, "logit").normal(V) * scale).astype(np.float32)
+        lp = O.log_softmax(l)
+        ref = l.astype(np.float64) - _lse64(l)
+        m, lam, Z = O.log_softmax_norm(l)
+        assert m == float(l.max())
+        tol = _lp_tolerance(l, lp, Z)
+        assert np.all(np.abs(lp - ref) <= tol), float(np.max(np.abs(lp - ref) - tol))
+        # probabilities sum to one (to the same bound)
+        assert abs(math.log(np.exp(lp.astype(np.float64)).sum())) <= float(np.max(tol)) * 1.01
+
+
+def test_log_softmax_equal_row_is_minus_ln_v():
+    """All logits equal: every weight is exactly 2^24, Z = V 2^24, lambda = ln V."""
+    for V in (4, 8000, 32000):
+        l = np.full(V, 1.375, np.float32)
+        m, lam, Z = O.log_softmax_norm(l)
+        assert Z == V * 2 ** 24
+        assert abs(lam - math.log(V)) <= ulp32(math.log(V))
+        lp = O.log_softmax(l)
+        assert np.all(lp == np.float32(-lam))
+
+
+def test_log_softmax_spikes():
+    """One logit far above the rest: Z = 2^24, lambda = 0 (to double rounding),
+    lp = 0 at the spike and l - m elsewhere; two equal spikes: lambda = ln 2."""
+    l = np.full(32000, -50.0, np.float32); l[123] = 60.0
+    m, lam, Z = O.log_softmax_norm(l)
+    assert Z == 2 ** 24 and abs(lam) <= 1e-14
+    lp = O.log_softmax(l)
+    assert abs(float(lp[123])) <= 1e-14 and np.all(lp[np.arange(32000) != 123] == np.float32(-110.0))
+    l[9] = 60.0
+    m, lam, Z = O.log_softmax_norm(l)
+    assert Z == 2 ** 25 and lam == f32(math.log(2.0))
+    lp = O.log_softmax(l)
+    assert lp[9] == lp[123] == np.float32(-f32(math.log(2.0)))
+
+
+def test_beam_search_scores_use_the_pinned_log_softmax():
+    """The cumulative score of a beam-1 search is the sum of the pinned
+    log-probabilities of its own tokens along the teacher-forced trace."""
+    cfg = synth.ModelConfig(1, 1, 64, 2, 128, 300, 64, 1, 1, max_pos=32)
+    blob = synth.build_blob(cfg, 5)
+    ids, lens = synth.source_batch(cfg.vocab, 1, 6, 6, 8)
+    T = 6
+    out, olen, sc = O.translate(blob, ids, lens, -1, T)
+    n = int(olen[0])
+    tgt = np.concatenate([[cfg.bos_id], out[0, :n - 1]]).astype(np.int32)
+    logits, _ = O.decode_trace(blob, ids[0], lens[0], tgt, cfg)
+    cum = np.float32(0.0)
+    for t in range(n):
+        cum = np.float32(cum + O.log_softmax(logits[t])[out[0, t]])
+    ref = sum(float(l[out[0, t]]) - _lse64(l) for t, l in enumerate(logits[:n]))
+    assert sc[0] == cum
+    assert abs(float(sc[0]) - ref) <= 1e-4 * n
