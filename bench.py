@@ -20,6 +20,17 @@ tokens.  Metric: decoded tokens per second (whole job over all GPUs).
             flushed before each; algorithmic bytes = the weights, scales and
             biases every step must read plus its K/V cache reads
   cpu_baseline  the CPU oracle on a bounded sample of the same workload
+  batched   the batched half of the metric on the two batched-beam workloads
+            (12+2-layer d=256 model, batch 32 x beam 4; 6+6-layer d=512 model,
+            batch 128 x beam 4): tokens/s (device-resident and end to end),
+            decode-step p50/p90, encode time, the encoder's operations per
+            second as a fraction of the measured dense fp16/bf16 tensor peak
+            (the exact int8 route: int8 codes carried as fp16, see the
+            tensor-core linear), and the decode step's fraction of HBM
+  microbench  the int8 linear sweep M in {1..4096} x five (K, N) shapes and
+            the wide encoder's linears, each with TOPS and GB/s and its
+            fraction of the bounding peak, plus incremental attention over
+            caches of 1..512 keys (GB/s)
 
 --impl reference runs the CPU oracle (the reference of this path) on the host
 cores with the same metric and config.  Under torchrun every rank translates
@@ -55,6 +66,24 @@ def _peaks():
         return float(p["hbm_gbs"]), "measured"
     except Exception:
         return 6800.0, "fallback"
+
+
+def _tensor_peak():
+    """Dense fp16/bf16 tensor peak (TFLOP/s): the measured burst figure, else the fallback."""
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def _source_hash(files):
+    import hashlib
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2306_04235_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 class ClockSampler:
@@ -152,6 +181,18 @@ def decode_step_bytes(cfg, R, B, S, t):
     return w + 8 * rows + 4 * inv + ln + proj + vocab + emb + kv
 
 
+def encoder_ops(cfg, B, S):
+    """Operations (2 per multiply-add) of one encode of B sentences padded to S:
+    the factorised embedding projection, every encoder layer's QKV, W_o, FFN1,
+    FFN2 linears and its attention (Q K^T and P V over S keys per query row),
+    and every decoder layer's cross key/value projection."""
+    d, F, E, M = cfg.d_model, cfg.d_ffn, cfg.d_embed, B * S
+    ops = 2 * M * d * E if E != d else 0
+    ops += cfg.n_enc * (2 * M * (4 * d * d + 2 * d * F) + 4 * B * S * S * d)
+    ops += cfg.n_dec * 2 * M * 2 * d * d
+    return ops
+
+
 def cpu_sample(workload, n_sent, threads):
     """The oracle translating n_sent sentences drawn like the workload's (batch-1
     translations, one per thread at a time)."""
@@ -203,6 +244,319 @@ def run_reference(args):
     return 0
 
 
+class Workload:
+    """One workload's model, session, device buffers and pinned host buffers."""
+
+    def __init__(self, name, mnmt, torch, stream, rank):
+        self.wl = synth.WORKLOADS[name]
+        self.cfg = synth.MODELS[self.wl.model]
+        self.blob = synth.build_blob(self.cfg, self.wl.model_seed)
+        # every rank translates its own replica batch (independent sentences)
+        self.ids, self.lens = synth.source_batch(self.cfg.vocab, self.wl.batch, self.wl.src_len[0],
+                                                 self.wl.src_len[1], self.wl.src_seed + 101 * rank)
+        self.B, self.S = self.ids.shape
+        self.T = self.wl.max_len
+        self.mnmt, self.torch, self.stream = mnmt, torch, stream
+        self.tr = mnmt.Translator(self.blob, self.B, self.S, self.wl.beam, self.T, stream)
+        self.sess = self.tr.session
+        dev = "cuda"
+        self.d_ids = torch.from_numpy(self.ids).to(dev)
+        self.d_lens = torch.from_numpy(self.lens).to(dev)
+        self.o_ids = torch.zeros((self.B, self.T), dtype=torch.int32, device=dev)
+        self.o_len = torch.zeros(self.B, dtype=torch.int32, device=dev)
+        self.o_sc = torch.zeros(self.B, dtype=torch.float32, device=dev)
+        torch.cuda.synchronize()
+
+    def translate(self):
+        self.mnmt.mnmt_translate(self.sess, self.d_ids, self.d_lens, self.B, self.S, self.T,
+                                 self.mnmt.DEVICE_PTRS, self.o_ids, self.o_len, self.o_sc)
+
+    def close(self):
+        self.tr.close()
+
+
+def _event(torch):
+    return torch.cuda.Event(enable_timing=True)
+
+
+def time_translations(w, flush, steps, warmup, dist=None):
+    """`steps` translations timed one by one with CUDA events on the library's
+    stream, L2 flushed (outside the events) before each."""
+    torch, stream = w.torch, w.stream
+    for _ in range(warmup):
+        with torch.cuda.stream(stream):
+            flush.fill_(1)
+        w.translate()
+    stream.synchronize()
+    evs = [(_event(torch), _event(torch)) for _ in range(steps)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(steps):
+        with torch.cuda.stream(stream):
+            flush.fill_(i & 0xFF)
+            evs[i][0].record(stream)
+        w.translate()
+        with torch.cuda.stream(stream):
+            evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    return [a.elapsed_time(b) for a, b in evs]
+
+
+def time_encode(w, flush, n=5):
+    torch, stream, mnmt = w.torch, w.stream, w.mnmt
+    out = []
+    for i in range(n):
+        e0, e1 = _event(torch), _event(torch)
+        with torch.cuda.stream(stream):
+            flush.fill_(i & 0xFF)
+            e0.record(stream)
+        mnmt.mnmt_encode(w.sess, w.d_ids, w.d_lens, w.B, w.S, mnmt.DEVICE_PTRS)
+        with torch.cuda.stream(stream):
+            e1.record(stream)
+        stream.synchronize()
+        out.append(e0.elapsed_time(e1))
+    return statistics.median(out)
+
+
+def time_e2e(w, flush, steps, warmup, world):
+    """The same translation through the C ABI with pinned host buffers: the
+    host->device copy of the sources and the device->host copy of the outputs
+    are inside the timed region."""
+    torch, stream, mnmt = w.torch, w.stream, w.mnmt
+    h_ids = torch.from_numpy(w.ids).pin_memory()
+    h_lens = torch.from_numpy(w.lens).pin_memory()
+    h_out = torch.zeros((w.B, w.T), dtype=torch.int32).pin_memory()
+    h_olen = torch.zeros(w.B, dtype=torch.int32).pin_memory()
+    h_osc = torch.zeros(w.B, dtype=torch.float32).pin_memory()
+    times = []
+    for i in range(warmup + steps):
+        with torch.cuda.stream(stream):
+            flush.fill_(i & 0xFF)
+        stream.synchronize()
+        t0 = time.perf_counter()
+        mnmt.mnmt_translate(w.sess, h_ids.data_ptr(), h_lens.data_ptr(), w.B, w.S, w.T, 0, h_out.data_ptr(),
+                            h_olen.data_ptr(), h_osc.data_ptr())
+        if i >= warmup:
+            times.append(time.perf_counter() - t0)
+    toks = int(h_olen.sum().item())
+    assert torch.equal(h_out, w.o_ids.cpu()), "host and device paths disagree"
+    return {"value": toks * world * len(times) / sum(times), "unit": "tokens/s",
+            "h2d_bytes_per_step": int(w.ids.nbytes + w.lens.nbytes),
+            "d2h_bytes_per_step": int(w.B * w.T * 4 + w.B * 8)}
+
+
+# DRAM bytes of one decode step (dram__bytes_read.sum + dram__bytes_write.sum of
+# its kernels, from single-kernel ncu captures of this bench's command), with
+# the hash of the step kernels' sources they were taken on: a stale figure
+# (sources changed since) is reported as null
+STEP_TRAFFIC = {("small-b1-s10to50-greedy64", True): (10_582_950, None)}
+STEP_SOURCES = ["decode_cluster.cu", "common.cuh", "mbarrier.cuh"]
+
+
+def measure_decode_step(w, flush, steps_run, cluster):
+    """Decode steps of one encoded batch timed with CUDA events on the
+    library's stream: one step per event pair with L2 flushed before each
+    (cold: the weights come from HBM, as the roofline assumes), then the same
+    number of steps back to back (warm: the weights stay in the 129 MB L2)."""
+    torch, stream, mnmt, cfg, wl = w.torch, w.stream, w.mnmt, w.cfg, w.wl
+    R = w.B * wl.beam
+    n = max(1, min(steps_run, wl.max_len))
+    mnmt.mnmt_encode(w.sess, w.d_ids, w.d_lens, w.B, w.S, mnmt.DEVICE_PTRS)
+    cold = []
+    for t in range(n):
+        with torch.cuda.stream(stream):
+            flush.fill_(t & 0xFF)
+            e0, e1 = _event(torch), _event(torch)
+            e0.record(stream)
+        mnmt.mnmt_decode_steps(w.sess, 1)
+        with torch.cuda.stream(stream):
+            e1.record(stream)
+        cold.append((e0, e1))
+    mnmt.mnmt_encode(w.sess, w.d_ids, w.d_lens, w.B, w.S, mnmt.DEVICE_PTRS)
+    with torch.cuda.stream(stream):
+        w0, w1 = _event(torch), _event(torch)
+        w0.record(stream)
+    mnmt.mnmt_decode_steps(w.sess, n)
+    with torch.cuda.stream(stream):
+        w1.record(stream)
+    stream.synchronize()
+    cold_us = [a.elapsed_time(b) * 1e3 for a, b in cold]
+    avg_us = sum(cold_us) / len(cold_us)
+    warm_us = w0.elapsed_time(w1) * 1e3 / n
+    algo = sum(decode_step_bytes(cfg, R, w.B, w.S, t) for t in range(n)) / n
+    peak, kind = _peaks()
+    achieved = algo / (avg_us * 1e-6) / 1e9
+    unit = ("decode_cluster_kernel + vocab_greedy_kernel (one graph launch)" if cluster
+            else "multi-kernel decode step (one graph launch)")
+    traffic, stamp = STEP_TRAFFIC.get((wl.name, cluster), (None, None))
+    if traffic is not None and stamp != _source_hash(STEP_SOURCES):
+        traffic = None
+    srt = sorted(cold_us)
+    return {"kernel": f"decode step: {unit}, R={R} rows, S={w.S}", "bound": "hbm", "achieved": achieved,
+            "peak": peak, "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{kind} hbm_gbs (burst)",
+            "traffic": traffic, "algorithmic_bytes": int(algo), "avg_us": avg_us,
+            "p50_us": srt[len(srt) // 2], "warm_avg_us": warm_us, "launches": len(cold_us)}
+
+
+def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None):
+    """tokens/s (device-resident and end to end), decode-step latency, encode
+    time and the decode step's roofline for one workload."""
+    w = Workload(name, mnmt, torch, stream, rank)
+    try:
+        step_ms = time_translations(w, flush, steps, warmup, dist)
+        toks_per_step = int(w.o_len.sum().item())
+        total_ms = sum(step_ms)
+        if dist:
+            t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            total_ms = float(t.item())
+            nt = torch.tensor([toks_per_step], dtype=torch.float64, device="cuda")
+            dist.all_reduce(nt, op=dist.ReduceOp.SUM)
+            job_toks = float(nt.item())
+        else:
+            job_toks = float(toks_per_step)
+        value = job_toks * steps / (total_ms / 1e3)
+        enc_ms = time_encode(w, flush)
+        # decode steps actually executed per translation (greedy stops when
+        # every sentence has emitted EOS; the beam workloads run all T)
+        steps_run = int(w.o_len.max().item()) if w.wl.beam == 1 else w.T
+        step_us = sorted(1e3 * (t - enc_ms) / max(steps_run, 1) for t in step_ms)
+        e2e = time_e2e(w, flush, steps, warmup, world)
+        cluster = mnmt.mnmt_session_decode_path(w.sess) == 1
+        roof = measure_decode_step(w, flush, steps_run, cluster)
+        return {"w": w, "value": value, "total_ms": total_ms, "toks_per_step": toks_per_step,
+                "steps_run": steps_run, "enc_ms": enc_ms, "step_us": step_us, "e2e": e2e,
+                "roofline": roof, "cluster": cluster}
+    finally:
+        w.close()
+
+
+def batched_entry(name, mnmt, torch, stream, flush, steps, warmup):
+    r = measure_workload(name, mnmt, torch, stream, flush, steps, warmup)
+    w = r["w"]
+    peak_t, kind_t = _tensor_peak()
+    ops = encoder_ops(w.cfg, w.B, w.S)
+    enc_tops = ops / (r["enc_ms"] * 1e-3) / 1e12
+    su = r["step_us"]
+    roof = r["roofline"]
+    return {
+        "workload": name, "model": w.wl.model, "batch": w.B, "beam": w.wl.beam, "s_pad": w.S, "max_len": w.T,
+        "tokens_per_translation": r["toks_per_step"], "translations_timed": steps,
+        "value": r["value"], "unit": "tokens/s", "ms_per_translation": r["total_ms"] / steps,
+        "e2e": r["e2e"],
+        "decode_step_us_p50": su[len(su) // 2], "decode_step_us_p90": su[min(len(su) - 1, int(0.9 * len(su)))],
+        "encode_ms_p50": r["enc_ms"],
+        "encoder": {"bound": "tensor", "ops": ops, "achieved": enc_tops, "peak": peak_t, "unit": "TOPS",
+                    "frac": enc_tops / peak_t,
+                    "peak_kind": f"{kind_t} bf16_tflops (burst); int8 codes run as exact fp16 on tcgen05 "
+                                 "kind::f16, which has no int8 kind on sm_103a"},
+        "decode_step": {"bound": "hbm", "achieved": roof["achieved"], "peak": roof["peak"], "unit": "GB/s",
+                        "frac": roof["frac"], "algorithmic_bytes": roof["algorithmic_bytes"],
+                        "cold_avg_us": roof["avg_us"], "cold_p50_us": roof["p50_us"],
+                        "warm_avg_us": roof["warm_avg_us"], "kernel": roof["kernel"]},
+    }
+
+
+SWEEP_M = [1, 4, 16, 64, 256, 1024, 4096]
+SWEEP_KN = [(256, 1024), (1024, 256), (512, 2048), (2048, 512), (256, 32000)]
+WIDE_ENCODER_LINEARS = [("qkv", 512, 1536), ("o", 512, 512), ("ffn1", 512, 2048), ("ffn2", 2048, 512)]
+
+
+def _time_cold(torch, stream, flush, fn, reps=5, warm=2):
+    for _ in range(warm):
+        fn()
+    evs = []
+    for i in range(reps):
+        with torch.cuda.stream(stream):
+            flush.fill_(i & 0xFF)
+            e0, e1 = _event(torch), _event(torch)
+            e0.record(stream)
+        fn()
+        with torch.cuda.stream(stream):
+            e1.record(stream)
+        evs.append((e0, e1))
+    stream.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e3  # us
+
+
+def microbench(mnmt, torch, stream, flush):
+    """The int8 linear sweep (E1 epilogue: int8 output) on the kernel the
+    translation path uses at each M (<= 16 rows: the int8 GEMV; more: the
+    tcgen05 kernel over fp16 copies of the codes), the wide encoder's linears at
+    M = 16384, and incremental attention.  Cold L2 (flushed before each rep)."""
+    peak_b, kind_b = _peaks()
+    peak_t, kind_t = _tensor_peak()
+    ridge = peak_t * 1e12 / (peak_b * 1e9)  # ops per byte where the bounds cross
+    dev = "cuda"
+    torch.manual_seed(5)
+    Mmax, Kmax, Nmax = 16384, 2048, 32000
+    max_out = max([M * N for (K, N) in SWEEP_KN for M in SWEEP_M] + [16384 * N for _, K, N in WIDE_ENCODER_LINEARS])
+    max_w = max([K * N for (K, N) in SWEEP_KN] + [K * N for _, K, N in WIDE_ENCODER_LINEARS])
+    A8 = torch.randint(-127, 128, (Mmax * Kmax,), dtype=torch.int8, device=dev)
+    W8 = torch.randint(-127, 128, (max_w,), dtype=torch.int8, device=dev)
+    A16 = torch.empty(Mmax * Kmax, dtype=torch.int16, device=dev)
+    W16 = torch.empty(max_w, dtype=torch.int16, device=dev)
+    s_w = torch.rand(Nmax, device=dev) * 2e-4 + 1e-4
+    bias = torch.rand(Nmax, device=dev) - 0.5
+    inv = torch.full((Nmax,), 50.0, device=dev)
+    out_q = torch.empty(max_out, dtype=torch.int8, device=dev)
+    torch.cuda.synchronize()
+    mnmt.mnmt_codes_to_f16(A8, A16, A8.numel(), stream)
+    mnmt.mnmt_codes_to_f16(W8, W16, W8.numel(), stream)
+    stream.synchronize()
+
+    def lin_entry(M, K, N, label=None):
+        if M <= 16:
+            fn = lambda: mnmt.mnmt_linear(A8, W8, s_w, bias, 0.03, inv, 1.0, M, N, K, mnmt.EPI_Q8,  # noqa: E731
+                                         out_q, None, stream)
+            kern = "linear_smallm (int8 dp4a GEMV)"
+        else:
+            fn = lambda: mnmt.mnmt_linear_tc(A16, W16, s_w, bias, 0.03, inv, 1.0, M, N, K,  # noqa: E731
+                                            mnmt.EPI_Q8, out_q=out_q, stream=stream)
+            kern = "linear_tc (tcgen05 kind::f16 on exact fp16 codes)"
+        us = _time_cold(torch, stream, flush, fn)
+        ops = 2 * M * N * K
+        byts = M * K + K * N + 8 * N + M * N
+        tops = ops / (us * 1e-6) / 1e12
+        gbs = byts / (us * 1e-6) / 1e9
+        bound = "hbm" if ops / byts < ridge else "tensor"
+        frac = gbs / peak_b if bound == "hbm" else tops / peak_t
+        e = {"M": M, "K": K, "N": N, "us": round(us, 2), "TOPS": round(tops, 2), "GBps": round(gbs, 1),
+             "bound": bound, "frac": round(frac, 4), "kernel": kern}
+        if label:
+            e["layer"] = label
+        return e
+
+    sweep = [lin_entry(M, K, N) for (K, N) in SWEEP_KN for M in SWEEP_M]
+    wide = [lin_entry(16384, K, N, lab) for lab, K, N in WIDE_ENCODER_LINEARS]
+
+    attn = []
+    for R, H, T in [(1, 4, 512), (128, 4, 512), (512, 8, 512)]:
+        dh = 64
+        Kc = torch.randint(-127, 128, (R * H * T * dh,), dtype=torch.int8, device=dev)
+        Vc = torch.randint(-127, 128, (R * H * T * dh,), dtype=torch.int8, device=dev)
+        q = torch.randint(-127, 128, (R * H * dh,), dtype=torch.int8, device=dev)
+        ctx = torch.empty(R * H * dh, dtype=torch.int8, device=dev)
+        torch.cuda.synchronize()
+        for t in [1, 16, 64, 256, 512]:
+            nk = torch.full((R,), t, dtype=torch.int32, device=dev)
+            fn = lambda: mnmt.mnmt_attention_decode(q, Kc, Vc, nk, R, H, dh, T, 0.001, 0.9, ctx,  # noqa: E731
+                                                    stream)
+            us = _time_cold(torch, stream, flush, fn)
+            byts = 2 * R * H * t * dh + 2 * R * H * dh + 4 * R
+            gbs = byts / (us * 1e-6) / 1e9
+            attn.append({"R": R, "H": H, "dh": dh, "cache": t, "us": round(us, 2), "GBps": round(gbs, 1),
+                         "bound": "hbm", "frac": round(gbs / peak_b, 4)})
+        del Kc, Vc
+    return {"linear_sweep": sweep, "wide_encoder_linears_M16384": wide, "attention_decode": attn,
+            "peaks": {"hbm_gbs": peak_b, "hbm_kind": kind_b, "tensor_tflops": peak_t, "tensor_kind": kind_t},
+            "bytes": "int8 algorithmic bytes M*K + K*N + 8*N + M*N (the tensor-core kernel reads 2-byte "
+                     "fp16 copies of the codes)", "l2": "flushed before each rep; median of 5"}
+
+
 def run_gpu(args):
     import torch
 
@@ -216,101 +570,24 @@ def run_gpu(args):
     torch.cuda.set_device(local)
     from paper_2306_04235_gb300 import mnmt
 
-    wl = synth.WORKLOADS[args.workload]
-    cfg = synth.MODELS[wl.model]
-    blob = synth.build_blob(cfg, wl.model_seed)
-    # every rank translates its own replica batch (independent sentences)
-    ids, lens = synth.source_batch(cfg.vocab, wl.batch, wl.src_len[0], wl.src_len[1], wl.src_seed + 101 * rank)
-    B, S = ids.shape
     stream = torch.cuda.Stream()
-    tr = mnmt.Translator(blob, B, S, wl.beam, wl.max_len, stream)
-    sess = tr.session
-    T = wl.max_len
-    d_ids = torch.from_numpy(ids).cuda()
-    d_lens = torch.from_numpy(lens).cuda()
-    o_ids = torch.zeros((B, T), dtype=torch.int32, device="cuda")
-    o_len = torch.zeros(B, dtype=torch.int32, device="cuda")
-    o_sc = torch.zeros(B, dtype=torch.float32, device="cuda")
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-    torch.cuda.synchronize()
-
-    def step():
-        mnmt.mnmt_translate(sess, d_ids, d_lens, B, S, T, mnmt.DEVICE_PTRS, o_ids, o_len, o_sc)
-
-    for _ in range(args.warmup):
-        with torch.cuda.stream(stream):
-            flush.fill_(1)
-        step()
-    stream.synchronize()
-
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    toks = 0
-    if dist:
-        dist.barrier()
-    torch.cuda.synchronize()
     with ClockSampler(local) as clk:
-        for i in range(args.steps):
-            with torch.cuda.stream(stream):
-                flush.fill_(i & 0xFF)
-                evs[i][0].record(stream)
-            step()
-            with torch.cuda.stream(stream):
-                evs[i][1].record(stream)
-        torch.cuda.synchronize()
-    if dist:
-        dist.barrier()
-    step_ms = [a.elapsed_time(b) for a, b in evs]
-    toks_per_step = int(o_len.sum().item())
-    total_ms = sum(step_ms)
-    if dist:
-        t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-        n = torch.tensor([toks_per_step], dtype=torch.float64, device="cuda")
-        dist.all_reduce(n, op=dist.ReduceOp.SUM)
-        job_toks_per_step = float(n.item())
-    else:
-        job_toks_per_step = float(toks_per_step)
-    value = job_toks_per_step * args.steps / (total_ms / 1e3)
+        r = measure_workload(args.workload, mnmt, torch, stream, flush, args.steps, args.warmup, rank, world,
+                             dist)
+    w = r["w"]
+    cfg, wl, B, S, T = w.cfg, w.wl, w.B, w.S, w.T
+    step_us = r["step_us"]
 
-    # per decode-step latency: translation time minus the encoder's, over the steps
-    enc_ms = []
-    for _ in range(5):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-        mnmt.mnmt_encode(sess, d_ids, d_lens, B, S, mnmt.DEVICE_PTRS)
-        with torch.cuda.stream(stream):
-            e1.record(stream)
-        stream.synchronize()
-        enc_ms.append(e0.elapsed_time(e1))
-    steps_run = int(o_len.max().item()) if wl.beam == 1 else T
-    enc_med = statistics.median(enc_ms)
-    step_us = sorted(1e3 * (t - enc_med) / max(steps_run, 1) for t in step_ms)
-
-    # end to end through the C ABI with pinned host buffers
-    h_ids = torch.from_numpy(ids).pin_memory()
-    h_lens = torch.from_numpy(lens).pin_memory()
-    h_out = torch.zeros((B, T), dtype=torch.int32).pin_memory()
-    h_olen = torch.zeros(B, dtype=torch.int32).pin_memory()
-    h_osc = torch.zeros(B, dtype=torch.float32).pin_memory()
-    e2e_times = []
-    for i in range(args.warmup + args.steps):
-        with torch.cuda.stream(stream):
-            flush.fill_(i & 0xFF)
-        stream.synchronize()
-        t0 = time.perf_counter()
-        mnmt.mnmt_translate(sess, h_ids.data_ptr(), h_lens.data_ptr(), B, S, T, 0, h_out.data_ptr(),
-                            h_olen.data_ptr(), h_osc.data_ptr())
-        if i >= args.warmup:
-            e2e_times.append(time.perf_counter() - t0)
-    e2e_tok = int(h_olen.sum().item())
-    e2e_value = e2e_tok * world * len(e2e_times) / sum(e2e_times)
-    assert torch.equal(h_out, o_ids.cpu()), "host and device paths disagree"
-
-    # the decode step, one at a time (cold L2) and back to back (warm)
-    cluster = mnmt.mnmt_session_decode_path(sess) == 1
-    roof = measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster)
+    batched = micro = None
+    if rank == 0 and world == 1 and not args.no_batched:
+        with ClockSampler(local) as bclk:
+            batched = {"entries": [batched_entry(n, mnmt, torch, stream, flush, 5, 3) for n in BATCHED]}
+        batched["clocks"] = bclk.summary()
+    if rank == 0 and world == 1 and not args.no_micro:
+        with ClockSampler(local) as mclk:
+            micro = microbench(mnmt, torch, stream, flush)
+        micro["clocks"] = mclk.summary()
 
     if rank == 0:
         cpu = None
@@ -322,78 +599,37 @@ def run_gpu(args):
                    "kind": "oracle",
                    "sample": f"{n_sent} translation(s) of {wl.batch} sentence(s) drawn like the workload, "
                              f"one per thread ({cdt:.1f} s)"}
+        steps_run = r["steps_run"]
         # translate queues steps in chunks of 16 with one chunk of look-ahead:
         # a translation that finishes early has one more (no-op) chunk queued
         launched = T if steps_run >= T else min(T, -(-steps_run // 16) * 16 + 16)
-        launches = kernels_per_translation(cfg, B, S, wl.beam, launched, cluster) * args.steps
+        launches = kernels_per_translation(cfg, B, S, wl.beam, launched, r["cluster"]) * args.steps
         line = {
-            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "metric": METRIC, "value": r["value"], "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": r["total_ms"] / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
             "config": {"workload": args.workload, "model": wl.model, "batch": B, "beam": wl.beam,
-                       "max_len": T, "src_len": list(wl.src_len), "s_pad": S, "tokens_per_step": toks_per_step,
+                       "max_len": T, "src_len": list(wl.src_len), "s_pad": S,
+                       "tokens_per_step": r["toks_per_step"],
                        "l2": "flushed between steps (256 MB write, outside the timed events)",
                        "decode_step_us_p50": step_us[len(step_us) // 2],
                        "decode_step_us_p90": step_us[min(len(step_us) - 1, int(0.9 * len(step_us)))],
-                       "encode_ms_p50": enc_med, "parallelism": f"replicas x{world}"},
-            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": int(ids.nbytes + lens.nbytes),
-                    "d2h_bytes_per_step": int(B * T * 4 + B * 8)},
-            "roofline": roof,
+                       "encode_ms_p50": r["enc_ms"], "parallelism": f"replicas x{world}"},
+            "e2e": r["e2e"],
+            "roofline": r["roofline"],
             "cpu_baseline": cpu,
             "clocks": clk.summary(),
             "gpu_launches": launches,
+            "batched": batched,
+            "microbench": micro,
         }
         print(json.dumps(line), flush=True)
-    tr.close()
     if dist:
         dist.destroy_process_group()
     return 0
 
 
-# DRAM bytes of one decode step (dram__bytes_read.sum + dram__bytes_write.sum
-# of its kernels, one ncu capture of this bench's command); only for the step
-# kernels they were taken on -- refresh whenever those kernels change
-STEP_TRAFFIC = {("small-b1-s10to50-greedy64", True): 10_582_950}
-
-
-def measure_decode_step(cfg, wl, mnmt, torch, stream, flush, sess, d_ids, d_lens, B, S, steps_run, cluster):
-    """Decode steps of one encoded batch timed with CUDA events on the
-    library's stream: one step per event pair with L2 flushed before each
-    (cold: the weights come from HBM, as the roofline assumes), then the same
-    number of steps back to back (warm: the weights stay in the 129 MB L2)."""
-    R = B * wl.beam
-    n = max(1, min(steps_run, wl.max_len))
-    mnmt.mnmt_encode(sess, d_ids, d_lens, B, S, mnmt.DEVICE_PTRS)
-    cold = []
-    for t in range(n):
-        with torch.cuda.stream(stream):
-            flush.fill_(t & 0xFF)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-        mnmt.mnmt_decode_steps(sess, 1)
-        with torch.cuda.stream(stream):
-            e1.record(stream)
-        cold.append((e0, e1))
-    mnmt.mnmt_encode(sess, d_ids, d_lens, B, S, mnmt.DEVICE_PTRS)
-    with torch.cuda.stream(stream):
-        w0, w1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        w0.record(stream)
-    mnmt.mnmt_decode_steps(sess, n)
-    with torch.cuda.stream(stream):
-        w1.record(stream)
-    stream.synchronize()
-    cold_us = [a.elapsed_time(b) * 1e3 for a, b in cold]
-    avg_us = sum(cold_us) / len(cold_us)
-    warm_us = w0.elapsed_time(w1) * 1e3 / n
-    algo = sum(decode_step_bytes(cfg, R, B, S, t) for t in range(n)) / n
-    peak, kind = _peaks()
-    achieved = algo / (avg_us * 1e-6) / 1e9
-    unit = ("decode_cluster_kernel + vocab_greedy_kernel (one graph launch)" if cluster
-            else "multi-kernel decode step (one graph launch)")
-    return {"kernel": f"decode step: {unit}, R={R} rows, S={S}", "bound": "hbm", "achieved": achieved, "peak": peak,
-            "unit": "GB/s", "frac": achieved / peak, "peak_kind": f"{kind} hbm_gbs (burst)",
-            "traffic": STEP_TRAFFIC.get((wl.name, cluster)), "algorithmic_bytes": int(algo), "avg_us": avg_us, "warm_avg_us": warm_us,
-            "launches": len(cold_us)}
+BATCHED = ["small-b32-s10to80-beam4-t128", "wide-b128-s20to128-beam4-t160"]
 
 
 def main():
@@ -404,6 +640,8 @@ def main():
     ap.add_argument("--impl", default="mnmt", choices=["mnmt", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-batched", action="store_true", help="skip the batched-beam workloads")
+    ap.add_argument("--no-micro", action="store_true", help="skip the linear / attention sweep")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -134,6 +134,9 @@ int mnmt_decode_step(mnmt_session *s, int32_t *tokens, int32_t *parents, float *
                      int32_t *all_done);
 
 /* encode + decode until every sentence has emitted EOS or max_len steps ran.
+ * The beam width is the session's (fixed by mnmt_session_create): translating
+ * with another width needs another session.  max_len may not exceed the
+ * session's. 
  * out_ids [B][max_len]: tokens of the best hypothesis, EOS included, PAD after;
  * out_lens [B]: number of tokens up to and including EOS (max_len if none);
  * out_scores [B]: cumulative log-probability of the best beam (0 for greedy).

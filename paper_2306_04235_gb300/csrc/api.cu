@@ -52,19 +52,27 @@ static int fail(int code, const char *fmt, ...) {
                         __LINE__);                                                                \
     } while (0)
 
-static std::once_flag g_init_once;
-static cudaError_t g_init_err = cudaSuccess;
+// Kernel set-up (dynamic shared-memory opt-ins, the SM count) applies to the
+// device current at the time, so it runs once for every device a call is
+// made on, with that device current.
+static std::mutex g_init_mu;
+static constexpr int MAX_INIT_DEVICES = 64;
+static bool g_init_done[MAX_INIT_DEVICES] = {false};
 
 static int lib_init() {
-    std::call_once(g_init_once, [] {
-        g_init_err = linear_init();
-        if (g_init_err == cudaSuccess) g_init_err = attention_init();
-        if (g_init_err == cudaSuccess) g_init_err = rows_init();
-        if (g_init_err == cudaSuccess) g_init_err = decode_cluster_init();
-        if (g_init_err == cudaSuccess) g_init_err = linear_tc_init();
-    });
-    if (g_init_err != cudaSuccess)
-        return fail(MNMT_ECUDA, "kernel set-up failed: %s", cudaGetErrorString(g_init_err));
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return fail(MNMT_ECUDA, "no usable current device: %s", cudaGetErrorString(e));
+    if (dev < 0 || dev >= MAX_INIT_DEVICES) return fail(MNMT_ECUDA, "device index %d out of range", dev);
+    std::lock_guard<std::mutex> lk(g_init_mu);
+    if (g_init_done[dev]) return MNMT_OK;
+    e = linear_init();
+    if (e == cudaSuccess) e = attention_init();
+    if (e == cudaSuccess) e = rows_init();
+    if (e == cudaSuccess) e = decode_cluster_init();
+    if (e == cudaSuccess) e = linear_tc_init();
+    if (e != cudaSuccess) return fail(MNMT_ECUDA, "kernel set-up failed: %s", cudaGetErrorString(e));
+    g_init_done[dev] = true;
     return MNMT_OK;
 }
 

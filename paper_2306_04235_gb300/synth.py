@@ -219,15 +219,33 @@ class _BlobWriter:
         return b"".join(self.parts)
 
 
-def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None) -> bytes:
+# Weight-std multipliers of the decoder's cross-attention projections.  With
+# every weight drawn N(0, 0.02) the cross-attention scores are ~0.1 (a flat
+# softmax) and its output is a small average of source values, so a random
+# model decodes almost the same tokens whatever the source (with a tied output
+# matrix it repeats its input token).  A translation model's output depends on
+# its source through this sublayer, so the synthetic models sharpen it: the
+# query and key projections are drawn with std 0.02*qk, the value projection
+# 0.02*v, the output projection 0.02*o.  The activation scales of the points
+# these weights feed follow the same multipliers.  With these values every
+# workload model decodes a different token sequence for each of 8 random
+# sources (at most 1 of 8 distinct without them).
+CROSS_GAINS = {"qk": 10.0, "v": 3.0, "o": 40.0}
+NO_GAINS = {"qk": 1.0, "v": 1.0, "o": 1.0}
+
+
+def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cross_gains=None) -> bytes:
     """Write a seeded synthetic model in the MNMT v1 blob format.
 
     gamma_range: None for gamma_i = 1 on every sublayer, or (lo, hi) to draw each
     sublayer's residual weight uniformly.  out_bias: optional dict {token: value}
-    added to the output bias (used to force e.g. immediate EOS).
+    added to the output bias (used to force e.g. immediate EOS).  cross_gains:
+    the cross-attention weight-std multipliers (default CROSS_GAINS; NO_GAINS
+    draws every weight N(0, 0.02)).
     """
     d, F, V, E = cfg.d_model, cfg.d_ffn, cfg.vocab, cfg.d_embed
     sc = activation_scales(cfg)
+    cg = dict(CROSS_GAINS if cross_gains is None else cross_gains)
     w = _BlobWriter()
     hdr = struct.pack("<4sI13i", b"MNMT", 1, *cfg.as_ints())
     hdr += b"\0" * (64 - len(hdr))
@@ -240,9 +258,9 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None) -> 
         lo, hi = gamma_range
         return _f32(lo + (hi - lo) * st.uniform(1)[0])
 
-    def linear(name, n, k):
+    def linear(name, n, k, std=0.02):
         st = Stream(seed, name)
-        q, s = int8_weight(st, n, k)
+        q, s = int8_weight(st, n, k, std)
         b = f32_normal(Stream(seed, name + ".b"), n, 0.0, 0.02)
         w.put(q)
         w.put(s)
@@ -268,11 +286,19 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None) -> 
     def cross_attn(prefix):
         ln(prefix + ".ln")
         g = gamma(Stream(seed, prefix + ".gamma"))
-        w.put(np.array([sc["ln"], sc["lin"], sc["lin"], sc["lin"], sc["lin"], g, 0, 0],
-                       dtype=np.float32))
-        linear(prefix + ".q", d, d)
-        linear(prefix + ".kv", 2 * d, d)
-        linear(prefix + ".o", d, d)
+        s_qk = _f32(sc["lin"] * cg["qk"])
+        s_v = _f32(sc["lin"] * cg["v"])
+        w.put(np.array([sc["ln"], s_qk, s_qk, s_v, s_v, g, 0, 0], dtype=np.float32))
+        linear(prefix + ".q", d, d, 0.02 * cg["qk"])
+        if cg["qk"] == cg["v"]:
+            linear(prefix + ".kv", 2 * d, d, 0.02 * cg["qk"])
+        else:  # key rows and value rows drawn with their own std, stored as one [2d][d] linear
+            qk_, sk_ = int8_weight(Stream(seed, prefix + ".kv"), d, d, 0.02 * cg["qk"])
+            qv_, sv_ = int8_weight(Stream(seed, prefix + ".kv.v"), d, d, 0.02 * cg["v"])
+            w.put(np.concatenate([qk_, qv_]))
+            w.put(np.concatenate([sk_, sv_]))
+            w.put(f32_normal(Stream(seed, prefix + ".kv.b"), 2 * d, 0.0, 0.02))
+        linear(prefix + ".o", d, d, 0.02 * cg["o"])
 
     def ffn(prefix):
         ln(prefix + ".ln")

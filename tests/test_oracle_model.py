@@ -157,3 +157,20 @@ def test_malformed_blobs_are_rejected():
     assert O.check_blob(blob + b"\0" * 16)[0] == O.EFORMAT
     assert O.check_blob(b"XNMT" + blob[4:])[0] == O.EFORMAT
     assert O.check_blob(blob[:40])[0] == O.EFORMAT
+
+
+@pytest.mark.parametrize("workload,T", [("tiny-b1-s16-greedy16", 16), ("small-b1-s10to50-greedy64", 10),
+                                        ("wide-b128-s20to128-beam4-t160", 6)])
+def test_workload_models_translate_each_source_differently(workload, T):
+    """The synthetic workload models decode a source-dependent sequence: six
+    random sources give six different greedy translations, so a wrong encoder
+    output, cross key/value or cross-attention value changes the tokens."""
+    wl = synth.WORKLOADS[workload]
+    cfg = synth.MODELS[wl.model]
+    blob = synth.build_blob(cfg, wl.model_seed)
+    ids, lens = synth.source_batch(cfg.vocab, 6, 10, 40, 4242)
+    out, olen, _ = O.translate(blob, ids, lens, 1, T, n_threads=6)
+    seqs = {tuple(out[b, :olen[b]]) for b in range(6)}
+    assert len(seqs) == 6
+    # and a sequence is not one token repeated
+    assert sum(len(set(s)) > 1 for s in seqs) >= 4
