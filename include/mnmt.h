@@ -54,7 +54,7 @@
  *   Scales s_* are the per-tensor activation scales of the quantisation points
  *   of Fig. 5; pre_ln = 0 selects post-LN sublayers (LayerNorm after the
  *   residual add, no final LayerNorm).  Constraints checked at load: d_model a
- *   power of two in [64, 2048], d_ffn a multiple of 64, d_embed a multiple of
+ *   multiple of 64 in [64, 2048], d_ffn a multiple of 64, d_embed a multiple of
  *   16, d_model / n_heads in {32, 64, 128}, at most 16 heads, vocab >= 4.
  */
 #ifndef MNMT_H

@@ -220,10 +220,15 @@ static void linear_row(const int8_t *a, float s_x, const olin *L, float *y) {
         y[n] = dequant_bias(dot_i8(a, L->w + (size_t)n * L->k, L->k), s_x, L->s[n], L->b[n]);
 }
 
-/* Nearest float (ties to even) to the exact value s 2^e / d.  The long double
- * quotient (64-bit significand on x86, 113-bit on Arm) is exact for the
- * power-of-two d of every model here, so the one rounding to float is the
- * correct rounding of the exact value, subnormals included. */
+/* Nearest float (ties to even) to the exact value s 2^e / d, |s| < 2^63,
+ * 1 <= d <= 2048.  For a power-of-two d the long double quotient (64-bit
+ * significand on x86, 113-bit on Arm) is exact.  Otherwise s 2^e / d is
+ * either a midpoint between two floats (then the quotient, an odd multiple of
+ * a power of two with at most 26 significant bits, is exact in long double
+ * too) or at least 2^-36 (relative) away from every midpoint (its distance
+ * to M 2^E is a nonzero multiple of 2^E / d, and M < 2^25, d < 2^11), while
+ * the long double quotient is within 2^-64 of it: either way the one rounding
+ * to float is the correct rounding of the exact value, subnormals included. */
 static float rn32_scaled(int64_t s, int e, int d) {
     return (float)(ldexpl((long double)s, e) / (long double)d);
 }
@@ -247,7 +252,7 @@ static float rn32_quotient(int64_t n, int64_t z) {
  * 2^eb > max|c_i| every c_i^2 2^(52-2eb) is below 2^52, so d <= 2048 terms
  * cannot overflow int64 and every term keeps its leading 24+ bits.
  * rstd = 1 / sqrt(var + 1e-5) in IEEE fp32.  |r_i| >= 2^32 is rejected. */
-static int layer_norm(const float *r, int d, const oln *ln, float *out) {
+static int ln_stats(const float *r, int d, float *mu_out, float *var_out) {
     float amax = 0.0f;
     for (int i = 0; i < d; i++) {
         float v = fabsf(r[i]);
@@ -273,6 +278,15 @@ static int layer_norm(const float *r, int d, const oln *ln, float *out) {
         s2 += llrint(ldexp((double)c2, 52 - 2 * eb));
     }
     float var = rn32_scaled(s2, 2 * eb - 52, d);
+    *mu_out = mu;
+    *var_out = var;
+    return OR_OK;
+}
+
+static int layer_norm(const float *r, int d, const oln *ln, float *out) {
+    float mu, var;
+    int st = ln_stats(r, d, &mu, &var);
+    if (st) return st;
     float rstd = 1.0f / sqrtf(var + 1e-5f);
     for (int i = 0; i < d; i++) {
         float c = r[i] - mu;
@@ -838,6 +852,15 @@ int oracle_check_blob(const void *blob, size_t bytes, int32_t *cfg_out) {
 }
 
 float oracle_q8(float x, float inv) { return (float)q8(x, inv); }
+
+/* The LayerNorm's mean and biased variance of M rows of length d. */
+int oracle_ln_stats(const float *r, int M, int d, float *mu, float *var) {
+    for (int m = 0; m < M; m++) {
+        int st = ln_stats(r + (size_t)m * d, d, mu + m, var + m);
+        if (st) return st;
+    }
+    return OR_OK;
+}
 float oracle_exp(float x) { return exp_own(x); }
 double oracle_log(double z) { return log_own(z); }
 

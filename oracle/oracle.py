@@ -69,10 +69,11 @@ def _declare(L):
     L.oracle_embed.argtypes = [_p, _sz, _p, _p, _i, _p]
     L.oracle_log_softmax.argtypes = [_p, _i, _p]
     L.oracle_log_softmax_norm.argtypes = [_p, _i, _p, _p, _p]
+    L.oracle_ln_stats.argtypes = [_p, _i, _i, _p, _p]
     L.oracle_translate.argtypes = [_p, _sz, _p, _p, _i, _i, _i, _i, _i, _p, _p, _p]
     for name in ["oracle_check_blob", "oracle_linear", "oracle_layernorm", "oracle_attention_decode",
                  "oracle_attention_probs", "oracle_encode", "oracle_decode_trace",
-                 "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_log_softmax_norm",
+                 "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_log_softmax_norm", "oracle_ln_stats",
                  "oracle_translate"]:
         getattr(L, name).restype = _i
 
@@ -156,6 +157,15 @@ def layernorm(r, g, b, inv=1.0):
     if st != OK:
         raise OracleError(f"oracle returned {st}")
     return of, oq
+
+
+def ln_stats(r):
+    """(mean, biased variance) per row as the LayerNorm computes them."""
+    r = np.ascontiguousarray(r, np.float32)
+    M, d = r.shape
+    mu = np.zeros(M, np.float32); var = np.zeros(M, np.float32)
+    _chk(lib().oracle_ln_stats(_ptr(r), M, d, _ptr(mu), _ptr(var)))
+    return mu, var
 
 
 def attention_decode(q, Kc, Vc, n_keys, sigma_, rho):

@@ -147,8 +147,9 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
     c.pad_id = h[10]; c.bos_id = h[11]; c.eos_id = h[12];
     const int d = c.d_model, F = c.d_ffn, V = c.vocab, E = c.d_embed;
     if (c.n_enc < 1 || c.n_enc > 64 || c.n_dec < 1 || c.n_dec > 64) return fail(MNMT_EFORMAT, "layer counts out of range");
-    if (!pow2_in(d, 64, 2048) || c.n_heads < 1 || d % c.n_heads)
-        return fail(MNMT_EFORMAT, "d_model %d / heads %d unsupported (d_model: a power of two in [64, 2048])", d, c.n_heads);
+    if (d < 64 || d > 2048 || d % 64 || c.n_heads < 1 || d % c.n_heads)
+        return fail(MNMT_EFORMAT, "d_model %d / heads %d unsupported (d_model: a multiple of 64 in [64, 2048])", d,
+                    c.n_heads);
     if (!pow2_in(d / c.n_heads, 32, 128)) return fail(MNMT_EFORMAT, "head dim %d not in {32,64,128}", d / c.n_heads);
     if (c.n_heads > 16) return fail(MNMT_EFORMAT, "more than 16 heads");
     if (F < 64 || F % 64 || F > 8192) return fail(MNMT_EFORMAT, "d_ffn %d unsupported", F);
@@ -1025,8 +1026,13 @@ int setup_cluster_step(mnmt_session *s) {
     const int d = c.d_model, F = c.d_ffn, H = c.n_heads, dh = d / H;
     const int R = s->B * s->k;
     const int nc = dc_cluster_size(d);
+    // the step's slice GEMV spreads each K-long row over K/64 lanes (a power
+    // of two) and a residual slice over at most 32 lanes: d, F and the
+    // factorised embedding width must be powers of two
+    const int E = c.d_embed;
     if (s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
-        F % (16 * nc) || (3 * d) % (16 * nc))
+        F % (16 * nc) || (3 * d) % (16 * nc) || !pow2_in(d, 64, 512) || !pow2_in(F, 64, 2048) ||
+        (m->factorised && !pow2_in(E, 16, 512)))
         return MNMT_OK;
     DcParams P;
     std::memset(&P, 0, sizeof(P));
@@ -1544,8 +1550,8 @@ extern "C" int mnmt_layernorm(const float *r, const float *g, const float *b, in
                               float *out_f, int8_t *out_q, int32_t *status, void *cuda_stream) {
     int rc = lib_init();
     if (rc) return rc;
-    if (!r || !g || !b || M < 1 || d < 1 || d > 2048 || (d & (d - 1)))
-        return fail(MNMT_EINVAL, "layernorm: d must be a power of two <= 2048");
+    if (!r || !g || !b || M < 1 || d < 1 || d > 2048)
+        return fail(MNMT_EINVAL, "layernorm: d must be in [1, 2048]");
     LnArgs a;
     std::memset(&a, 0, sizeof(a));
     a.r = r;

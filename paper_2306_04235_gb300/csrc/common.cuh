@@ -250,6 +250,28 @@ MNMT_DEV float rn32_pow2(long long S, int e) {
     return __uint_as_float(bits);
 }
 
+// nearest float (ties to even) to S * 2^e / d for 1 <= d <= 2048 and
+// |S| < 2^63: the LayerNorm's mean and variance, S an exact fixed-point sum of
+// d terms.  With d = z 2^k (z odd) and z = 1 this is rn32_pow2.  Otherwise
+// |S| is shifted so the integer quotient q = floor(|S| 2^t / z) keeps at least
+// 50 significant bits; the float keeps at most 24 of them, so the remainder
+// only decides whether the value lies exactly on q or strictly above it, which
+// one appended sticky bit (2q + [r != 0]) tells rn32_pow2 without moving the
+// value across a rounding boundary.
+MNMT_DEV float rn32_scaled_div(long long S, int e, int d) {
+    const int k = __ffs(d) - 1;
+    const unsigned z = (unsigned)d >> k;
+    if (z == 1u) return rn32_pow2(S, e - k);
+    if (S == 0) return 0.0f;
+    const unsigned long long a = S < 0 ? 0ull - (unsigned long long)S : (unsigned long long)S;
+    const int nb = 64 - __clzll(a);
+    const int t = nb < 62 ? 62 - nb : 0;
+    const unsigned long long num = a << t;
+    const unsigned long long q = num / z, r = num - q * z;
+    const float f = rn32_pow2((long long)(2ull * q + (r != 0ull ? 1ull : 0ull)), e - k - t - 1);
+    return S < 0 ? -f : f;
+}
+
 // sign of a - X * 2^E for a < 2^62, X < 2^63
 MNMT_DEV int cmp_scaled(unsigned long long a, unsigned long long X, int E) {
     if (E >= 0) {
@@ -317,7 +339,7 @@ MNMT_DEV int8_t q8_quotient(long long n, long long z, float rho, ExactDiv exact)
 // variance are exact fixed-point sums: the row's largest magnitude (an
 // order-free maximum) sets a power-of-two grid on which every term is an
 // integer below 2^52, summed in int64, so any reduction order gives the same
-// bits; each sum / d is rounded once to fp32 (d a power of two); rstd =
+// bits; each sum / d is rounded once to fp32 (rn32_scaled_div); rstd =
 // 1 / sqrt(var + 1e-5) in IEEE fp32; returns false if |x| >= 2^32.
 // warp LayerNorm over a row held as VPL values per lane (element u*32 + lane)
 // ---------------------------------------------------------------------------
@@ -343,13 +365,12 @@ MNMT_DEV bool warp_layernorm_v(const float (&x)[VPL], int d, const float (&gv)[V
     const float amax = __uint_as_float(__reduce_max_sync(0xFFFFFFFFu, amax_bits));
     if (!(amax < 0x1p32f)) return false;
     const int ea = exp_bound(amax);
-    const int log2d = 31 - __clz(d);  // d is a power of two
     long long s1 = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
     s1 = warp_sum_exact(s1);
-    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    const float mu = rn32_scaled_div(s1, ea - 52, d);
     float c[VPL];
     unsigned bmax_bits = 0;
 #pragma unroll
@@ -363,7 +384,7 @@ MNMT_DEV bool warp_layernorm_v(const float (&x)[VPL], int d, const float (&gv)[V
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
     s2 = warp_sum_exact(s2);
-    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float var = rn32_scaled_div(s2, 2 * eb - 52, d);
     const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
 #pragma unroll
     for (int u = 0; u < VPL; u++) out[u] = __fadd_rn(__fmul_rn(__fmul_rn(c[u], rstd), gv[u]), bv[u]);
@@ -380,13 +401,12 @@ MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restri
     const float amax = __uint_as_float(__reduce_max_sync(0xFFFFFFFFu, amax_bits));
     if (!(amax < 0x1p32f)) return false;
     const int ea = exp_bound(amax);
-    const int log2d = 31 - __clz(d);  // d is a power of two
     long long s1 = 0;
 #pragma unroll
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s1 += fx_scale(x[u], 52 - ea);
     s1 = warp_sum_exact(s1);
-    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    const float mu = rn32_scaled_div(s1, ea - 52, d);
     float c[VPL];
     unsigned bmax_bits = 0;
 #pragma unroll
@@ -400,7 +420,7 @@ MNMT_DEV bool warp_layernorm(const float (&x)[VPL], int d, const float *__restri
     for (int u = 0; u < VPL; u++)
         if (u * 32 + lane < d) s2 += fx_scale(__fmul_rn(c[u], c[u]), 52 - 2 * eb);
     s2 = warp_sum_exact(s2);
-    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float var = rn32_scaled_div(s2, 2 * eb - 52, d);
     const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
 #pragma unroll
     for (int u = 0; u < VPL; u++) {

@@ -56,7 +56,6 @@ __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
         return;
     }
     const int ea = exp_bound(amax);
-    const int log2d = 31 - __clz(d);  // d is a power of two
     long long s1 = 0;
 #pragma unroll
     for (int v = 0; v < VPT; v++) s1 += fx_scale(x[v], 52 - ea);  // padding adds 0
@@ -66,7 +65,7 @@ __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     s1 = 0;
 #pragma unroll
     for (int k = 0; k < LN_T / 32; k++) s1 += s_s1[k];
-    const float mu = rn32_pow2(s1, ea - 52 - log2d);
+    const float mu = rn32_scaled_div(s1, ea - 52, d);
     // centred values -> their maximum magnitude -> the grid of the variance sum
     float c[VPT];
     unsigned bm = 0;
@@ -92,7 +91,7 @@ __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     s2 = 0;
 #pragma unroll
     for (int k = 0; k < LN_T / 32; k++) s2 += s_s2[k];
-    const float var = rn32_pow2(s2, 2 * eb - 52 - log2d);
+    const float var = rn32_scaled_div(s2, 2 * eb - 52, d);
     const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
 #pragma unroll
     for (int v = 0; v < VPT; v++) {

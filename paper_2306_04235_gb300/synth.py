@@ -120,6 +120,12 @@ MODELS = {
     "small-12x2-d256-v32k-e128": ModelConfig(12, 2, 256, 4, 1024, 32000, 128, 1, 0),
     # 6+6 layers, d=512, tied 32000-entry vocabulary
     "wide-6x6-d512-v32k": ModelConfig(6, 6, 512, 8, 2048, 32000, 512, 1, 1),
+    # the paper's two models (Table "detailed settings of MobileNMT"): 12+2
+    # layers, a shared 8000-entry vocabulary tied to the output, no embedding
+    # factorisation, pre-LN; 10MB: d=256, 4 heads, FFN 512; 20MB: d=384,
+    # 6 heads, FFN 768
+    "mobilenmt-10mb": ModelConfig(12, 2, 256, 4, 512, 8000, 256, 1, 1),
+    "mobilenmt-20mb": ModelConfig(12, 2, 384, 6, 768, 8000, 384, 1, 1),
 }
 
 
@@ -143,6 +149,9 @@ WORKLOADS = {
         Workload("wide-b128-s20to128-beam4-t160", "wide-6x6-d512-v32k", 4, 128, (20, 128), 4, 160, 1004),
         # the paper's own measurement shape: one sentence, source and target length 30
         Workload("small-b1-s30-greedy30", "small-12x2-d256-v32k-e128", 1, 1, (30, 30), 1, 30, 1005),
+        # the paper's models at its measurement shape (src/tgt 30, batch 1, greedy)
+        Workload("mobilenmt10-b1-s30-greedy30", "mobilenmt-10mb", 10, 1, (30, 30), 1, 30, 1010),
+        Workload("mobilenmt20-b1-s30-greedy30", "mobilenmt-20mb", 20, 1, (30, 30), 1, 30, 1020),
     ]
 }
 

@@ -139,7 +139,9 @@ def test_attention_decode_full_size_sampled():
     assert np.array_equal(got[rows], ref)
 
 
-LN_CASES = [(1, 128, 1.0), (7, 256, 30.0), (33, 512, 700.0), (5, 2048, 1e-3), (100, 1024, 3.0), (1, 64, 1e6)]
+LN_CASES = [(1, 128, 1.0), (7, 256, 30.0), (33, 512, 700.0), (5, 2048, 1e-3), (100, 1024, 3.0), (1, 64, 1e6),
+            # widths with an odd factor (the 20MB model's d = 384), decode and encoder block sizes
+            (3, 384, 1.0), (1500, 384, 30.0), (9, 768, 1e-3), (4, 1152, 700.0), (2, 96, 3e6), (5, 1536, 1e-30)]
 
 
 @pytest.mark.parametrize("M,d,scale", LN_CASES)

@@ -128,3 +128,40 @@ def test_greedy_batch_of_four_taps(stream):
     ids, lens = synth.source_batch(cfg.vocab, 4, 10, 50, 4711)
     kind, n = _check_taps(blob, cfg, ids, lens, 1, 40, 40, [0, 1, 2, 3], stream)
     assert kind == 1 and n == 4
+
+
+@pytest.mark.parametrize("name", ["mobilenmt10-b1-s30-greedy30", "mobilenmt20-b1-s30-greedy30"])
+def test_paper_models_tokens_and_taps(name, stream):
+    """The paper's two models (Table "detailed settings of MobileNMT") at its
+    measurement shape: src/tgt 30, batch 1, greedy.  The 20MB model's width
+    384 = 3 x 128 exercises the LayerNorm's exact division by a width with an
+    odd factor in every kernel that normalises."""
+    cfg, blob, ids, lens, beam, T = synth.workload_inputs(name)
+    _check_taps(blob, cfg, ids, lens, beam, T, T, [0], stream)
+    tr = mnmt.Translator(blob, 1, ids.shape[1], beam, T, stream)
+    try:
+        g_ids, g_len, _ = tr.translate(ids, lens, T)
+    finally:
+        tr.close()
+    o_ids, o_len, _ = O.translate(blob, ids, lens, beam, T)
+    assert np.array_equal(g_ids, o_ids) and np.array_equal(g_len, o_len)
+
+
+@pytest.mark.parametrize("beam,B", [(1, 160), (4, 40)])
+def test_paper_20mb_model_batched(beam, B, stream):
+    """The 20MB model with >= 128 decoder rows (tensor-core linears at K = 384
+    and 768) under greedy and beam search; 4 sentences checked."""
+    cfg = synth.MODELS["mobilenmt-20mb"]
+    blob = synth.build_blob(cfg, 20)
+    ids, lens = synth.source_batch(cfg.vocab, B, 10, 40, 2020)
+    T = 16
+    tr = mnmt.Translator(blob, B, ids.shape[1], beam, T, stream)
+    try:
+        g_ids, g_len, g_sc = tr.translate(ids, lens, T)
+    finally:
+        tr.close()
+    pick = [0, 1, B // 2, B - 1]
+    o_ids, o_len, o_sc = O.translate(blob, ids[pick], lens[pick], beam, T, n_threads=4)
+    assert np.array_equal(g_ids[pick], o_ids) and np.array_equal(g_len[pick], o_len)
+    assert np.array_equal(g_sc[pick].view(np.uint32), o_sc.view(np.uint32))
+    _check_taps(blob, cfg, ids, lens, beam, T, 8, [0, B - 1], stream)

@@ -338,3 +338,46 @@ def test_beam_search_scores_use_the_pinned_log_softmax():
     ref = sum(float(l[out[0, t]]) - _lse64(l) for t, l in enumerate(logits[:n]))
     assert sc[0] == cum
     assert abs(float(sc[0]) - ref) <= 1e-4 * n
+
+
+# ------------------------------------------- LayerNorm statistics, any width
+def _grid_sum(vals, shift):
+    """Exact sum of round-half-even(v * 2^shift) over float32 values v."""
+    from fractions import Fraction
+    tot = 0
+    for v in vals:
+        x = Fraction(float(v)) * (Fraction(2) ** shift)
+        fl = x.numerator // x.denominator
+        rem = x - fl
+        if rem > Fraction(1, 2) or (rem == Fraction(1, 2) and fl % 2 == 1):
+            fl += 1
+        tot += fl
+    return tot
+
+
+@pytest.mark.parametrize("d", [96, 128, 384, 640, 768, 1152, 1536, 2048])
+@pytest.mark.parametrize("scale", [1e-30, 1e-3, 1.0, 700.0, 3e6])
+def test_layernorm_statistics_are_nearest_floats_of_exact_sums(d, scale):
+    """Mean and biased variance (R5): each the nearest float to its exact
+    fixed-point sum over d, for widths with odd factors (d = 384, 768, ... of
+    the 20MB model) as well as powers of two; and within half an ulp plus the
+    grid's rounding of the exact mean of the row."""
+    from fractions import Fraction
+    r = (synth.Stream(d, f"ln{scale}").normal(4 * d).reshape(4, d) * scale + scale * 0.25).astype(np.float32)
+    r[3, ::7] = np.float32(-scale * 2.5)
+    mu, var = O.ln_stats(r)
+    for m in range(4):
+        row = r[m]
+        amax = float(np.max(np.abs(row)))
+        ea = math.frexp(amax)[1]
+        s1 = _grid_sum(row, 52 - ea)
+        exact_mu = Fraction(s1) * Fraction(2) ** (ea - 52) / d
+        assert mu[m] == _nearest_f32(exact_mu), (d, scale, m)
+        true_mean = sum(Fraction(float(v)) for v in row) / d
+        assert abs(Fraction(float(mu[m])) - true_mean) <= Fraction(ulp32(float(mu[m]))) / 2 + \
+            Fraction(2) ** (ea - 52)
+        c = (row - mu[m]).astype(np.float32)
+        c2 = (c * c).astype(np.float32)
+        eb = math.frexp(float(np.max(np.abs(c))))[1]
+        s2 = _grid_sum(c2, 52 - 2 * eb)
+        assert var[m] == _nearest_f32(Fraction(s2) * Fraction(2) ** (2 * eb - 52) / d), (d, scale, m)

@@ -31,3 +31,22 @@ def test_printed_sizes(row):
     if row["flops"] != "-":
         macs = structure.macs(row["V"], row["d"], row["F"], row["ne"], row["nd"], 30, 30)
         assert abs(macs / 1e9 - float(row["flops"])) <= 0.05 + 1e-9
+
+
+def test_synthetic_paper_models_have_the_printed_sizes():
+    """The synthetic MobileNMT-10MB / -20MB models have the shapes of the
+    paper's table and hence its printed parameter counts (10M / 20M)."""
+    from paper_2306_04235_gb300 import synth
+    rows = {r["name"]: r for r in _rows()}
+    for name in ("mobilenmt-10mb", "mobilenmt-20mb"):
+        cfg = synth.MODELS[name]
+        row = rows[name]
+        assert (cfg.vocab, cfg.d_model, cfg.d_ffn, cfg.n_enc, cfg.n_dec) == \
+            (row["V"], row["d"], row["F"], row["ne"], row["nd"])
+        assert cfg.tied_output == 1 and cfg.d_embed == cfg.d_model and cfg.pre_ln == 1
+        total, _ = structure.params(cfg.vocab, cfg.d_model, cfg.d_ffn, cfg.n_enc, cfg.n_dec)
+        assert abs(total / 1e6 - float(row["params"])) <= row["tol"] * float(row["params"])
+        # int8 weights: the model's weight bytes are its size in MB (Table 5 "8-8-8")
+        blob = synth.build_blob(cfg, 1)
+        assert abs(total - float(row["params"]) * 1e6) <= 0.04 * float(row["params"]) * 1e6
+        assert len(blob) > total
