@@ -27,6 +27,9 @@ tokens.  Metric: decoded tokens per second (whole job over all GPUs).
             second as a fraction of the measured dense fp16/bf16 tensor peak
             (the exact int8 route: int8 codes carried as fp16, see the
             tensor-core linear), and the decode step's fraction of HBM
+  paper_models  the paper's MobileNMT-10MB / -20MB shapes at its measurement
+            setting (src/tgt 30, batch 1, greedy): latency per translation and
+            the library's device memory, default and memory-minimal (lean)
   microbench  the int8 linear sweep M in {1..4096} x five (K, N) shapes and
             the wide encoder's linears, each with TOPS and GB/s and its
             fraction of the bounding peak, plus incremental attention over
@@ -247,7 +250,7 @@ def run_reference(args):
 class Workload:
     """One workload's model, session, device buffers and pinned host buffers."""
 
-    def __init__(self, name, mnmt, torch, stream, rank):
+    def __init__(self, name, mnmt, torch, stream, rank, lean=False):
         self.wl = synth.WORKLOADS[name]
         self.cfg = synth.MODELS[self.wl.model]
         self.blob = synth.build_blob(self.cfg, self.wl.model_seed)
@@ -257,7 +260,9 @@ class Workload:
         self.B, self.S = self.ids.shape
         self.T = self.wl.max_len
         self.mnmt, self.torch, self.stream = mnmt, torch, stream
-        self.tr = mnmt.Translator(self.blob, self.B, self.S, self.wl.beam, self.T, stream)
+        self.tr = mnmt.Translator(self.blob, self.B, self.S, self.wl.beam, self.T, stream, lean=lean)
+        self.model_bytes = mnmt.mnmt_model_device_bytes(self.tr.model)
+        self.session_bytes = mnmt.mnmt_session_device_bytes(self.tr.session)
         self.sess = self.tr.session
         dev = "cuda"
         self.d_ids = torch.from_numpy(self.ids).to(dev)
@@ -401,10 +406,10 @@ def measure_decode_step(w, flush, steps_run, cluster):
             "p50_us": srt[len(srt) // 2], "warm_avg_us": warm_us, "launches": len(cold_us)}
 
 
-def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None):
+def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None, lean=False):
     """tokens/s (device-resident and end to end), decode-step latency, encode
     time and the decode step's roofline for one workload."""
-    w = Workload(name, mnmt, torch, stream, rank)
+    w = Workload(name, mnmt, torch, stream, rank, lean)
     try:
         step_ms = time_translations(w, flush, steps, warmup, dist)
         toks_per_step = int(w.o_len.sum().item())
@@ -458,6 +463,30 @@ def batched_entry(name, mnmt, torch, stream, flush, steps, warmup):
                         "cold_avg_us": roof["avg_us"], "cold_p50_us": roof["p50_us"],
                         "warm_avg_us": roof["warm_avg_us"], "kernel": roof["kernel"]},
     }
+
+
+# the paper's on-device figures for its two models (Google Pixel 4 ARM CPU,
+# src/tgt length 30, batch 1, greedy): context, not a target
+PAPER_PIXEL4 = {"mobilenmt10-b1-s30-greedy30": {"latency_ms": 27.3, "memory_mb": 14.9},
+                "mobilenmt20-b1-s30-greedy30": {"latency_ms": 46.3, "memory_mb": 26.0}}
+
+
+def paper_entry(name, mnmt, torch, stream, flush, steps, warmup):
+    """One translation of the paper's measurement shape, default and lean:
+    per-translation latency (encode + 30 greedy steps) and the library's
+    device memory (model + session)."""
+    out = {"workload": name, "paper_pixel4_context": PAPER_PIXEL4[name]}
+    for lean in (False, True):
+        r = measure_workload(name, mnmt, torch, stream, flush, steps, warmup, lean=lean)
+        w = r["w"]
+        su = r["step_us"]
+        out["lean" if lean else "default"] = {
+            "ms_per_translation": r["total_ms"] / steps, "value": r["value"], "unit": "tokens/s",
+            "e2e": r["e2e"]["value"], "decode_step_us_p50": su[len(su) // 2], "encode_ms_p50": r["enc_ms"],
+            "decode_path": "cluster" if r["cluster"] else "multi-kernel",
+            "model_mb": w.model_bytes / 1e6, "session_mb": w.session_bytes / 1e6,
+            "device_mb": (w.model_bytes + w.session_bytes) / 1e6}
+    return out
 
 
 SWEEP_M = [1, 4, 16, 64, 256, 1024, 4096]
@@ -615,6 +644,9 @@ def run_gpu(args):
         with ClockSampler(local) as bclk:
             batched = {"entries": [batched_entry(n, mnmt, torch, stream, flush, 5, 3) for n in BATCHED]}
         batched["clocks"] = bclk.summary()
+    paper = None
+    if rank == 0 and world == 1 and not args.no_batched:
+        paper = [paper_entry(n, mnmt, torch, stream, flush, 10, 3) for n in PAPER_PIXEL4]
     if rank == 0 and world == 1 and not args.no_micro:
         with ClockSampler(local) as mclk:
             micro = microbench(mnmt, torch, stream, flush)
@@ -651,7 +683,9 @@ def run_gpu(args):
             "cpu_baseline": cpu,
             "clocks": clk.summary(),
             "gpu_launches": launches,
+            "device_memory_mb": {"model": w.model_bytes / 1e6, "session": w.session_bytes / 1e6},
             "batched": batched,
+            "paper_models": paper,
             "microbench": micro,
         }
         print(json.dumps(line), flush=True)

@@ -97,6 +97,15 @@ int mnmt_blob_check(const void *blob, size_t bytes, mnmt_config *cfg_out);
  * cuda_stream: cudaStream_t the model and its sessions run on.
  * *out receives the model on success. */
 int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stream, mnmt_model **out);
+
+/* Memory-minimal operation (Sec. 4 "Memory Optimization"; the running memory
+ * column of Table 2).  MNMT_LOAD_LEAN keeps only the int8 blob and the derived
+ * per-column constants on the device (no fp16 copy of the weight codes): every
+ * linear of the model's sessions runs on the int8 GEMV / IMMA kernels, with
+ * results identical to the default load.  flags = 0 is mnmt_load_weights.
+ * MNMT_EINVAL for unknown flags. */
+#define MNMT_LOAD_LEAN 1
+int mnmt_load_weights_ex(const void *blob, size_t bytes, void *cuda_stream, int32_t flags, mnmt_model **out);
 void mnmt_model_free(mnmt_model *model);
 int mnmt_model_config(const mnmt_model *model, mnmt_config *cfg_out);
 
@@ -106,7 +115,26 @@ int mnmt_model_config(const mnmt_model *model, mnmt_config *cfg_out);
  * no later call allocates. */
 int mnmt_session_create(mnmt_model *model, int32_t max_batch, int32_t max_src_len, int32_t beam,
                         int32_t max_len, mnmt_session **out);
+
+/* mnmt_session_create with flags.  MNMT_SESSION_LEAN shares the activation
+ * memory the way the paper's engine does (Sec. 4: operations that are never
+ * live at the same time share one buffer): the encoder and the decoder step
+ * use two int8 buffers -- LayerNorm output / attention context, and QKV
+ * output / FFN hidden -- plus the fp32 residual stream, and no fp16 mirrors
+ * (every linear on the int8 kernels).  Results are identical to the default
+ * session.  MNMT_EINVAL for unknown flags. */
+#define MNMT_SESSION_LEAN 1
+int mnmt_session_create_ex(mnmt_model *model, int32_t max_batch, int32_t max_src_len, int32_t beam,
+                           int32_t max_len, int32_t flags, mnmt_session **out);
 void mnmt_session_free(mnmt_session *s);
+
+/* Device bytes held by a model (blob, derived constants, fp16 operand copy
+ * unless lean) or by a session (its one arena: caches, activations, search
+ * state).  Nothing else is allocated on the device by the library after these
+ * objects are created, so model + session bytes are the library's peak device
+ * memory for a translation.  Negative MNMT_EINVAL for a null handle. */
+int64_t mnmt_model_device_bytes(const mnmt_model *model);
+int64_t mnmt_session_device_bytes(const mnmt_session *s);
 
 /* Encoder (App. A): src_ids [B][S_pad] right-padded with PAD, src_lens [B]
  * (1 <= len <= S_pad).  Runs the encoder stack and the cross-attention key /

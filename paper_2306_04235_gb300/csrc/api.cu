@@ -257,9 +257,11 @@ struct mnmt_model {
     cudaStream_t stream;
     bool own_stream;
     uint8_t *d_blob;
-    __half *d_blob16;  // fp16 copy of every blob byte read as an int8 code (tensor-core operands)
+    __half *d_blob16;  // fp16 copy of every blob byte read as an int8 code (tensor-core operands); null when lean
     float *d_aux;
     size_t bytes;
+    size_t device_bytes;  // every byte of device memory the model holds
+    bool lean;            // loaded with MNMT_LOAD_LEAN: int8 blob only, no fp16 operand copy
     const int8_t *emb_q;
     const float *emb_s;
     bool factorised;
@@ -292,8 +294,14 @@ extern "C" int mnmt_model_config(const mnmt_model *m, mnmt_config *cfg_out) {
 }
 
 extern "C" int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stream, mnmt_model **out) {
+    return mnmt_load_weights_ex(blob, bytes, cuda_stream, 0, out);
+}
+
+extern "C" int mnmt_load_weights_ex(const void *blob, size_t bytes, void *cuda_stream, int32_t flags,
+                                    mnmt_model **out) {
     if (!out) return fail(MNMT_EINVAL, "out is null");
     *out = nullptr;
+    if (flags & ~MNMT_LOAD_LEAN) return fail(MNMT_EINVAL, "unknown load flags 0x%x", flags);
     Layout L;
     int st = parse_layout(blob, bytes, &L);
     if (st) return st;
@@ -302,6 +310,7 @@ extern "C" int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stre
     if (!m) return fail(MNMT_ENOMEM, "host allocation failed");
     m->c = L.c;
     m->bytes = bytes;
+    m->lean = (flags & MNMT_LOAD_LEAN) != 0;
     if (cuda_stream) {
         m->stream = static_cast<cudaStream_t>(cuda_stream);
         m->own_stream = false;
@@ -425,15 +434,20 @@ extern "C" int mnmt_load_weights(const void *blob, size_t bytes, void *cuda_stre
     m->out.k = d;
     // the tensor-core linears read the weight codes as fp16: convert the whole
     // blob once (the fp32 regions become unused garbage); offsets stay 16-byte
-    // aligned, so W16 = d_blob16 + (W - d_blob) is 32-byte aligned
-    if (cudaMalloc(&m->d_blob16, bytes * 2) != cudaSuccess) {
-        mnmt_model_free(m);
-        return fail(MNMT_ENOMEM, "cudaMalloc of %zu fp16 weight bytes failed", bytes * 2);
-    }
-    if (launch_codes_to_f16_flat(reinterpret_cast<const int8_t *>(m->d_blob), m->d_blob16, bytes, m->stream) !=
-        cudaSuccess) {
-        mnmt_model_free(m);
-        return fail(MNMT_ECUDA, "fp16 weight conversion failed");
+    // aligned, so W16 = d_blob16 + (W - d_blob) is 32-byte aligned.  A lean
+    // model keeps the int8 blob only and runs every linear on the int8 kernels.
+    m->device_bytes = bytes + aux.size() * 4;
+    if (!m->lean) {
+        if (cudaMalloc(&m->d_blob16, bytes * 2) != cudaSuccess) {
+            mnmt_model_free(m);
+            return fail(MNMT_ENOMEM, "cudaMalloc of %zu fp16 weight bytes failed", bytes * 2);
+        }
+        m->device_bytes += bytes * 2;
+        if (launch_codes_to_f16_flat(reinterpret_cast<const int8_t *>(m->d_blob), m->d_blob16, bytes, m->stream) !=
+            cudaSuccess) {
+            mnmt_model_free(m);
+            return fail(MNMT_ECUDA, "fp16 weight conversion failed");
+        }
     }
     if (cudaMalloc(&m->d_aux, aux.size() * 4) != cudaSuccess) {
         mnmt_model_free(m);
@@ -509,9 +523,21 @@ static int poison(mnmt_session *s, int code) {
 
 extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max_src_len, int32_t beam,
                                    int32_t max_len, mnmt_session **out) {
+    return mnmt_session_create_ex(m, max_batch, max_src_len, beam, max_len, 0, out);
+}
+
+extern "C" int mnmt_session_create_ex(mnmt_model *m, int32_t max_batch, int32_t max_src_len, int32_t beam,
+                                      int32_t max_len, int32_t flags, mnmt_session **out) {
     if (!out) return fail(MNMT_EINVAL, "out is null");
     *out = nullptr;
     if (!m) return fail(MNMT_EINVAL, "model is null");
+    if (flags & ~MNMT_SESSION_LEAN) return fail(MNMT_EINVAL, "unknown session flags 0x%x", flags);
+    // lean: the encoder and decoder share two int8 activation buffers and the
+    // fp32 residual (the context aliases the LayerNorm output, the FFN hidden
+    // aliases the QKV output: never live at the same time), no fp16 mirrors;
+    // a lean model's sessions run every linear on the int8 kernels
+    const bool lean = (flags & MNMT_SESSION_LEAN) != 0;
+    const bool tc_ok = !lean && !m->lean;
     const mnmt_config &c = m->c;
     if (max_batch < 1 || max_src_len < 1 || max_src_len > 512 || max_src_len > c.max_pos || beam < 1 ||
         beam > 16 || beam > c.vocab || max_len < 1 || max_len > c.max_pos || max_len > 1024)
@@ -536,8 +562,10 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
         off += (bytes + 255) & ~(size_t)255;
         return at;
     };
-    size_t o_resid = piece(rows * d * 4), o_act = piece(rows * (d > F ? d : F)), o_qkv = piece(ME * 3 * d),
-           o_ctx = piece(rows * d), o_hid = piece(rows * F), o_qbuf = piece(R * d), o_encq = piece(ME * d),
+    const size_t qkv_bytes = lean ? std::max(ME * 3 * d, rows * F) : ME * 3 * d;
+    size_t o_resid = piece(rows * d * 4), o_act = piece(rows * (d > F ? d : F)), o_qkv = piece(qkv_bytes),
+           o_ctx = lean ? o_act : piece(rows * d), o_hid = lean ? o_qkv : piece(rows * F), o_qbuf = piece(R * d),
+           o_encq = piece(ME * d),
            o_ck = piece(L * s->ck_layer), o_cv = piece(L * s->ck_layer), o_sk = piece(L * s->sk_layer),
            o_sv = piece(L * s->sk_layer), o_ids = piece(ME * 4), o_lens = piece((size_t)max_batch * 4),
            o_tok = piece(R * 4), o_fin = piece(R * 4), o_cum = piece(R * 4),
@@ -547,7 +575,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
            o_outlens = piece((size_t)max_batch * 4), o_outsc = piece((size_t)max_batch * 4),
            o_state = piece(ST_N * 4), o_dc = piece(sizeof(DcParams)), o_dcln = piece((6 * L + 2) * d * 4);
     const size_t kmax = std::max(d, std::max(F, (size_t)c.d_embed));
-    const bool tc_any = rows >= TC_MIN_ROWS;
+    const bool tc_any = tc_ok && rows >= TC_MIN_ROWS;
     size_t o_a16 = piece(tc_any ? rows * kmax * 2 : 256);
     size_t o_act16 = piece(tc_any ? rows * kmax * 2 : 256), o_ctx16 = piece(tc_any ? rows * d * 2 : 256),
            o_hid16 = piece(tc_any ? rows * F * 2 : 256), o_encq16 = piece(tc_any ? ME * d * 2 : 256);
@@ -603,7 +631,7 @@ extern "C" int mnmt_session_create(mnmt_model *m, int32_t max_batch, int32_t max
     s->encq16 = reinterpret_cast<__half *>(a + o_encq16);
     {
         const char *v = std::getenv("MNMT_TC");
-        s->use_tc = !(v && v[0] == '0') && rows >= TC_MIN_ROWS;
+        s->use_tc = tc_ok && !(v && v[0] == '0') && rows >= TC_MIN_ROWS;
     }
     if (cudaMemsetAsync(s->arena, 0, off, m->stream) != cudaSuccess ||
         cudaStreamSynchronize(m->stream) != cudaSuccess) {
@@ -1380,6 +1408,16 @@ extern "C" int64_t mnmt_debug_tap(mnmt_session *s, int32_t tap, int32_t layer, v
 }
 
 extern "C" const char *mnmt_last_error(void) { return g_err.c_str(); }
+
+extern "C" int64_t mnmt_model_device_bytes(const mnmt_model *m) {
+    if (!m) return fail(MNMT_EINVAL, "model is null");
+    return (int64_t)m->device_bytes;
+}
+
+extern "C" int64_t mnmt_session_device_bytes(const mnmt_session *s) {
+    if (!s) return fail(MNMT_EINVAL, "session is null");
+    return (int64_t)s->arena_bytes;
+}
 
 extern "C" int mnmt_session_decode_path(mnmt_session *s) {
     if (!s) return fail(MNMT_EINVAL, "session is null");

@@ -59,6 +59,10 @@ def _declare(L):
     p, i32, sz, f = C.c_void_p, C.c_int32, C.c_size_t, C.c_float
     L.mnmt_blob_check.argtypes = [p, sz, C.POINTER(_Config)]
     L.mnmt_load_weights.argtypes = [p, sz, p, C.POINTER(p)]
+    L.mnmt_load_weights_ex.argtypes = [p, sz, p, i32, C.POINTER(p)]
+    L.mnmt_session_create_ex.argtypes = [p, i32, i32, i32, i32, i32, C.POINTER(p)]
+    L.mnmt_model_device_bytes.argtypes = [p]; L.mnmt_model_device_bytes.restype = C.c_int64
+    L.mnmt_session_device_bytes.argtypes = [p]; L.mnmt_session_device_bytes.restype = C.c_int64
     L.mnmt_model_free.argtypes = [p]; L.mnmt_model_free.restype = None
     L.mnmt_model_config.argtypes = [p, C.POINTER(_Config)]
     L.mnmt_session_create.argtypes = [p, i32, i32, i32, i32, C.POINTER(p)]
@@ -79,7 +83,8 @@ def _declare(L):
     L.mnmt_linear_tc.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p, p]
     L.mnmt_codes_to_f16.argtypes = [p, p, sz, p]
     L.mnmt_wait_timeout_selftest.argtypes = [p, p]
-    for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
+    for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_load_weights_ex", "mnmt_session_create_ex",
+              "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
               "mnmt_decode_step", "mnmt_translate", "mnmt_linear", "mnmt_linear_argmax", "mnmt_attention_decode", "mnmt_layernorm",
               "mnmt_linear_tc", "mnmt_codes_to_f16", "mnmt_wait_timeout_selftest"]:
         getattr(L, n).restype = C.c_int
@@ -121,10 +126,31 @@ def mnmt_blob_check(blob: bytes) -> dict:
     return {n: getattr(cfg, n) for n, _ in _Config._fields_}
 
 
-def mnmt_load_weights(blob: bytes, stream=None) -> int:
+LOAD_LEAN = 1
+SESSION_LEAN = 1
+
+
+def mnmt_load_weights(blob: bytes, stream=None, flags: int = 0) -> int:
     h = C.c_void_p()
-    _chk(lib().mnmt_load_weights(blob, len(blob), _stream_handle(stream), C.byref(h)))
+    if flags:
+        _chk(lib().mnmt_load_weights_ex(blob, len(blob), _stream_handle(stream), flags, C.byref(h)))
+    else:
+        _chk(lib().mnmt_load_weights(blob, len(blob), _stream_handle(stream), C.byref(h)))
     return h.value
+
+
+def mnmt_model_device_bytes(model: int) -> int:
+    r = lib().mnmt_model_device_bytes(model)
+    if r < 0:
+        raise MnmtError(int(r), last_error())
+    return int(r)
+
+
+def mnmt_session_device_bytes(session: int) -> int:
+    r = lib().mnmt_session_device_bytes(session)
+    if r < 0:
+        raise MnmtError(int(r), last_error())
+    return int(r)
 
 
 def mnmt_model_free(model: int):
@@ -137,9 +163,13 @@ def mnmt_model_config(model: int) -> dict:
     return {n: getattr(cfg, n) for n, _ in _Config._fields_}
 
 
-def mnmt_session_create(model: int, max_batch: int, max_src_len: int, beam: int, max_len: int) -> int:
+def mnmt_session_create(model: int, max_batch: int, max_src_len: int, beam: int, max_len: int,
+                        flags: int = 0) -> int:
     h = C.c_void_p()
-    _chk(lib().mnmt_session_create(model, max_batch, max_src_len, beam, max_len, C.byref(h)))
+    if flags:
+        _chk(lib().mnmt_session_create_ex(model, max_batch, max_src_len, beam, max_len, flags, C.byref(h)))
+    else:
+        _chk(lib().mnmt_session_create(model, max_batch, max_src_len, beam, max_len, C.byref(h)))
     return h.value
 
 
@@ -244,10 +274,13 @@ def mnmt_layernorm(r, g, b, M, d, inv, out_f, out_q, status=None, stream=None):
 class Translator:
     """A loaded model plus one session (owner of both handles)."""
 
-    def __init__(self, blob: bytes, max_batch: int, max_src_len: int, beam: int, max_len: int, stream=None):
-        self.model = mnmt_load_weights(blob, stream)
+    def __init__(self, blob: bytes, max_batch: int, max_src_len: int, beam: int, max_len: int, stream=None,
+                 lean: bool = False):
+        """lean=True: memory-minimal model and session (MNMT_LOAD_LEAN, MNMT_SESSION_LEAN)."""
+        self.model = mnmt_load_weights(blob, stream, LOAD_LEAN if lean else 0)
         try:
-            self.session = mnmt_session_create(self.model, max_batch, max_src_len, beam, max_len)
+            self.session = mnmt_session_create(self.model, max_batch, max_src_len, beam, max_len,
+                                               SESSION_LEAN if lean else 0)
         except Exception:
             mnmt_model_free(self.model)
             raise

@@ -42,3 +42,15 @@ def test_unsupported_shapes_are_rejected_on_host():
     with pytest.raises(mnmt.MnmtError) as ei:
         mnmt.mnmt_blob_check(synth.build_blob(cfg, 3))
     assert ei.value.code == mnmt.EFORMAT
+
+
+def test_paper_model_shapes_pass_host_validation():
+    """d_model = 384 (MobileNMT-20MB, 6 heads of 64) is a supported width."""
+    for name in ("mobilenmt-10mb", "mobilenmt-20mb"):
+        cfg = synth.MODELS[name]
+        got = mnmt.mnmt_blob_check(synth.build_blob(cfg, 1))
+        assert got["d_model"] == cfg.d_model and got["n_heads"] == cfg.n_heads and got["vocab"] == 8000
+    cfg = synth.ModelConfig(1, 1, 352, 4, 128, 300, 352, 1, 1, max_pos=64)   # not a multiple of 64
+    with pytest.raises(mnmt.MnmtError) as ei:
+        mnmt.mnmt_blob_check(synth.build_blob(cfg, 3))
+    assert ei.value.code == mnmt.EFORMAT
