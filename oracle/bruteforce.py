@@ -8,8 +8,11 @@ hidden layer; softmax, biases, residuals and LayerNorm in full precision), so
 its int8 codes agree with the oracle's except where a value lies within
 rounding distance of a .5 boundary, and its float outputs agree to ~1e-6.
 
-It also parses the MNMT v1 blob on its own (numpy views), sharing no code
-with either the C oracle or the CUDA library.
+It also parses the MNMT blob on its own (numpy views), sharing no code
+with either the C oracle or the CUDA library.  Every linear is held as its
+dequantised float64 weight matrix: s_n * code for int8 and symmetric 4-bit
+rows (4-bit codes stored as v + 8), s_n * u + r_n for 4-bit min-max rows
+(App. B Eq. quant).
 """
 from __future__ import annotations
 
@@ -25,14 +28,16 @@ class Blob:
     def __init__(self, blob: bytes):
         self.buf = memoryview(blob)
         magic, ver, *cfg = struct.unpack_from("<4sI13i", blob, 0)
-        assert magic == b"MNMT" and ver == 1
+        assert magic == b"MNMT" and ver in (1, 2)
         (self.n_enc, self.n_dec, self.d, self.H, self.F, self.V, self.E, self.pre_ln,
          self.tied, self.max_pos, self.pad, self.bos, self.eos) = cfg
+        self.wq = struct.unpack_from("<i", blob, 60)[0] if ver == 2 else 8
+        assert self.wq in (8, 4, 4 | 0x100)
         self.off = 64
         d, F, V, E = self.d, self.F, self.V, self.E
         self.emb_q = self._arr(np.int8, (V, E))
         self.emb_s = self._arr(np.float32, (V,))
-        self.proj = self._lin(d, E) if E != d else None
+        self.proj = self._lin(d, E, 8) if E != d else None
         g = self._arr(np.float32, (4,))
         self.emb_scale, self.s_enc, self.s_dout = float(g[0]), float(g[1]), float(g[2])
         self.pe = self._arr(np.float32, (self.max_pos, d))
@@ -45,10 +50,10 @@ class Blob:
             self.dec.append((self._self_attn(), self._cross(), self._ffn()))
         self.dec_final = self._ln() if self.pre_ln else None
         if self.tied:
-            self.out = (self.emb_q, self.emb_s)
+            self.out = self.emb_q.astype(np.float64) * self.emb_s.astype(np.float64)[:, None]
+            self.out_b = self._arr(np.float32, (V,))
         else:
-            self.out = (self._arr(np.int8, (V, d)), self._arr(np.float32, (V,)))
-        self.out_b = self._arr(np.float32, (V,))
+            self.out, self.out_b = self._lin(V, d, 8)
         assert self.off == len(blob), (self.off, len(blob))
 
     def _arr(self, dt, shape):
@@ -58,8 +63,21 @@ class Blob:
         self.off = (self.off + 15) // 16 * 16
         return a
 
-    def _lin(self, n, k):
-        return (self._arr(np.int8, (n, k)), self._arr(np.float32, (n,)), self._arr(np.float32, (n,)))
+    def _lin(self, n, k, wq=None):
+        """(dequantised weight float64 [n][k], bias [n]); wq: the format (the
+        blob's for the attention / FFN linears, 8 for the embedding's)"""
+        wq = self.wq if wq is None else wq
+        if wq == 8:
+            w = self._arr(np.int8, (n, k)).astype(np.float64)
+            s_w = self._arr(np.float32, (n,)).astype(np.float64)
+            return w * s_w[:, None], self._arr(np.float32, (n,))
+        packed = self._arr(np.uint8, (n, k // 2)).reshape(n, k // 32, 16)
+        codes = np.concatenate([packed & 15, packed >> 4], axis=2).reshape(n, k).astype(np.float64)
+        s_w = self._arr(np.float32, (n,)).astype(np.float64)
+        if wq == 4:
+            return (codes - 8.0) * s_w[:, None], self._arr(np.float32, (n,))
+        r = self._arr(np.float32, (n,)).astype(np.float64)
+        return codes * s_w[:, None] + r[:, None], self._arr(np.float32, (n,))
 
     def _ln(self):
         return (self._arr(np.float32, (self.d,)), self._arr(np.float32, (self.d,)))
@@ -90,8 +108,8 @@ def quant(x, s):
 
 
 def linear(codes, s_x, lin):
-    w, s_w, b = lin
-    return (codes @ w.astype(np.float64).T) * (float(s_x) * s_w.astype(np.float64)) + b
+    w, b = lin
+    return (codes * float(s_x)) @ w.T + b
 
 
 def layernorm(x, ln, eps=1e-5):
@@ -123,9 +141,8 @@ class Model:
         if b.proj is None:
             x = rows * b.emb_s[ids].astype(np.float64)[:, None]
         else:
-            w, s_w, bias = b.proj
-            x = (rows @ w.astype(np.float64).T) * (b.emb_s[ids].astype(np.float64)[:, None]
-                                                   * s_w.astype(np.float64)[None, :]) + bias
+            w, bias = b.proj
+            x = (rows * b.emb_s[ids].astype(np.float64)[:, None]) @ w.T + bias
         return x * b.emb_scale + b.pe[pos].astype(np.float64)
 
     def _sub_in(self, r, blk):
@@ -198,5 +215,4 @@ class Model:
             r = self._ffn_block(r, ffn)
         x = layernorm(r, b.dec_final) if b.pre_ln else r
         a = quant(x, b.s_dout)
-        w, s_w = b.out
-        return (a @ w.astype(np.float64).T) * (b.s_dout * s_w.astype(np.float64)) + b.out_b
+        return (a * b.s_dout) @ b.out.T + b.out_b

@@ -30,6 +30,13 @@
  *                       factorisation V*E + E*H (Sec. 2.1 "Scaling E")
  *   greedy / beam ..... greedy search (App. D) and beam search (Table 6 row
  *                       "+Greedy Search" implies beam was the default)
+ *   4-bit weights ..... row-wise low-bit quantisation of the attention and
+ *                       FFN linears (Sec. 3.3 "lower-bit quantization ...
+ *                       row-wise"; the embedding stays 8-bit; Table
+ *                       "quantizing weights to lower bits", 4-8-8): per
+ *                       output row either a symmetric scale (codes -7..7) or
+ *                       the min-max scale and offset of App. B Eq. scale /
+ *                       Eq. quant (codes 0..15, offset r_m = the row minimum)
  *
  * Where the paper is silent (rounding ties, LN epsilon and arithmetic,
  * softmax arithmetic, exp/log, beam details) the reading implemented here is
@@ -55,7 +62,10 @@ typedef struct {
     int n_enc, n_dec, d, H, F, V, E, pre_ln, tied, max_pos, pad, bos, eos;
 } ocfg;
 
-typedef struct { const int8_t *w; const float *s, *b; int n, k; } olin;
+/* A linear: int8 codes w [n][k] (bits 8), or 4-bit codes packed two per byte
+ * in wp (bits 4; see lin_code), with per-row scale s, bias b and, for the
+ * min-max form (asym), per-row offset m. */
+typedef struct { const int8_t *w; const uint8_t *wp; const float *s, *b, *m; int n, k, bits, asym; } olin;
 typedef struct { const float *g, *b; } oln;
 typedef struct { oln ln; float s_in, s_q, s_k, s_v, s_ctx, gamma; olin qkv, o; } oself;
 typedef struct { oln ln; float s_in, s_q, s_k, s_v, s_ctx, gamma; olin q, kv, o; } ocross;
@@ -63,6 +73,7 @@ typedef struct { oln ln; float s_in, s_h, gamma; olin w1, w2; } offn;
 
 typedef struct {
     ocfg c;
+    int wq;
     const int8_t *emb_q;
     const float *emb_s;
     int factorised;
@@ -90,11 +101,22 @@ static const void *take(cursor *cu, size_t bytes) {
     return p;
 }
 
-static olin take_lin(cursor *cu, int n, int k) {
+/* weight format of the blob's linears: 8 = int8 symmetric per row, 4 =
+ * int4 symmetric per row, 4 | WQ_ASYM = int4 min-max per row */
+#define WQ_ASYM 0x100
+static olin take_lin_q(cursor *cu, int n, int k, int wq) {
     olin l;
+    memset(&l, 0, sizeof(l));
     l.n = n; l.k = k;
-    l.w = (const int8_t *)take(cu, (size_t)n * k);
+    l.bits = wq & 0xFF;
+    l.asym = (wq & WQ_ASYM) != 0;
+    if (l.bits == 4) {
+        l.wp = (const uint8_t *)take(cu, (size_t)n * k / 2);
+    } else {
+        l.w = (const int8_t *)take(cu, (size_t)n * k);
+    }
     l.s = (const float *)take(cu, (size_t)n * 4);
+    if (l.asym) l.m = (const float *)take(cu, (size_t)n * 4);
     l.b = (const float *)take(cu, (size_t)n * 4);
     return l;
 }
@@ -113,9 +135,13 @@ static int parse(const void *blob, size_t bytes, omodel *m) {
     if (memcmp(p, "MNMT", 4) != 0) return OR_EFORMAT;
     uint32_t ver;
     memcpy(&ver, p + 4, 4);
-    if (ver != 1) return OR_EFORMAT;
+    if (ver != 1 && ver != 2) return OR_EFORMAT;
     int32_t h[13];
     memcpy(h, p + 8, sizeof(h));
+    int32_t wq = 8; /* version 2 names the linears' weight format at byte 60 */
+    if (ver == 2) memcpy(&wq, p + 60, 4);
+    if (wq != 8 && wq != 4 && wq != (4 | WQ_ASYM)) return OR_EFORMAT;
+    m->wq = wq;
     ocfg *c = &m->c;
     c->n_enc = h[0]; c->n_dec = h[1]; c->d = h[2]; c->H = h[3]; c->F = h[4]; c->V = h[5];
     c->E = h[6]; c->pre_ln = h[7]; c->tied = h[8]; c->max_pos = h[9];
@@ -126,25 +152,28 @@ static int parse(const void *blob, size_t bytes, omodel *m) {
     if (c->tied && c->E != c->d) return OR_EFORMAT;
     if (c->max_pos < 1) return OR_EFORMAT;
     int d = c->d, F = c->F, V = c->V, E = c->E;
+    if (wq != 8 && (d % 32 || F % 32)) return OR_EFORMAT; /* 32-code chunks */
     cursor cu = {p, 64, bytes, 0};
     m->emb_q = (const int8_t *)take(&cu, (size_t)V * E);
     m->emb_s = (const float *)take(&cu, (size_t)V * 4);
     m->factorised = (E != d);
-    if (m->factorised) m->proj = take_lin(&cu, d, E);
+    /* the embedding (its table, factorised projection and an untied output
+     * projection: the "E" of W-E-A) stays 8-bit whatever the linears' format */
+    if (m->factorised) m->proj = take_lin_q(&cu, d, E, 8);
     const float *gl = (const float *)take(&cu, 16);
     m->pe = (const float *)take(&cu, (size_t)c->max_pos * d * 4);
     for (int l = 0; l < c->n_enc; l++) {
         oself *a = &m->enc_self[l];
         a->ln = take_ln(&cu, d);
         const float *s = (const float *)take(&cu, 32);
-        a->qkv = take_lin(&cu, 3 * d, d);
-        a->o = take_lin(&cu, d, d);
+        a->qkv = take_lin_q(&cu, 3 * d, d, wq);
+        a->o = take_lin_q(&cu, d, d, wq);
         if (s) { a->s_in = s[0]; a->s_q = s[1]; a->s_k = s[2]; a->s_v = s[3]; a->s_ctx = s[4]; a->gamma = s[5]; }
         offn *f = &m->enc_ffn[l];
         f->ln = take_ln(&cu, d);
         s = (const float *)take(&cu, 16);
-        f->w1 = take_lin(&cu, F, d);
-        f->w2 = take_lin(&cu, d, F);
+        f->w1 = take_lin_q(&cu, F, d, wq);
+        f->w2 = take_lin_q(&cu, d, F, wq);
         if (s) { f->s_in = s[0]; f->s_h = s[1]; f->gamma = s[2]; }
     }
     if (c->pre_ln) m->enc_final = take_ln(&cu, d);
@@ -152,33 +181,34 @@ static int parse(const void *blob, size_t bytes, omodel *m) {
         oself *a = &m->dec_self[l];
         a->ln = take_ln(&cu, d);
         const float *s = (const float *)take(&cu, 32);
-        a->qkv = take_lin(&cu, 3 * d, d);
-        a->o = take_lin(&cu, d, d);
+        a->qkv = take_lin_q(&cu, 3 * d, d, wq);
+        a->o = take_lin_q(&cu, d, d, wq);
         if (s) { a->s_in = s[0]; a->s_q = s[1]; a->s_k = s[2]; a->s_v = s[3]; a->s_ctx = s[4]; a->gamma = s[5]; }
         ocross *x = &m->dec_cross[l];
         x->ln = take_ln(&cu, d);
         s = (const float *)take(&cu, 32);
-        x->q = take_lin(&cu, d, d);
-        x->kv = take_lin(&cu, 2 * d, d);
-        x->o = take_lin(&cu, d, d);
+        x->q = take_lin_q(&cu, d, d, wq);
+        x->kv = take_lin_q(&cu, 2 * d, d, wq);
+        x->o = take_lin_q(&cu, d, d, wq);
         if (s) { x->s_in = s[0]; x->s_q = s[1]; x->s_k = s[2]; x->s_v = s[3]; x->s_ctx = s[4]; x->gamma = s[5]; }
         offn *f = &m->dec_ffn[l];
         f->ln = take_ln(&cu, d);
         s = (const float *)take(&cu, 16);
-        f->w1 = take_lin(&cu, F, d);
-        f->w2 = take_lin(&cu, d, F);
+        f->w1 = take_lin_q(&cu, F, d, wq);
+        f->w2 = take_lin_q(&cu, d, F, wq);
         if (s) { f->s_in = s[0]; f->s_h = s[1]; f->gamma = s[2]; }
     }
     if (c->pre_ln) m->dec_final = take_ln(&cu, d);
     m->out.n = V; m->out.k = d;
     if (c->tied) {
+        /* the output projection is the 8-bit embedding table (the "E" of W-E-A) */
+        m->out.bits = 8;
         m->out.w = m->emb_q;
         m->out.s = m->emb_s;
     } else {
-        m->out.w = (const int8_t *)take(&cu, (size_t)V * d);
-        m->out.s = (const float *)take(&cu, (size_t)V * 4);
+        m->out = take_lin_q(&cu, V, d, 8);
     }
-    m->out.b = (const float *)take(&cu, (size_t)V * 4);
+    if (c->tied) m->out.b = (const float *)take(&cu, (size_t)V * 4);
     if (cu.bad || cu.off != bytes) return OR_EFORMAT;
     m->emb_scale = gl[0]; m->s_enc = gl[1]; m->s_dout = gl[2];
     return OR_OK;
@@ -214,10 +244,42 @@ static float dequant_bias(int32_t acc, float s_x, float s_w, float b) {
     return t + b;
 }
 
+/* The 4-bit code of weight (n, k): the codes of a row are packed in chunks of
+ * 32 codes held in 16 bytes, code j of a chunk in the low nibble of byte j
+ * (j < 16) or the high nibble of byte j - 16.  Symmetric rows store v + 8 for
+ * a code v in [-7, 7]; min-max rows store u in [0, 15]. */
+static int lin_code(const olin *L, int n, int k) {
+    const uint8_t byte = L->wp[(size_t)n * L->k / 2 + (size_t)(k / 32) * 16 + (k % 32) % 16];
+    return (k % 32) < 16 ? (byte & 15) : (byte >> 4);
+}
+
+/* Output n of a quantised linear on the int8 row a at activation scale s_x.
+ *   8-bit and 4-bit symmetric rows (codes v): the dequant-then-bias of
+ *     dequant_bias on the exact integer sum of a_k v_nk.
+ *   4-bit min-max rows, W_nk = s_n u_nk + r_n (App. B Eq. quant with the row
+ *     minimum r_n as offset): x W_n = s_x (s_n sum a_k u_nk + r_n sum a_k)
+ *     exactly, so with the two integer sums A_u and A_1,
+ *     y = fl(fl(fl(A_u fl(s_x s_n)) + fl(A_1 fl(s_x r_n))) + b_n). */
+static float lin_out(const olin *L, int n, const int8_t *a, float s_x) {
+    if (L->bits == 8) return dequant_bias(dot_i8(a, L->w + (size_t)n * L->k, L->k), s_x, L->s[n], L->b[n]);
+    int32_t acc = 0, a1 = 0;
+    for (int k = 0; k < L->k; k++) {
+        int u = lin_code(L, n, k);
+        acc += (int32_t)a[k] * (L->asym ? u : u - 8);
+        a1 += a[k];
+    }
+    if (!L->asym) return dequant_bias(acc, s_x, L->s[n], L->b[n]);
+    float sc = s_x * L->s[n];
+    float mc = s_x * L->m[n];
+    float t = (float)acc * sc;
+    float o = (float)a1 * mc;
+    float y = t + o;
+    return y + L->b[n];
+}
+
 /* Quantised linear on one row: y[n] for n in [0, N). */
 static void linear_row(const int8_t *a, float s_x, const olin *L, float *y) {
-    for (int n = 0; n < L->n; n++)
-        y[n] = dequant_bias(dot_i8(a, L->w + (size_t)n * L->k, L->k), s_x, L->s[n], L->b[n]);
+    for (int n = 0; n < L->n; n++) y[n] = lin_out(L, n, a, s_x);
 }
 
 /* Nearest float (ties to even) to the exact value s 2^e / d, |s| < 2^63,
@@ -394,8 +456,7 @@ static void embed(const omodel *m, int id, int pos, float *x) {
         }
     } else {
         for (int n = 0; n < c->d; n++) {
-            int32_t acc = dot_i8(row, m->proj.w + (size_t)n * c->E, c->E);
-            float y = dequant_bias(acc, m->emb_s[id], m->proj.s[n], m->proj.b[n]);
+            float y = lin_out(&m->proj, n, row, m->emb_s[id]);
             float t = y * m->emb_scale;
             x[n] = t + pe[n];
         }
@@ -852,6 +913,79 @@ int oracle_check_blob(const void *blob, size_t bytes, int32_t *cfg_out) {
 }
 
 float oracle_q8(float x, float inv) { return (float)q8(x, inv); }
+
+/* Row-wise quantisation of a float64 matrix W [N][K] to `bits` bits (App. B
+ * Eq. scale / Eq. quant; Sec. 3.3 per-row "row-wise" scales for low bits).
+ *   symmetric (asym = 0): s_n = fl32(max_k |W_nk| / (2^(bits-1) - 1)), code
+ *     v = clamp(rne(W_nk / s_n), -(2^(bits-1) - 1), 2^(bits-1) - 1): Eq. quant
+ *     with the range [-max|W_n|, max|W_n|] and zero offset.
+ *   min-max (asym = 1): r_n = fl32(min_k W_nk), s_n = fl32((max_k W_nk - r_n) /
+ *     (2^bits - 1)), code u = clamp(rne((W_nk - r_n) / s_n), 0, 2^bits - 1);
+ *     the dequantised weight is s_n u + r_n.
+ * codes [N][K] receive v or u; s [N], m [N] (r_n; 0 when symmetric).  A row
+ * of zeros (or a constant row, min-max) gets scale 1. */
+int oracle_quantise_rows(const double *W, int N, int K, int bits, int asym, int32_t *codes, float *s,
+                         float *m) {
+    if (bits < 2 || bits > 8 || N < 1 || K < 1) return OR_EINVAL;
+    for (int n = 0; n < N; n++) {
+        const double *w = W + (size_t)n * K;
+        double lo = w[0], hi = w[0], amax = 0.0;
+        for (int k = 0; k < K; k++) {
+            if (w[k] < lo) lo = w[k];
+            if (w[k] > hi) hi = w[k];
+            if (fabs(w[k]) > amax) amax = fabs(w[k]);
+        }
+        if (!asym) {
+            int qmax = (1 << (bits - 1)) - 1;
+            float sn = amax > 0.0 ? (float)(amax / qmax) : 1.0f;
+            s[n] = sn;
+            m[n] = 0.0f;
+            for (int k = 0; k < K; k++) {
+                double t = rint(w[k] / (double)sn);
+                if (t > qmax) t = qmax;
+                if (t < -qmax) t = -qmax;
+                codes[(size_t)n * K + k] = (int32_t)t;
+            }
+        } else {
+            int qmax = (1 << bits) - 1;
+            float rn = (float)lo;
+            float sn = hi > (double)rn ? (float)((hi - (double)rn) / qmax) : 1.0f;
+            if (sn == 0.0f) sn = 1.0f;
+            s[n] = sn;
+            m[n] = rn;
+            for (int k = 0; k < K; k++) {
+                double t = rint((w[k] - (double)rn) / (double)sn);
+                if (t > qmax) t = qmax;
+                if (t < 0) t = 0;
+                codes[(size_t)n * K + k] = (int32_t)t;
+            }
+        }
+    }
+    return OR_OK;
+}
+
+/* A 4-bit quantised linear on M int8 rows (kernel-level parity): Wp [N][K/2]
+ * packed as in the blob (lin_code), s / m / b [N] (m only if asym); mode as
+ * oracle_linear. */
+int oracle_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s_w, const float *m_w, const float *b,
+                     float s_x, const float *inv_out, float gamma, int M, int N, int K, int asym, int mode,
+                     int8_t *out_q, float *out_f) {
+    if (K % 32) return OR_EINVAL;
+    olin L;
+    memset(&L, 0, sizeof(L));
+    L.wp = Wp; L.s = s_w; L.m = m_w; L.b = b; L.n = N; L.k = K; L.bits = 4; L.asym = asym;
+    for (int mm = 0; mm < M; mm++) {
+        for (int n = 0; n < N; n++) {
+            float y = lin_out(&L, n, A + (size_t)mm * K, s_x);
+            size_t o = (size_t)mm * N + n;
+            if (mode == 0) out_q[o] = q8(y, inv_out[n]);
+            else if (mode == 1) out_q[o] = q8(y > 0.0f ? y : 0.0f, inv_out[n]);
+            else if (mode == 2) { float t = gamma * out_f[o]; out_f[o] = t + y; }
+            else out_f[o] = y;
+        }
+    }
+    return OR_OK;
+}
 
 /* The LayerNorm's mean and biased variance of M rows of length d. */
 int oracle_ln_stats(const float *r, int M, int d, float *mu, float *var) {

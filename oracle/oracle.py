@@ -70,10 +70,13 @@ def _declare(L):
     L.oracle_log_softmax.argtypes = [_p, _i, _p]
     L.oracle_log_softmax_norm.argtypes = [_p, _i, _p, _p, _p]
     L.oracle_ln_stats.argtypes = [_p, _i, _i, _p, _p]
+    L.oracle_quantise_rows.argtypes = [_p, _i, _i, _i, _i, _p, _p, _p]
+    L.oracle_linear_w4.argtypes = [_p, _p, _p, _p, _p, _f, _p, _f, _i, _i, _i, _i, _i, _p, _p]
     L.oracle_translate.argtypes = [_p, _sz, _p, _p, _i, _i, _i, _i, _i, _p, _p, _p]
     for name in ["oracle_check_blob", "oracle_linear", "oracle_layernorm", "oracle_attention_decode",
                  "oracle_attention_probs", "oracle_encode", "oracle_decode_trace",
                  "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_log_softmax_norm", "oracle_ln_stats",
+                 "oracle_quantise_rows", "oracle_linear_w4",
                  "oracle_translate"]:
         getattr(L, name).restype = _i
 
@@ -157,6 +160,35 @@ def layernorm(r, g, b, inv=1.0):
     if st != OK:
         raise OracleError(f"oracle returned {st}")
     return of, oq
+
+
+def quantise_rows(W, bits, asym):
+    """Row-wise quantisation (App. B Eq. scale / Eq. quant): (codes int32 [N][K], s [N], m [N])."""
+    W = np.ascontiguousarray(W, np.float64)
+    N, K = W.shape
+    codes = np.zeros((N, K), np.int32); s_ = np.zeros(N, np.float32); m_ = np.zeros(N, np.float32)
+    _chk(lib().oracle_quantise_rows(_ptr(W), N, K, int(bits), int(asym), _ptr(codes), _ptr(s_), _ptr(m_)))
+    return codes, s_, m_
+
+
+def linear_w4(A, Wp, s_w, m_w, b, s_x, mode, asym, inv_out=None, gamma=1.0, resid=None):
+    """4-bit linear; Wp [N][K/2] packed as in the blob."""
+    A = np.ascontiguousarray(A, np.int8); Wp = np.ascontiguousarray(Wp, np.uint8)
+    s_w = np.ascontiguousarray(s_w, np.float32); b = np.ascontiguousarray(b, np.float32)
+    m_w = None if m_w is None else np.ascontiguousarray(m_w, np.float32)
+    M, K = A.shape; N = Wp.shape[0]
+    out_q = out_f = None
+    if mode in (MODE_Q8, MODE_RELU_Q8):
+        inv_out = np.ascontiguousarray(np.broadcast_to(np.float32(inv_out) if np.isscalar(inv_out)
+                                                       else inv_out, (N,)), np.float32)
+        out_q = np.zeros((M, N), np.int8)
+    elif mode == MODE_RESID:
+        out_f = np.array(resid, dtype=np.float32, copy=True).reshape(M, N)
+    else:
+        out_f = np.zeros((M, N), np.float32)
+    _chk(lib().oracle_linear_w4(_ptr(A), _ptr(Wp), _ptr(s_w), _ptr(m_w), _ptr(b), float(s_x), _ptr(inv_out),
+                                float(gamma), M, N, K, int(asym), mode, _ptr(out_q), _ptr(out_f)))
+    return out_q if out_q is not None else out_f
 
 
 def ln_stats(r):

@@ -163,13 +163,50 @@ def _f32(x: float) -> float:
     return struct.unpack("<f", struct.pack("<f", float(x)))[0]
 
 
+# weight formats of the linears (the blob header's wq field): int8 symmetric
+# per row, int4 symmetric per row, int4 min-max (scale and offset) per row
+WQ_INT8, WQ_INT4, WQ_INT4_MINMAX = 8, 4, 4 | 0x100
+
+
+def weight_draw(st: Stream, n: int, k: int, std: float = 0.02) -> np.ndarray:
+    """The float64 N(0, std) [n][k] matrix a quantised weight is made from."""
+    return st.normal(n * k).reshape(n, k) * std
+
+
+def int4_weight(w: np.ndarray, minmax: bool):
+    """Per-row 4-bit codes of a float matrix (row-wise low-bit quantisation):
+    symmetric: s = fl32(max|w|/7), v = clip(rint(w/s), -7, 7), stored as v + 8;
+    min-max: r = fl32(min w), s = fl32((max w - r)/15), u = clip(rint((w - r)/s), 0, 15).
+    Returns (stored codes uint8 [n][k] in 0..15, s f32 [n], r f32 [n] or None)."""
+    if not minmax:
+        amax = np.abs(w).max(axis=1)
+        s = np.where(amax > 0, amax / 7.0, 1.0).astype(np.float32)
+        v = np.clip(np.rint(w / s.astype(np.float64)[:, None]), -7, 7)
+        return (v + 8).astype(np.uint8), s, None
+    r = w.min(axis=1).astype(np.float32)
+    span = w.max(axis=1) - r.astype(np.float64)
+    s = np.where(span > 0, span / 15.0, 1.0).astype(np.float32)
+    s = np.where(s > 0, s, np.float32(1.0)).astype(np.float32)
+    u = np.clip(np.rint((w - r.astype(np.float64)[:, None]) / s.astype(np.float64)[:, None]), 0, 15)
+    return u.astype(np.uint8), s, r
+
+
+def pack4(codes: np.ndarray) -> np.ndarray:
+    """Pack 4-bit codes [n][k] (k a multiple of 32) two per byte: each run of 32
+    codes fills 16 bytes, code j in the low nibble of byte j (j < 16) and code
+    16 + j in its high nibble."""
+    n, k = codes.shape
+    c = codes.reshape(n, k // 32, 2, 16).astype(np.uint8)
+    return np.ascontiguousarray((c[:, :, 0, :] | (c[:, :, 1, :] << 4)).reshape(n, k // 2))
+
+
 def int8_weight(st: Stream, n: int, k: int, std: float = 0.02):
     """Per-row symmetric int8 codes of an N(0, std) [n][k] matrix and the row scales.
 
     The codes are the row-absmax normalised rounding of the Gaussian draw, which
     is how a per-output-channel quantised checkpoint looks; they are data here.
     """
-    w = st.normal(n * k).reshape(n, k) * std
+    w = weight_draw(st, n, k, std)
     amax = np.abs(w).max(axis=1)
     amax = np.where(amax > 0, amax, 1.0)
     s = (amax / 127.0).astype(np.float32)
@@ -243,20 +280,28 @@ CROSS_GAINS = {"qk": 10.0, "v": 3.0, "o": 40.0}
 NO_GAINS = {"qk": 1.0, "v": 1.0, "o": 1.0}
 
 
-def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cross_gains=None) -> bytes:
+def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cross_gains=None,
+               wq: int = WQ_INT8) -> bytes:
     """Write a seeded synthetic model in the MNMT v1 blob format.
 
     gamma_range: None for gamma_i = 1 on every sublayer, or (lo, hi) to draw each
     sublayer's residual weight uniformly.  out_bias: optional dict {token: value}
     added to the output bias (used to force e.g. immediate EOS).  cross_gains:
     the cross-attention weight-std multipliers (default CROSS_GAINS; NO_GAINS
-    draws every weight N(0, 0.02)).
+    draws every weight N(0, 0.02)).  wq: the weight format of every linear
+    (WQ_INT8; WQ_INT4 / WQ_INT4_MINMAX write a version-2 blob whose attention
+    and FFN linears hold 4-bit codes; the embedding -- table, factorised
+    projection, untied output projection -- stays int8).
     """
+    assert wq in (WQ_INT8, WQ_INT4, WQ_INT4_MINMAX)
     d, F, V, E = cfg.d_model, cfg.d_ffn, cfg.vocab, cfg.d_embed
     sc = activation_scales(cfg)
     cg = dict(CROSS_GAINS if cross_gains is None else cross_gains)
     w = _BlobWriter()
-    hdr = struct.pack("<4sI13i", b"MNMT", 1, *cfg.as_ints())
+    if wq == WQ_INT8:
+        hdr = struct.pack("<4sI13i", b"MNMT", 1, *cfg.as_ints())
+    else:
+        hdr = struct.pack("<4sI13ii", b"MNMT", 2, *cfg.as_ints(), wq)
     hdr += b"\0" * (64 - len(hdr))
     w.parts.append(hdr)
     w.size = 64
@@ -267,13 +312,23 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cro
         lo, hi = gamma_range
         return _f32(lo + (hi - lo) * st.uniform(1)[0])
 
-    def linear(name, n, k, std=0.02):
+    def put_weight(st, n, k, std):
+        """codes [+ row offsets] and row scales of one linear's weight, in blob order"""
+        if wq == WQ_INT8:
+            q, s_ = int8_weight(st, n, k, std)
+            return [q, s_]
+        u, s_, r = int4_weight(weight_draw(st, n, k, std), wq == WQ_INT4_MINMAX)
+        return [pack4(u), s_] + ([r] if r is not None else [])
+
+    def linear(name, n, k, std=0.02, embedding=False):
         st = Stream(seed, name)
-        q, s = int8_weight(st, n, k, std)
-        b = f32_normal(Stream(seed, name + ".b"), n, 0.0, 0.02)
-        w.put(q)
-        w.put(s)
-        w.put(b)
+        if embedding:  # part of the embedding: 8-bit in every format
+            for arr in int8_weight(st, n, k, std):
+                w.put(arr)
+        else:
+            for arr in put_weight(st, n, k, std):
+                w.put(arr)
+        w.put(f32_normal(Stream(seed, name + ".b"), n, 0.0, 0.02))
 
     def ln(name):
         w.put(f32_normal(Stream(seed, name + ".g"), d, 1.0, 0.02))
@@ -302,10 +357,10 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cro
         if cg["qk"] == cg["v"]:
             linear(prefix + ".kv", 2 * d, d, 0.02 * cg["qk"])
         else:  # key rows and value rows drawn with their own std, stored as one [2d][d] linear
-            qk_, sk_ = int8_weight(Stream(seed, prefix + ".kv"), d, d, 0.02 * cg["qk"])
-            qv_, sv_ = int8_weight(Stream(seed, prefix + ".kv.v"), d, d, 0.02 * cg["v"])
-            w.put(np.concatenate([qk_, qv_]))
-            w.put(np.concatenate([sk_, sv_]))
+            pk = put_weight(Stream(seed, prefix + ".kv"), d, d, 0.02 * cg["qk"])
+            pv = put_weight(Stream(seed, prefix + ".kv.v"), d, d, 0.02 * cg["v"])
+            for a_, b_ in zip(pk, pv):
+                w.put(np.concatenate([a_, b_]))
             w.put(f32_normal(Stream(seed, prefix + ".kv.b"), 2 * d, 0.0, 0.02))
         linear(prefix + ".o", d, d, 0.02 * cg["o"])
 
@@ -320,7 +375,7 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cro
     w.put(eq)
     w.put(es)
     if E != d:
-        linear("embed.proj", d, E)
+        linear("embed.proj", d, E, embedding=True)
     # emb_scale = fl32(sqrt(d)); s_enc, s_dout: quant scales of the encoder
     # output (cross K/V input) and of the decoder output (vocab input)
     w.put(np.array([_f32(math.sqrt(d)), sc["ln"], sc["ln"], 0], dtype=np.float32))
@@ -336,7 +391,7 @@ def build_blob(cfg: ModelConfig, seed: int, gamma_range=None, out_bias=None, cro
         ffn(f"dec{l}.ffn")
     if cfg.pre_ln:
         ln("dec.final")
-    if not cfg.tied_output:
+    if not cfg.tied_output:  # the output embedding: 8-bit in every format
         oq, os_ = int8_weight(Stream(seed, "out"), V, d)
         w.put(oq)
         w.put(os_)
