@@ -27,6 +27,8 @@ tokens.  Metric: decoded tokens per second (whole job over all GPUs).
             second as a fraction of the measured dense fp16/bf16 tensor peak
             (the exact int8 route: int8 codes carried as fp16, see the
             tensor-core linear), and the decode step's fraction of HBM
+  w4        the batch-1 workload with row-wise 4-bit attention / FFN weights
+            (symmetric, and min-max scale + offset), 8-bit embedding
   paper_models  the paper's MobileNMT-10MB / -20MB shapes at its measurement
             setting (src/tgt 30, batch 1, greedy): latency per translation and
             the library's device memory, default and memory-minimal (lean)
@@ -164,7 +166,7 @@ def kernels_per_translation(cfg, B, S, beam, steps_launched, cluster):
     return enc + 1 + step * steps_launched + 1
 
 
-def decode_step_bytes(cfg, R, B, S, t):
+def decode_step_bytes(cfg, R, B, S, t, wq=8):
     """Algorithmic bytes one decode step must move for R hypotheses of B
     sentences (padded source length S) at step t: every decoder weight (int8),
     its per-output-channel scale and bias (fp32) and the requantisation
@@ -174,6 +176,8 @@ def decode_step_bytes(cfg, R, B, S, t):
     per hypothesis, cross [S] per sentence)."""
     d, F, V, E, L = cfg.d_model, cfg.d_ffn, cfg.vocab, cfg.d_embed, cfg.n_dec
     w = L * (6 * d * d + 2 * F * d)
+    if wq != 8:  # 4-bit attention / FFN codes (+ a row offset per output row in the min-max form)
+        w = w // 2 + (4 * L * (7 * d + F) if wq & 0x100 else 0)
     rows = L * (6 * d + F)
     inv = L * (4 * d + F)
     ln = (3 * L + (1 if cfg.pre_ln else 0)) * 2 * d * 4
@@ -250,10 +254,11 @@ def run_reference(args):
 class Workload:
     """One workload's model, session, device buffers and pinned host buffers."""
 
-    def __init__(self, name, mnmt, torch, stream, rank, lean=False):
+    def __init__(self, name, mnmt, torch, stream, rank, lean=False, wq=8):
         self.wl = synth.WORKLOADS[name]
         self.cfg = synth.MODELS[self.wl.model]
-        self.blob = synth.build_blob(self.cfg, self.wl.model_seed)
+        self.wq = wq
+        self.blob = synth.build_blob(self.cfg, self.wl.model_seed, wq=wq)
         # every rank translates its own replica batch (independent sentences)
         self.ids, self.lens = synth.source_batch(self.cfg.vocab, self.wl.batch, self.wl.src_len[0],
                                                  self.wl.src_len[1], self.wl.src_seed + 101 * rank)
@@ -391,7 +396,7 @@ def measure_decode_step(w, flush, steps_run, cluster):
     cold_us = [a.elapsed_time(b) * 1e3 for a, b in cold]
     avg_us = sum(cold_us) / len(cold_us)
     warm_us = w0.elapsed_time(w1) * 1e3 / n
-    algo = sum(decode_step_bytes(cfg, R, w.B, w.S, t) for t in range(n)) / n
+    algo = sum(decode_step_bytes(cfg, R, w.B, w.S, t, w.wq) for t in range(n)) / n
     peak, kind = _peaks()
     achieved = algo / (avg_us * 1e-6) / 1e9
     unit = ("decode_cluster_kernel + vocab_greedy_kernel (one graph launch)" if cluster
@@ -406,10 +411,11 @@ def measure_decode_step(w, flush, steps_run, cluster):
             "p50_us": srt[len(srt) // 2], "warm_avg_us": warm_us, "launches": len(cold_us)}
 
 
-def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None, lean=False):
+def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None, lean=False,
+                     wq=8):
     """tokens/s (device-resident and end to end), decode-step latency, encode
     time and the decode step's roofline for one workload."""
-    w = Workload(name, mnmt, torch, stream, rank, lean)
+    w = Workload(name, mnmt, torch, stream, rank, lean, wq)
     try:
         step_ms = time_translations(w, flush, steps, warmup, dist)
         toks_per_step = int(w.o_len.sum().item())
@@ -487,6 +493,22 @@ def paper_entry(name, mnmt, torch, stream, flush, steps, warmup):
             "model_mb": w.model_bytes / 1e6, "session_mb": w.session_bytes / 1e6,
             "device_mb": (w.model_bytes + w.session_bytes) / 1e6}
     return out
+
+
+def w4_entry(name, wq, mnmt, torch, stream, flush, steps, warmup):
+    """The batch-1 workload's model with 4-bit attention / FFN weights."""
+    r = measure_workload(name, mnmt, torch, stream, flush, steps, warmup, wq=wq)
+    w = r["w"]
+    su = r["step_us"]
+    roof = r["roofline"]
+    return {"workload": name, "weights": "4-bit symmetric rows" if wq == synth.WQ_INT4 else "4-bit min-max rows",
+            "value": r["value"], "unit": "tokens/s", "e2e": r["e2e"]["value"],
+            "decode_step_us_p50": su[len(su) // 2], "encode_ms_p50": r["enc_ms"],
+            "decode_path": "cluster" if r["cluster"] else "multi-kernel",
+            "model_mb": w.model_bytes / 1e6, "blob_mb": len(w.blob) / 1e6,
+            "decode_step": {"bound": "hbm", "achieved": roof["achieved"], "peak": roof["peak"], "unit": "GB/s",
+                            "frac": roof["frac"], "algorithmic_bytes": roof["algorithmic_bytes"],
+                            "cold_avg_us": roof["avg_us"], "warm_avg_us": roof["warm_avg_us"]}}
 
 
 SWEEP_M = [1, 4, 16, 64, 256, 1024, 4096]
@@ -644,9 +666,11 @@ def run_gpu(args):
         with ClockSampler(local) as bclk:
             batched = {"entries": [batched_entry(n, mnmt, torch, stream, flush, 5, 3) for n in BATCHED]}
         batched["clocks"] = bclk.summary()
-    paper = None
+    paper = w4 = None
     if rank == 0 and world == 1 and not args.no_batched:
         paper = [paper_entry(n, mnmt, torch, stream, flush, 10, 3) for n in PAPER_PIXEL4]
+        w4 = [w4_entry(DEFAULT_WORKLOAD, q, mnmt, torch, stream, flush, 10, 3)
+              for q in (synth.WQ_INT4, synth.WQ_INT4_MINMAX)]
     if rank == 0 and world == 1 and not args.no_micro:
         with ClockSampler(local) as mclk:
             micro = microbench(mnmt, torch, stream, flush)
@@ -686,6 +710,7 @@ def run_gpu(args):
             "device_memory_mb": {"model": w.model_bytes / 1e6, "session": w.session_bytes / 1e6},
             "batched": batched,
             "paper_models": paper,
+            "w4": w4,
             "microbench": micro,
         }
         print(json.dumps(line), flush=True)

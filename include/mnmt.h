@@ -24,8 +24,16 @@
  *   - Token ids are in [0, vocab); PAD = 0, BOS = 1 (decoder start), EOS = 2
  *     (the ids the blob header carries).
  *
- * MNMT v1 weight blob (little endian).  64-byte header: char magic[4] = "MNMT",
- * uint32 version = 1, int32 config[13] in mnmt_config field order, zero padding.
+ * MNMT weight blob (little endian).  64-byte header: char magic[4] = "MNMT",
+ * uint32 version (1 or 2), int32 config[13] in mnmt_config field order, then
+ * (version 2 only) int32 wq at byte 60, zero padding.  wq is the format of the
+ * attention and FFN linears (Sec. 3.3, table "quantizing weights to lower
+ * bits"): 8 = int8 (version 1), 4 = 4-bit symmetric rows, 0x104 = 4-bit
+ * min-max rows (App. B Eq. scale / Eq. quant); see mnmt_linear_w4 for the
+ * 4-bit codes.  In a 4-bit linear the codes are packed [N][K/2] and the
+ * min-max form stores f32 m[N] (row offsets) between s_w and b.  The
+ * embedding table, its factorised projection and an untied output projection
+ * (the embedding of W-E-A) are int8 in every format.
  * Then the arrays below in this order, each starting at a 16-byte aligned
  * offset (zero padding between arrays), the blob ending right after the last
  * array's padding.  A "linear" is {int8 W[N][K] (row n = output channel,
@@ -256,6 +264,23 @@ enum { MNMT_EPI_ARGMAX = 4 };
 int mnmt_linear_tc(const uint16_t *A16, const uint16_t *W16, const float *s_w, const float *bias, float s_x,
                    const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
                    int8_t *out_q, float *out_f, uint64_t *keys, int32_t *status, void *cuda_stream);
+
+/* Quantised linear with row-wise 4-bit weights (Sec. 3.3: low-bit weights are
+ * quantised row-wise; table "quantizing weights to lower bits", 4-8-8).
+ * Wp [N][K/2] holds each row's K codes packed in runs of 32 codes per 16
+ * bytes: code j of a run in the low nibble of byte j (j < 16), code 16 + j in
+ * the high nibble of byte j.  m_w == NULL: symmetric rows, stored code
+ * c = v + 8 for v in [-7, 7], W[n][k] = s_w[n] v, and every mode is exactly
+ * mnmt_linear's on the codes v.  m_w != NULL: min-max rows (App. B Eq. scale /
+ * Eq. quant), code u in [0, 15], W[n][k] = s_w[n] u + m_w[n]; with
+ * A_u = sum_k A[m][k] u and A_1 = sum_k A[m][k] (exact int32)
+ *   y = fl(fl(fl(A_u fl(s_x s_w[n])) + fl(A_1 fl(s_x m_w[n]))) + bias[n]),
+ * then mode as in mnmt_linear, or MNMT_EPI_ARGMAX into keys (as in
+ * mnmt_linear_tc).  K a multiple of 32 in [32, 3072]; A and Wp 16-byte
+ * aligned; any M (rows beyond 16 are taken 16 at a time). */
+int mnmt_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s_w, const float *m_w, const float *bias,
+                   float s_x, const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
+                   int8_t *out_q, float *out_f, uint64_t *keys, void *cuda_stream);
 
 /* dst[i] = the fp16 value of the int8 code src[i] (exact), i < n.  Device
  * pointers, src and dst 16-byte aligned. */

@@ -18,7 +18,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libmnmt.so")
-SOURCES = ["api.cu", "linear.cu", "gemm_tc.cu", "attention.cu", "rows.cu", "decode_cluster.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "linear.cu", "linear_w4.cu", "gemm_tc.cu", "attention.cu", "rows.cu", "decode_cluster.cu",
+           "noalloc.cu"]
 HEADERS = ["common.cuh", "epilogue.cuh", "internal.h", "mbarrier.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -81,9 +81,12 @@ static int lib_init() {
 // ---------------------------------------------------------------------------
 namespace {
 
+constexpr int WQ_MINMAX = 0x100;  // blob v2: 4-bit rows with a min-max scale and offset
+
 struct LinOff {
-    size_t w, s, b;
-    int n, k;
+    size_t w, s, b, m;
+    int n, k, bits;
+    bool minmax;
 };
 struct SelfOff {
     size_t ln_g, ln_b, sc;
@@ -99,6 +102,7 @@ struct FfnOff {
 };
 struct Layout {
     mnmt_config c;
+    int wq;  // weight format of the attention / FFN linears: 8, 4, or 4 | WQ_MINMAX
     size_t emb_q, emb_s, globals, pe, enc_ln_g, enc_ln_b, dec_ln_g, dec_ln_b, out_w, out_s, out_b;
     LinOff proj;
     std::vector<SelfOff> enc_self, dec_self;
@@ -119,12 +123,17 @@ struct Walker {
         if (off > size) off = size;
         return at;
     }
-    LinOff lin(int n, int k) {
+    // a linear of format wq: codes (int8 [n][k], or 4-bit packed [n][k/2]),
+    // row scales, row offsets (min-max form only), biases
+    LinOff lin(int n, int k, int wq = 8) {
         LinOff l;
         l.n = n;
         l.k = k;
-        l.w = take((size_t)n * k);
+        l.bits = wq & 0xFF;
+        l.minmax = (wq & WQ_MINMAX) != 0;
+        l.w = take(l.bits == 4 ? (size_t)n * k / 2 : (size_t)n * k);
         l.s = take((size_t)n * 4);
+        l.m = l.minmax ? take((size_t)n * 4) : 0;
         l.b = take((size_t)n * 4);
         return l;
     }
@@ -138,7 +147,11 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
     if (std::memcmp(p, "MNMT", 4) != 0) return fail(MNMT_EFORMAT, "bad magic");
     uint32_t ver;
     std::memcpy(&ver, p + 4, 4);
-    if (ver != 1) return fail(MNMT_EFORMAT, "unsupported blob version %u", ver);
+    if (ver != 1 && ver != 2) return fail(MNMT_EFORMAT, "unsupported blob version %u", ver);
+    L->wq = 8;
+    if (ver == 2) std::memcpy(&L->wq, p + 60, 4);
+    if (L->wq != 8 && L->wq != 4 && L->wq != (4 | WQ_MINMAX))
+        return fail(MNMT_EFORMAT, "unsupported weight format 0x%x", L->wq);
     int32_t h[13];
     std::memcpy(h, p + 8, sizeof(h));
     mnmt_config &c = L->c;
@@ -169,8 +182,8 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
         s.ln_g = w.take((size_t)d * 4);
         s.ln_b = w.take((size_t)d * 4);
         s.sc = w.take(32);
-        s.qkv = w.lin(3 * d, d);
-        s.o = w.lin(d, d);
+        s.qkv = w.lin(3 * d, d, L->wq);
+        s.o = w.lin(d, d, L->wq);
         return s;
     };
     auto ffn_blk = [&]() {
@@ -178,8 +191,8 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
         f.ln_g = w.take((size_t)d * 4);
         f.ln_b = w.take((size_t)d * 4);
         f.sc = w.take(16);
-        f.w1 = w.lin(F, d);
-        f.w2 = w.lin(d, F);
+        f.w1 = w.lin(F, d, L->wq);
+        f.w2 = w.lin(d, F, L->wq);
         return f;
     };
     for (int l = 0; l < c.n_enc; l++) {
@@ -196,9 +209,9 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
         x.ln_g = w.take((size_t)d * 4);
         x.ln_b = w.take((size_t)d * 4);
         x.sc = w.take(32);
-        x.q = w.lin(d, d);
-        x.kv = w.lin(2 * d, d);
-        x.o = w.lin(d, d);
+        x.q = w.lin(d, d, L->wq);
+        x.kv = w.lin(2 * d, d, L->wq);
+        x.o = w.lin(d, d, L->wq);
         L->dec_cross.push_back(x);
         L->dec_ffn.push_back(ffn_blk());
     }
@@ -225,9 +238,12 @@ int parse_layout(const void *blob, size_t bytes, Layout *L) {
 // ---------------------------------------------------------------------------
 namespace {
 struct Lin {
-    const int8_t *w;
+    const int8_t *w;  // int8 codes [n][k] (4-bit symmetric rows: the unpacked copy, or null when lean)
     const float *s, *b;
     int n, k;
+    int bits;                 // 8 or 4
+    const uint8_t *wp;        // 4-bit: packed codes [n][k/2]
+    const float *m;           // 4-bit min-max rows: row offsets (null: symmetric)
 };
 struct LnP {
     const float *g, *b;
@@ -258,6 +274,10 @@ struct mnmt_model {
     bool own_stream;
     uint8_t *d_blob;
     __half *d_blob16;  // fp16 copy of every blob byte read as an int8 code (tensor-core operands); null when lean
+    int wq;            // weight format of the attention / FFN linears (8, 4, 4 | WQ_MINMAX)
+    int8_t *d_w8;      // symmetric 4-bit linears unpacked to int8 (the IMMA / tensor-core operands); null when lean
+    __half *d_w8_16;   // its fp16 copy
+    size_t w8_codes;
     float *d_aux;
     size_t bytes;
     size_t device_bytes;  // every byte of device memory the model holds
@@ -339,13 +359,49 @@ extern "C" int mnmt_load_weights_ex(const void *blob, size_t bytes, void *cuda_s
         std::memcpy(&v, hb + off + 4 * i, 4);
         return v;
     };
+    // 4-bit linears: rows of at most 16 (and min-max rows always) run on the
+    // 4-bit GEMV kernel; for more rows symmetric linears use an int8 copy of
+    // their codes on the IMMA / tensor-core kernels (not kept when lean)
+    m->wq = L.wq;
+    if (L.wq == 4 && !m->lean) {
+        size_t codes = 0;
+        auto add = [&](const LinOff &o) { codes += (size_t)o.n * o.k; };
+        for (const auto &x : L.enc_self) { add(x.qkv); add(x.o); }
+        for (const auto &x : L.enc_ffn) { add(x.w1); add(x.w2); }
+        for (const auto &x : L.dec_self) { add(x.qkv); add(x.o); }
+        for (const auto &x : L.dec_cross) { add(x.q); add(x.kv); add(x.o); }
+        for (const auto &x : L.dec_ffn) { add(x.w1); add(x.w2); }
+        if (cudaMalloc(&m->d_w8, codes) != cudaSuccess) {
+            mnmt_model_free(m);
+            return fail(MNMT_ENOMEM, "cudaMalloc of %zu unpacked weight codes failed", codes);
+        }
+        m->w8_codes = codes;
+    }
+    size_t w8_at = 0;
+    cudaError_t unpack_err = cudaSuccess;
     auto dlin = [&](const LinOff &o) {
         Lin l;
-        l.w = reinterpret_cast<const int8_t *>(m->d_blob + o.w);
         l.s = reinterpret_cast<const float *>(m->d_blob + o.s);
         l.b = reinterpret_cast<const float *>(m->d_blob + o.b);
         l.n = o.n;
         l.k = o.k;
+        l.bits = o.bits;
+        l.wp = nullptr;
+        l.m = nullptr;
+        if (o.bits == 4) {
+            l.wp = m->d_blob + o.w;
+            l.m = o.minmax ? reinterpret_cast<const float *>(m->d_blob + o.m) : nullptr;
+            l.w = nullptr;
+            if (m->d_w8 && !o.minmax) {
+                int8_t *dst = m->d_w8 + w8_at;
+                w8_at += (size_t)o.n * o.k;
+                if (unpack_err == cudaSuccess)
+                    unpack_err = launch_unpack_w4_sym(l.wp, (size_t)o.n * o.k, dst, m->stream);
+                l.w = dst;
+            }
+        } else {
+            l.w = reinterpret_cast<const int8_t *>(m->d_blob + o.w);
+        }
         return l;
     };
     auto dln = [&](size_t g, size_t b) {
@@ -436,7 +492,22 @@ extern "C" int mnmt_load_weights_ex(const void *blob, size_t bytes, void *cuda_s
     // blob once (the fp32 regions become unused garbage); offsets stay 16-byte
     // aligned, so W16 = d_blob16 + (W - d_blob) is 32-byte aligned.  A lean
     // model keeps the int8 blob only and runs every linear on the int8 kernels.
-    m->device_bytes = bytes + aux.size() * 4;
+    if (unpack_err != cudaSuccess) {
+        mnmt_model_free(m);
+        return fail(MNMT_ECUDA, "unpacking the 4-bit weights failed");
+    }
+    m->device_bytes = bytes + aux.size() * 4 + m->w8_codes;
+    if (m->d_w8) {
+        if (cudaMalloc(&m->d_w8_16, m->w8_codes * 2) != cudaSuccess) {
+            mnmt_model_free(m);
+            return fail(MNMT_ENOMEM, "cudaMalloc of %zu fp16 weight bytes failed", m->w8_codes * 2);
+        }
+        m->device_bytes += m->w8_codes * 2;
+        if (launch_codes_to_f16_flat(m->d_w8, m->d_w8_16, m->w8_codes, m->stream) != cudaSuccess) {
+            mnmt_model_free(m);
+            return fail(MNMT_ECUDA, "fp16 weight conversion failed");
+        }
+    }
     if (!m->lean) {
         if (cudaMalloc(&m->d_blob16, bytes * 2) != cudaSuccess) {
             mnmt_model_free(m);
@@ -468,6 +539,8 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
     if (m->stream) cudaStreamSynchronize(m->stream);
     if (m->d_blob) cudaFree(m->d_blob);
     if (m->d_blob16) cudaFree(m->d_blob16);
+    if (m->d_w8) cudaFree(m->d_w8);
+    if (m->d_w8_16) cudaFree(m->d_w8_16);
     if (m->d_aux) cudaFree(m->d_aux);
     if (m->own_stream && m->stream) cudaStreamDestroy(m->stream);
     delete m;
@@ -670,6 +743,7 @@ Epi base_epi(int mode, float s_x, const Lin &l) {
 
 // fp16 copy of the codes of weight w (tensor-core operand)
 const __half *w16_of(const mnmt_model *m, const int8_t *w) {
+    if (m->d_w8 && w >= m->d_w8 && w < m->d_w8 + m->w8_codes) return m->d_w8_16 + (w - m->d_w8);
     return m->d_blob16 + (w - reinterpret_cast<const int8_t *>(m->d_blob));
 }
 
@@ -696,6 +770,7 @@ __half *out16_for(mnmt_session *s, const int8_t *buf, int M) { return tc_rows(s,
 cudaError_t run_linear(mnmt_session *s, const int8_t *A, int lda, const Lin &l, int M, const Epi &e,
                        cudaStream_t st) {
     const mnmt_model *m = s->m;
+    if (l.bits == 4 && ((size_t)M <= 16 || !l.w)) return launch_linear_w4(A, lda, l.wp, l.m, M, l.n, l.k, e, st);
     if (tc_rows(s, M) && l.k % 16 == 0) {
         const __half *w16 = w16_of(m, l.w);
         const __half *a16 = mirror16(s, A);
@@ -1058,7 +1133,7 @@ int setup_cluster_step(mnmt_session *s) {
     // of two) and a residual slice over at most 32 lanes: d, F and the
     // factorised embedding width must be powers of two
     const int E = c.d_embed;
-    if (s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
+    if (m->wq != 8 || s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
         F % (16 * nc) || (3 * d) % (16 * nc) || !pow2_in(d, 64, 512) || !pow2_in(F, 64, 2048) ||
         (m->factorised && !pow2_in(E, 16, 512)))
         return MNMT_OK;
@@ -1469,6 +1544,51 @@ extern "C" int mnmt_linear(const int8_t *A, const int8_t *W, const float *s_w, c
     }
     cudaError_t err = launch_linear(A, K, W, M, N, K, e, static_cast<cudaStream_t>(cuda_stream));
     if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear launch: %s", cudaGetErrorString(err));
+    return MNMT_OK;
+}
+
+extern "C" int mnmt_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s_w, const float *m_w,
+                              const float *bias, float s_x, const float *inv_out, float gamma, int32_t M, int32_t N,
+                              int32_t K, int32_t mode, int8_t *out_q, float *out_f, uint64_t *keys,
+                              void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!A || !Wp || !s_w || !bias || M < 1 || N < 1 || K < 32 || K % 32 || K > 3072)
+        return fail(MNMT_EINVAL, "linear_w4: bad shape M=%d N=%d K=%d", M, N, K);
+    if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(Wp)) & 15)
+        return fail(MNMT_EINVAL, "linear_w4: A and Wp must be 16-byte aligned");
+    Epi e;
+    std::memset(&e, 0, sizeof(e));
+    e.s_x = s_x;
+    e.s_w = s_w;
+    e.bias = bias;
+    switch (mode) {
+        case MNMT_EPI_Q8:
+        case MNMT_EPI_RELU_Q8:
+            if (!out_q || !inv_out) return fail(MNMT_EINVAL, "linear_w4: int8 output needs out_q and inv_out");
+            e.mode = mode == MNMT_EPI_Q8 ? EPI_Q8 : EPI_RELU_Q8;
+            e.out = out_q;
+            e.ldo = N;
+            e.inv_out = inv_out;
+            break;
+        case MNMT_EPI_RESID:
+        case MNMT_EPI_F32:
+            if (!out_f) return fail(MNMT_EINVAL, "linear_w4: fp32 output needs out_f");
+            e.mode = mode == MNMT_EPI_RESID ? EPI_RESID : EPI_F32;
+            e.f32 = out_f;
+            e.ldf = N;
+            e.gamma = gamma;
+            break;
+        case MNMT_EPI_ARGMAX:
+            if (!keys) return fail(MNMT_EINVAL, "linear_w4: argmax needs keys");
+            e.mode = EPI_ARGMAX;
+            e.keys = reinterpret_cast<unsigned long long *>(keys);
+            break;
+        default:
+            return fail(MNMT_EINVAL, "linear_w4: unknown mode %d", mode);
+    }
+    cudaError_t err = launch_linear_w4(A, K, Wp, m_w, M, N, K, e, static_cast<cudaStream_t>(cuda_stream));
+    if (err != cudaSuccess) return fail(MNMT_ECUDA, "linear_w4 launch: %s", cudaGetErrorString(err));
     return MNMT_OK;
 }
 

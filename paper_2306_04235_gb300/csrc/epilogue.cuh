@@ -9,10 +9,9 @@
 
 namespace mnmt {
 
-// epilogue of one output element; accf = fl(acc), the accumulator rounded to
-// fp32 (exact for |acc| <= 2^24); t: decode step
-MNMT_DEV void epi_store_f(const Epi &e, int m, int n, float accf, int t) {
-    float y = __fadd_rn(__fmul_rn(accf, __fmul_rn(e.s_x, e.s_w[n])), e.bias[n]);
+// epilogue of one output element from its dequantised, biased value y;
+// t: decode step
+MNMT_DEV void epi_store_y(const Epi &e, int m, int n, float y, int t) {
     switch (e.mode) {
         case EPI_Q8:
         case EPI_RELU_Q8: {
@@ -55,6 +54,12 @@ MNMT_DEV void epi_store_f(const Epi &e, int m, int n, float accf, int t) {
         default:
             break;
     }
+}
+
+// epilogue of one output element; accf = fl(acc), the accumulator rounded to
+// fp32 (exact for |acc| <= 2^24)
+MNMT_DEV void epi_store_f(const Epi &e, int m, int n, float accf, int t) {
+    epi_store_y(e, m, n, __fadd_rn(__fmul_rn(accf, __fmul_rn(e.s_x, e.s_w[n])), e.bias[n]), t);
 }
 
 // the same from the exact int32 accumulator

@@ -76,6 +76,12 @@ cudaError_t rows_init();
 // ---- launchers (stream-ordered, no synchronisation) ----
 cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int N, int K, const Epi &e,
                           cudaStream_t st);
+// row-wise 4-bit weights Wp [N][K/2] (packed runs of 32 codes); m_w: row
+// offsets of the min-max form, null for symmetric rows (stored code v + 8)
+cudaError_t launch_linear_w4(const int8_t *A, int lda, const uint8_t *Wp, const float *m_w, int M, int N, int K,
+                             const Epi &e, cudaStream_t st);
+// symmetric 4-bit rows (codes elements) unpacked to int8 v = c - 8
+cudaError_t launch_unpack_w4_sym(const uint8_t *Wp, size_t codes, int8_t *out, cudaStream_t st);
 
 // tensor-core (tcgen05) linear over fp16 copies of the int8 codes: A16 [M][lda],
 // W16 [N][ldw]; K <= 2048 and a multiple of 8; *status (device, may be null)

@@ -82,6 +82,8 @@ def _declare(L):
     L.mnmt_layernorm.argtypes = [p, p, p, i32, i32, f, p, p, p, p]
     L.mnmt_linear_tc.argtypes = [p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p, p]
     L.mnmt_codes_to_f16.argtypes = [p, p, sz, p]
+    L.mnmt_linear_w4.argtypes = [p, p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p]
+    L.mnmt_linear_w4.restype = C.c_int
     L.mnmt_wait_timeout_selftest.argtypes = [p, p]
     for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_load_weights_ex", "mnmt_session_create_ex",
               "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
@@ -241,6 +243,14 @@ def mnmt_linear_tc(A16, W16, s_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_
     """Tensor-core quantised linear over fp16 copies of the int8 codes (see mnmt_codes_to_f16)."""
     _chk(lib().mnmt_linear_tc(_ptr(A16), _ptr(W16), _ptr(s_w), _ptr(bias), float(s_x), _ptr(inv_out), float(gamma),
                               M, N, K, mode, _ptr(out_q), _ptr(out_f), _ptr(keys), _ptr(status),
+                              _stream_handle(stream)))
+
+
+def mnmt_linear_w4(A, Wp, s_w, m_w, bias, s_x, inv_out, gamma, M, N, K, mode, out_q=None, out_f=None, keys=None,
+                   stream=None):
+    """Quantised linear with row-wise 4-bit weights (m_w None: symmetric rows)."""
+    _chk(lib().mnmt_linear_w4(_ptr(A), _ptr(Wp), _ptr(s_w), _ptr(m_w), _ptr(bias), float(s_x), _ptr(inv_out),
+                              float(gamma), M, N, K, mode, _ptr(out_q), _ptr(out_f), _ptr(keys),
                               _stream_handle(stream)))
 
 
