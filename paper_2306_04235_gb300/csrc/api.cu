@@ -946,7 +946,7 @@ int issue_decode_step(mnmt_session *s) {
         g.eos = c.eos_id;
         g.pad = c.pad_id;
         LK(launch_vocab_greedy(s->act, m->out.w, m->out.s, m->out.b, m->s_dout, R, c.vocab, d, s->keys,
-                               s->state + ST_TICKET, g, st));
+                               s->state + ST_TICKET, g, s->dc_nc, st));
         return MNMT_OK;
     }
     {

@@ -837,11 +837,16 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
 
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
-                                cudaStream_t st) {
+                                int reserved_sms, cudaStream_t st) {
     const int kc = K / 16;
     if (M < 1 || M > 4 || K % 16 || (kc & (kc - 1))) return cudaErrorInvalidValue;
-    // two blocks per SM, each holding its contiguous rows in shared memory
-    int blocks = 2 * 152;
+    // two blocks per SM, each holding its contiguous rows in shared memory, on
+    // the SMs the step's cluster does not occupy: every block is resident (and
+    // prefetching its rows) while the step runs, and the next step's cluster
+    // finds its SMs free and runs its prologue while this kernel finishes
+    int free_sms = device_sm_count() - reserved_sms;
+    if (free_sms < 16) free_sms = 16;
+    int blocks = 2 * free_sms;
     int rows = (N + blocks - 1) / blocks;
     if ((size_t)rows * K > 96 * 1024) rows = (96 * 1024) / K;
     blocks = (N + rows - 1) / rows;

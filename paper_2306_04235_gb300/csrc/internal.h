@@ -261,8 +261,9 @@ size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
 bool decode_cluster_fits(int dh, int nc, size_t smem);
 cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, cudaStream_t st);
+// reserved_sms: SMs the step kernel that precedes the launch occupies
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
-                                cudaStream_t st);
+                                int reserved_sms, cudaStream_t st);
 
 }  // namespace mnmt
