@@ -479,9 +479,16 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const float *sw = reinterpret_cast<const float *>(slot + rows * K);
             const float *bb = sw + rows;
             const float *iv = bb + rows;
-            const int kc = K / 16;                 // 16-byte chunks per row
-            const int lpr = kc >= 4 ? kc / 4 : 1;  // lanes per row: each lane takes kc / lpr chunks
-            const int cpl = kc / lpr;
+            const int kc = K / 16;  // 16-byte chunks per row (a power of two)
+            // lanes per row: as many as spread the slice's rows * kc chunks over
+            // all 8 warps, at most 32 (each lane takes kc / lpr chunks)
+            int cpl = 1;
+            while (rows * kc > DC_THREADS * cpl && cpl < kc) cpl *= 2;
+            int lpr = kc / cpl;
+            if (lpr > 32) {
+                lpr = 32;
+                cpl = kc / 32;
+            }
             const int rpw = 32 / lpr;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
             const int sub = lane % lpr;
@@ -820,13 +827,18 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
     cfg.blockDim = dim3(DC_THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    // a programmatic dependent of the previous step's vocabulary kernel: the
+    // cluster launches as soon as its SMs are free and runs its prologue
+    // (parameters, LayerNorm vectors, cross keys / values) before it waits
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = nc;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     switch (dh) {
         case 32: return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<32>, dP);
         case 64: return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<64>, dP);
