@@ -282,6 +282,38 @@ int mnmt_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s_w, const f
                    float s_x, const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K, int32_t mode,
                    int8_t *out_q, float *out_f, uint64_t *keys, void *cuda_stream);
 
+/* Fake quantisation for quantisation-aware training (App. B "PTQ and QAT":
+ * the quantiser of Eq. quant inserted into the float model; besides the
+ * weights, its scale s is learnable).  Element-wise over x [n] (fp32):
+ *   minmax = 0: q = clamp(rne(fl(x fl(1/s))), -(2^(bits-1)-1), 2^(bits-1)-1),
+ *               y = fl(q s)
+ *   minmax = 1: q = clamp(rne(fl(fl(x - r_m) fl(1/s))), 0, 2^bits - 1),
+ *               y = fl(fl(q s) + r_m)            (Eq. scale / Eq. quant)
+ * y [n] (fp32) and codes [n] (int32) are optional outputs (at least one).
+ * 2 <= bits <= 8, s > 0 finite.  Device pointers; asynchronous on cuda_stream. */
+int mnmt_fake_quant(const float *x, size_t n, float s, float r_m, int32_t bits, int32_t minmax, float *y,
+                    int32_t *codes, void *cuda_stream);
+
+/* Backward of mnmt_fake_quant for the upstream gradient g [n]: with t the
+ * unrounded code and in = (qmin <= t <= qmax), gx = in ? g : 0 (straight
+ * through), *gs = sum g (in ? q - t : q) (the learnable scale's gradient),
+ * *gr = sum g (1 - in) (the offset's, min-max form; 0 otherwise).  gs / gr are
+ * device doubles (gr may be NULL), accumulated in fp64 (summation order not
+ * fixed). */
+int mnmt_fake_quant_backward(const float *x, const float *g, size_t n, float s, float r_m, int32_t bits,
+                             int32_t minmax, float *gx, double *gs, double *gr, void *cuda_stream);
+
+/* QAT forward of one linear: X [M][K] fp32 fake-quantised per tensor to 8-bit
+ * symmetric codes at s_x, W [N][K] fp32 per row to `wbits`-bit symmetric codes
+ * at the learnable row scales s_w [N]; y [M][N] fp32 = X_q W_q^T + bias with the
+ * products exact, i.e. mnmt_linear's MNMT_EPI_F32 on the two code tensors.
+ * workspace: caller-allocated device scratch of at least
+ * round_up(M*K, 16) + N*K bytes, 16-byte aligned, holding the codes.  K a
+ * multiple of 16 (of 64 when M > 16), K <= 2048 when M <= 16. */
+int mnmt_fake_quant_linear(const float *X, const float *W, float s_x, const float *s_w, const float *bias,
+                           int32_t M, int32_t N, int32_t K, int32_t wbits, void *workspace, float *y,
+                           void *cuda_stream);
+
 /* dst[i] = the fp16 value of the int8 code src[i] (exact), i < n.  Device
  * pointers, src and dst 16-byte aligned. */
 int mnmt_codes_to_f16(const int8_t *src, uint16_t *dst, size_t n, void *cuda_stream);

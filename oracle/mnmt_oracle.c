@@ -987,6 +987,85 @@ int oracle_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s_w, const
     return OR_OK;
 }
 
+/* ---- fake quantisation (QAT forward / backward; App. B "PTQ and QAT") ----
+ * The quantiser of Eq. quant inserted into a float model, with a learnable
+ * scale s (and, min-max form, offset r_m):
+ *   symmetric, n bits: q = clamp(rne(fl(x fl(1/s))), -(2^(n-1)-1), 2^(n-1)-1),
+ *                      y = fl(q s)
+ *   min-max,   n bits: q = clamp(rne(fl(fl(x - r_m) fl(1/s))), 0, 2^n - 1),
+ *                      y = fl(fl(q s) + r_m)
+ * Backward (straight-through estimator for x; the scale and offset gradients
+ * of the same expression, rounding held fixed): with t = the unrounded code
+ * above and `in` = qmin <= t <= qmax,
+ *   dy/dx = in,  dy/ds = in ? q - t : q,  dy/dr_m = in ? 0 : 1. */
+static void fq_range(int bits, int minmax, int *qmin, int *qmax) {
+    if (minmax) { *qmin = 0; *qmax = (1 << bits) - 1; }
+    else { *qmax = (1 << (bits - 1)) - 1; *qmin = -*qmax; }
+}
+
+int oracle_fake_quant(const float *x, int n, float s, float r_m, int bits, int minmax, float *y, int32_t *codes) {
+    if (bits < 2 || bits > 8 || !(s > 0.0f)) return OR_EINVAL;
+    int qmin, qmax;
+    fq_range(bits, minmax, &qmin, &qmax);
+    float inv = 1.0f / s;
+    for (int i = 0; i < n; i++) {
+        float t = minmax ? (x[i] - r_m) * inv : x[i] * inv;
+        float q = rintf(t);
+        if (q < qmin) q = (float)qmin;
+        if (q > qmax) q = (float)qmax;
+        if (codes) codes[i] = (int32_t)q;
+        if (y) {
+            float v = q * s;
+            y[i] = minmax ? v + r_m : v;
+        }
+    }
+    return OR_OK;
+}
+
+int oracle_fake_quant_backward(const float *x, const float *g, int n, float s, float r_m, int bits, int minmax,
+                               float *gx, double *gs, double *gr) {
+    if (bits < 2 || bits > 8 || !(s > 0.0f)) return OR_EINVAL;
+    int qmin, qmax;
+    fq_range(bits, minmax, &qmin, &qmax);
+    float inv = 1.0f / s;
+    double as = 0.0, ar = 0.0;
+    for (int i = 0; i < n; i++) {
+        float t = minmax ? (x[i] - r_m) * inv : x[i] * inv;
+        int in = t >= (float)qmin && t <= (float)qmax;
+        float q = rintf(t);
+        if (q < qmin) q = (float)qmin;
+        if (q > qmax) q = (float)qmax;
+        gx[i] = in ? g[i] : 0.0f;
+        as += (double)g[i] * (in ? (double)q - (double)t : (double)q);
+        if (!in) ar += (double)g[i];
+    }
+    *gs = as;
+    if (gr) *gr = minmax ? ar : 0.0;
+    return OR_OK;
+}
+
+/* QAT forward of one linear: X [M][K] float fake-quantised per tensor to
+ * 8-bit codes at scale s_x, W [N][K] float fake-quantised per row to `wbits`
+ * symmetric codes at scales s_w[n]; y = the quantised linear of the codes
+ * (dequantise with fl(s_x s_w[n]), add the bias), i.e. X_q W_q^T + b with the
+ * products exact. */
+int oracle_fake_quant_linear(const float *X, const float *W, float s_x, const float *s_w, const float *b, int M,
+                             int N, int K, int wbits, float *y) {
+    if (wbits < 2 || wbits > 8 || !(s_x > 0.0f)) return OR_EINVAL;
+    int32_t *qx = malloc(sizeof(int32_t) * (size_t)M * K), *qw = malloc(sizeof(int32_t) * (size_t)N * K);
+    if (!qx || !qw) { free(qx); free(qw); return OR_ENOMEM; }
+    int st = oracle_fake_quant(X, M * K, s_x, 0.0f, 8, 0, NULL, qx);
+    for (int n = 0; !st && n < N; n++) st = oracle_fake_quant(W + (size_t)n * K, K, s_w[n], 0.0f, wbits, 0, NULL, qw + (size_t)n * K);
+    for (int m = 0; !st && m < M; m++)
+        for (int n = 0; n < N; n++) {
+            int32_t acc = 0;
+            for (int k = 0; k < K; k++) acc += qx[(size_t)m * K + k] * qw[(size_t)n * K + k];
+            y[(size_t)m * N + n] = dequant_bias(acc, s_x, s_w[n], b[n]);
+        }
+    free(qx); free(qw);
+    return st;
+}
+
 /* The LayerNorm's mean and biased variance of M rows of length d. */
 int oracle_ln_stats(const float *r, int M, int d, float *mu, float *var) {
     for (int m = 0; m < M; m++) {

@@ -71,12 +71,16 @@ def _declare(L):
     L.oracle_log_softmax_norm.argtypes = [_p, _i, _p, _p, _p]
     L.oracle_ln_stats.argtypes = [_p, _i, _i, _p, _p]
     L.oracle_quantise_rows.argtypes = [_p, _i, _i, _i, _i, _p, _p, _p]
+    L.oracle_fake_quant.argtypes = [_p, _i, _f, _f, _i, _i, _p, _p]
+    L.oracle_fake_quant_backward.argtypes = [_p, _p, _i, _f, _f, _i, _i, _p, _p, _p]
+    L.oracle_fake_quant_linear.argtypes = [_p, _p, _f, _p, _p, _i, _i, _i, _i, _p]
     L.oracle_linear_w4.argtypes = [_p, _p, _p, _p, _p, _f, _p, _f, _i, _i, _i, _i, _i, _p, _p]
     L.oracle_translate.argtypes = [_p, _sz, _p, _p, _i, _i, _i, _i, _i, _p, _p, _p]
     for name in ["oracle_check_blob", "oracle_linear", "oracle_layernorm", "oracle_attention_decode",
                  "oracle_attention_probs", "oracle_encode", "oracle_decode_trace",
                  "oracle_decode_forced", "oracle_embed", "oracle_log_softmax", "oracle_log_softmax_norm", "oracle_ln_stats",
-                 "oracle_quantise_rows", "oracle_linear_w4",
+                 "oracle_quantise_rows", "oracle_linear_w4", "oracle_fake_quant",
+                 "oracle_fake_quant_backward", "oracle_fake_quant_linear",
                  "oracle_translate"]:
         getattr(L, name).restype = _i
 
@@ -189,6 +193,32 @@ def linear_w4(A, Wp, s_w, m_w, b, s_x, mode, asym, inv_out=None, gamma=1.0, resi
     _chk(lib().oracle_linear_w4(_ptr(A), _ptr(Wp), _ptr(s_w), _ptr(m_w), _ptr(b), float(s_x), _ptr(inv_out),
                                 float(gamma), M, N, K, int(asym), mode, _ptr(out_q), _ptr(out_f)))
     return out_q if out_q is not None else out_f
+
+
+def fake_quant(x, s, bits=8, r_m=0.0, minmax=False):
+    """QAT fake quantisation (App. B Eq. quant, scale s, offset r_m): (y f32, codes int32)."""
+    x = np.ascontiguousarray(x, np.float32)
+    y = np.zeros_like(x); q = np.zeros(x.shape, np.int32)
+    _chk(lib().oracle_fake_quant(_ptr(x), x.size, float(s), float(r_m), int(bits), int(minmax), _ptr(y), _ptr(q)))
+    return y, q
+
+
+def fake_quant_backward(x, g, s, bits=8, r_m=0.0, minmax=False):
+    """(dL/dx f32, dL/ds, dL/dr_m) of the fake quantiser for upstream gradient g."""
+    x = np.ascontiguousarray(x, np.float32); g = np.ascontiguousarray(g, np.float32)
+    gx = np.zeros_like(x); gs = np.zeros(1, np.float64); gr = np.zeros(1, np.float64)
+    _chk(lib().oracle_fake_quant_backward(_ptr(x), _ptr(g), x.size, float(s), float(r_m), int(bits), int(minmax),
+                                          _ptr(gx), _ptr(gs), _ptr(gr)))
+    return gx, float(gs[0]), float(gr[0])
+
+
+def fake_quant_linear(X, W, s_x, s_w, b, wbits=8):
+    X = np.ascontiguousarray(X, np.float32); W = np.ascontiguousarray(W, np.float32)
+    M, K = X.shape; N = W.shape[0]
+    y = np.zeros((M, N), np.float32)
+    _chk(lib().oracle_fake_quant_linear(_ptr(X), _ptr(W), float(s_x), _ptr(np.ascontiguousarray(s_w, np.float32)),
+                                        _ptr(np.ascontiguousarray(b, np.float32)), M, N, K, int(wbits), _ptr(y)))
+    return y
 
 
 def ln_stats(r):

@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB = os.path.join(OUT_DIR, "libmnmt.so")
 SOURCES = ["api.cu", "linear.cu", "linear_w4.cu", "gemm_tc.cu", "attention.cu", "rows.cu", "decode_cluster.cu",
-           "noalloc.cu"]
+           "noalloc.cu", "fakequant.cu"]
 HEADERS = ["common.cuh", "epilogue.cuh", "internal.h", "mbarrier.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

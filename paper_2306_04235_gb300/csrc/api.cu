@@ -1592,6 +1592,45 @@ extern "C" int mnmt_linear_w4(const int8_t *A, const uint8_t *Wp, const float *s
     return MNMT_OK;
 }
 
+extern "C" int mnmt_fake_quant(const float *x, size_t n, float s, float r_m, int32_t bits, int32_t minmax, float *y,
+                               int32_t *codes, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!x || (!y && !codes) || bits < 2 || bits > 8 || !(s > 0.0f) || !std::isfinite(s) || !std::isfinite(r_m))
+        return fail(MNMT_EINVAL, "fake_quant: bad argument");
+    cudaError_t err = launch_fake_quant(x, n, s, r_m, bits, minmax ? 1 : 0, y, codes,
+                                        static_cast<cudaStream_t>(cuda_stream));
+    return err == cudaSuccess ? MNMT_OK : fail(MNMT_ECUDA, "fake_quant: %s", cudaGetErrorString(err));
+}
+
+extern "C" int mnmt_fake_quant_backward(const float *x, const float *g, size_t n, float s, float r_m, int32_t bits,
+                                        int32_t minmax, float *gx, double *gs, double *gr, void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!x || !g || !gx || !gs || bits < 2 || bits > 8 || !(s > 0.0f) || !std::isfinite(s) || !std::isfinite(r_m))
+        return fail(MNMT_EINVAL, "fake_quant_backward: bad argument");
+    cudaError_t err = launch_fake_quant_backward(x, g, n, s, r_m, bits, minmax ? 1 : 0, gx, gs, gr,
+                                                 static_cast<cudaStream_t>(cuda_stream));
+    return err == cudaSuccess ? MNMT_OK : fail(MNMT_ECUDA, "fake_quant_backward: %s", cudaGetErrorString(err));
+}
+
+extern "C" int mnmt_fake_quant_linear(const float *X, const float *W, float s_x, const float *s_w, const float *bias,
+                                      int32_t M, int32_t N, int32_t K, int32_t wbits, void *workspace, float *y,
+                                      void *cuda_stream) {
+    int rc = lib_init();
+    if (rc) return rc;
+    if (!X || !W || !s_w || !bias || !workspace || !y || M < 1 || N < 1 || K < 16 || K % 16 || (M > 16 && K % 64) ||
+        (M <= 16 && K > 2048) || wbits < 2 || wbits > 8 || !(s_x > 0.0f) || !std::isfinite(s_x))
+        return fail(MNMT_EINVAL, "fake_quant_linear: bad argument or shape (M=%d N=%d K=%d)", M, N, K);
+    if (reinterpret_cast<uintptr_t>(workspace) & 15)
+        return fail(MNMT_EINVAL, "fake_quant_linear: workspace must be 16-byte aligned");
+    int8_t *qx = static_cast<int8_t *>(workspace);
+    int8_t *qw = qx + (((size_t)M * K + 15) & ~(size_t)15);
+    cudaError_t err = launch_fake_quant_linear(X, W, s_x, s_w, bias, M, N, K, wbits, qx, qw, y,
+                                               static_cast<cudaStream_t>(cuda_stream));
+    return err == cudaSuccess ? MNMT_OK : fail(MNMT_ECUDA, "fake_quant_linear: %s", cudaGetErrorString(err));
+}
+
 extern "C" int mnmt_linear_tc(const uint16_t *A16, const uint16_t *W16, const float *s_w, const float *bias,
                               float s_x, const float *inv_out, float gamma, int32_t M, int32_t N, int32_t K,
                               int32_t mode, int8_t *out_q, float *out_f, uint64_t *keys, int32_t *status,

@@ -80,6 +80,14 @@ cudaError_t launch_linear(const int8_t *A, int lda, const int8_t *W, int M, int 
 // offsets of the min-max form, null for symmetric rows (stored code v + 8)
 cudaError_t launch_linear_w4(const int8_t *A, int lda, const uint8_t *Wp, const float *m_w, int M, int N, int K,
                              const Epi &e, cudaStream_t st);
+// fake quantisation (QAT forward / backward) and the QAT forward of a linear
+cudaError_t launch_fake_quant(const float *x, size_t n, float s, float r, int bits, int minmax, float *y,
+                              int32_t *codes, cudaStream_t st);
+cudaError_t launch_fake_quant_backward(const float *x, const float *g, size_t n, float s, float r, int bits,
+                                       int minmax, float *gx, double *gs, double *gr, cudaStream_t st);
+cudaError_t launch_fake_quant_linear(const float *X, const float *W, float s_x, const float *s_w, const float *bias,
+                                     int M, int N, int K, int wbits, int8_t *qx, int8_t *qw, float *y,
+                                     cudaStream_t st);
 // symmetric 4-bit rows (codes elements) unpacked to int8 v = c - 8
 cudaError_t launch_unpack_w4_sym(const uint8_t *Wp, size_t codes, int8_t *out, cudaStream_t st);
 

@@ -84,6 +84,11 @@ def _declare(L):
     L.mnmt_codes_to_f16.argtypes = [p, p, sz, p]
     L.mnmt_linear_w4.argtypes = [p, p, p, p, p, f, p, f, i32, i32, i32, i32, p, p, p, p]
     L.mnmt_linear_w4.restype = C.c_int
+    L.mnmt_fake_quant.argtypes = [p, sz, f, f, i32, i32, p, p, p]
+    L.mnmt_fake_quant_backward.argtypes = [p, p, sz, f, f, i32, i32, p, p, p, p]
+    L.mnmt_fake_quant_linear.argtypes = [p, p, f, p, p, i32, i32, i32, i32, p, p, p]
+    for n in ["mnmt_fake_quant", "mnmt_fake_quant_backward", "mnmt_fake_quant_linear"]:
+        getattr(L, n).restype = C.c_int
     L.mnmt_wait_timeout_selftest.argtypes = [p, p]
     for n in ["mnmt_blob_check", "mnmt_load_weights", "mnmt_load_weights_ex", "mnmt_session_create_ex",
               "mnmt_model_config", "mnmt_session_create", "mnmt_encode",
@@ -252,6 +257,24 @@ def mnmt_linear_w4(A, Wp, s_w, m_w, bias, s_x, inv_out, gamma, M, N, K, mode, ou
     _chk(lib().mnmt_linear_w4(_ptr(A), _ptr(Wp), _ptr(s_w), _ptr(m_w), _ptr(bias), float(s_x), _ptr(inv_out),
                               float(gamma), M, N, K, mode, _ptr(out_q), _ptr(out_f), _ptr(keys),
                               _stream_handle(stream)))
+
+
+def mnmt_fake_quant(x, n, s, r_m=0.0, bits=8, minmax=False, y=None, codes=None, stream=None):
+    """QAT fake quantisation (device buffers): y = Q(x), codes = q (int32)."""
+    _chk(lib().mnmt_fake_quant(_ptr(x), n, float(s), float(r_m), bits, int(minmax), _ptr(y), _ptr(codes),
+                               _stream_handle(stream)))
+
+
+def mnmt_fake_quant_backward(x, g, n, s, gx, gs, gr=None, r_m=0.0, bits=8, minmax=False, stream=None):
+    """STE gradient gx and the scale / offset gradients gs, gr (device fp64 scalars)."""
+    _chk(lib().mnmt_fake_quant_backward(_ptr(x), _ptr(g), n, float(s), float(r_m), bits, int(minmax), _ptr(gx),
+                                        _ptr(gs), _ptr(gr), _stream_handle(stream)))
+
+
+def mnmt_fake_quant_linear(X, W, s_x, s_w, bias, M, N, K, wbits, workspace, y, stream=None):
+    """QAT forward of a linear from fp32 input and weights (learnable scales)."""
+    _chk(lib().mnmt_fake_quant_linear(_ptr(X), _ptr(W), float(s_x), _ptr(s_w), _ptr(bias), M, N, K, wbits,
+                                      _ptr(workspace), _ptr(y), _stream_handle(stream)))
 
 
 def mnmt_codes_to_f16(src, dst, n, stream=None):
