@@ -1128,14 +1128,10 @@ int setup_cluster_step(mnmt_session *s) {
     if (env && env[0] == '0') return MNMT_OK;
     const int d = c.d_model, F = c.d_ffn, H = c.n_heads, dh = d / H;
     const int R = s->B * s->k;
-    const int nc = dc_cluster_size(d);
-    // the step's slice GEMV spreads each K-long row over K/64 lanes (a power
-    // of two) and a residual slice over at most 32 lanes: d, F and the
-    // factorised embedding width must be powers of two
     const int E = c.d_embed;
+    const int nc = dc_cluster_size(d, F, E);
     if (m->wq != 8 || s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
-        F % (16 * nc) || (3 * d) % (16 * nc) || !pow2_in(d, 64, 512) || !pow2_in(F, 64, 2048) ||
-        (m->factorised && !pow2_in(E, 16, 512)))
+        F % (16 * nc) || (3 * d) % (16 * nc))
         return MNMT_OK;
     DcParams P;
     std::memset(&P, 0, sizeof(P));

@@ -63,6 +63,14 @@ MNMT_DEV float dc_rn32_pow2(long long s, int e) {
     return dc_rn32_pow2_full(s, e);
 }
 
+// nearest float to s 2^e / (dodd 2^kd): the power-of-two case inline, an odd
+// factor (widths such as 384 = 3 * 128) out of line
+__device__ __noinline__ float dc_rn32_scaled_div(long long s, int e, int d) { return rn32_scaled_div(s, e, d); }
+MNMT_DEV float dc_rn32_scaled(long long s, int e, int kd, int dodd) {
+    if (dodd == 1) return dc_rn32_pow2(s, e - kd);
+    return dc_rn32_scaled_div(s, e, dodd << kd);
+}
+
 // signed bytes of a 32-bit word
 MNMT_DEV int sb0(int x) { return (x << 24) >> 24; }
 MNMT_DEV int sb1(int x) { return (x << 16) >> 24; }
@@ -139,7 +147,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
                                           long long *part_l) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int n = R * d, spr = d / 32;  // partial slots (warps) per row
-    const int log2d = 31 - __clz(d);
+    const int kd = __ffs(d) - 1, dodd = d >> kd;  // d = dodd 2^kd
     // pass 1: exact sum of x on the grid of max |x|
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
@@ -158,7 +166,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
         float hi, lo;
         dc_row_extremes(mm, row, nc, hi, lo);
         const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
-        const float mu = dc_rn32_pow2(dc_row_sum(part_l, row, spr), ea - 52 - log2d);
+        const float mu = dc_rn32_scaled(dc_row_sum(part_l, row, spr), ea - 52, kd, dodd);
         const int eb = exp_bound(fmaxf(fabsf(__fsub_rn(hi, mu)), fabsf(__fsub_rn(lo, mu))));
         const float cv = __fsub_rn(r[e0 + lane], mu);
         const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
@@ -175,7 +183,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
         const int row = e0 / d, e = e0 + lane, i = e - row * d;
         const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
         const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
-        const float var = dc_rn32_pow2(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52 - log2d);
+        const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd);
         const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
         const float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(r[e], mu), rstd), g[i]), b[i]);
         a[e] = q8(y, inv);
@@ -479,16 +487,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const float *sw = reinterpret_cast<const float *>(slot + rows * K);
             const float *bb = sw + rows;
             const float *iv = bb + rows;
-            const int kc = K / 16;  // 16-byte chunks per row (a power of two)
-            // lanes per row: as many as spread the slice's rows * kc chunks over
-            // all 8 warps, at most 32 (each lane takes kc / lpr chunks)
-            int cpl = 1;
-            while (rows * kc > DC_THREADS * cpl && cpl < kc) cpl *= 2;
-            int lpr = kc / cpl;
-            if (lpr > 32) {
-                lpr = 32;
-                cpl = kc / 32;
-            }
+            const int kc = K / 16;  // 16-byte chunks per row
+            // lanes per row: a power of two dividing kc, at most 32, and no more
+            // than spreads the slice's rows over the block's 256 threads (each
+            // lane takes kc / lpr chunks)
+            int lpr = kc & -kc;
+            if (lpr > 32) lpr = 32;
+            while (lpr > 1 && rows * lpr > DC_THREADS) lpr >>= 1;
+            const int cpl = kc / lpr;
             const int rpw = 32 / lpr;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
             const int sub = lane % lpr;
@@ -543,9 +549,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // for the next LayerNorm's grids
             if (threadIdx.x < 32 * R) {
                 const int m = threadIdx.x >> 5, ln = threadIdx.x & 31;
-                const unsigned k = ln < rows ? ordered_bits(stf[m * rows + ln]) : 0u;
-                const unsigned kh = __reduce_max_sync(0xFFFFFFFFu, k);
-                const unsigned kl = __reduce_min_sync(0xFFFFFFFFu, ln < rows ? k : 0xFFFFFFFFu);
+                unsigned kmax = 0u, kmin = 0xFFFFFFFFu;
+                for (int i = ln; i < rows; i += 32) {
+                    const unsigned k = ordered_bits(stf[m * rows + i]);
+                    kmax = k > kmax ? k : kmax;
+                    kmin = k < kmin ? k : kmin;
+                }
+                const unsigned kh = __reduce_max_sync(0xFFFFFFFFu, kmax);
+                const unsigned kl = __reduce_min_sync(0xFFFFFFFFu, kmin);
                 if (ln < nc) {
                     unsigned *dst = cl.map_shared_rank(mm + (m * nc + c) * 2, ln);
                     dst[0] = kh;
@@ -621,7 +632,8 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
     asm volatile("cp.async.wait_all;\n" ::);
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int lpr = kc >= 32 ? 32 : kc;  // lanes per weight row (kc is a power of two)
+    int lpr = kc & -kc;  // lanes per weight row: the largest power of two dividing kc, at most 32
+    if (lpr > 32) lpr = 32;
     const int rpw = 32 / lpr;            // rows per warp and pass
     const int grp = lane / lpr, sl = lane % lpr;
     unsigned long long best[MT];
@@ -700,14 +712,16 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
 // ---------------------------------------------------------------------------
 // CTAs per cluster: a slice of at least 16 columns of d per CTA, at most
 // MNMT_DC_MAX_CTAS (default 16, the largest cluster; measured fastest) CTAs
-int dc_cluster_size(int d) {
+int dc_cluster_size(int d, int F, int E) {
     int cap = 16;
     if (const char *e = getenv("MNMT_DC_MAX_CTAS")) cap = atoi(e);
     if (cap < 2) cap = 2;
     if (cap > 16) cap = 16;
-    int nc = d / 16;
-    if (nc > cap) nc = cap;
-    return nc >= 2 ? nc : 0;
+    // every phase's slice (d, 3d, F or the factorised width's d columns per
+    // CTA, as int8 or fp32) must be a whole number of 16-byte chunks
+    for (int nc = cap; nc >= 2; nc--)
+        if (d % (16 * nc) == 0 && (3 * d) % (16 * nc) == 0 && F % (16 * nc) == 0 && E % 16 == 0) return nc;
+    return 0;
 }
 
 // Fills the phase table and the shared-memory carve-up; returns the bytes of
@@ -850,8 +864,7 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
                                 int reserved_sms, cudaStream_t st) {
-    const int kc = K / 16;
-    if (M < 1 || M > 4 || K % 16 || (kc & (kc - 1))) return cudaErrorInvalidValue;
+    if (M < 1 || M > 4 || K % 16) return cudaErrorInvalidValue;
     // two blocks per SM, each holding its contiguous rows in shared memory, on
     // the SMs the step's cluster does not occupy: every block is resident (and
     // prefetching its rows) while the step runs, and the next step's cluster

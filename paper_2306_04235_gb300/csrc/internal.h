@@ -264,7 +264,7 @@ struct alignas(16) DcParams {
     DcPhase phase[1 + 6 * DC_LMAX];
 };
 static_assert(sizeof(DcParams) % 16 == 0, "the parameter block is copied in 16-byte chunks");
-int dc_cluster_size(int d);
+int dc_cluster_size(int d, int F, int E);
 size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
 bool decode_cluster_fits(int dh, int nc, size_t smem);

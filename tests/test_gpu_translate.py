@@ -14,6 +14,7 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 MINI = {
+    "odd": synth.ModelConfig(2, 2, 192, 3, 384, 300, 192, 1, 1, max_pos=64),   # d = 3 x 64: 4-CTA cluster step
     "pre": synth.ModelConfig(2, 2, 64, 2, 128, 300, 64, 1, 1, max_pos=64),
     "post": synth.ModelConfig(2, 1, 64, 1, 128, 300, 64, 0, 1, max_pos=64),
     "fact": synth.ModelConfig(3, 2, 128, 4, 256, 500, 32, 1, 0, max_pos=96),
