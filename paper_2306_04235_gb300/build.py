@@ -47,16 +47,24 @@ def _stale():
     return any(os.path.getmtime(p) > t for p in deps)
 
 
-def build(force: bool = False, verbose_ptxas: bool = False) -> str:
-    if not force and not _stale():
+STAMPS_LIB = os.path.join(OUT_DIR, "libmnmt_stamps.so")
+
+
+def build(force: bool = False, verbose_ptxas: bool = False, stamps: bool = False) -> str:
+    """Build libmnmt.so; stamps=True builds the phase-timing debug variant
+    libmnmt_stamps.so instead (the cluster decode step compiled with
+    -DMNMT_DC_STAMPS; see phase_profile.py)."""
+    lib = STAMPS_LIB if stamps else LIB
+    if not force and not stamps and not _stale():
         return LIB
     os.makedirs(OUT_DIR, exist_ok=True)
     nvcc = _nvcc()
     flags = _flags(verbose_ptxas)
 
     def compile_one(src):
-        obj = os.path.join(OUT_DIR, src.replace(".cu", ".o"))
-        cmd = [nvcc] + flags + ["-c", os.path.join(CSRC, src), "-o", obj]
+        obj = os.path.join(OUT_DIR, src.replace(".cu", ".stamps.o" if stamps else ".o"))
+        extra = ["-DMNMT_DC_STAMPS"] if stamps and src == "decode_cluster.cu" else []
+        cmd = [nvcc] + flags + extra + ["-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed on {src}:\n{r.stderr}")
@@ -67,14 +75,14 @@ def build(force: bool = False, verbose_ptxas: bool = False) -> str:
     if verbose_ptxas:
         for _, err in results:
             sys.stderr.write(err)
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     cmd = [nvcc] + ARCH + ["-shared", "-o", tmp] + [o for o, _ in results]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose_ptxas="-v" in sys.argv))
+    print(build(force="--force" in sys.argv, verbose_ptxas="-v" in sys.argv, stamps="--stamps" in sys.argv))

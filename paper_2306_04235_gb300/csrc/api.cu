@@ -932,7 +932,7 @@ int issue_decode_step(mnmt_session *s) {
     int *t_ptr = s->state + ST_T;
     int *status = s->state + ST_STATUS;
     if (s->use_cluster) {
-        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, st));
+        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, st));
         GreedyArgs g;
         g.keys = s->keys;
         g.tok = s->tok;
@@ -1130,7 +1130,7 @@ int setup_cluster_step(mnmt_session *s) {
     const int R = s->B * s->k;
     const int E = c.d_embed;
     const int nc = dc_cluster_size(d, F, E);
-    if (m->wq != 8 || s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
+    if (s->k != 1 || R > DC_RMAX || c.n_dec > DC_LMAX || nc == 0 || d > 512 || F > 2048 || d % (16 * nc) ||
         F % (16 * nc) || (3 * d) % (16 * nc))
         return MNMT_OK;
     DcParams P;
@@ -1138,7 +1138,7 @@ int setup_cluster_step(mnmt_session *s) {
     P.R = R; P.d = d; P.H = H; P.dh = dh; P.F = F; P.E = c.d_embed; P.V = c.vocab; P.T = s->Tcap; P.S = s->S;
     P.n_dec = c.n_dec; P.pre_ln = c.pre_ln; P.factorised = m->factorised; P.nc = nc;
     P.emb_q = m->emb_q; P.emb_s = m->emb_s;
-    if (m->factorised) P.proj = DcLin{m->proj.w, m->proj.s, m->proj.b};
+    if (m->factorised) P.proj = DcLin{m->proj.w, m->proj.s, m->proj.b, nullptr, 8};
     P.emb_scale = m->emb_scale; P.pe = m->pe;
     P.fin_g = m->dec_final.g; P.fin_b = m->dec_final.b; P.s_dout = m->s_dout;
     P.tok = s->tok; P.t_ptr = s->state + ST_T; P.done = s->state + ST_DONE; P.src_len = s->src_lens;
@@ -1152,9 +1152,14 @@ int setup_cluster_step(mnmt_session *s) {
         Y.s_in1 = A.s_in; Y.s_ctx1 = A.s_ctx; Y.gamma1 = A.gamma; Y.sigma1 = A.sigma; Y.rho1 = A.rho;
         Y.s_in2 = X.s_in; Y.s_ctx2 = X.s_ctx; Y.gamma2 = X.gamma; Y.sigma2 = X.sigma; Y.rho2 = X.rho;
         Y.s_in3 = Fb.s_in; Y.s_h = Fb.s_h; Y.gamma3 = Fb.gamma;
-        Y.qkv = DcLin{A.qkv.w, A.qkv.s, A.qkv.b}; Y.o = DcLin{A.o.w, A.o.s, A.o.b};
-        Y.q2 = DcLin{X.q.w, X.q.s, X.q.b}; Y.o2 = DcLin{X.o.w, X.o.s, X.o.b};
-        Y.w1 = DcLin{Fb.w1.w, Fb.w1.s, Fb.w1.b}; Y.w2 = DcLin{Fb.w2.w, Fb.w2.s, Fb.w2.b};
+        // 4-bit linears stream their packed codes (half the ring bytes)
+        auto dl = [](const Lin &x) {
+            if (x.bits == 4) return DcLin{reinterpret_cast<const int8_t *>(x.wp), x.s, x.b, x.m, 4};
+            return DcLin{x.w, x.s, x.b, nullptr, 8};
+        };
+        Y.qkv = dl(A.qkv); Y.o = dl(A.o);
+        Y.q2 = dl(X.q); Y.o2 = dl(X.o);
+        Y.w1 = dl(Fb.w1); Y.w2 = dl(Fb.w2);
         Y.inv_qkv = A.inv_qkv; Y.inv_q2 = X.inv_q; Y.inv_h = Fb.inv_h;
         Y.self_k = s->sk + l * s->sk_layer; Y.self_v = s->sv + l * s->sk_layer;
         Y.cross_k = s->ck + l * s->ck_layer; Y.cross_v = s->cv + l * s->ck_layer;
@@ -1181,7 +1186,7 @@ int setup_cluster_step(mnmt_session *s) {
     P.S = s->Smax;
     size_t smem = dc_layout(P, 227 * 1024);
     P.S = s->S;
-    if (!decode_cluster_fits(dh, nc, smem)) return MNMT_OK;
+    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8)) return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
     s->use_cluster = true;

@@ -31,6 +31,32 @@
 
 namespace cg = cooperative_groups;
 
+// Phase timing for the debug build (compiled with -DMNMT_DC_STAMPS only): CTA 0,
+// thread 0 records %globaltimer at the phase boundaries of decode step
+// DC_STAMP_STEP, and the vocabulary kernel of the step before records its
+// start, the end of its wait and its end.  Slots: 0 kernel start, 1 / 2
+// around the grid wait, 3 phase loop start, 4 + 4 ph .. 7 + 4 ph the phase's
+// ring wait / input prep / slice GEMV / broadcast + cluster barrier ends, 100
+// / 101 / 102 final LayerNorm start / end / kernel end, 110 .. 113 vocabulary
+// kernel (block 0 start, before / after its wait, last block's end).
+constexpr int DC_STAMP_STEP = 20;
+#ifdef MNMT_DC_STAMPS
+__device__ unsigned long long g_dc_ns[128];
+extern "C" int mnmt_dc_stamps(unsigned long long *out) {
+    return (int)cudaMemcpyFromSymbol(out, g_dc_ns, sizeof(g_dc_ns));
+}
+__device__ __forceinline__ unsigned long long dc_gtime() {
+    unsigned long long x;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(x));
+    return x;
+}
+#define DC_STAMP(cond, id) \
+    do { if ((cond) && (id) < 128) g_dc_ns[id] = dc_gtime(); } while (0)
+#else
+#define DC_STAMP(cond, id) \
+    do { } while (0)
+#endif
+
 namespace mnmt {
 
 constexpr int DC_THREADS = 256;
@@ -89,11 +115,12 @@ __device__ __noinline__ void dc_prefetch(const DcParams &P, int ph, int c, uint8
         const DcPhase &f = P.phase[ph];
         if (f.rows) {
             uint8_t *dst = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
-            const int wb = f.rows * f.K, vb = f.rows * 4;
+            const int wb = f.rows * (f.bits == 4 ? f.K / 2 : f.K), vb = f.rows * 4;
             dc_copy(dst, f.w + (size_t)c * wb, wb);
             dc_copy(dst + wb, f.s + c * f.rows, vb);
             dc_copy(dst + wb + vb, f.b + c * f.rows, vb);
             if (f.inv) dc_copy(dst + wb + 2 * vb, f.inv + c * f.rows, vb);
+            if (f.m) dc_copy(dst + wb + 3 * vb, f.m + c * f.rows, vb);
         }
     }
     dc_commit();
@@ -332,7 +359,9 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
 // ---------------------------------------------------------------------------
 enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
 
-template <int DH>
+// W4: the model's attention / FFN linears hold 4-bit codes (a separate
+// instantiation, so the int8 step carries no 4-bit code)
+template <int DH, bool W4>
 __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcParams *__restrict__ Pp) {
     // Launched as a programmatic dependent of the previous step's vocabulary
     // kernel: everything up to dc_grid_wait() reads only data that no kernel
@@ -340,6 +369,9 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     // encoder's cross keys / values), so it overlaps the previous kernel.
     // `done` only turns 0 -> 1 within a translation: seen set, it is final.
     if (*Pp->done) return;  // uniform for the whole cluster
+#ifdef MNMT_DC_STAMPS
+    const unsigned long long ns_start = dc_gtime();
+#endif
     extern __shared__ __align__(16) uint8_t smem[];
     {
         // the parameter block lives in shared memory for the whole step
@@ -387,12 +419,24 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
     }
     // ---- the previous step's results: token, position, self keys / values ----
+#ifdef MNMT_DC_STAMPS
+    const unsigned long long ns_w0 = dc_gtime();
+#endif
     dc_grid_wait();
     if (*P.done) {  // uniform for the whole cluster; no copy may outlive the CTA
         asm volatile("cp.async.wait_all;\n" ::);
         return;
     }
     const int t = *P.t_ptr;
+    const bool stamp = c == 0 && threadIdx.x == 0 && t == DC_STAMP_STEP;
+    (void)stamp;
+#ifdef MNMT_DC_STAMPS
+    if (stamp) {
+        g_dc_ns[0] = ns_start;
+        g_dc_ns[1] = ns_w0;
+        g_dc_ns[2] = dc_gtime();
+    }
+#endif
     if (threadIdx.x < R) {
         int id = P.tok[threadIdx.x];
         if (id < 0 || id >= P.V) {
@@ -415,6 +459,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
     }
     dc_prefetch(P, 1, c, ring);
+    DC_STAMP(stamp, 3);
 
     for (int ph = 0; ph < nphase; ph++) {
         const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
@@ -424,6 +469,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         if (ph == nphase - 1) dc_launch_dependents();
         dc_wait_ring();
         __syncthreads();
+        DC_STAMP(stamp, 4 + 4 * ph);
         dc_prefetch(P, ph + DC_NB - 1, c, ring);
         const uint8_t *slot = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
         const float *lnl = lnp + (size_t)6 * l * d;
@@ -459,6 +505,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             K = F;
         }
         __syncthreads();
+        DC_STAMP(stamp, 5 + 4 * ph);
 
         // ---- the phase's slice of outputs ----
         const int rows = ph == 0 ? d / nc : P.phase[ph].rows;
@@ -483,11 +530,18 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 stf[i] = __fadd_rn(v, P.pe[(size_t)t * d + n]);
             }
         } else {
+            // the slot: W rows (rows * K int8 codes, or rows * K / 2 bytes of
+            // packed 4-bit codes), then s, b, inv [rows] and, for min-max
+            // 4-bit rows, the offsets m [rows]
+            const DcPhase &f = P.phase[ph];
+            const bool w4 = W4 && kind != K_EMB && f.bits == 4;
+            const int rb = w4 ? K / 2 : K;  // weight bytes per row
             const int8_t *W = reinterpret_cast<const int8_t *>(slot);
-            const float *sw = reinterpret_cast<const float *>(slot + rows * K);
+            const float *sw = reinterpret_cast<const float *>(slot + rows * rb);
             const float *bb = sw + rows;
             const float *iv = bb + rows;
-            const int kc = K / 16;  // 16-byte chunks per row
+            const float *mw = (w4 && f.m) ? iv + rows : nullptr;
+            const int kc = rb / 16;  // 16-byte weight chunks per row (4-bit: one run of 32 codes each)
             // lanes per row: a power of two dividing kc, at most 32, and no more
             // than spreads the slice's rows over the block's 256 threads (each
             // lane takes kc / lpr chunks)
@@ -498,23 +552,44 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int rpw = 32 / lpr;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
             const int sub = lane % lpr;
+            const int4 ones = make_int4(0x01010101, 0x01010101, 0x01010101, 0x01010101);
             for (int r0 = warp * rpw; r0 < rows; r0 += DC_WARPS * rpw) {
                 const int nl = r0 + lane / lpr;
                 int acc[DC_RMAX] = {0, 0, 0, 0};
+                int a1[DC_RMAX] = {0, 0, 0, 0};  // 4-bit rows: the activation codes' sums
                 if (nl < rows) {
-                    const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * K);
+                    const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * rb);
                     for (int q = 0; q < cpl; q++) {
                         const int k = q * lpr + sub;  // consecutive lanes read consecutive chunks
                         const int4 w = wr[k];
+                        if (w4) {
+                            const int4 lo = make_int4(w.x & 0x0F0F0F0F, w.y & 0x0F0F0F0F, w.z & 0x0F0F0F0F,
+                                                      w.w & 0x0F0F0F0F);
+                            const int4 hi = make_int4((w.x >> 4) & 0x0F0F0F0F, (w.y >> 4) & 0x0F0F0F0F,
+                                                      (w.z >> 4) & 0x0F0F0F0F, (w.w >> 4) & 0x0F0F0F0F);
 #pragma unroll
-                        for (int m = 0; m < DC_RMAX; m++)
-                            if (m < R) acc[m] = dot16(reinterpret_cast<const int4 *>(A + (size_t)m * K)[k], w, acc[m]);
+                            for (int m = 0; m < DC_RMAX; m++)
+                                if (m < R) {
+                                    const int4 *am = reinterpret_cast<const int4 *>(A + (size_t)m * K);
+                                    const int4 x0 = am[2 * k], x1 = am[2 * k + 1];
+                                    acc[m] = dot16(x1, hi, dot16(x0, lo, acc[m]));
+                                    a1[m] = dot16(x1, ones, dot16(x0, ones, a1[m]));
+                                }
+                        } else {
+#pragma unroll
+                            for (int m = 0; m < DC_RMAX; m++)
+                                if (m < R)
+                                    acc[m] = dot16(reinterpret_cast<const int4 *>(A + (size_t)m * K)[k], w, acc[m]);
+                        }
                     }
                 }
 #pragma unroll
                 for (int m = 0; m < DC_RMAX; m++)
                     if (m < R)
-                        for (int o = lpr / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
+                        for (int o = lpr / 2; o > 0; o >>= 1) {
+                            acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
+                            if (w4) a1[m] += __shfl_xor_sync(0xFFFFFFFFu, a1[m], o);
+                        }
                 if (sub == 0 && nl < rows) {
                     const int n = n0 + nl;
 #pragma unroll
@@ -525,7 +600,16 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                             stf[m * rows + nl] = __fadd_rn(__fmul_rn(y, P.emb_scale), P.pe[(size_t)t * d + n]);
                             continue;
                         }
-                        const float y = dequant_bias(acc[m], sx, sw[nl], bb[nl]);
+                        float y;
+                        if (!w4) {
+                            y = dequant_bias(acc[m], sx, sw[nl], bb[nl]);
+                        } else if (!mw) {  // symmetric 4-bit rows: stored code v + 8
+                            y = dequant_bias(acc[m] - 8 * a1[m], sx, sw[nl], bb[nl]);
+                        } else {  // min-max rows: W = s u + r
+                            const float tt = __fmul_rn(__int2float_rn(acc[m]), __fmul_rn(sx, sw[nl]));
+                            const float oo = __fmul_rn(__int2float_rn(a1[m]), __fmul_rn(sx, mw[nl]));
+                            y = __fadd_rn(__fadd_rn(tt, oo), bb[nl]);
+                        }
                         if (out_f32) {
                             stf[m * rows + nl] = __fadd_rn(__fmul_rn(gam, r_full[(size_t)m * d + n]), y);
                         } else {
@@ -543,6 +627,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             }
         }
         __syncthreads();
+        DC_STAMP(stamp, 6 + 4 * ph);
         // ---- publish the slice to every CTA ----
         if (out_f32) {
             // the slice's largest and smallest residual value per row (rows <= 32),
@@ -570,6 +655,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             dc_bcast(cl, stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc);
         }
         cl.sync();
+        DC_STAMP(stamp, 7 + 4 * ph);
         if (kind == K_W2 && !P.pre_ln) {
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
@@ -577,6 +663,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l);
         }
     }
+    DC_STAMP(stamp, 100);
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
@@ -588,8 +675,10 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             if (P.resid_out) P.resid_out[i] = r_full[i];
         }
     }
+    DC_STAMP(stamp, 101);
     // every CTA must still hold its shared memory while others may write to it
     cl.sync();
+    DC_STAMP(stamp, 102);
 }
 
 // ---------------------------------------------------------------------------
@@ -605,6 +694,9 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
     // Launched as a programmatic dependent of the step kernel: the block's
     // weight rows, scales and biases (static) are fetched into shared memory
     // while the step kernel finishes; only the input row waits for it.
+#ifdef MNMT_DC_STAMPS
+    const unsigned long long v_start = dc_gtime();
+#endif
     dc_launch_dependents();
     extern __shared__ __align__(16) int4 vsm[];  // [rows][K/16] weights, [MT][K/16] input, [rows] scale, [rows] bias
     const int kc = K >> 4;
@@ -620,7 +712,17 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
         scs[i] = __fmul_rn(s_x, s_w[n0 + i]);
         bss[i] = bias[n0 + i];
     }
+#ifdef MNMT_DC_STAMPS
+    const unsigned long long v_w0 = dc_gtime();
+#endif
     dc_grid_wait();
+#ifdef MNMT_DC_STAMPS
+    if (blockIdx.x == 0 && threadIdx.x == 0 && *g.t_ptr == DC_STAMP_STEP - 1) {
+        g_dc_ns[110] = v_start;
+        g_dc_ns[111] = v_w0;
+        g_dc_ns[112] = dc_gtime();
+    }
+#endif
     if (*g.done) {  // no copy may outlive the block
         asm volatile("cp.async.wait_all;\n" ::);
         return;
@@ -700,6 +802,7 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
         fin_all &= f;
     }
     int all = __syncthreads_and(fin_all);
+    DC_STAMP(threadIdx.x == 0 && t == DC_STAMP_STEP - 1, 113);
     if (threadIdx.x == 0) {
         if (all || t + 1 >= *g.tmax_ptr) *g.done = 1;
         *g.t_ptr = t + 1;
@@ -730,18 +833,21 @@ int dc_cluster_size(int d, int F, int E) {
 size_t dc_layout(DcParams &P, size_t max_smem) {
     const int R = P.R, d = P.d, F = P.F, nc = P.nc;
     // phase table: slices of CTA c are rows [c * rows, (c + 1) * rows)
-    DcPhase z = {nullptr, nullptr, nullptr, nullptr, 0, 0};
+    DcPhase z = {nullptr, nullptr, nullptr, nullptr, nullptr, 0, 0, 8};
     P.phase[0] = z;
-    if (P.factorised) P.phase[0] = DcPhase{P.proj.w, P.proj.s, P.proj.b, nullptr, d / nc, P.E};
+    if (P.factorised) P.phase[0] = DcPhase{P.proj.w, P.proj.s, P.proj.b, nullptr, nullptr, d / nc, P.E, 8};
+    auto ph = [](const DcLin &x, const float *inv, int rows, int K) {
+        return DcPhase{x.w, x.s, x.b, inv, x.m, rows, K, x.bits};
+    };
     for (int l = 0; l < P.n_dec; l++) {
         const DcLayer &Y = P.layer[l];
         DcPhase *f = &P.phase[1 + 6 * l];
-        f[0] = DcPhase{Y.qkv.w, Y.qkv.s, Y.qkv.b, Y.inv_qkv, 3 * d / nc, d};
-        f[1] = DcPhase{Y.o.w, Y.o.s, Y.o.b, nullptr, d / nc, d};
-        f[2] = DcPhase{Y.q2.w, Y.q2.s, Y.q2.b, Y.inv_q2, d / nc, d};
-        f[3] = DcPhase{Y.o2.w, Y.o2.s, Y.o2.b, nullptr, d / nc, d};
-        f[4] = DcPhase{Y.w1.w, Y.w1.s, Y.w1.b, Y.inv_h, F / nc, d};
-        f[5] = DcPhase{Y.w2.w, Y.w2.s, Y.w2.b, nullptr, d / nc, F};
+        f[0] = ph(Y.qkv, Y.inv_qkv, 3 * d / nc, d);
+        f[1] = ph(Y.o, nullptr, d / nc, d);
+        f[2] = ph(Y.q2, Y.inv_q2, d / nc, d);
+        f[3] = ph(Y.o2, nullptr, d / nc, d);
+        f[4] = ph(Y.w1, Y.inv_h, F / nc, d);
+        f[5] = ph(Y.w2, nullptr, d / nc, F);
     }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;
@@ -770,7 +876,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const DcPhase &f = P.phase[ph];
-        int b = f.rows * f.K + 12 * f.rows;
+        int b = f.rows * (f.bits == 4 ? f.K / 2 : f.K) + (f.m ? 16 : 12) * f.rows;
         if (b > slot) slot = b;
     }
     P.slot_bytes = (slot + 15) & ~15;
@@ -793,9 +899,12 @@ cudaError_t decode_cluster_init() {
         if (err == cudaSuccess) err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem);
         if (err == cudaSuccess) err = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     };
-    setk((const void *)decode_cluster_kernel<32>);
-    setk((const void *)decode_cluster_kernel<64>);
-    setk((const void *)decode_cluster_kernel<128>);
+    setk((const void *)decode_cluster_kernel<32, false>);
+    setk((const void *)decode_cluster_kernel<64, false>);
+    setk((const void *)decode_cluster_kernel<128, false>);
+    setk((const void *)decode_cluster_kernel<32, true>);
+    setk((const void *)decode_cluster_kernel<64, true>);
+    setk((const void *)decode_cluster_kernel<128, true>);
     // the vocabulary kernel keeps its SMs in the largest shared-memory
     // configuration, so the next step's cluster (about 200 KB per CTA) can
     // become resident beside it as soon as it is allowed to launch
@@ -810,10 +919,19 @@ cudaError_t decode_cluster_init() {
 }
 
 // can one cluster of nc CTAs with smem bytes each be resident?
-bool decode_cluster_fits(int dh, int nc, size_t smem) {
+static const void *dc_kernel(int dh, bool w4) {
+    if (w4)
+        return dh == 32 ? (const void *)decode_cluster_kernel<32, true>
+                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, true>
+                                    : (const void *)decode_cluster_kernel<128, true>);
+    return dh == 32 ? (const void *)decode_cluster_kernel<32, false>
+                    : (dh == 64 ? (const void *)decode_cluster_kernel<64, false>
+                                : (const void *)decode_cluster_kernel<128, false>);
+}
+
+bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4) {
     if (smem > 227 * 1024) return false;
-    const void *k = dh == 32 ? (const void *)decode_cluster_kernel<32>
-                             : (dh == 64 ? (const void *)decode_cluster_kernel<64> : (const void *)decode_cluster_kernel<128>);
+    const void *k = dc_kernel(dh, w4);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -835,7 +953,7 @@ bool decode_cluster_fits(int dh, int nc, size_t smem) {
     return clusters >= 1;
 }
 
-cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, cudaStream_t st) {
+cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -853,12 +971,9 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    switch (dh) {
-        case 32: return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<32>, dP);
-        case 64: return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<64>, dP);
-        case 128: return cudaLaunchKernelEx(&cfg, decode_cluster_kernel<128>, dP);
-        default: return cudaErrorInvalidValue;
-    }
+    if (dh != 32 && dh != 64 && dh != 128) return cudaErrorInvalidValue;
+    void *args[] = {(void *)&dP};
+    return cudaLaunchKernelExC(&cfg, dc_kernel(dh, w4), args);
 }
 
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,

@@ -218,8 +218,10 @@ constexpr int DC_RMAX = 4;   // rows (sentences) per step
 constexpr int DC_LMAX = 16;  // decoder layers
 
 struct DcLin {
-    const int8_t *w;
+    const int8_t *w;  // int8 codes, or packed 4-bit codes when bits == 4
     const float *s, *b;
+    const float *m;   // 4-bit min-max rows: row offsets (else null)
+    int bits;         // 8 or 4
 };
 struct DcLayer {
     const float *ln1_g, *ln1_b, *ln2_g, *ln2_b, *ln3_g, *ln3_b;
@@ -235,9 +237,10 @@ struct DcLayer {
 // projection, then per layer qkv, o, q2, o2, w1, w2); CTA c's slice is rows
 // [c * rows, (c + 1) * rows) of the [N][K] matrix
 struct DcPhase {
-    const int8_t *w;
-    const float *s, *b, *inv;  // inv: per-column requantisation constants (or null)
-    int rows, K;
+    const int8_t *w;             // int8 codes or (bits == 4) packed 4-bit codes
+    const float *s, *b, *inv;    // inv: per-column requantisation constants (or null)
+    const float *m;              // 4-bit min-max rows: row offsets (else null)
+    int rows, K, bits;
 };
 struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
@@ -267,8 +270,8 @@ static_assert(sizeof(DcParams) % 16 == 0, "the parameter block is copied in 16-b
 int dc_cluster_size(int d, int F, int E);
 size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
-bool decode_cluster_fits(int dh, int nc, size_t smem);
-cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, cudaStream_t st);
+bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4);
+cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, cudaStream_t st);
 // reserved_sms: SMs the step kernel that precedes the launch occupies
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,

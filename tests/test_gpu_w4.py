@@ -101,7 +101,8 @@ def test_w4_batch1_workload_matches_oracle(wq, stream):
     g = _translate(blob, ids, lens, 1, wl.max_len, stream)
     o = O.translate(blob, ids, lens, 1, wl.max_len)
     assert np.array_equal(g[0], o[0]) and np.array_equal(g[1], o[1])
-    check_taps(blob, cfg, ids, lens, 1, wl.max_len, 24, [0], stream)
+    kind, _ = check_taps(blob, cfg, ids, lens, 1, wl.max_len, 24, [0], stream)
+    assert kind == 1  # the cluster decode step streams the packed 4-bit slices
     gl = _translate(blob, ids, lens, 1, wl.max_len, stream, lean=True)
     assert np.array_equal(gl[0], o[0])
 
@@ -129,3 +130,23 @@ def test_w4_paper_20mb_model(wq, stream):
     g = _translate(blob, ids, lens, beam, T, stream)
     o = O.translate(blob, ids, lens, beam, T)
     assert np.array_equal(g[0], o[0]) and np.array_equal(g[1], o[1])
+
+
+@pytest.mark.parametrize("wq", [synth.WQ_INT4, synth.WQ_INT4_MINMAX])
+@pytest.mark.parametrize("B", [1, 4])
+@pytest.mark.parametrize("shape", [(2, 2, 64, 2, 128, 300, 64, 1, 1), (3, 2, 128, 4, 256, 500, 32, 1, 0),
+                                   (2, 2, 192, 3, 384, 300, 192, 1, 1), (2, 1, 64, 1, 128, 300, 64, 0, 1)])
+def test_w4_cluster_step_matches_oracle(wq, B, shape, stream):
+    """Greedy batches of <= 4 run the single-cluster step on 4-bit slices."""
+    cfg = synth.ModelConfig(*shape, max_pos=64)
+    blob = synth.build_blob(cfg, 71, gamma_range=(0.5, 1.5), wq=wq)
+    ids, lens = synth.source_batch(cfg.vocab, B, 1, 40, 72)
+    T = 20
+    tr = mnmt.Translator(blob, B, ids.shape[1], 1, T, stream)
+    try:
+        g_ids, g_len, _ = tr.translate(ids, lens, T)
+        assert mnmt.mnmt_session_decode_path(tr.session) == 1
+    finally:
+        tr.close()
+    o_ids, o_len, _ = O.translate(blob, ids, lens, 1, T, n_threads=B)
+    assert np.array_equal(g_ids, o_ids) and np.array_equal(g_len, o_len)
