@@ -38,7 +38,6 @@ MNMT_DEV uint32_t vec_word(const uint4 &v, int k) { return k == 0 ? v.x : k == 1
 // then fetches from L2 once and serves from L1.
 template <int DH, bool XS>
 __global__ void __launch_bounds__(XS ? 32 * 32 : 32 * 16) attn_decode(AttnDecArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (a.skip && *a.skip) return;
     extern __shared__ int dsm[];
@@ -195,7 +194,6 @@ constexpr int ENC_QCHUNK = 32;
 
 template <int DH>
 __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, int qchunk) {
-    pdl_allow_next();
     pdl_grid_wait();
     extern __shared__ __align__(16) uint8_t esm[];
     constexpr int KS = DH + 16;  // padded key row: conflict-free 16-byte lane reads

@@ -249,7 +249,6 @@ template <int BN, int NCH, int STAGES, int NBUF>
 __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant__ CUtensorMap tmA,
                                                            const __grid_constant__ CUtensorMap tmB, int M, int N,
                                                            int K, Epi e, int *status) {
-    pdl_allow_next();
     pdl_grid_wait();
     using L = TcLayout<BN, STAGES>;
     constexpr int ACC_COLS = NCH * BN;  // one accumulator buffer (NBUF of them)
@@ -359,6 +358,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
             if (failed) break;
             mma_commit(accf_bar(buf));
         }
+        // every MMA of this CTA is issued: the stream's next kernel may launch
+        // (it waits for this grid's completion before it reads anything)
+        pdl_allow_next();
         misc[2] = it;          // k-blocks whose copies this thread saw land
         mma_commit(done_bar);  // arrives once every MMA issued above has completed
     } else if (warp >= 2) {
@@ -471,7 +473,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc(const __grid_constant
 // ---------------------------------------------------------------------------
 __global__ void codes_to_f16_kernel(const int8_t *__restrict__ src, int ld_src, __half *__restrict__ dst, int ld_dst,
                                     int rows, int cols) {
-    pdl_allow_next();
     pdl_grid_wait();
     const int per_row = cols >> 4;
     const long total = (long)rows * per_row;
@@ -489,7 +490,6 @@ __global__ void codes_to_f16_kernel(const int8_t *__restrict__ src, int ld_src, 
 }
 
 __global__ void codes_to_f16_tail(const int8_t *src, __half *dst, size_t from, size_t n) {
-    pdl_allow_next();
     pdl_grid_wait();
     size_t i = from + blockIdx.x * (size_t)blockDim.x + threadIdx.x;
     if (i < n) dst[i] = __short2half_rn((short)src[i]);
@@ -559,7 +559,6 @@ template <int S>
 __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc_sk(const __grid_constant__ CUtensorMap tmA,
                                                               const __grid_constant__ CUtensorMap tmB, int M, int N,
                                                               int K, Epi e, int *status) {
-    pdl_allow_next();
     pdl_grid_wait();
     using L = SkLayout<S>;
     constexpr int SW = SK_BN / S;  // columns this CTA finishes
@@ -643,6 +642,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1) linear_tc_sk(const __grid_const
                 mma_f16(tbase, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), IDESC, (uint32_t)(it | k));
             mma_commit(empty_bar(s));
         }
+        pdl_allow_next();  // every MMA of this CTA is issued
         misc[2] = it;
         mma_commit(accf_bar);  // also after a timed-out wait: the epilogue reaches the cluster barrier
         mma_commit(done_bar);

@@ -35,7 +35,6 @@ template <int MT, int LPC, int U>
 __global__ void __launch_bounds__(SM_THREADS) linear_smallm(const int8_t *__restrict__ A, int lda,
                                                            const int8_t *__restrict__ W, int M, int N,
                                                            int K, Epi e) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (e.skip && *e.skip) return;
     extern __shared__ int4 smA[];  // [MT][K/16]
@@ -176,7 +175,6 @@ __global__ void __launch_bounds__(WARPS_M *WARPS_N * 32)
     constexpr int WTM = BM / WARPS_M, WTN = BN / WARPS_N;
     constexpr int MI = WTM / 16, NI = WTN / 8;
     static_assert(NI % 2 == 0, "B fragments are loaded two n8 tiles at a time");
-    pdl_allow_next();
     pdl_grid_wait();
     if (e.skip && *e.skip) return;
     extern __shared__ __align__(128) uint8_t smem[];

@@ -40,7 +40,6 @@ __global__ void __launch_bounds__(W4_THREADS) linear_w4_small(const int8_t *__re
                                                              const uint8_t *__restrict__ Wp,
                                                              const float *__restrict__ m_w, int M, int N, int K,
                                                              Epi e) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (e.skip && *e.skip) return;
     extern __shared__ int4 smA[];  // [MT][K/16]

@@ -23,7 +23,6 @@ namespace mnmt {
 // ---------------------------------------------------------------------------
 template <int VPT, int LN_T>
 __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     __shared__ unsigned s_amax[LN_T / 32], s_bmax[LN_T / 32];
     __shared__ long long s_s1[LN_T / 32], s_s2[LN_T / 32];
@@ -93,6 +92,7 @@ __global__ void __launch_bounds__(LN_T) layernorm_kernel(LnArgs a) {
     for (int k = 0; k < LN_T / 32; k++) s2 += s_s2[k];
     const float var = rn32_scaled_div(s2, 2 * eb - 52, d);
     const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
+    pdl_allow_next();  // only the normalise-and-store pass is left
 #pragma unroll
     for (int v = 0; v < VPT; v++) {
         const int i = i0 + v;
@@ -135,7 +135,6 @@ cudaError_t launch_layernorm(const LnArgs &a, cudaStream_t st) {
 // ---------------------------------------------------------------------------
 template <int VPL>
 __global__ void __launch_bounds__(256) embed_kernel(EmbedArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (a.skip && *a.skip) return;
     const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -214,7 +213,6 @@ cudaError_t launch_embed(const EmbedArgs &a, cudaStream_t st) {
 // search state
 // ---------------------------------------------------------------------------
 __global__ void search_init_kernel(InitArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < a.R) {
@@ -247,7 +245,6 @@ cudaError_t launch_search_init(const InitArgs &a, cudaStream_t st) {
 
 // greedy: argmax key -> token; after EOS a sentence emits PAD
 __global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (*a.done) return;
     const int t = *a.t_ptr;
@@ -359,7 +356,6 @@ MNMT_DEV float warp_list_insert(unsigned long long &wl, unsigned long long key, 
 // simpler passes: better where a few rows leave the SMs short of warps).
 template <int KM, int NT, bool CAND>
 __global__ void __launch_bounds__(NT) beam_rows_kernel(BeamArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (*a.done) return;
     constexpr int KC = KM + 4;
@@ -532,7 +528,6 @@ __global__ void __launch_bounds__(NT) beam_rows_kernel(BeamArgs a) {
 
 // per sentence: best k of the k*k row candidates; reorder state
 __global__ void __launch_bounds__(256) beam_select_kernel(BeamArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     if (*a.done) return;
     const int b = blockIdx.x;
@@ -638,7 +633,6 @@ cudaError_t launch_beam_step(const BeamArgs &a, cudaStream_t st) {
 // backtracked through the parent pointers
 // ---------------------------------------------------------------------------
 __global__ void finalize_kernel(FinalArgs a) {
-    pdl_allow_next();
     pdl_grid_wait();
     const int b = blockIdx.x;
     if (threadIdx.x != 0) return;
