@@ -549,7 +549,10 @@ extern "C" void mnmt_model_free(mnmt_model *m) {
 // ---------------------------------------------------------------------------
 // session
 // ---------------------------------------------------------------------------
-enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_STATUS = 5, ST_N = 8 };
+// state words: step counter, done flag, step limit, beam tickets [3..4] (the
+// cluster step's pending greedy selection shares [4]: search init clears
+// both), status
+enum { ST_T = 0, ST_DONE = 1, ST_TMAX = 2, ST_TICKET = 3, ST_PENDING = 4, ST_STATUS = 5, ST_N = 8 };
 // layers of more rows than the GEMV kernel takes (16) run on the tensor cores
 constexpr size_t TC_MIN_ROWS = 17;
 // steps per multi-step decode graph (and per completion check of translate)
@@ -945,6 +948,7 @@ int issue_decode_step(mnmt_session *s) {
         g.T = s->Tcap;
         g.eos = c.eos_id;
         g.pad = c.pad_id;
+        g.pending = s->state + ST_PENDING;
         LK(launch_vocab_greedy(s->act, m->out.w, m->out.s, m->out.b, m->s_dout, R, c.vocab, d, s->keys,
                                s->state + ST_TICKET, g, s->dc_nc, st));
         return MNMT_OK;
@@ -1142,6 +1146,9 @@ int setup_cluster_step(mnmt_session *s) {
     P.emb_scale = m->emb_scale; P.pe = m->pe;
     P.fin_g = m->dec_final.g; P.fin_b = m->dec_final.b; P.s_dout = m->s_dout;
     P.tok = s->tok; P.t_ptr = s->state + ST_T; P.done = s->state + ST_DONE; P.src_len = s->src_lens;
+    P.keys = s->keys; P.tok_w = s->tok; P.fin = s->fin; P.hist = s->hist; P.t_w = s->state + ST_T;
+    P.done_w = s->state + ST_DONE; P.pending = s->state + ST_PENDING; P.tmax_ptr = s->state + ST_TMAX;
+    P.eos = c.eos_id; P.pad = c.pad_id;
     P.act_out = s->act; P.resid_out = s->resid; P.status = s->state + ST_STATUS;
     for (int l = 0; l < c.n_dec; l++) {
         const SelfBlk &A = m->dec_self[l];
@@ -1202,6 +1209,25 @@ int capture_steps(mnmt_session *s, int steps, cudaGraphExec_t *out) {
     CK(cudaStreamBeginCapture(st, cudaStreamCaptureModeThreadLocal));
     int rc = MNMT_OK;
     for (int i = 0; i < steps && !rc; i++) rc = issue_decode_step(s);
+    if (!rc && s->use_cluster) {
+        // the last step's greedy selection is still pending: apply it, so the
+        // step counter, done flag and history are current when the graph ends
+        GreedyArgs ga;
+        ga.keys = s->keys;
+        ga.tok = s->tok;
+        ga.fin = s->fin;
+        ga.hist = s->hist;
+        ga.t_ptr = s->state + ST_T;
+        ga.done = s->state + ST_DONE;
+        ga.tmax_ptr = s->state + ST_TMAX;
+        ga.R = s->B * s->k;
+        ga.T = s->Tcap;
+        ga.eos = s->m->c.eos_id;
+        ga.pad = s->m->c.pad_id;
+        ga.pending = s->state + ST_PENDING;
+        cudaError_t le = launch_greedy_update(ga, st);
+        if (le != cudaSuccess) rc = fail(MNMT_ECUDA, "greedy update launch failed: %s", cudaGetErrorString(le));
+    }
     cudaError_t ce = cudaStreamEndCapture(st, &g);
     if (rc) {
         if (g) cudaGraphDestroy(g);

@@ -357,6 +357,21 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
 // ---------------------------------------------------------------------------
 // the step kernel: one generic phase body run 1 + 6 * n_dec times
 // ---------------------------------------------------------------------------
+// commit the greedy selection of decode step tp (one thread): the token per
+// row into the history and the next input, the finished flags, the cleared
+// keys for the next vocabulary kernel, the step counter; done if requested
+__device__ __noinline__ void dc_commit_greedy(const DcParams &P, int tp, const int *out, const int *fin, int done) {
+    for (int m = 0; m < P.R; m++) {
+        P.hist[(size_t)tp * P.R + m] = out[m];
+        P.tok_w[m] = out[m];
+        P.fin[m] = fin[m];
+        P.keys[m] = 0ull;
+    }
+    *P.t_w = tp + 1;
+    if (done) *P.done_w = 1;
+    *P.pending = 0;
+}
+
 enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
 
 // W4: the model's attention / FFN linears hold 4-bit codes (a separate
@@ -427,7 +442,33 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         asm volatile("cp.async.wait_all;\n" ::);
         return;
     }
-    const int t = *P.t_ptr;
+    int t = *P.t_ptr;
+    // The previous step's vocabulary kernel left its greedy selection pending
+    // (row maxima in keys): apply it here -- every CTA computes the same
+    // tokens and finished flags from the same data; CTA 0 commits them (token,
+    // history, flags, step counter, cleared keys) at the end of this step, or
+    // at once if the translation has just finished.
+    static_assert(3 * DC_RMAX <= 16, "tokens, pending tokens and flags share the 16-int token area");
+    int *s_out = tok_s + DC_RMAX, *s_fin = tok_s + 2 * DC_RMAX;  // no static shared memory: the
+                                                                 // dynamic carve-up may take all 227 KB
+    const bool pend = *P.pending != 0;
+    if (pend) {
+        if (threadIdx.x < R) {
+            const int y = (int)key_index(P.keys[threadIdx.x]);
+            const int f = P.fin[threadIdx.x];
+            s_out[threadIdx.x] = f ? P.pad : y;
+            s_fin[threadIdx.x] = (f || y == P.eos) ? 1 : 0;
+        }
+        __syncthreads();
+        int all = 1;
+        for (int m = 0; m < R; m++) all &= s_fin[m];
+        if (all || t + 1 >= *P.tmax_ptr) {  // uniform over the cluster
+            if (c == 0 && threadIdx.x == 0) dc_commit_greedy(P, t, s_out, s_fin, 1);
+            asm volatile("cp.async.wait_all;\n" ::);
+            return;
+        }
+        t = t + 1;
+    }
     const bool stamp = c == 0 && threadIdx.x == 0 && t == DC_STAMP_STEP;
     (void)stamp;
 #ifdef MNMT_DC_STAMPS
@@ -438,7 +479,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
 #endif
     if (threadIdx.x < R) {
-        int id = P.tok[threadIdx.x];
+        int id = pend ? s_out[threadIdx.x] : P.tok[threadIdx.x];
         if (id < 0 || id >= P.V) {
             set_status(P.status, MNMT_EINVAL);
             id = 0;
@@ -676,6 +717,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
     }
     DC_STAMP(stamp, 101);
+    if (pend && c == 0 && threadIdx.x == 0) dc_commit_greedy(P, t - 1, s_out, s_fin, 0);
     // every CTA must still hold its shared memory while others may write to it
     cl.sync();
     DC_STAMP(stamp, 102);
@@ -767,7 +809,6 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
         }
     }
     __shared__ unsigned long long red[8][MT];
-    __shared__ int s_last;
 #pragma unroll
     for (int m = 0; m < MT; m++) {
         unsigned long long v = warp_max_u64(best[m]);
@@ -779,35 +820,13 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
         for (int w = 0; w < 8; w++) v = red[w][threadIdx.x] > v ? red[w][threadIdx.x] : v;
         atomicMax(keys + threadIdx.x, v);
     }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        __threadfence();
-        s_last = atomicAdd(ticket, 1) == (int)gridDim.x - 1;
-    }
-    __syncthreads();
-    if (!s_last) return;
-    // last block: greedy update of every row (keys read and cleared atomically)
-    __threadfence();
-    const int t = *g.t_ptr;
-    int fin_all = 1;
-    for (int r = threadIdx.x; r < g.R; r += 256) {
-        unsigned long long k = atomicExch(keys + r, 0ull);
-        int y = (int)key_index(k);
-        int f = g.fin[r];
-        int out = f ? g.pad : y;
-        g.hist[(size_t)t * g.R + r] = out;
-        g.tok[r] = out;
-        if (!f && y == g.eos) f = 1;
-        g.fin[r] = f;
-        fin_all &= f;
-    }
-    int all = __syncthreads_and(fin_all);
-    DC_STAMP(threadIdx.x == 0 && t == DC_STAMP_STEP - 1, 113);
-    if (threadIdx.x == 0) {
-        if (all || t + 1 >= *g.tmax_ptr) *g.done = 1;
-        *g.t_ptr = t + 1;
-        *ticket = 0;
-    }
+    // The greedy bookkeeping of this step (token, history, finished flags,
+    // step counter) is left to the next step kernel, which reads the keys
+    // after waiting for this grid anyway, or to the greedy update closing a
+    // run of steps: no fence, ticket or last-block pass on the step's path.
+    if (blockIdx.x == 0 && threadIdx.x == 0) *g.pending = 1;
+    DC_STAMP(blockIdx.x == 0 && threadIdx.x == 0 && *g.t_ptr == DC_STAMP_STEP - 1, 113);
+    (void)ticket;
 }
 
 // ---------------------------------------------------------------------------

@@ -180,6 +180,10 @@ struct GreedyArgs {
     int *t_ptr, *done;
     const int *tmax_ptr;       // steps of this translation (device)
     int R, T, eos, pad;
+    // cluster step: 1 while a vocabulary kernel's maxima wait in keys for their
+    // bookkeeping (done by the next step kernel, or by the greedy update as
+    // the flush at the end of a run of steps, which then does nothing when 0)
+    int *pending = nullptr;
 };
 cudaError_t launch_greedy_update(const GreedyArgs &a, cudaStream_t st);
 
@@ -258,6 +262,12 @@ struct alignas(16) DcParams {
     float s_dout;
     const int32_t *tok;
     const int *t_ptr, *done;
+    // the previous step's greedy selection, applied by this step (CTA 0 writes)
+    unsigned long long *keys;
+    int32_t *tok_w, *fin, *hist;
+    int *t_w, *done_w, *pending;
+    const int *tmax_ptr;
+    int eos, pad;
     const int32_t *src_len;
     int8_t *act_out;
     float *resid_out;

@@ -247,6 +247,7 @@ cudaError_t launch_search_init(const InitArgs &a, cudaStream_t st) {
 __global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
     pdl_grid_wait();
     if (*a.done) return;
+    if (a.pending && !*a.pending) return;  // the cluster step applied it already
     const int t = *a.t_ptr;
     int fin_all = 1;
     for (int r = threadIdx.x; r < a.R; r += blockDim.x) {
@@ -265,6 +266,7 @@ __global__ void __launch_bounds__(1024) greedy_update_kernel(GreedyArgs a) {
     if (threadIdx.x == 0) {
         if (all || t + 1 >= *a.tmax_ptr) *a.done = 1;
         *a.t_ptr = t + 1;
+        if (a.pending) *a.pending = 0;
     }
 }
 
