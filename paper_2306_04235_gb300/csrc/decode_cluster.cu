@@ -28,6 +28,7 @@
 
 #include "common.cuh"
 #include "internal.h"
+#include "mbarrier.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -38,7 +39,7 @@ namespace cg = cooperative_groups;
 // around the grid wait, 3 phase loop start, 4 + 4 ph .. 7 + 4 ph the phase's
 // ring wait / input prep / slice GEMV / broadcast + cluster barrier ends, 100
 // / 101 / 102 final LayerNorm start / end / kernel end, 110 .. 113 vocabulary
-// kernel (block 0 start, before / after its wait, last block's end).
+// kernel (block 0 start, before / after its wait, end).
 constexpr int DC_STAMP_STEP = 20;
 #ifdef MNMT_DC_STAMPS
 __device__ unsigned long long g_dc_ns[128];
@@ -68,7 +69,6 @@ MNMT_DEV void dc_cp16(void *dst_smem, const void *src) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16;\n" ::"r"(dc_smem_u32(dst_smem)), "l"(src));
 }
 MNMT_DEV void dc_commit() { asm volatile("cp.async.commit_group;\n" ::); }
-MNMT_DEV void dc_wait_ring() { asm volatile("cp.async.wait_group %0;\n" ::"n"(DC_NB - 2)); }
 
 // programmatic dependent launch: wait for the preceding kernel of the stream
 // (and the memory it wrote); allow the following kernel to launch
@@ -110,20 +110,37 @@ MNMT_DEV void dc_copy(void *dst, const void *src, int bytes) {
 }
 
 // ring slot layout: W rows (rows * K bytes), then s[rows], b[rows], inv[rows] (fp32)
-__device__ __noinline__ void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring) {
-    if (ph < 1 + 6 * P.n_dec) {
-        const DcPhase &f = P.phase[ph];
-        if (f.rows) {
-            uint8_t *dst = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
-            const int wb = f.rows * (f.bits == 4 ? f.K / 2 : f.K), vb = f.rows * 4;
-            dc_copy(dst, f.w + (size_t)c * wb, wb);
-            dc_copy(dst + wb, f.s + c * f.rows, vb);
-            dc_copy(dst + wb + vb, f.b + c * f.rows, vb);
-            if (f.inv) dc_copy(dst + wb + 2 * vb, f.inv + c * f.rows, vb);
-            if (f.m) dc_copy(dst + wb + 3 * vb, f.m + c * f.rows, vb);
-        }
+// Phase ph's slice goes to slot ph % DC_NB as up to five 1-D bulk copies (the
+// copy engine moves them: no per-thread copy instructions queue ahead of the
+// phase's own shared-memory work) that complete on the slot's mbarrier; the
+// barrier gets one arrival per phase, copies or not, so phase ph always waits
+// for parity (ph / DC_NB) & 1.  Issued by thread `who`; slices, offsets and
+// sizes are whole 16-byte chunks (the cluster size is chosen so).
+MNMT_DEV void dc_prefetch(const DcParams &P, int ph, int c, uint8_t *ring, uint32_t bars, int who = 0) {
+    if ((int)threadIdx.x != who || ph >= 1 + 6 * P.n_dec) return;
+    const DcPhase &f = P.phase[ph];
+    const uint32_t bar = bars + 8u * (uint32_t)(ph % DC_NB);
+    if (!f.rows) {
+        mbar_arrive(bar);
+        return;
     }
-    dc_commit();
+    const uint32_t dst = dc_smem_u32(ring + (size_t)(ph % DC_NB) * P.slot_bytes);
+    const uint32_t wb = (uint32_t)(f.rows * (f.bits == 4 ? f.K / 2 : f.K)), vb = (uint32_t)f.rows * 4u;
+    const uint32_t total = wb + vb * (2u + (f.inv ? 1u : 0u) + (f.m ? 1u : 0u));
+    // the slot's previous contents were read by ordinary loads before the
+    // block barrier that precedes this call; order them before the copy's writes
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+    mbar_expect_tx(bar, total);
+    bulk_load(dst, f.w + (size_t)c * wb, wb, bar);
+    bulk_load(dst + wb, f.s + c * f.rows, vb, bar);
+    bulk_load(dst + wb + vb, f.b + c * f.rows, vb, bar);
+    if (f.inv) bulk_load(dst + wb + 2 * vb, f.inv + c * f.rows, vb, bar);
+    if (f.m) bulk_load(dst + wb + 3 * vb, f.m + c * f.rows, vb, bar);
+}
+
+// wait for phase ph's slice; a wait that gives up records MNMT_ETIMEOUT
+MNMT_DEV void dc_wait_slice(const DcParams &P, int ph, uint32_t bars) {
+    if (!mbar_wait(bars + 8u * (uint32_t)(ph % DC_NB), (uint32_t)(ph / DC_NB) & 1u)) set_status(P.status, MNMT_ETIMEOUT);
 }
 
 // copy stage [R][row_bytes] into every CTA's full buffer at column offset
@@ -393,9 +410,15 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const int n16 = (int)(sizeof(DcParams) / 16);
         for (int i = threadIdx.x; i < n16; i += DC_THREADS)
             reinterpret_cast<int4 *>(smem)[i] = reinterpret_cast<const int4 *>(Pp)[i];
+        if (threadIdx.x == 0) {  // the weight ring's mbarriers, one arrival per phase
+            const uint32_t b0 = dc_smem_u32(smem + Pp->off_bar);
+            for (int i = 0; i < DC_NB; i++) mbar_init(b0 + 8u * (uint32_t)i, 1u);
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
         __syncthreads();
     }
     const DcParams &P = *reinterpret_cast<const DcParams *>(smem);
+    const uint32_t bars = dc_smem_u32(smem + P.off_bar);
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
     const int nc = P.nc;
@@ -421,7 +444,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
 
     // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
     dc_copy(lnp, P.ln_all, (6 * P.n_dec + 2) * d * 4);
-    dc_prefetch(P, 0, c, ring);
+    dc_prefetch(P, 0, c, ring, bars);
     // group 1: the second weight slice and the keys / values the step attends to
     if (P.kv_staged) {
         // one layer's cross K (or V) is one contiguous [R][H][S][dh] block: the
@@ -440,6 +463,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     dc_grid_wait();
     if (*P.done) {  // uniform for the whole cluster; no copy may outlive the CTA
         asm volatile("cp.async.wait_all;\n" ::);
+        dc_wait_slice(P, 0, bars);
         return;
     }
     int t = *P.t_ptr;
@@ -465,6 +489,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         if (all || t + 1 >= *P.tmax_ptr) {  // uniform over the cluster
             if (c == 0 && threadIdx.x == 0) dc_commit_greedy(P, t, s_out, s_fin, 1);
             asm volatile("cp.async.wait_all;\n" ::);
+            dc_wait_slice(P, 0, bars);
             return;
         }
         t = t + 1;
@@ -499,7 +524,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                     (lkv & 1 ? Y.self_v : Y.self_k) + (size_t)mh * P.T * (d / H) + (size_t)ch * 16);
         }
     }
-    dc_prefetch(P, 1, c, ring);
+    dc_prefetch(P, 1, c, ring, bars);
+    dc_prefetch(P, 2, c, ring, bars);
     DC_STAMP(stamp, 3);
 
     for (int ph = 0; ph < nphase; ph++) {
@@ -508,10 +534,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const DcLayer &Y = P.layer[l];
         // from the last phase on, the vocabulary kernel may launch and fetch its weights
         if (ph == nphase - 1) dc_launch_dependents();
-        dc_wait_ring();
-        __syncthreads();
+        // Each thread waits for the slice itself; the cluster barrier that ended
+        // the previous phase already orders this CTA's threads.  Phase 0 reads
+        // the tokens of the prologue, phase 1 on the LayerNorm vectors and
+        // (phase 2 on) the staged keys / values: both cross a block barrier.
+        if (ph == 1) asm volatile("cp.async.wait_all;\n" ::: "memory");
+        dc_wait_slice(P, ph, bars);
+        if (ph <= 1) __syncthreads();
         DC_STAMP(stamp, 4 + 4 * ph);
-        dc_prefetch(P, ph + DC_NB - 1, c, ring);
         const uint8_t *slot = ring + (size_t)(ph % DC_NB) * P.slot_bytes;
         const float *lnl = lnp + (size_t)6 * l * d;
 
@@ -669,6 +699,10 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         }
         __syncthreads();
         DC_STAMP(stamp, 6 + 4 * ph);
+        // the slot is free again: the slice of phase ph + DC_NB goes into it,
+        // issued by the last warp, which the small broadcasts leave idle (a
+        // thread issuing bulk copies is held for a few hundred ns)
+        dc_prefetch(P, ph + DC_NB, c, ring, bars, DC_THREADS - 32);
         // ---- publish the slice to every CTA ----
         if (out_f32) {
             // the slice's largest and smallest residual value per row (rows <= 32),
@@ -892,6 +926,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
     P.off_part = take(512 + 1024 + 64);  // slice extremes [R][nc][2], LN partials [2][64], per-row (mu, eb)
     if (R * d > 64 * 32) return (size_t)-1;                         // 64 warp chunks of partials
+    P.off_bar = take(8 * DC_NB);
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const DcPhase &f = P.phase[ph];
