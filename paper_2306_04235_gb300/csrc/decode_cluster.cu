@@ -143,17 +143,43 @@ MNMT_DEV void dc_wait_slice(const DcParams &P, int ph, uint32_t bars) {
     if (!mbar_wait(bars + 8u * (uint32_t)(ph % DC_NB), (uint32_t)(ph / DC_NB) & 1u)) set_status(P.status, MNMT_ETIMEOUT);
 }
 
-// copy stage [R][row_bytes] into every CTA's full buffer at column offset
-__device__ __noinline__ void dc_bcast(cg::cluster_group &cl, const uint8_t *stage, int R, int row_bytes, uint8_t *full,
-                       int full_row_bytes, int col_off, int nc) {
+// Exchange between the CTAs of the cluster.  A phase's slice goes to every
+// CTA (itself included) as st.async stores, each completing its bytes on the
+// receiver's exchange mbarrier for that phase (two, used by alternate
+// phases); a CTA waits on its own barrier until the whole vector has arrived
+// instead of a cluster-wide barrier.  No store can overwrite data a receiver
+// still reads: a CTA sends phase ph + 1 only after receiving phase ph from
+// every CTA, i.e. after every CTA finished the GEMV of phase ph (and with it
+// every read of the buffers that phase ph + 1 overwrites).
+MNMT_DEV uint32_t dc_mapa(uint32_t local, int rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;\n" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+MNMT_DEV void dc_st_async4(uint32_t remote, int4 v, uint32_t remote_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];\n" ::"r"(
+                     remote),
+                 "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(remote_bar)
+                 : "memory");
+}
+MNMT_DEV void dc_st_async2(uint32_t remote, unsigned x, unsigned y, uint32_t remote_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v2.b32 [%0], {%1, %2}, [%3];\n" ::"r"(remote),
+                 "r"(x), "r"(y), "r"(remote_bar)
+                 : "memory");
+}
+
+// copy stage [R][row_bytes] into every CTA's full buffer at column offset,
+// completing on each receiver's exchange barrier xbar (local address)
+__device__ __noinline__ void dc_bcast(const uint8_t *stage, int R, int row_bytes, uint8_t *full, int full_row_bytes,
+                                      int col_off, int nc, uint32_t xbar) {
     const int cpr = row_bytes / 16;
     const int total = nc * R * cpr;
     for (int i = threadIdx.x; i < total; i += DC_THREADS) {
         const int dst = i / (R * cpr), rem = i - dst * R * cpr;
         const int m = rem / cpr, ch = rem - m * cpr;
-        int4 v = reinterpret_cast<const int4 *>(stage + (size_t)m * row_bytes)[ch];
-        uint8_t *local = full + (size_t)m * full_row_bytes + col_off + ch * 16;
-        *reinterpret_cast<int4 *>(cl.map_shared_rank(local, dst)) = v;
+        const int4 v = reinterpret_cast<const int4 *>(stage + (size_t)m * row_bytes)[ch];
+        const uint32_t local = dc_smem_u32(full + (size_t)m * full_row_bytes + col_off + ch * 16);
+        dc_st_async4(dc_mapa(local, dst), v, dc_mapa(xbar, dst));
     }
 }
 
@@ -391,6 +417,18 @@ __device__ __noinline__ void dc_commit_greedy(const DcParams &P, int tp, const i
 
 enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
 
+// bytes a CTA receives in the exchange of phase ph: the full int8 vector
+// (qkv, q2, h) or the fp32 residual plus every slice's [R] max / min pair
+MNMT_DEV uint32_t dc_xbytes(const DcParams &P, int ph) {
+    const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
+    switch (kind) {
+        case K_QKV: return (uint32_t)(P.R * 3 * P.d);
+        case K_Q2: return (uint32_t)(P.R * P.d);
+        case K_W1: return (uint32_t)(P.R * P.F);
+        default: return (uint32_t)(P.R * P.d * 4 + P.R * P.nc * 8);
+    }
+}
+
 // W4: the model's attention / FFN linears hold 4-bit codes (a separate
 // instantiation, so the int8 step carries no 4-bit code)
 template <int DH, bool W4>
@@ -410,15 +448,22 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const int n16 = (int)(sizeof(DcParams) / 16);
         for (int i = threadIdx.x; i < n16; i += DC_THREADS)
             reinterpret_cast<int4 *>(smem)[i] = reinterpret_cast<const int4 *>(Pp)[i];
-        if (threadIdx.x == 0) {  // the weight ring's mbarriers, one arrival per phase
+        if (threadIdx.x == 0) {
+            // the weight ring's mbarriers and the two exchange barriers, one
+            // arrival per phase each; the exchange barriers of phases 0 and 1
+            // are armed with the bytes they receive
             const uint32_t b0 = dc_smem_u32(smem + Pp->off_bar);
-            for (int i = 0; i < DC_NB; i++) mbar_init(b0 + 8u * (uint32_t)i, 1u);
+            for (int i = 0; i < DC_NB + 2; i++) mbar_init(b0 + 8u * (uint32_t)i, 1u);
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+            for (int i = 0; i < 2; i++) mbar_expect_tx(b0 + 8u * (uint32_t)(DC_NB + i), dc_xbytes(*Pp, i));
         }
         __syncthreads();
+        // the barriers are set before any CTA of the cluster may store into
+        // this one (each waits for every arrival before its first exchange)
+        asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
     }
     const DcParams &P = *reinterpret_cast<const DcParams *>(smem);
-    const uint32_t bars = dc_smem_u32(smem + P.off_bar);
+    const uint32_t bars = dc_smem_u32(smem + P.off_bar), xbars = bars + 8u * DC_NB;
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
     const int nc = P.nc;
@@ -527,6 +572,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     dc_prefetch(P, 1, c, ring, bars);
     dc_prefetch(P, 2, c, ring, bars);
     DC_STAMP(stamp, 3);
+    asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
 
     for (int ph = 0; ph < nphase; ph++) {
         const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
@@ -704,6 +750,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         // thread issuing bulk copies is held for a few hundred ns)
         dc_prefetch(P, ph + DC_NB, c, ring, bars, DC_THREADS - 32);
         // ---- publish the slice to every CTA ----
+        const uint32_t xbar = xbars + 8u * (uint32_t)(ph & 1);
         if (out_f32) {
             // the slice's largest and smallest residual value per row (rows <= 32),
             // for the next LayerNorm's grids
@@ -717,19 +764,18 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 }
                 const unsigned kh = __reduce_max_sync(0xFFFFFFFFu, kmax);
                 const unsigned kl = __reduce_min_sync(0xFFFFFFFFu, kmin);
-                if (ln < nc) {
-                    unsigned *dst = cl.map_shared_rank(mm + (m * nc + c) * 2, ln);
-                    dst[0] = kh;
-                    dst[1] = kl;
-                }
+                if (ln < nc)
+                    dc_st_async2(dc_mapa(dc_smem_u32(mm + (m * nc + c) * 2), ln), kh, kl, dc_mapa(xbar, ln));
             }
-            dc_bcast(cl, stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc);
+            dc_bcast(stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc, xbar);
         } else {
             int8_t *full = kind == K_QKV ? qkv_full : (kind == K_Q2 ? q2_full : h_full);
             const int width = kind == K_QKV ? 3 * d : (kind == K_Q2 ? d : F);
-            dc_bcast(cl, stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc);
+            dc_bcast(stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc, xbar);
         }
-        cl.sync();
+        // the whole vector of this phase, from every CTA
+        if (!mbar_wait(xbar, (uint32_t)(ph >> 1) & 1u)) set_status(P.status, MNMT_ETIMEOUT);
+        if (threadIdx.x == 0 && ph + 2 < nphase) mbar_expect_tx(xbar, dc_xbytes(P, ph + 2));
         DC_STAMP(stamp, 7 + 4 * ph);
         if (kind == K_W2 && !P.pre_ln) {
             // post-LN: the FFN's LayerNorm normalises the stream in place
@@ -752,8 +798,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
     DC_STAMP(stamp, 101);
     if (pend && c == 0 && threadIdx.x == 0) dc_commit_greedy(P, t - 1, s_out, s_fin, 0);
-    // every CTA must still hold its shared memory while others may write to it
-    cl.sync();
+    // no closing cluster barrier: the last exchange has delivered everything
+    // any CTA stores into this one
     DC_STAMP(stamp, 102);
 }
 
@@ -926,7 +972,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens
     P.off_part = take(512 + 1024 + 64);  // slice extremes [R][nc][2], LN partials [2][64], per-row (mu, eb)
     if (R * d > 64 * 32) return (size_t)-1;                         // 64 warp chunks of partials
-    P.off_bar = take(8 * DC_NB);
+    P.off_bar = take(8 * (DC_NB + 2));  // weight ring, then the two exchange barriers
     int slot = 0;
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const DcPhase &f = P.phase[ph];

@@ -50,7 +50,7 @@ def main(argv):
     print(f"{name}: S_pad {ids.shape[1]}, decode step 20 (ns from the step kernel's start)")
     print(f"previous vocabulary kernel: start {ns[110] - t0}, wait ends {ns[112] - t0}, ends {ns[113] - t0}")
     print(f"step kernel: grid wait {ns[1] - t0}..{ns[2] - t0}, phase loop starts {ns[3] - t0}")
-    print("| phase | kind | ring wait | prep | slice GEMV | broadcast + barrier |")
+    print("| phase | kind | ring wait | prep | slice GEMV | exchange |")
     print("|---:|---|---:|---:|---:|---:|")
     prev = ns[3]
     tot = np.zeros(4, np.int64)
