@@ -487,10 +487,10 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     long long *part_l = reinterpret_cast<long long *>(smem + P.off_part + 512);    // [2][64] LN partials, [R] (mu, eb)
     const int nphase = 1 + 6 * P.n_dec;
 
-    // group 0: LayerNorm vectors of every layer (+ the final LN) and the first weight slice
+    // the LayerNorm vectors of every layer (+ the final LN), the first DC_NB
+    // weight slices and the cross keys / values the step attends to
     dc_copy(lnp, P.ln_all, (6 * P.n_dec + 2) * d * 4);
-    dc_prefetch(P, 0, c, ring, bars);
-    // group 1: the second weight slice and the keys / values the step attends to
+    for (int i = 0; i < DC_NB; i++) dc_prefetch(P, i, c, ring, bars);
     if (P.kv_staged) {
         // one layer's cross K (or V) is one contiguous [R][H][S][dh] block: the
         // 2 * n_dec blocks go in one flat loop of 16-byte chunks
@@ -506,12 +506,21 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     const unsigned long long ns_w0 = dc_gtime();
 #endif
     dc_grid_wait();
-    if (*P.done) {  // uniform for the whole cluster; no copy may outlive the CTA
+    // every word of the decode state this step reads, in one round of loads
+    const int done_v = *P.done, t_v = *P.t_ptr, pend_v = *P.pending, tmax_v = *P.tmax_ptr;
+    unsigned long long key_v = 0ull;
+    int fin_v = 0, tok_v = 0;
+    if (threadIdx.x < R) {
+        key_v = P.keys[threadIdx.x];
+        fin_v = P.fin[threadIdx.x];
+        tok_v = P.tok[threadIdx.x];
+    }
+    if (done_v) {  // uniform for the whole cluster; no copy may outlive the CTA
         asm volatile("cp.async.wait_all;\n" ::);
-        dc_wait_slice(P, 0, bars);
+        for (int i = 0; i < DC_NB; i++) dc_wait_slice(P, i, bars);
         return;
     }
-    int t = *P.t_ptr;
+    int t = t_v;
     // The previous step's vocabulary kernel left its greedy selection pending
     // (row maxima in keys): apply it here -- every CTA computes the same
     // tokens and finished flags from the same data; CTA 0 commits them (token,
@@ -520,21 +529,20 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     static_assert(3 * DC_RMAX <= 16, "tokens, pending tokens and flags share the 16-int token area");
     int *s_out = tok_s + DC_RMAX, *s_fin = tok_s + 2 * DC_RMAX;  // no static shared memory: the
                                                                  // dynamic carve-up may take all 227 KB
-    const bool pend = *P.pending != 0;
+    const bool pend = pend_v != 0;
     if (pend) {
         if (threadIdx.x < R) {
-            const int y = (int)key_index(P.keys[threadIdx.x]);
-            const int f = P.fin[threadIdx.x];
-            s_out[threadIdx.x] = f ? P.pad : y;
-            s_fin[threadIdx.x] = (f || y == P.eos) ? 1 : 0;
+            const int y = (int)key_index(key_v);
+            s_out[threadIdx.x] = fin_v ? P.pad : y;
+            s_fin[threadIdx.x] = (fin_v || y == P.eos) ? 1 : 0;
         }
         __syncthreads();
         int all = 1;
         for (int m = 0; m < R; m++) all &= s_fin[m];
-        if (all || t + 1 >= *P.tmax_ptr) {  // uniform over the cluster
+        if (all || t + 1 >= tmax_v) {  // uniform over the cluster
             if (c == 0 && threadIdx.x == 0) dc_commit_greedy(P, t, s_out, s_fin, 1);
             asm volatile("cp.async.wait_all;\n" ::);
-            dc_wait_slice(P, 0, bars);
+            for (int i = 0; i < DC_NB; i++) dc_wait_slice(P, i, bars);
             return;
         }
         t = t + 1;
@@ -549,7 +557,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
 #endif
     if (threadIdx.x < R) {
-        int id = pend ? s_out[threadIdx.x] : P.tok[threadIdx.x];
+        int id = pend ? s_out[threadIdx.x] : tok_v;
         if (id < 0 || id >= P.V) {
             set_status(P.status, MNMT_EINVAL);
             id = 0;
@@ -569,8 +577,6 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                     (lkv & 1 ? Y.self_v : Y.self_k) + (size_t)mh * P.T * (d / H) + (size_t)ch * 16);
         }
     }
-    dc_prefetch(P, 1, c, ring, bars);
-    dc_prefetch(P, 2, c, ring, bars);
     DC_STAMP(stamp, 3);
     asm volatile("barrier.cluster.wait.acquire;\n" ::: "memory");
 
@@ -838,6 +844,11 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
     const unsigned long long v_w0 = dc_gtime();
 #endif
     dc_grid_wait();
+    // the done flag and the first chunk of input rows in one round of loads
+    const int done_v = *g.done;
+    int4 a0 = make_int4(0, 0, 0, 0);
+    if ((int)threadIdx.x < MT * kc && (int)threadIdx.x / kc < M)
+        a0 = reinterpret_cast<const int4 *>(A + (size_t)(threadIdx.x / kc) * K)[threadIdx.x % kc];
 #ifdef MNMT_DC_STAMPS
     if (blockIdx.x == 0 && threadIdx.x == 0 && *g.t_ptr == DC_STAMP_STEP - 1) {
         g_dc_ns[110] = v_start;
@@ -845,11 +856,12 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
         g_dc_ns[112] = dc_gtime();
     }
 #endif
-    if (*g.done) {  // no copy may outlive the block
+    if (done_v) {  // no copy may outlive the block
         asm volatile("cp.async.wait_all;\n" ::);
         return;
     }
-    for (int i = threadIdx.x; i < MT * kc; i += 256) {
+    if ((int)threadIdx.x < MT * kc) as[threadIdx.x] = a0;
+    for (int i = threadIdx.x + 256; i < MT * kc; i += 256) {
         const int m = i / kc, c = i - m * kc;
         as[i] = m < M ? reinterpret_cast<const int4 *>(A + (size_t)m * K)[c] : make_int4(0, 0, 0, 0);
     }
