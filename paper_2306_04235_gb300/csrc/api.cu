@@ -1144,7 +1144,7 @@ int setup_cluster_step(mnmt_session *s) {
     P.emb_q = m->emb_q; P.emb_s = m->emb_s;
     if (m->factorised) P.proj = DcLin{m->proj.w, m->proj.s, m->proj.b, nullptr, 8};
     P.emb_scale = m->emb_scale; P.pe = m->pe;
-    P.fin_g = m->dec_final.g; P.fin_b = m->dec_final.b; P.s_dout = m->s_dout;
+    P.fin_g = m->dec_final.g; P.fin_b = m->dec_final.b; P.s_dout = m->s_dout; P.inv_dout = 1.0f / m->s_dout;
     P.tok = s->tok; P.t_ptr = s->state + ST_T; P.done = s->state + ST_DONE; P.src_len = s->src_lens;
     P.keys = s->keys; P.tok_w = s->tok; P.fin = s->fin; P.hist = s->hist; P.t_w = s->state + ST_T;
     P.done_w = s->state + ST_DONE; P.pending = s->state + ST_PENDING; P.tmax_ptr = s->state + ST_TMAX;
@@ -1159,6 +1159,7 @@ int setup_cluster_step(mnmt_session *s) {
         Y.s_in1 = A.s_in; Y.s_ctx1 = A.s_ctx; Y.gamma1 = A.gamma; Y.sigma1 = A.sigma; Y.rho1 = A.rho;
         Y.s_in2 = X.s_in; Y.s_ctx2 = X.s_ctx; Y.gamma2 = X.gamma; Y.sigma2 = X.sigma; Y.rho2 = X.rho;
         Y.s_in3 = Fb.s_in; Y.s_h = Fb.s_h; Y.gamma3 = Fb.gamma;
+        Y.inv_in1 = 1.0f / A.s_in; Y.inv_in2 = 1.0f / X.s_in; Y.inv_in3 = 1.0f / Fb.s_in;
         // 4-bit linears stream their packed codes (half the ring bytes)
         auto dl = [](const Lin &x) {
             if (x.bits == 4) return DcLin{reinterpret_cast<const int8_t *>(x.wp), x.s, x.b, x.m, 4};

@@ -109,6 +109,19 @@ MNMT_DEV void dc_copy(void *dst, const void *src, int bytes) {
         dc_cp16(static_cast<uint8_t *>(dst) + i * 16, static_cast<const uint8_t *>(src) + i * 16);
 }
 
+// Index arithmetic of the step avoids integer division by run-time values
+// (a multi-instruction sequence on the critical path of every phase):
+// quotients come from multiply-high by a host-computed ceil(2^32 / d) (exact
+// for i, d < 2^16; mg == 0 stands for d == 1), from shifts by powers of two,
+// or from a few compares when the quotient is a row index below DC_RMAX.
+MNMT_DEV int dc_udiv(int i, uint32_t mg) { return mg ? (int)__umulhi((uint32_t)i, mg) : i; }
+MNMT_DEV int dc_row_of(int i, int d, int R) {  // i / d for i < R d, R <= DC_RMAX
+    int r = 0;
+#pragma unroll
+    for (int k = 1; k < DC_RMAX; k++) r += (k < R && i >= k * d) ? 1 : 0;
+    return r;
+}
+
 // ring slot layout: W rows (rows * K bytes), then s[rows], b[rows], inv[rows] (fp32)
 // Phase ph's slice goes to slot ph % DC_NB as up to five 1-D bulk copies (the
 // copy engine moves them: no per-thread copy instructions queue ahead of the
@@ -170,13 +183,13 @@ MNMT_DEV void dc_st_async2(uint32_t remote, unsigned x, unsigned y, uint32_t rem
 
 // copy stage [R][row_bytes] into every CTA's full buffer at column offset,
 // completing on each receiver's exchange barrier xbar (local address)
-__device__ __noinline__ void dc_bcast(const uint8_t *stage, int R, int row_bytes, uint8_t *full, int full_row_bytes,
-                                      int col_off, int nc, uint32_t xbar) {
-    const int cpr = row_bytes / 16;
+__device__ __noinline__ void dc_bcast(const DcPhase &f, const uint8_t *stage, int R, int row_bytes, uint8_t *full,
+                                      int full_row_bytes, int col_off, int nc, uint32_t xbar) {
+    const int cpr = f.cpr;  // row_bytes / 16
     const int total = nc * R * cpr;
     for (int i = threadIdx.x; i < total; i += DC_THREADS) {
-        const int dst = i / (R * cpr), rem = i - dst * R * cpr;
-        const int m = rem / cpr, ch = rem - m * cpr;
+        const int dst = dc_udiv(i, f.mg_rc), rem = i - dst * R * cpr;
+        const int m = dc_udiv(rem, f.mg_c), ch = rem - m * cpr;
         const int4 v = reinterpret_cast<const int4 *>(stage + (size_t)m * row_bytes)[ch];
         const uint32_t local = dc_smem_u32(full + (size_t)m * full_row_bytes + col_off + ch * 16);
         dc_st_async4(dc_mapa(local, dst), v, dc_mapa(xbar, dst));
@@ -222,7 +235,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
         float hi, lo;
-        dc_row_extremes(mm, e0 / d, nc, hi, lo);
+        dc_row_extremes(mm, dc_row_of(e0, d, R), nc, hi, lo);
         const float am = fmaxf(fabsf(hi), fabsf(lo));
         if (!(am < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
         const long long s = warp_sum_exact(fx_scale(r[e0 + lane], 52 - exp_bound(am)));
@@ -232,7 +245,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     // pass 2: exact sum of c^2 = fl(x - mean)^2 on the grid of max |c|
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
-        const int row = e0 / d;
+        const int row = dc_row_of(e0, d, R);
         float hi, lo;
         dc_row_extremes(mm, row, nc, hi, lo);
         const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
@@ -241,7 +254,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
         const float cv = __fsub_rn(r[e0 + lane], mu);
         const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
         if (lane == 0) part_l[64 + e0 / 32] = s;
-        if (lane == 0 && (e0 % d) == 0) {
+        if (lane == 0 && e0 == row * d) {
             reinterpret_cast<float *>(part_l + 128)[2 * row] = mu;  // per row: mu, 2^eb grid
             reinterpret_cast<int *>(part_l + 128)[2 * row + 1] = eb;
         }
@@ -250,7 +263,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     // pass 3: normalise, scale, shift, quantise
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
-        const int row = e0 / d, e = e0 + lane, i = e - row * d;
+        const int row = dc_row_of(e0, d, R), e = e0 + lane, i = e - row * d;
         const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
         const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
         const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd);
@@ -279,12 +292,13 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
     const float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
     const int items = R * H;
     const int ip = items >= DC_WARPS ? DC_WARPS : (items > 4 ? 8 : (items > 2 ? 4 : (items > 1 ? 2 : 1)));
-    const int wpi = DC_WARPS / ip;  // warps per item in a round of ip items
+    const int wpi = DC_WARPS / ip;  // warps per item in a round of ip items (a power of two)
+    const int lw = __ffs(wpi) - 1;
     constexpr int QC = DH / 16;
     for (int base = 0; base < items; base += ip) {
-        const int it = base + warp / wpi, part = warp % wpi;
+        const int it = base + (warp >> lw), part = warp & (wpi - 1);
         const bool live = it < items;
-        const int m = live ? it / H : 0, h = live ? it - m * H : 0;
+        const int m = live ? dc_row_of(it, H, R) : 0, h = live ? it - m * H : 0;
         int n;
         const int8_t *kb, *vb;
         if (cross) {
@@ -309,9 +323,9 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                 vb = Y.self_v + ((size_t)m * H + h) * T * DH;
             }
         }
-        const int per = (n + wpi - 1) / wpi;
+        const int per = (n + wpi - 1) >> lw;
         const int j0 = part * per, j1 = min(n, j0 + per);
-        int *sc = att + (warp / wpi) * P.att_cap;
+        int *sc = att + (warp >> lw) * P.att_cap;
         float mx = -INFINITY;
         if (live) {
             int4 qv[QC];
@@ -333,7 +347,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
         if (lane == 0) red_f[warp] = mx;
         __syncthreads();
         mx = -INFINITY;
-        for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp / wpi) * wpi + w]);
+        for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp >> lw) * wpi + w]);
         int zl = 0;
         if (live)
             for (int j = j0 + lane; j < j1; j += 32) {
@@ -389,7 +403,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                     N += pn[(ii * wpi + w) * DH + e];
                     Z += pz[ii * wpi + w];
                 }
-                const int m2 = it2 / H, h2 = it2 - m2 * H;
+                const int m2 = dc_row_of(it2, H, R), h2 = it2 - m2 * H;
                 ctx[(size_t)m2 * P.d + h2 * DH + e] = q8_quotient(N, Z, rho, dc_rn32_div);
             }
         }
@@ -495,10 +509,11 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         // one layer's cross K (or V) is one contiguous [R][H][S][dh] block: the
         // 2 * n_dec blocks go in one flat loop of 16-byte chunks
         const int cpb = R * P.S * d / 16;
-        for (int i = threadIdx.x; i < 2 * P.n_dec * cpb; i += DC_THREADS) {
-            const int blk = i / cpb, ch = i - blk * cpb;
+        for (int blk = 0; blk < 2 * P.n_dec; blk++) {
             const DcLayer &Y = P.layer[blk >> 1];
-            dc_cp16(smem + P.off_kvc + (size_t)i * 16, (blk & 1 ? Y.cross_v : Y.cross_k) + (size_t)ch * 16);
+            const int8_t *src = blk & 1 ? Y.cross_v : Y.cross_k;
+            uint8_t *dst = smem + P.off_kvc + (size_t)blk * cpb * 16;
+            for (int ch = threadIdx.x; ch < cpb; ch += DC_THREADS) dc_cp16(dst + (size_t)ch * 16, src + (size_t)ch * 16);
         }
     }
     // ---- the previous step's results: token, position, self keys / values ----
@@ -566,15 +581,17 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
     if (P.kv_staged && t > 0) {
         // positions 0..t-1 of every (layer, K/V, row, head): segments of t * dh
-        // bytes, [T][dh] apart in the cache, in one flat loop of 16-byte chunks
-        const int cps = t * (d / H) / 16, nseg = 2 * P.n_dec * R * H;
-        for (int i = threadIdx.x; i < nseg * cps; i += DC_THREADS) {
-            const int sg = i / cps, ch = i - sg * cps;
-            const int lkv = sg / (R * H), mh = sg - lkv * R * H;
+        // bytes, [T][dh] apart in the cache, one warp per segment
+        const int cps = t * (DH / 16), RH = R * H;
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        for (int lkv = 0; lkv < 2 * P.n_dec; lkv++) {
             const DcLayer &Y = P.layer[lkv >> 1];
-            const size_t off = ((size_t)lkv * R * H + mh) * P.T * (d / H);
-            dc_cp16(smem + P.off_kvs + off + (size_t)ch * 16,
-                    (lkv & 1 ? Y.self_v : Y.self_k) + (size_t)mh * P.T * (d / H) + (size_t)ch * 16);
+            const int8_t *src0 = lkv & 1 ? Y.self_v : Y.self_k;
+            for (int mh = warp; mh < RH; mh += DC_WARPS) {
+                uint8_t *dst = smem + P.off_kvs + ((size_t)lkv * RH + mh) * P.T * DH;
+                const int8_t *src = src0 + (size_t)mh * P.T * DH;
+                for (int ch = lane; ch < cps; ch += 32) dc_cp16(dst + (size_t)ch * 16, src + (size_t)ch * 16);
+            }
         }
     }
     DC_STAMP(stamp, 3);
@@ -603,19 +620,20 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         if (kind == K_EMB) {
             if (P.factorised)
                 for (int i = threadIdx.x; i < R * P.E; i += DC_THREADS)
-                    a_full[i] = P.emb_q[(size_t)tok_s[i / P.E] * P.E + (i % P.E)];
+                for (int m = 0; m < R; m++)
+                    if (i >= m * P.E && i < (m + 1) * P.E) a_full[i] = P.emb_q[(size_t)tok_s[m] * P.E + (i - m * P.E)];
             K = P.E;
         } else if (kind == K_QKV || kind == K_Q2 || kind == K_W1) {
             // pre-LN: LN of this sublayer; post-LN: LN of the previous sublayer's
             // residual (written back), or plain quantisation for the first one
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
-            const float s_in = kind == K_QKV ? Y.s_in1 : (kind == K_Q2 ? Y.s_in2 : Y.s_in3);
+            const float inv_in = kind == K_QKV ? Y.inv_in1 : (kind == K_Q2 ? Y.inv_in2 : Y.inv_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, 1.0f / s_in, a_full, 0, P.status, mm, nc, part_l);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l);
             } else if (kind == K_QKV) {
-                for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], 1.0f / s_in);
+                for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], inv_in);
             } else {
-                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, 1.0f / s_in, a_full, 1, P.status, mm, nc,
+                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, inv_in, a_full, 1, P.status, mm, nc,
                              part_l);
             }
         } else if (kind == K_O || kind == K_O2) {
@@ -631,7 +649,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         DC_STAMP(stamp, 5 + 4 * ph);
 
         // ---- the phase's slice of outputs ----
-        const int rows = ph == 0 ? d / nc : P.phase[ph].rows;
+        const int rows = ph == 0 ? P.phase[0].cpr * 4 : P.phase[ph].rows;  // phase 0: d / nc fp32 values
         const int n0 = c * rows;
         int out_f32;
         float sx, gam;
@@ -648,7 +666,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
         if (kind == K_EMB && !P.factorised) {
             for (int i = threadIdx.x; i < R * rows; i += DC_THREADS) {
-                const int m = i / rows, nl = i - m * rows, n = n0 + nl, id = tok_s[m];
+                const int m = dc_row_of(i, rows, R), nl = i - m * rows, n = n0 + nl, id = tok_s[m];
                 const float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
                 stf[i] = __fadd_rn(v, P.pe[(size_t)t * d + n]);
             }
@@ -671,13 +689,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             int lpr = kc & -kc;
             if (lpr > 32) lpr = 32;
             while (lpr > 1 && rows * lpr > DC_THREADS) lpr >>= 1;
-            const int cpl = kc / lpr;
-            const int rpw = 32 / lpr;              // rows per warp pass
+            const int lg = __ffs(lpr) - 1;         // lpr = 2^lg
+            const int cpl = kc >> lg;
+            const int rpw = 32 >> lg;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-            const int sub = lane % lpr;
+            const int sub = lane & (lpr - 1);
             const int4 ones = make_int4(0x01010101, 0x01010101, 0x01010101, 0x01010101);
             for (int r0 = warp * rpw; r0 < rows; r0 += DC_WARPS * rpw) {
-                const int nl = r0 + lane / lpr;
+                const int nl = r0 + (lane >> lg);
                 int acc[DC_RMAX] = {0, 0, 0, 0};
                 int a1[DC_RMAX] = {0, 0, 0, 0};  // 4-bit rows: the activation codes' sums
                 if (nl < rows) {
@@ -773,11 +792,11 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 if (ln < nc)
                     dc_st_async2(dc_mapa(dc_smem_u32(mm + (m * nc + c) * 2), ln), kh, kl, dc_mapa(xbar, ln));
             }
-            dc_bcast(stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc, xbar);
+            dc_bcast(P.phase[ph], stage, R, rows * 4, reinterpret_cast<uint8_t *>(r_full), d * 4, n0 * 4, nc, xbar);
         } else {
             int8_t *full = kind == K_QKV ? qkv_full : (kind == K_Q2 ? q2_full : h_full);
             const int width = kind == K_QKV ? 3 * d : (kind == K_Q2 ? d : F);
-            dc_bcast(stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc, xbar);
+            dc_bcast(P.phase[ph], stage, R, rows, reinterpret_cast<uint8_t *>(full), width, n0, nc, xbar);
         }
         // the whole vector of this phase, from every CTA
         if (!mbar_wait(xbar, (uint32_t)(ph >> 1) & 1u)) set_status(P.status, MNMT_ETIMEOUT);
@@ -786,7 +805,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         if (kind == K_W2 && !P.pre_ln) {
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
-            const float inv = last ? 1.0f / P.s_dout : 1.0f / P.layer[l + 1].s_in1;
+            const float inv = last ? P.inv_dout : P.layer[l + 1].inv_in1;
             dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l);
         }
     }
@@ -794,7 +813,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     1.0f / P.s_dout, a_full, 0, P.status, mm, nc, part_l);
+                     P.inv_dout, a_full, 0, P.status, mm, nc, part_l);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -843,12 +862,14 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
 #ifdef MNMT_DC_STAMPS
     const unsigned long long v_w0 = dc_gtime();
 #endif
+    const int am = dc_row_of((int)threadIdx.x, kc, MT <= DC_RMAX ? MT : DC_RMAX);  // row of this thread's input chunk
+    const bool aload = (int)threadIdx.x < MT * kc && am < M;
+    const int4 *asrc = reinterpret_cast<const int4 *>(A + (size_t)am * K) + ((int)threadIdx.x - am * kc);
     dc_grid_wait();
     // the done flag and the first chunk of input rows in one round of loads
     const int done_v = *g.done;
     int4 a0 = make_int4(0, 0, 0, 0);
-    if ((int)threadIdx.x < MT * kc && (int)threadIdx.x / kc < M)
-        a0 = reinterpret_cast<const int4 *>(A + (size_t)(threadIdx.x / kc) * K)[threadIdx.x % kc];
+    if (aload) a0 = *asrc;
 #ifdef MNMT_DC_STAMPS
     if (blockIdx.x == 0 && threadIdx.x == 0 && *g.t_ptr == DC_STAMP_STEP - 1) {
         g_dc_ns[110] = v_start;
@@ -870,8 +891,9 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int lpr = kc & -kc;  // lanes per weight row: the largest power of two dividing kc, at most 32
     if (lpr > 32) lpr = 32;
-    const int rpw = 32 / lpr;            // rows per warp and pass
-    const int grp = lane / lpr, sl = lane % lpr;
+    const int lg = __ffs(lpr) - 1;       // lpr = 2^lg
+    const int rpw = 32 >> lg;            // rows per warp and pass
+    const int grp = lane >> lg, sl = lane & (lpr - 1);
     unsigned long long best[MT];
 #pragma unroll
     for (int m = 0; m < MT; m++) best[m] = 0ull;
@@ -959,6 +981,18 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
         f[3] = ph(Y.o2, nullptr, d / nc, d);
         f[4] = ph(Y.w1, Y.inv_h, F / nc, d);
         f[5] = ph(Y.w2, nullptr, d / nc, F);
+    }
+    // exchange geometry: slices of fp32 residual values (embedding, O, O2, W2)
+    // or int8 codes (qkv, q2, h)
+    auto magic = [](int v) { return v > 1 ? (uint32_t)((0x100000000ull + (uint64_t)v - 1) / (uint64_t)v) : 0u; };
+    for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
+        const int kind = ph == 0 ? -1 : (ph - 1) % 6;
+        const bool f32 = kind == -1 || kind == 1 || kind == 3 || kind == 5;
+        const int rows = ph == 0 ? d / nc : P.phase[ph].rows;
+        const int cpr = f32 ? rows / 4 : rows / 16;
+        P.phase[ph].cpr = cpr;
+        P.phase[ph].mg_rc = magic(R * cpr);
+        P.phase[ph].mg_c = magic(cpr);
     }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;

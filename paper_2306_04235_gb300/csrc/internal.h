@@ -236,6 +236,7 @@ struct DcLayer {
     float s_in1, s_ctx1, gamma1, sigma1, rho1;
     float s_in2, s_ctx2, gamma2, sigma2, rho2;
     float s_in3, s_h, gamma3;
+    float inv_in1, inv_in2, inv_in3;  // fl(1 / s_in) of the three sublayer inputs
     DcLin qkv, o, q2, o2, w1, w2;
     const float *inv_qkv, *inv_q2, *inv_h;
     int8_t *self_k, *self_v;          // [R][H][T][dh]
@@ -249,6 +250,11 @@ struct DcPhase {
     const float *s, *b, *inv;    // inv: per-column requantisation constants (or null)
     const float *m;              // 4-bit min-max rows: row offsets (else null)
     int rows, K, bits;
+    // the exchange of the phase's output: 16-byte chunks per row of a slice
+    // (cpr) and ceil(2^32 / d) multipliers for d = R * cpr and d = cpr
+    // (quotients of chunk indices below 2^16 by one multiply-high)
+    int cpr;
+    uint32_t mg_rc, mg_c;
 };
 struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
@@ -259,7 +265,7 @@ struct alignas(16) DcParams {
     const float *pe;
     const float *fin_g, *fin_b;
     const float *ln_all;  // every LayerNorm vector of the step, contiguous: [n_dec][6][d] then final [2][d]
-    float s_dout;
+    float s_dout, inv_dout;  // inv_dout = fl(1 / s_dout)
     const int32_t *tok;
     const int *t_ptr, *done;
     // the previous step's greedy selection, applied by this step (CTA 0 writes)
