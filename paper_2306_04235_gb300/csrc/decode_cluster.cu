@@ -285,7 +285,7 @@ template <int DH>
 __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
                                           const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx,
                                           int *att, float *red_f, long long *pz, long long *pn,
-                                          const uint8_t *smem) {
+                                          const uint8_t *smem, const int *src_len_s) {
     const DcLayer &Y = P.layer[l];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int H = P.H, T = P.T, S = P.S, R = P.R;
@@ -302,7 +302,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
         int n;
         const int8_t *kb, *vb;
         if (cross) {
-            n = P.src_len[m];
+            n = src_len_s[m];
             n = n < 1 ? 1 : (n > S ? S : n);
             if (P.kv_staged) {
                 const int8_t *cb = reinterpret_cast<const int8_t *>(smem + P.off_kvc);
@@ -357,41 +357,37 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
             }
         const long long z = warp_sum_exact(zl);
         __syncwarp();
-        // context: lane l owns elements [l * EPL, (l + 1) * EPL) of the head and
-        // walks the warp's keys (consecutive lanes read consecutive bytes)
-        constexpr int EPL = DH / 32;
-        int hi[EPL], lo[EPL];
-#pragma unroll
-        for (int u = 0; u < EPL; u++) hi[u] = lo[u] = 0;
+        // context: the warp's keys KPI at a time, LPK lanes per key and 4
+        // consecutive elements of the head per lane; the key groups' exact
+        // integer partial sums meet by shuffles
+        constexpr int LPK = DH / 4, KPI = 32 / LPK;
+        const int kg = lane / LPK, el = (lane % LPK) * 4;
+        int hi[4] = {0, 0, 0, 0}, lo[4] = {0, 0, 0, 0};
         if (live) {
 #pragma unroll 2
-            for (int j = j0; j < j1; j++) {
+            for (int j = j0 + kg; j < j1; j += KPI) {
                 const int E = sc[j];
                 const int Eh = E >> 12, El = E & 4095;
                 const int8_t *vr = (!cross && j == t) ? vnew + (size_t)m * kv_ld + h * DH : vb + (size_t)j * DH;
-                int v[EPL];
-                if constexpr (EPL == 1) {
-                    v[0] = vr[lane];
-                } else if constexpr (EPL == 2) {
-                    const char2 x2 = reinterpret_cast<const char2 *>(vr)[lane];
-                    v[0] = x2.x;
-                    v[1] = x2.y;
-                } else {
-                    const char4 x4 = reinterpret_cast<const char4 *>(vr)[lane];
-                    v[0] = x4.x;
-                    v[1] = x4.y;
-                    v[2] = x4.z;
-                    v[3] = x4.w;
-                }
+                const char4 x4 = *reinterpret_cast<const char4 *>(vr + el);
+                const int v[4] = {x4.x, x4.y, x4.z, x4.w};
 #pragma unroll
-                for (int u = 0; u < EPL; u++) {
+                for (int u = 0; u < 4; u++) {
                     hi[u] += Eh * v[u];
                     lo[u] += El * v[u];
                 }
             }
         }
 #pragma unroll
-        for (int u = 0; u < EPL; u++) pn[warp * DH + lane * EPL + u] = (long long)hi[u] * 4096 + lo[u];
+        for (int o = LPK; o < 32; o <<= 1)
+#pragma unroll
+            for (int u = 0; u < 4; u++) {
+                hi[u] += __shfl_xor_sync(0xFFFFFFFFu, hi[u], o);
+                lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
+            }
+        if (kg == 0)
+#pragma unroll
+            for (int u = 0; u < 4; u++) pn[warp * DH + el + u] = (long long)hi[u] * 4096 + lo[u];
         if (lane == 0) pz[warp] = z;
         __syncthreads();
         for (int x = threadIdx.x; x < ip * DH; x += DC_THREADS) {
@@ -524,11 +520,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     // every word of the decode state this step reads, in one round of loads
     const int done_v = *P.done, t_v = *P.t_ptr, pend_v = *P.pending, tmax_v = *P.tmax_ptr;
     unsigned long long key_v = 0ull;
-    int fin_v = 0, tok_v = 0;
+    int fin_v = 0, tok_v = 0, srcl_v = 0;
     if (threadIdx.x < R) {
         key_v = P.keys[threadIdx.x];
         fin_v = P.fin[threadIdx.x];
         tok_v = P.tok[threadIdx.x];
+        srcl_v = P.src_len[threadIdx.x];
     }
     if (done_v) {  // uniform for the whole cluster; no copy may outlive the CTA
         asm volatile("cp.async.wait_all;\n" ::);
@@ -541,9 +538,11 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     // tokens and finished flags from the same data; CTA 0 commits them (token,
     // history, flags, step counter, cleared keys) at the end of this step, or
     // at once if the translation has just finished.
-    static_assert(3 * DC_RMAX <= 16, "tokens, pending tokens and flags share the 16-int token area");
+    static_assert(4 * DC_RMAX <= 16, "tokens, pending tokens, flags and source lengths share the 16-int token area");
     int *s_out = tok_s + DC_RMAX, *s_fin = tok_s + 2 * DC_RMAX;  // no static shared memory: the
                                                                  // dynamic carve-up may take all 227 KB
+    int *src_len_s = tok_s + 3 * DC_RMAX;
+    if (threadIdx.x < R) src_len_s[threadIdx.x] = srcl_v;  // read from phase 0 on (after its block barrier)
     const bool pend = pend_v != 0;
     if (pend) {
         if (threadIdx.x < R) {
@@ -639,7 +638,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
             dc_attention<DH>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
-                             qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn, smem);
+                             qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn, smem, src_len_s);
             A = ctx_full;
         } else {  // K_W2
             A = h_full;
