@@ -9,16 +9,19 @@
 //   * every CTA holds the full activation vectors of the step in shared memory
 //     (residual stream fp32 [R][d], LN output, q/k/v, context, FFN hidden);
 //   * a linear layer is split by output columns: CTA c computes its column
-//     slice from its weight slice and writes the result into the shared
-//     memory of every CTA of the cluster (distributed shared memory), then a
-//     hardware cluster barrier publishes it;
+//     slice from its weight slice and stores it into the shared memory of
+//     every CTA of the cluster (distributed shared memory) with st.async,
+//     whose bytes complete on the receiver's exchange mbarrier: each CTA waits
+//     only until its own copy of the vector is whole;
 //   * LayerNorm and attention (all heads of the step's rows) are computed
-//     redundantly by every CTA, which removes two barriers per attention;
-//   * weight slices stream from L2/HBM into a 3-slot shared-memory ring with
-//     cp.async, two phases ahead of use; the keys and values the step attends
-//     to are staged into shared memory at kernel start when they fit.
-// The step is one compact phase loop (the instruction cache holds it) with
-// 1 + 6 * n_dec cluster barriers, no global synchronisation and no spin loop.
+//     redundantly by every CTA, which removes two exchanges per attention;
+//   * weight slices stream from L2/HBM into a 3-slot shared-memory ring by 1-D
+//     bulk copies (an mbarrier per slot), three phases ahead of use; the keys
+//     and values the step attends to are staged into shared memory at kernel
+//     start when they fit.
+// The step is one compact phase loop with one exchange per phase, a single
+// cluster barrier (every CTA's mbarriers are set before the first exchange),
+// no global synchronisation and only bounded waits.
 // The arithmetic is exactly that of the other kernels (Fig. 5 quantisation
 // points, fixed-point LayerNorm and softmax), so the step is bit-identical to
 // the multi-kernel path.
@@ -37,7 +40,7 @@ namespace cg = cooperative_groups;
 // DC_STAMP_STEP, and the vocabulary kernel of the step before records its
 // start, the end of its wait and its end.  Slots: 0 kernel start, 1 / 2
 // around the grid wait, 3 phase loop start, 4 + 4 ph .. 7 + 4 ph the phase's
-// ring wait / input prep / slice GEMV / broadcast + cluster barrier ends, 100
+// ring wait / input prep / slice GEMV / exchange ends, 100
 // / 101 / 102 final LayerNorm start / end / kernel end, 110 .. 113 vocabulary
 // kernel (block 0 start, before / after its wait, end).
 constexpr int DC_STAMP_STEP = 20;
@@ -485,7 +488,10 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     int8_t *ctx_full = reinterpret_cast<int8_t *>(smem + P.off_ctx);
     int8_t *q2_full = reinterpret_cast<int8_t *>(smem + P.off_q2);
     int8_t *h_full = reinterpret_cast<int8_t *>(smem + P.off_h);
-    uint8_t *stage = smem + P.off_stage;
+    // the slice's staging buffer alternates by phase: a thread may still be
+    // storing the previous phase's slice to other CTAs (the exchange only
+    // waits for what this CTA receives) when a faster one writes the next
+    uint8_t *const stage2 = smem + P.off_stage;
     int *att = reinterpret_cast<int *>(smem + P.off_att);
     uint8_t *ring = smem + P.off_ring;
     float *lnp = reinterpret_cast<float *>(smem + P.off_ln);                  // [n_dec][6][d] + final [2][d]
@@ -602,10 +608,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const DcLayer &Y = P.layer[l];
         // from the last phase on, the vocabulary kernel may launch and fetch its weights
         if (ph == nphase - 1) dc_launch_dependents();
-        // Each thread waits for the slice itself; the cluster barrier that ended
-        // the previous phase already orders this CTA's threads.  Phase 0 reads
-        // the tokens of the prologue, phase 1 on the LayerNorm vectors and
-        // (phase 2 on) the staged keys / values: both cross a block barrier.
+        // Each thread waits for the slice itself.  Every buffer this phase's
+        // prep writes was last read before the block barrier that follows the
+        // previous phase's GEMV; what this CTA receives is complete once the
+        // exchange wait that ended that phase returns.  Phase 0 reads the
+        // tokens of the prologue, phase 1 on the LayerNorm vectors and (phase 2
+        // on) the staged keys / values: both cross a block barrier.
         if (ph == 1) asm volatile("cp.async.wait_all;\n" ::: "memory");
         dc_wait_slice(P, ph, bars);
         if (ph <= 1) __syncthreads();
@@ -661,6 +669,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             case K_W1: out_f32 = 0; sx = Y.s_in3; gam = 0.0f; break;
             default: out_f32 = 1; sx = Y.s_h; gam = Y.gamma3; break;
         }
+        uint8_t *stage = stage2 + (ph & 1) * P.stage_bytes;
         float *stf = reinterpret_cast<float *>(stage);
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
         if (kind == K_EMB && !P.factorised) {
@@ -1011,7 +1020,8 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     int stage_bytes = R * (d / nc) * 4;
     if (R * 3 * d / nc > stage_bytes) stage_bytes = R * 3 * d / nc;
     if (R * F / nc > stage_bytes) stage_bytes = R * F / nc;
-    P.off_stage = take(stage_bytes);
+    P.stage_bytes = (stage_bytes + 15) & ~15;
+    P.off_stage = take(2 * (size_t)P.stage_bytes);  // two, alternating by phase
     P.att_cap = P.T > P.S ? P.T : P.S;
     P.off_att = take((size_t)DC_WARPS * P.att_cap * 4);
     P.off_red = take(128 + (size_t)DC_WARPS * P.dh * 8 + 16 * 4);  // reductions, context partials, tokens

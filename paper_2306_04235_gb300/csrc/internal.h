@@ -281,7 +281,8 @@ struct alignas(16) DcParams {
     // shared-memory carve-up (bytes), filled by dc_layout
     int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, off_ln, off_red, slot_bytes,
         att_cap;
-    int kv_staged, off_kvs, off_kvc;  // self / cross keys and values staged in shared memory
+    int kv_staged, off_kvs, off_kvc;
+    int stage_bytes;  // one of the two slice staging buffers  // self / cross keys and values staged in shared memory
     int off_part, off_bar;  // off_bar: mbarriers of the weight ring [DC_NB] and of the exchange [2]
     DcLayer layer[DC_LMAX];
     DcPhase phase[1 + 6 * DC_LMAX];
