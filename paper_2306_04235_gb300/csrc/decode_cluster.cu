@@ -658,17 +658,8 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         // ---- the phase's slice of outputs ----
         const int rows = ph == 0 ? P.phase[0].cpr * 4 : P.phase[ph].rows;  // phase 0: d / nc fp32 values
         const int n0 = c * rows;
-        int out_f32;
-        float sx, gam;
-        switch (kind) {
-            case K_EMB: out_f32 = 1; sx = 0.0f; gam = 0.0f; break;
-            case K_QKV: out_f32 = 0; sx = Y.s_in1; gam = 0.0f; break;
-            case K_O: out_f32 = 1; sx = Y.s_ctx1; gam = Y.gamma1; break;
-            case K_Q2: out_f32 = 0; sx = Y.s_in2; gam = 0.0f; break;
-            case K_O2: out_f32 = 1; sx = Y.s_ctx2; gam = Y.gamma2; break;
-            case K_W1: out_f32 = 0; sx = Y.s_in3; gam = 0.0f; break;
-            default: out_f32 = 1; sx = Y.s_h; gam = Y.gamma3; break;
-        }
+        const int out_f32 = P.phase[ph].out_f32;
+        const float sx = P.phase[ph].sx, gam = P.phase[ph].gam;
         uint8_t *stage = stage2 + (ph & 1) * P.stage_bytes;
         float *stf = reinterpret_cast<float *>(stage);
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
@@ -691,13 +682,10 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const float *iv = bb + rows;
             const float *mw = (w4 && f.m) ? iv + rows : nullptr;
             const int kc = rb / 16;  // 16-byte weight chunks per row (4-bit: one run of 32 codes each)
-            // lanes per row: a power of two dividing kc, at most 32, and no more
-            // than spreads the slice's rows over the block's 256 threads (each
-            // lane takes kc / lpr chunks)
-            int lpr = kc & -kc;
-            if (lpr > 32) lpr = 32;
-            while (lpr > 1 && rows * lpr > DC_THREADS) lpr >>= 1;
-            const int lg = __ffs(lpr) - 1;         // lpr = 2^lg
+            // lpr = 2^lg lanes per row (host-chosen: a power of two dividing kc,
+            // at most 32, no more than spreads the slice's rows over the block's
+            // 256 threads; each lane takes kc / lpr chunks)
+            const int lg = f.lg, lpr = 1 << lg;
             const int cpl = kc >> lg;
             const int rpw = 32 >> lg;              // rows per warp pass
             const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -991,7 +979,8 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
         f[5] = ph(Y.w2, nullptr, d / nc, F);
     }
     // exchange geometry: slices of fp32 residual values (embedding, O, O2, W2)
-    // or int8 codes (qkv, q2, h)
+    // or int8 codes (qkv, q2, h); the slice GEMV's lane groups and epilogue
+    // constants
     auto magic = [](int v) { return v > 1 ? (uint32_t)((0x100000000ull + (uint64_t)v - 1) / (uint64_t)v) : 0u; };
     for (int ph = 0; ph < 1 + 6 * P.n_dec; ph++) {
         const int kind = ph == 0 ? -1 : (ph - 1) % 6;
@@ -1001,6 +990,25 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
         P.phase[ph].cpr = cpr;
         P.phase[ph].mg_rc = magic(R * cpr);
         P.phase[ph].mg_c = magic(cpr);
+        DcPhase &f = P.phase[ph];
+        const int kc = (f.bits == 4 ? f.K / 2 : f.K) / 16;
+        int lpr = kc & -kc;
+        if (lpr > 32) lpr = 32;
+        while (lpr > 1 && f.rows * lpr > DC_THREADS) lpr >>= 1;
+        int lg = 0;
+        while ((1 << lg) < lpr) lg++;
+        f.lg = kc > 0 ? lg : 0;
+        f.out_f32 = f32 ? 1 : 0;
+        const DcLayer &Y = P.layer[ph == 0 ? 0 : (ph - 1) / 6];
+        switch (kind) {
+            case 0: f.sx = Y.s_in1; f.gam = 0.0f; break;
+            case 1: f.sx = Y.s_ctx1; f.gam = Y.gamma1; break;
+            case 2: f.sx = Y.s_in2; f.gam = 0.0f; break;
+            case 3: f.sx = Y.s_ctx2; f.gam = Y.gamma2; break;
+            case 4: f.sx = Y.s_in3; f.gam = 0.0f; break;
+            case 5: f.sx = Y.s_h; f.gam = Y.gamma3; break;
+            default: f.sx = 0.0f; f.gam = 0.0f; break;
+        }
     }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;

@@ -255,6 +255,10 @@ struct DcPhase {
     // (quotients of chunk indices below 2^16 by one multiply-high)
     int cpr;
     uint32_t mg_rc, mg_c;
+    // the slice GEMV: 2^lg lanes per weight row; the epilogue's input scale
+    // and residual gain, and whether it produces fp32 residual values
+    int lg, out_f32;
+    float sx, gam;
 };
 struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
