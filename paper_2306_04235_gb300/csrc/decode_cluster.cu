@@ -230,10 +230,9 @@ MNMT_DEV void dc_row_extremes(const unsigned *mm, int row, int nc, float &hi, fl
 
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
                                           int8_t *a, int write_back, int *status, const unsigned *mm, int nc,
-                                          long long *part_l) {
+                                          long long *part_l, int kd, int dodd) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int n = R * d, spr = d / 32;  // partial slots (warps) per row
-    const int kd = __ffs(d) - 1, dodd = d >> kd;  // d = dodd 2^kd
     // pass 1: exact sum of x on the grid of max |x|
 #pragma unroll 1
     for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
@@ -294,9 +293,8 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
     const int H = P.H, T = P.T, S = P.S, R = P.R;
     const float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
     const int items = R * H;
-    const int ip = items >= DC_WARPS ? DC_WARPS : (items > 4 ? 8 : (items > 2 ? 4 : (items > 1 ? 2 : 1)));
-    const int wpi = DC_WARPS / ip;  // warps per item in a round of ip items (a power of two)
-    const int lw = __ffs(wpi) - 1;
+    const int ip = P.att_ip, lw = P.att_lw;  // items per round; 2^lw warps per item
+    const int wpi = 1 << lw;
     constexpr int QC = DH / 16;
     for (int base = 0; base < items; base += ip) {
         const int it = base + (warp >> lw), part = warp & (wpi - 1);
@@ -430,17 +428,10 @@ __device__ __noinline__ void dc_commit_greedy(const DcParams &P, int tp, const i
 
 enum { K_EMB = -1, K_QKV = 0, K_O = 1, K_Q2 = 2, K_O2 = 3, K_W1 = 4, K_W2 = 5 };
 
-// bytes a CTA receives in the exchange of phase ph: the full int8 vector
-// (qkv, q2, h) or the fp32 residual plus every slice's [R] max / min pair
-MNMT_DEV uint32_t dc_xbytes(const DcParams &P, int ph) {
-    const int kind = ph == 0 ? K_EMB : (ph - 1) % 6;
-    switch (kind) {
-        case K_QKV: return (uint32_t)(P.R * 3 * P.d);
-        case K_Q2: return (uint32_t)(P.R * P.d);
-        case K_W1: return (uint32_t)(P.R * P.F);
-        default: return (uint32_t)(P.R * P.d * 4 + P.R * P.nc * 8);
-    }
-}
+// bytes a CTA receives in the exchange of phase ph (host-computed): the full
+// int8 vector (qkv, q2, h) or the fp32 residual plus every slice's [R]
+// max / min pair
+MNMT_DEV uint32_t dc_xbytes(const DcParams &P, int ph) { return P.phase[ph].xbytes; }
 
 // W4: the model's attention / FFN linears hold 4-bit codes (a separate
 // instantiation, so the int8 step carries no 4-bit code)
@@ -636,12 +627,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float inv_in = kind == K_QKV ? Y.inv_in1 : (kind == K_Q2 ? Y.inv_in2 : Y.inv_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], inv_in);
             } else {
                 dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, inv_in, a_full, 1, P.status, mm, nc,
-                             part_l);
+                             part_l, P.ln_kd, P.ln_dodd);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
@@ -802,14 +793,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? P.inv_dout : P.layer[l + 1].inv_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l);
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
         }
     }
     DC_STAMP(stamp, 100);
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     P.inv_dout, a_full, 0, P.status, mm, nc, part_l);
+                     P.inv_dout, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -999,6 +990,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
         while ((1 << lg) < lpr) lg++;
         f.lg = kc > 0 ? lg : 0;
         f.out_f32 = f32 ? 1 : 0;
+        f.xbytes = (uint32_t)(f32 ? R * d * 4 + R * nc * 8 : R * (kind == 0 ? 3 * d : (kind == 2 ? d : F)));
         const DcLayer &Y = P.layer[ph == 0 ? 0 : (ph - 1) / 6];
         switch (kind) {
             case 0: f.sx = Y.s_in1; f.gam = 0.0f; break;
@@ -1009,6 +1001,18 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
             case 5: f.sx = Y.s_h; f.gam = Y.gamma3; break;
             default: f.sx = 0.0f; f.gam = 0.0f; break;
         }
+    }
+    {
+        const int items = R * P.H;
+        const int ip = items >= DC_WARPS ? DC_WARPS : (items > 4 ? 8 : (items > 2 ? 4 : (items > 1 ? 2 : 1)));
+        int lw = 0;
+        while ((DC_WARPS >> lw) > ip) lw++;  // DC_WARPS / ip = 2^lw warps per item
+        P.att_ip = ip;
+        P.att_lw = lw;
+        int kd = 0;
+        while (((d >> kd) & 1) == 0) kd++;
+        P.ln_kd = kd;
+        P.ln_dodd = d >> kd;
     }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;

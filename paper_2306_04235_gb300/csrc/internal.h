@@ -259,6 +259,7 @@ struct DcPhase {
     // and residual gain, and whether it produces fp32 residual values
     int lg, out_f32;
     float sx, gam;
+    uint32_t xbytes;  // bytes a CTA receives in the phase's exchange
 };
 struct alignas(16) DcParams {
     int R, d, H, dh, F, E, V, T, S, n_dec, pre_ln, factorised, nc;
@@ -286,7 +287,9 @@ struct alignas(16) DcParams {
     int off_r, off_a, off_qkv, off_ctx, off_q2, off_h, off_stage, off_att, off_ring, off_ln, off_red, slot_bytes,
         att_cap;
     int kv_staged, off_kvs, off_kvc;
-    int stage_bytes;  // one of the two slice staging buffers  // self / cross keys and values staged in shared memory
+    int stage_bytes;  // one of the two slice staging buffers
+    int att_ip, att_lw;  // attention: (row, head) items per round, log2 of warps per item
+    int ln_kd, ln_dodd;  // d = ln_dodd 2^ln_kd (ln_dodd odd)  // self / cross keys and values staged in shared memory
     int off_part, off_bar;  // off_bar: mbarriers of the weight ring [DC_NB] and of the exchange [2]
     DcLayer layer[DC_LMAX];
     DcPhase phase[1 + 6 * DC_LMAX];
