@@ -876,29 +876,33 @@ __global__ void __launch_bounds__(256) vocab_greedy_kernel(const int8_t *__restr
     asm volatile("cp.async.wait_all;\n" ::);
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    int lpr = kc & -kc;  // lanes per weight row: the largest power of two dividing kc, at most 32
-    if (lpr > 32) lpr = 32;
-    const int lg = __ffs(lpr) - 1;       // lpr = 2^lg
-    const int rpw = 32 >> lg;            // rows per warp and pass
-    const int grp = lane >> lg, sl = lane & (lpr - 1);
+    // a lane pair per weight row (16 rows per warp and pass): lane l takes the
+    // chunks k = (l & 1) + 2 j of its row, j rotated by the row so that the
+    // warp's 16-byte loads spread over the shared-memory banks; one shuffle
+    // joins the pair
+    const int half = lane & 1, hk = kc >> 1;
     unsigned long long best[MT];
 #pragma unroll
     for (int m = 0; m < MT; m++) best[m] = 0ull;
-    for (int r0 = warp * rpw; r0 < nr; r0 += 8 * rpw) {
-        const int row = r0 + grp;
+    for (int r0 = warp * 16; r0 < nr; r0 += 8 * 16) {
+        const int row = r0 + (lane >> 1);
         int acc[MT];
 #pragma unroll
         for (int m = 0; m < MT; m++) acc[m] = 0;
-        if (row < nr)
-            for (int cc = sl; cc < kc; cc += lpr) {
-                const int4 w = ws[(size_t)row * kc + cc];
+        if (row < nr) {
+            int jj = (hk & (hk - 1)) == 0 ? (row & (hk - 1)) : row % hk;
+            const int4 *wr = ws + (size_t)row * kc;
+            for (int j = 0; j < hk; j++) {
+                const int cc = half + 2 * jj;
+                const int4 w = wr[cc];
 #pragma unroll
                 for (int m = 0; m < MT; m++) acc[m] = dot16(as[m * kc + cc], w, acc[m]);
+                jj = jj + 1 == hk ? 0 : jj + 1;
             }
+        }
 #pragma unroll
-        for (int m = 0; m < MT; m++)
-            for (int o = lpr / 2; o > 0; o >>= 1) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
-        if (sl == 0 && row < nr) {
+        for (int m = 0; m < MT; m++) acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], 1);
+        if (half == 0 && row < nr) {
 #pragma unroll
             for (int m = 0; m < MT; m++) {
                 if (m < M) {
@@ -1146,7 +1150,7 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
                                 int reserved_sms, cudaStream_t st) {
-    if (M < 1 || M > 4 || K % 16) return cudaErrorInvalidValue;
+    if (M < 1 || M > 4 || K % 32) return cudaErrorInvalidValue;  // whole chunk pairs per row
     // two blocks per SM, each holding its contiguous rows in shared memory, on
     // the SMs the step's cluster does not occupy: every block is resident (and
     // prefetching its rows) while the step runs, and the next step's cluster
