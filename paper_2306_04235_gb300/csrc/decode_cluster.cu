@@ -93,11 +93,28 @@ MNMT_DEV float dc_rn32_pow2(long long s, int e) {
 }
 
 // nearest float to s 2^e / (dodd 2^kd): the power-of-two case inline, an odd
-// factor (widths such as 384 = 3 * 128) out of line
-__device__ __noinline__ float dc_rn32_scaled_div(long long s, int e, int d) { return rn32_scaled_div(s, e, d); }
-MNMT_DEV float dc_rn32_scaled(long long s, int e, int kd, int dodd) {
+// factor (widths such as 384 = 3 * 128) out of line.  The odd case is
+// rn32_scaled_div's method (an integer quotient of at least 50 significant
+// bits plus a sticky bit) with its 64-bit division replaced by a multiply-high
+// by zm = floor(2^64 / dodd) (host-computed): for num < 2^63 the estimate is
+// the quotient or one less, which the remainder corrects.
+__device__ __noinline__ float dc_rn32_scaled_div(long long S, int e, int kd, unsigned z, unsigned long long zm) {
+    if (S == 0) return 0.0f;
+    const unsigned long long a = S < 0 ? 0ull - (unsigned long long)S : (unsigned long long)S;
+    const int nb = 64 - __clzll(a);
+    const int t = nb < 62 ? 62 - nb : 0;
+    const unsigned long long num = a << t;
+    unsigned long long q = __umul64hi(num, zm), r = num - q * z;
+    if (r >= z) {
+        q++;
+        r -= z;
+    }
+    const float f = rn32_pow2((long long)(2ull * q + (r != 0ull ? 1ull : 0ull)), e - kd - t - 1);
+    return S < 0 ? -f : f;
+}
+MNMT_DEV float dc_rn32_scaled(long long s, int e, int kd, int dodd, unsigned long long zm) {
     if (dodd == 1) return dc_rn32_pow2(s, e - kd);
-    return dc_rn32_scaled_div(s, e, dodd << kd);
+    return dc_rn32_scaled_div(s, e, kd, (unsigned)dodd, zm);
 }
 
 // signed bytes of a 32-bit word
@@ -230,7 +247,7 @@ MNMT_DEV void dc_row_extremes(const unsigned *mm, int row, int nc, float &hi, fl
 
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
                                           int8_t *a, int write_back, int *status, const unsigned *mm, int nc,
-                                          long long *part_l, int kd, int dodd) {
+                                          long long *part_l, int kd, int dodd, unsigned long long zm) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int n = R * d, spr = d / 32;  // partial slots (warps) per row
     // pass 1: exact sum of x on the grid of max |x|
@@ -251,7 +268,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
         float hi, lo;
         dc_row_extremes(mm, row, nc, hi, lo);
         const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
-        const float mu = dc_rn32_scaled(dc_row_sum(part_l, row, spr), ea - 52, kd, dodd);
+        const float mu = dc_rn32_scaled(dc_row_sum(part_l, row, spr), ea - 52, kd, dodd, zm);
         const int eb = exp_bound(fmaxf(fabsf(__fsub_rn(hi, mu)), fabsf(__fsub_rn(lo, mu))));
         const float cv = __fsub_rn(r[e0 + lane], mu);
         const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
@@ -268,7 +285,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
         const int row = dc_row_of(e0, d, R), e = e0 + lane, i = e - row * d;
         const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
         const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
-        const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd);
+        const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd, zm);
         const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
         const float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(r[e], mu), rstd), g[i]), b[i]);
         a[e] = q8(y, inv);
@@ -627,12 +644,12 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float inv_in = kind == K_QKV ? Y.inv_in1 : (kind == K_Q2 ? Y.inv_in2 : Y.inv_in3);
             if (P.pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
+                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], inv_in);
             } else {
                 dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, inv_in, a_full, 1, P.status, mm, nc,
-                             part_l, P.ln_kd, P.ln_dodd);
+                             part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
@@ -793,14 +810,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? P.inv_dout : P.layer[l + 1].inv_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
+            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
         }
     }
     DC_STAMP(stamp, 100);
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (P.pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
-                     P.inv_dout, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd);
+                     P.inv_dout, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
     __syncthreads();
     if (c == 0) {
         for (int i = threadIdx.x; i < R * d; i += DC_THREADS) {
@@ -1017,6 +1034,7 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
         while (((d >> kd) & 1) == 0) kd++;
         P.ln_kd = kd;
         P.ln_dodd = d >> kd;
+        P.ln_zm = P.ln_dodd > 1 ? ~0ull / (unsigned long long)P.ln_dodd : 0ull;  // floor(2^64 / dodd), dodd odd
     }
     // shared-memory carve-up (16-byte aligned pieces)
     size_t off = 0;

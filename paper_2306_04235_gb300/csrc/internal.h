@@ -289,7 +289,8 @@ struct alignas(16) DcParams {
     int kv_staged, off_kvs, off_kvc;
     int stage_bytes;  // one of the two slice staging buffers
     int att_ip, att_lw;  // attention: (row, head) items per round, log2 of warps per item
-    int ln_kd, ln_dodd;  // d = ln_dodd 2^ln_kd (ln_dodd odd)  // self / cross keys and values staged in shared memory
+    int ln_kd, ln_dodd;  // d = ln_dodd 2^ln_kd (ln_dodd odd)
+    unsigned long long ln_zm;  // floor(2^64 / ln_dodd) when ln_dodd > 1  // self / cross keys and values staged in shared memory
     int off_part, off_bar;  // off_bar: mbarriers of the weight ring [DC_NB] and of the exchange [2]
     DcLayer layer[DC_LMAX];
     DcPhase phase[1 + 6 * DC_LMAX];

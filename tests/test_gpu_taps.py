@@ -71,7 +71,7 @@ def test_paper_models_tokens_and_taps(name, stream):
     odd factor in every kernel that normalises."""
     cfg, blob, ids, lens, beam, T = synth.workload_inputs(name)
     kind, _ = check_taps(blob, cfg, ids, lens, beam, T, T, [0], stream)
-    assert kind == 1  # the single-cluster decode step (8 CTAs of 48 columns at d = 384)
+    assert kind == 1  # the single-cluster decode step (12 CTAs of 32 columns at d = 384)
     tr = mnmt.Translator(blob, 1, ids.shape[1], beam, T, stream)
     try:
         g_ids, g_len, _ = tr.translate(ids, lens, T)
