@@ -152,6 +152,37 @@ def test_forced_eos_stops_at_once(beam, stream):
     assert np.all(g_len == 1) and np.all(g_ids[:, 0] == cfg.eos_id) and np.all(g_ids[:, 1:] == cfg.pad_id)
 
 
+@pytest.mark.parametrize("seed,bias,rows,lengths", [
+    (3, 0.15, None, [23, 1, 40, 40]),
+    (3, 0.2, None, [1, 1, 16, 40]),   # one sentence ends on a 16-step graph boundary
+    (5, 0.28, None, [1, 1, 24, 40]),
+    (3, 0.1, 0, [31]),
+    (3, 0.2, 2, [16]),
+])
+def test_cluster_step_mixed_lengths_match_oracle(seed, bias, rows, lengths, stream):
+    """The single-cluster step (greedy, <= 4 rows) with sentences that finish
+    at different steps, inside and at the end of a captured run of 16 steps:
+    the greedy selection left pending by the vocabulary kernel is applied by
+    the next step kernel or by the greedy update that closes the run."""
+    cfg = MINI["pre"]
+    blob = synth.build_blob(cfg, seed, out_bias={cfg.eos_id: bias})
+    ids, lens = synth.source_batch(cfg.vocab, 4, 2, 30, 4)
+    if rows is not None:
+        ids, lens = ids[rows:rows + 1], lens[rows:rows + 1]
+    T = 40
+    tr = mnmt.Translator(blob, ids.shape[0], ids.shape[1], 1, T, stream)
+    try:
+        g_ids, g_len, g_sc = tr.translate(ids, lens, T)
+        assert mnmt.mnmt_session_decode_path(tr.session) == 1
+    finally:
+        tr.close()
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, 1, T, n_threads=4)
+    assert o_len.tolist() == lengths
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_len, o_len)
+    assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
+
+
 @pytest.mark.parametrize("beam", [1, 3])
 def test_decode_step_api_matches_translate(beam, stream):
     cfg = MINI["fact"]
