@@ -248,31 +248,44 @@ MNMT_DEV void dc_row_extremes(const unsigned *mm, int row, int nc, float &hi, fl
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
                                           int8_t *a, int write_back, int *status, const unsigned *mm, int nc,
                                           long long *part_l, int kd, int dodd, unsigned long long zm) {
-    const int tid = threadIdx.x, lane = tid & 31;
-    const int n = R * d, spr = d / 32;  // partial slots (warps) per row
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    // a warp takes chunks of cw elements of one row: 32 (one per lane) up to
+    // 256 elements, else 64 (two per lane, independent chains), so rows of up
+    // to 512 elements still take one round per pass
+    const int n = R * d, two = n > DC_THREADS ? 1 : 0, cs = 5 + two, cw = 32 << two;
+    const int spr = d >> cs;  // partial slots (chunks) per row
     // pass 1: exact sum of x on the grid of max |x|
 #pragma unroll 1
-    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+    for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
         float hi, lo;
         dc_row_extremes(mm, dc_row_of(e0, d, R), nc, hi, lo);
         const float am = fmaxf(fabsf(hi), fabsf(lo));
         if (!(am < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
-        const long long s = warp_sum_exact(fx_scale(r[e0 + lane], 52 - exp_bound(am)));
-        if (lane == 0) part_l[e0 / 32] = s;
+        const int sh = 52 - exp_bound(am);
+        long long v = fx_scale(r[e0 + lane], sh);
+        if (two) v += fx_scale(r[e0 + 32 + lane], sh);
+        const long long s = warp_sum_exact(v);
+        if (lane == 0) part_l[e0 >> cs] = s;
     }
     __syncthreads();
     // pass 2: exact sum of c^2 = fl(x - mean)^2 on the grid of max |c|
 #pragma unroll 1
-    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+    for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
         const int row = dc_row_of(e0, d, R);
         float hi, lo;
         dc_row_extremes(mm, row, nc, hi, lo);
         const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
         const float mu = dc_rn32_scaled(dc_row_sum(part_l, row, spr), ea - 52, kd, dodd, zm);
         const int eb = exp_bound(fmaxf(fabsf(__fsub_rn(hi, mu)), fabsf(__fsub_rn(lo, mu))));
+        const int sh = 52 - 2 * eb;
         const float cv = __fsub_rn(r[e0 + lane], mu);
-        const long long s = warp_sum_exact(fx_scale(__fmul_rn(cv, cv), 52 - 2 * eb));
-        if (lane == 0) part_l[64 + e0 / 32] = s;
+        long long v = fx_scale(__fmul_rn(cv, cv), sh);
+        if (two) {
+            const float cw2 = __fsub_rn(r[e0 + 32 + lane], mu);
+            v += fx_scale(__fmul_rn(cw2, cw2), sh);
+        }
+        const long long s = warp_sum_exact(v);
+        if (lane == 0) part_l[64 + (e0 >> cs)] = s;
         if (lane == 0 && e0 == row * d) {
             reinterpret_cast<float *>(part_l + 128)[2 * row] = mu;  // per row: mu, 2^eb grid
             reinterpret_cast<int *>(part_l + 128)[2 * row + 1] = eb;
@@ -281,15 +294,21 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     __syncthreads();
     // pass 3: normalise, scale, shift, quantise
 #pragma unroll 1
-    for (int e0 = tid - lane; e0 < n; e0 += DC_THREADS) {
+    for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
         const int row = dc_row_of(e0, d, R), e = e0 + lane, i = e - row * d;
         const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
         const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
         const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd, zm);
         const float rstd = __fdiv_rn(1.0f, __fsqrt_rn(__fadd_rn(var, 1e-5f)));
         const float y = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(r[e], mu), rstd), g[i]), b[i]);
+        float y2 = 0.0f;
+        if (two) y2 = __fadd_rn(__fmul_rn(__fmul_rn(__fsub_rn(r[e + 32], mu), rstd), g[i + 32]), b[i + 32]);
         a[e] = q8(y, inv);
         if (write_back) r[e] = y;
+        if (two) {
+            a[e + 32] = q8(y2, inv);
+            if (write_back) r[e + 32] = y2;
+        }
     }
     __syncthreads();
 }
