@@ -152,6 +152,28 @@ def test_forced_eos_stops_at_once(beam, stream):
     assert np.all(g_len == 1) and np.all(g_ids[:, 0] == cfg.eos_id) and np.all(g_ids[:, 1:] == cfg.pad_id)
 
 
+@pytest.mark.parametrize("kind", list(MINI))
+@pytest.mark.parametrize("batch", [1, 3])
+def test_cluster_step_models_match_oracle(kind, batch, stream):
+    """Every small model shape (pre- and post-LN, factorised and plain
+    embedding, tied and untied output, d_h 64 and 128, d = 3 x 64) through
+    the single-cluster step: greedy batches of at most 4 rows."""
+    cfg = MINI[kind]
+    blob = synth.build_blob(cfg, 41, gamma_range=(0.5, 1.5))
+    ids, lens = synth.source_batch(cfg.vocab, batch, 1, 40, 42)
+    T = 24
+    tr = mnmt.Translator(blob, batch, ids.shape[1], 1, T, stream)
+    try:
+        g_ids, g_len, g_sc = tr.translate(ids, lens, T)
+        assert mnmt.mnmt_session_decode_path(tr.session) == 1
+    finally:
+        tr.close()
+    o_ids, o_len, o_sc = O.translate(blob, ids, lens, 1, T, n_threads=3)
+    assert np.array_equal(g_ids, o_ids)
+    assert np.array_equal(g_len, o_len)
+    assert np.array_equal(g_sc.view(np.uint32), o_sc.view(np.uint32))
+
+
 @pytest.mark.parametrize("seed,bias,rows,lengths", [
     (3, 0.15, None, [23, 1, 40, 40]),
     (3, 0.2, None, [1, 1, 16, 40]),   # one sentence ends on a 16-step graph boundary
