@@ -261,7 +261,7 @@ class Workload:
         self.blob = synth.build_blob(self.cfg, self.wl.model_seed, wq=wq)
         # every rank translates its own replica batch (independent sentences)
         self.ids, self.lens = synth.source_batch(self.cfg.vocab, self.wl.batch, self.wl.src_len[0],
-                                                 self.wl.src_len[1], self.wl.src_seed + 101 * rank)
+                                                 self.wl.src_len[1], replica_source_seed(self.wl.src_seed, rank))
         self.B, self.S = self.ids.shape
         self.T = self.wl.max_len
         self.mnmt, self.torch, self.stream = mnmt, torch, stream
@@ -411,6 +411,29 @@ def measure_decode_step(w, flush, steps_run, cluster):
             "p50_us": srt[len(srt) // 2], "warm_avg_us": warm_us, "launches": len(cold_us)}
 
 
+def replica_source_seed(src_seed, rank):
+    """Seed of the source batch rank `rank` translates (replicas: independent
+    sentences on every rank)."""
+    return src_seed + 101 * rank
+
+
+def aggregate_ranks(total_ms, toks_per_step, steps, dist=None, device="cuda"):
+    """Whole-job throughput of N replicas: every rank's tokens (SUM) over the
+    slowest rank's time (MAX).  Returns (tokens/s, time in ms, job tokens per
+    step)."""
+    import torch
+
+    job_toks = float(toks_per_step)
+    if dist:
+        t = torch.tensor([float(total_ms)], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+        nt = torch.tensor([job_toks], dtype=torch.float64, device=device)
+        dist.all_reduce(nt, op=dist.ReduceOp.SUM)
+        job_toks = float(nt.item())
+    return job_toks * steps / (total_ms / 1e3), total_ms, job_toks
+
+
 def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, world=1, dist=None, lean=False,
                      wq=8):
     """tokens/s (device-resident and end to end), decode-step latency, encode
@@ -419,17 +442,7 @@ def measure_workload(name, mnmt, torch, stream, flush, steps, warmup, rank=0, wo
     try:
         step_ms = time_translations(w, flush, steps, warmup, dist)
         toks_per_step = int(w.o_len.sum().item())
-        total_ms = sum(step_ms)
-        if dist:
-            t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            total_ms = float(t.item())
-            nt = torch.tensor([toks_per_step], dtype=torch.float64, device="cuda")
-            dist.all_reduce(nt, op=dist.ReduceOp.SUM)
-            job_toks = float(nt.item())
-        else:
-            job_toks = float(toks_per_step)
-        value = job_toks * steps / (total_ms / 1e3)
+        value, total_ms, _ = aggregate_ranks(sum(step_ms), toks_per_step, steps, dist)
         enc_ms = time_encode(w, flush)
         # decode steps actually executed per translation (greedy stops when
         # every sentence has emitted EOS; the beam workloads run all T)
