@@ -4,8 +4,9 @@ Builds libmnmt_stamps.so (the library with the cluster step compiled with
 -DMNMT_DC_STAMPS), translates a workload with it and prints, for decode step
 20, how long each of the step's phases spends waiting for its weight slice,
 preparing its input (LayerNorm or attention), in its slice GEMV and in the
-broadcast + cluster barrier, plus the prologue and the overlap with the
-previous step's vocabulary kernel.  Times in ns from %globaltimer at CTA 0.
+exchange (its slice stored to every CTA, then the wait until this CTA's copy
+of the vector is whole), plus the prologue and the overlap with the previous
+step's vocabulary kernel.  Times in ns from %globaltimer at CTA 0.
 
     python -m paper_2306_04235_gb300.phase_profile [workload]
 """
@@ -62,7 +63,7 @@ def main(argv):
         prev = d
         print(f"| {ph} | {kind} | {row[0]} | {row[1]} | {row[2]} | {row[3]} |")
     print(f"| all | | {tot[0]} | {tot[1]} | {tot[2]} | {tot[3]} |")
-    print(f"final LayerNorm {ns[101] - ns[100]}, last barrier {ns[102] - ns[101]}, kernel {ns[102] - t0}")
+    print(f"final LayerNorm {ns[101] - ns[100]}, output rows {ns[102] - ns[101]}, kernel {ns[102] - t0}")
     return 0
 
 
