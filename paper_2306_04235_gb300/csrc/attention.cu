@@ -18,6 +18,9 @@
 //   attn_encoder one block per (sentence, head, chunk of 4..32 queries): K and V of
 //                the head staged in shared memory, keys masked past the
 //                source length.
+//   attn_encoder_mma  the same on the int8 tensor cores (mma.sync, exact int32)
+//                for d_h = 64 and up to 256 keys: scores as one product, the
+//                weights split into bytes for the context products.
 #include <type_traits>
 
 #include "common.cuh"
@@ -272,6 +275,218 @@ __global__ void __launch_bounds__(32 * ENC_WARPS) attn_encoder(AttnEncArgs a, in
     }
 }
 
+// ---------------------------------------------------------------------------
+// encoder self-attention on the int8 tensor cores (mma.sync m16n8k32, exact
+// int32 accumulation), d_h = 64 and up to 256 keys.  Same arithmetic as
+// attn_encoder: the scores q . k_j are the same exact integers; the weights E_j
+// in [0, 2^24] are split into four bytes E_j = sum_k e_kj 2^(8k), each byte a
+// u8 operand of its own product with V (sum_j e_kj v_j[e] <= 256 * 255 * 128 <
+// 2^31: exact), and N_e = sum_k 2^(8k) (sum_j e_kj v_j[e]) is rebuilt in int64.
+//
+// One block per (sentence, head, 64 queries), four warps of 16 queries each.
+// Shared memory: Q [64][64] and K [Sp][64] in 64-byte rows, V^T [64][Sp], and
+// per warp the weight bytes [4][16][Sp] (Sp = key count padded to a power of
+// two >= 32), 16-byte chunks XOR-swizzled by row so that ldmatrix phases hit
+// distinct bank groups.  Keys past the source length score -inf (weight 0).
+// ---------------------------------------------------------------------------
+constexpr int ENC_MMA_WARPS = 4;
+
+MNMT_DEV uint32_t att_smem_u32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
+MNMT_DEV void att_ldmatrix_x4(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+MNMT_DEV void att_mma_s8(int (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k32.row.col.s32.s8.s8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+r"(c[0]), "+r"(c[1]), "+r"(c[2]), "+r"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+MNMT_DEV void att_mma_u8s8(int (&c)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k32.row.col.s32.u8.s8.s32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+        "{%0,%1,%2,%3};\n"
+        : "+r"(c[0]), "+r"(c[1]), "+r"(c[2]), "+r"(c[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+// byte offset of (row, 16-byte chunk) in 64-byte rows: chunk ^ (row / 2) % 4
+MNMT_DEV int sw64(int row, int chunk) { return row * 64 + ((chunk ^ ((row >> 1) & 3)) << 4); }
+// byte offset of (row, byte col) in rows of `len` bytes (len = 16 * nch, nch a
+// power of two): chunk ^ (row mod min(nch, 8))
+MNMT_DEV int swl(int row, int col, int len, int msk) {
+    return row * len + ((((col >> 4) ^ (row & msk))) << 4) + (col & 15);
+}
+
+__global__ void __launch_bounds__(32 * ENC_MMA_WARPS) attn_encoder_mma(AttnEncArgs a, int Sp) {
+    pdl_grid_wait();
+    extern __shared__ __align__(128) uint8_t emm[];
+    constexpr int DH = 64;
+    const int bh = blockIdx.x;
+    const int b = bh / a.H, h = bh - b * a.H;
+    const int S = a.S;
+    int len = a.len[b];
+    len = len < 1 ? 1 : (len > S ? S : len);
+    const int q0 = blockIdx.y * 64;
+    const int nch = Sp >> 4, msk = (nch < 8 ? nch : 8) - 1;
+    uint8_t *Qs = emm;                       // [64][64]
+    uint8_t *Ks = Qs + 64 * 64;              // [Sp][64]
+    uint8_t *Vt = Ks + (size_t)Sp * 64;      // [64][Sp]
+    uint8_t *Es = Vt + (size_t)64 * Sp;      // [warps][4][16][Sp]; first V row-major [Sp][64]
+    const int ld = 3 * a.d;
+    const int8_t *base = a.qkv + (size_t)b * S * ld;
+    // stage Q (64 queries), K and V (valid keys; the rest zero)
+    for (int i = threadIdx.x; i < 64 * 4; i += blockDim.x) {
+        const int r = i >> 2, c = i & 3, q = q0 + r;
+        int4 v = make_int4(0, 0, 0, 0);
+        if (q < S) v = reinterpret_cast<const int4 *>(base + (size_t)q * ld + h * DH)[c];
+        *reinterpret_cast<int4 *>(Qs + sw64(r, c)) = v;
+    }
+    for (int i = threadIdx.x; i < Sp * 4; i += blockDim.x) {
+        const int j = i >> 2, c = i & 3;
+        int4 kv = make_int4(0, 0, 0, 0), vv = make_int4(0, 0, 0, 0);
+        if (j < len) {
+            kv = reinterpret_cast<const int4 *>(base + (size_t)j * ld + a.d + h * DH)[c];
+            vv = reinterpret_cast<const int4 *>(base + (size_t)j * ld + 2 * a.d + h * DH)[c];
+        }
+        *reinterpret_cast<int4 *>(Ks + sw64(j, c)) = kv;
+        reinterpret_cast<int4 *>(Es + (size_t)j * DH)[c] = vv;
+    }
+    __syncthreads();
+    // V^T: word (e, keys 4w .. 4w + 3) from four rows of V
+    for (int i = threadIdx.x; i < DH * (Sp >> 2); i += blockDim.x) {
+        const int e = i & (DH - 1), j = 4 * (i >> 6);
+        const uint32_t x = (uint32_t)Es[(size_t)j * DH + e] | ((uint32_t)Es[(size_t)(j + 1) * DH + e] << 8) |
+                           ((uint32_t)Es[(size_t)(j + 2) * DH + e] << 16) |
+                           ((uint32_t)Es[(size_t)(j + 3) * DH + e] << 24);
+        *reinterpret_cast<uint32_t *>(Vt + swl(e, j, Sp, msk)) = x;
+    }
+    __syncthreads();
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int jq = lane >> 3, i8 = lane & 7, g = lane >> 2, tq = lane & 3;
+    uint8_t *Ew = Es + (size_t)warp * 4 * 16 * Sp;
+    // Q fragments of this warp's 16 queries (two k-steps of 32)
+    uint32_t af[2][4];
+#pragma unroll
+    for (int kk = 0; kk < 2; kk++)
+        att_ldmatrix_x4(af[kk], att_smem_u32(Qs + sw64(warp * 16 + (jq & 1) * 8 + i8, kk * 2 + (jq >> 1))));
+    // scores of 16 keys (two n-tiles) per call: exact int32, then fl(acc sigma),
+    // -inf past the source length
+    auto scores16 = [&](int k0, float (&sv)[2][4]) {
+        int acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
+#pragma unroll
+        for (int kk = 0; kk < 2; kk++) {
+            uint32_t r[4];
+            att_ldmatrix_x4(r, att_smem_u32(Ks + sw64(k0 + (jq >> 1) * 8 + i8, kk * 2 + (jq & 1))));
+            att_mma_s8(acc[0], af[kk], r[0], r[1]);
+            att_mma_s8(acc[1], af[kk], r[2], r[3]);
+        }
+#pragma unroll
+        for (int t = 0; t < 2; t++)
+#pragma unroll
+            for (int q = 0; q < 4; q++) {
+                const int key = k0 + t * 8 + tq * 2 + (q & 1);
+                sv[t][q] = key < len ? __fmul_rn(__int2float_rn(acc[t][q]), a.sigma) : -INFINITY;
+            }
+    };
+    // pass 1: each row's maximum score
+    float mx0 = -INFINITY, mx1 = -INFINITY;  // rows g and g + 8
+    for (int k0 = 0; k0 < Sp; k0 += 16) {
+        float sv[2][4];
+        scores16(k0, sv);
+#pragma unroll
+        for (int t = 0; t < 2; t++) {
+            mx0 = fmaxf(mx0, fmaxf(sv[t][0], sv[t][1]));
+            mx1 = fmaxf(mx1, fmaxf(sv[t][2], sv[t][3]));
+        }
+    }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+        mx0 = fmaxf(mx0, __shfl_xor_sync(0xFFFFFFFFu, mx0, o));
+        mx1 = fmaxf(mx1, __shfl_xor_sync(0xFFFFFFFFu, mx1, o));
+    }
+    // pass 2: weights E (the scores again), their bytes into shared memory, Z
+    long long z0 = 0, z1 = 0;
+    for (int k0 = 0; k0 < Sp; k0 += 16) {
+        float sv[2][4];
+        scores16(k0, sv);
+#pragma unroll
+        for (int t = 0; t < 2; t++) {
+            int E[4];
+#pragma unroll
+            for (int q = 0; q < 4; q++) E[q] = softmax_weight(__fadd_rn(sv[t][q], -(q < 2 ? mx0 : mx1)));
+            z0 += (long long)E[0] + E[1];
+            z1 += (long long)E[2] + E[3];
+            const int key = k0 + t * 8 + tq * 2;
+#pragma unroll
+            for (int L = 0; L < 4; L++) {
+                const uint32_t lo2 = ((uint32_t)(E[0] >> (8 * L)) & 255u) | (((uint32_t)(E[1] >> (8 * L)) & 255u) << 8);
+                const uint32_t hi2 = ((uint32_t)(E[2] >> (8 * L)) & 255u) | (((uint32_t)(E[3] >> (8 * L)) & 255u) << 8);
+                *reinterpret_cast<uint16_t *>(Ew + (size_t)L * 16 * Sp + swl(g, key, Sp, msk)) = (uint16_t)lo2;
+                *reinterpret_cast<uint16_t *>(Ew + (size_t)L * 16 * Sp + swl(g + 8, key, Sp, msk)) = (uint16_t)hi2;
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+        z0 += __shfl_xor_sync(0xFFFFFFFFu, z0, o);
+        z1 += __shfl_xor_sync(0xFFFFFFFFu, z1, o);
+    }
+    __syncwarp();
+    // context: per weight byte L, sum_j e_Lj v_j[e] on the tensor cores (u8 x s8)
+    long long N[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+        for (int q = 0; q < 4; q++) N[nt][q] = 0;
+#pragma unroll 1
+    for (int L = 0; L < 4; L++) {
+        int acc[8][4];
+#pragma unroll
+        for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+            for (int q = 0; q < 4; q++) acc[nt][q] = 0;
+        const uint8_t *EL = Ew + (size_t)L * 16 * Sp;
+        for (int ks = 0; ks < (Sp >> 5); ks++) {
+            uint32_t ea[4];
+            att_ldmatrix_x4(ea, att_smem_u32(EL + swl((jq & 1) * 8 + i8, (ks * 2 + (jq >> 1)) * 16, Sp, msk)));
+#pragma unroll
+            for (int nj = 0; nj < 4; nj++) {
+                uint32_t r[4];
+                att_ldmatrix_x4(r, att_smem_u32(Vt + swl(nj * 16 + (jq >> 1) * 8 + i8, (ks * 2 + (jq & 1)) * 16, Sp, msk)));
+                att_mma_u8s8(acc[2 * nj], ea, r[0], r[1]);
+                att_mma_u8s8(acc[2 * nj + 1], ea, r[2], r[3]);
+            }
+        }
+#pragma unroll
+        for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+            for (int q = 0; q < 4; q++) N[nt][q] += (long long)acc[nt][q] << (8 * L);
+    }
+    // row g (q < 2) or g + 8 of the warp's queries, element nt * 8 + 2 tq + (q & 1)
+#pragma unroll
+    for (int nt = 0; nt < 8; nt++)
+#pragma unroll
+        for (int q = 0; q < 4; q++) {
+            const int qrow = q0 + warp * 16 + g + (q >> 1) * 8;
+            if (qrow < S) {
+                const int e = nt * 8 + tq * 2 + (q & 1);
+                const int8_t v = q8_quotient(N[nt][q], q < 2 ? z0 : z1, a.rho, rn32_div);
+                const size_t o = ((size_t)b * S + qrow) * a.d + h * DH + e;
+                a.ctx[o] = v;
+                if (a.ctx16) a.ctx16[o] = __short2half_rn(v);
+            }
+        }
+}
+
+static int enc_mma_keys(int S) {
+    int sp = 32;
+    while (sp < S) sp <<= 1;
+    return sp;
+}
+static size_t enc_mma_smem(int Sp) { return 64 * 64 + (size_t)Sp * 64 * 2 + (size_t)ENC_MMA_WARPS * 4 * 16 * Sp; }
 template <int DH>
 static cudaError_t launch_enc(const AttnEncArgs &a, cudaStream_t st) {
     size_t smem = (size_t)a.S * (DH + 16) + (size_t)a.S * DH + (size_t)ENC_WARPS * a.S * sizeof(int);
@@ -287,6 +502,14 @@ static cudaError_t launch_enc(const AttnEncArgs &a, cudaStream_t st) {
 
 cudaError_t launch_attention_encoder(const AttnEncArgs &a, cudaStream_t st) {
     if (a.S < 1 || a.S > ENC_MAX_KEYS) return cudaErrorInvalidValue;
+    // the tensor-core kernel when its grid fills the GPU (a handful of
+    // sentences run faster on the dp4a kernel's finer query chunks)
+    if (a.dh == 64 && a.S <= 256 && (long)a.B * a.H * ((a.S + 63) / 64) >= device_sm_count()) {
+        const int Sp = enc_mma_keys(a.S);
+        dim3 grid(a.B * a.H, (a.S + 63) / 64);
+        launch_pdl(attn_encoder_mma, grid, 32 * ENC_MMA_WARPS, enc_mma_smem(Sp), st, a, Sp);
+        return cudaGetLastError();
+    }
     switch (a.dh) {
         case 32:
             return launch_enc<32>(a, st);
@@ -318,6 +541,9 @@ cudaError_t attention_init() {
     if (!err) err = cudaFuncSetAttribute(attn_encoder<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(32));
     if (!err) err = cudaFuncSetAttribute(attn_encoder<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(64));
     if (!err) err = cudaFuncSetAttribute(attn_encoder<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, enc(128));
+    if (!err)
+        err = cudaFuncSetAttribute(attn_encoder_mma, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   (int)enc_mma_smem(256));
     return err;
 }
 }  // namespace mnmt

@@ -99,3 +99,17 @@ def test_paper_20mb_model_batched(beam, B, stream):
     assert np.array_equal(g_ids[pick], o_ids) and np.array_equal(g_len[pick], o_len)
     assert np.array_equal(g_sc[pick].view(np.uint32), o_sc.view(np.uint32))
     check_taps(blob, cfg, ids, lens, beam, T, 8, [0, B - 1], stream)
+
+
+def test_encoder_attention_tensor_core_long_sources(stream):
+    """The tensor-core encoder attention at its largest key count: sources of
+    130-250 tokens (keys padded to 256, four 64-query blocks per head), d_h =
+    64, enough sentences that its grid fills the GPU; encoder output, cross
+    keys / values and two decode steps checked for the shortest and longest
+    sentence."""
+    cfg = synth.ModelConfig(2, 1, 192, 3, 384, 300, 192, 1, 1, max_pos=256)
+    blob = synth.build_blob(cfg, 77, gamma_range=(0.5, 1.5))
+    ids, lens = synth.source_batch(cfg.vocab, 16, 130, 250, 78)
+    assert ids.shape[1] > 128
+    picks = [int(np.argmin(lens)), int(np.argmax(lens))]
+    check_taps(blob, cfg, ids, lens, 1, 4, 2, picks, stream)
