@@ -471,7 +471,7 @@ MNMT_DEV uint32_t dc_xbytes(const DcParams &P, int ph) { return P.phase[ph].xbyt
 
 // W4: the model's attention / FFN linears hold 4-bit codes (a separate
 // instantiation, so the int8 step carries no 4-bit code)
-template <int DH, bool W4>
+template <int DH, bool W4, int RM>
 __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcParams *__restrict__ Pp) {
     // Launched as a programmatic dependent of the previous step's vocabulary
     // kernel: everything up to dc_grid_wait() reads only data that no kernel
@@ -720,8 +720,9 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int4 ones = make_int4(0x01010101, 0x01010101, 0x01010101, 0x01010101);
             for (int r0 = warp * rpw; r0 < rows; r0 += DC_WARPS * rpw) {
                 const int nl = r0 + (lane >> lg);
-                int acc[DC_RMAX] = {0, 0, 0, 0};
-                int a1[DC_RMAX] = {0, 0, 0, 0};  // 4-bit rows: the activation codes' sums
+                int acc[RM], a1[RM];  // a1: 4-bit rows, the activation codes' sums
+#pragma unroll
+                for (int m = 0; m < RM; m++) acc[m] = a1[m] = 0;
                 if (nl < rows) {
                     const int4 *wr = reinterpret_cast<const int4 *>(W + (size_t)nl * rb);
                     for (int q = 0; q < cpl; q++) {
@@ -733,7 +734,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                             const int4 hi = make_int4((w.x >> 4) & 0x0F0F0F0F, (w.y >> 4) & 0x0F0F0F0F,
                                                       (w.z >> 4) & 0x0F0F0F0F, (w.w >> 4) & 0x0F0F0F0F);
 #pragma unroll
-                            for (int m = 0; m < DC_RMAX; m++)
+                            for (int m = 0; m < RM; m++)
                                 if (m < R) {
                                     const int4 *am = reinterpret_cast<const int4 *>(A + (size_t)m * K);
                                     const int4 x0 = am[2 * k], x1 = am[2 * k + 1];
@@ -742,14 +743,14 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                                 }
                         } else {
 #pragma unroll
-                            for (int m = 0; m < DC_RMAX; m++)
+                            for (int m = 0; m < RM; m++)
                                 if (m < R)
                                     acc[m] = dot16(reinterpret_cast<const int4 *>(A + (size_t)m * K)[k], w, acc[m]);
                         }
                     }
                 }
 #pragma unroll
-                for (int m = 0; m < DC_RMAX; m++)
+                for (int m = 0; m < RM; m++)
                     if (m < R)
                         for (int o = lpr / 2; o > 0; o >>= 1) {
                             acc[m] += __shfl_xor_sync(0xFFFFFFFFu, acc[m], o);
@@ -758,7 +759,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
                 if (sub == 0 && nl < rows) {
                     const int n = n0 + nl;
 #pragma unroll
-                    for (int m = 0; m < DC_RMAX; m++) {
+                    for (int m = 0; m < RM; m++) {
                         if (m >= R) break;
                         if (kind == K_EMB) {
                             const float y = dequant_bias(acc[m], P.emb_s[tok_s[m]], sw[nl], bb[nl]);
@@ -1100,6 +1101,23 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
     return off;
 }
 
+// the step kernel of a head width, weight format and row count: int8 single-row
+// steps (greedy batch 1) run an instantiation whose slice GEMV keeps one row
+// of accumulators (a smaller kernel; the step is sensitive to its code size)
+static const void *dc_kernel(int dh, bool w4, bool one_row) {
+    if (w4)
+        return dh == 32 ? (const void *)decode_cluster_kernel<32, true, DC_RMAX>
+                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, true, DC_RMAX>
+                                    : (const void *)decode_cluster_kernel<128, true, DC_RMAX>);
+    if (one_row)
+        return dh == 32 ? (const void *)decode_cluster_kernel<32, false, 1>
+                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, 1>
+                                    : (const void *)decode_cluster_kernel<128, false, 1>);
+    return dh == 32 ? (const void *)decode_cluster_kernel<32, false, DC_RMAX>
+                    : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, DC_RMAX>
+                                : (const void *)decode_cluster_kernel<128, false, DC_RMAX>);
+}
+
 cudaError_t decode_cluster_init() {
     const int max_smem = 227 * 1024;
     cudaError_t err = cudaSuccess;
@@ -1107,12 +1125,8 @@ cudaError_t decode_cluster_init() {
         if (err == cudaSuccess) err = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem);
         if (err == cudaSuccess) err = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     };
-    setk((const void *)decode_cluster_kernel<32, false>);
-    setk((const void *)decode_cluster_kernel<64, false>);
-    setk((const void *)decode_cluster_kernel<128, false>);
-    setk((const void *)decode_cluster_kernel<32, true>);
-    setk((const void *)decode_cluster_kernel<64, true>);
-    setk((const void *)decode_cluster_kernel<128, true>);
+    for (int dh : {32, 64, 128})
+        for (int v = 0; v < 3; v++) setk(dc_kernel(dh, v == 1, v == 2));
     // the vocabulary kernel keeps its SMs in the largest shared-memory
     // configuration, so the next step's cluster (about 200 KB per CTA) can
     // become resident beside it as soon as it is allowed to launch
@@ -1127,19 +1141,9 @@ cudaError_t decode_cluster_init() {
 }
 
 // can one cluster of nc CTAs with smem bytes each be resident?
-static const void *dc_kernel(int dh, bool w4) {
-    if (w4)
-        return dh == 32 ? (const void *)decode_cluster_kernel<32, true>
-                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, true>
-                                    : (const void *)decode_cluster_kernel<128, true>);
-    return dh == 32 ? (const void *)decode_cluster_kernel<32, false>
-                    : (dh == 64 ? (const void *)decode_cluster_kernel<64, false>
-                                : (const void *)decode_cluster_kernel<128, false>);
-}
-
-bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4) {
+bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row) {
     if (smem > 227 * 1024) return false;
-    const void *k = dc_kernel(dh, w4);
+    const void *k = dc_kernel(dh, w4, one_row);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -1161,7 +1165,8 @@ bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4) {
     return clusters >= 1;
 }
 
-cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, cudaStream_t st) {
+cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, bool one_row,
+                                  cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -1181,7 +1186,7 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
     cfg.numAttrs = 2;
     if (dh != 32 && dh != 64 && dh != 128) return cudaErrorInvalidValue;
     void *args[] = {(void *)&dP};
-    return cudaLaunchKernelExC(&cfg, dc_kernel(dh, w4), args);
+    return cudaLaunchKernelExC(&cfg, dc_kernel(dh, w4, one_row), args);
 }
 
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
