@@ -935,7 +935,8 @@ int issue_decode_step(mnmt_session *s) {
     int *t_ptr = s->state + ST_T;
     int *status = s->state + ST_STATUS;
     if (s->use_cluster) {
-        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1, st));
+        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1,
+                                 (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0), st));
         GreedyArgs g;
         g.keys = s->keys;
         g.tok = s->tok;
@@ -1194,7 +1195,8 @@ int setup_cluster_step(mnmt_session *s) {
     P.S = s->Smax;
     size_t smem = dc_layout(P, 227 * 1024);
     P.S = s->S;
-    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1)) return MNMT_OK;
+    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1, (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0)))
+        return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
     s->use_cluster = true;

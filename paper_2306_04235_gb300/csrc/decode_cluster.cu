@@ -471,7 +471,7 @@ MNMT_DEV uint32_t dc_xbytes(const DcParams &P, int ph) { return P.phase[ph].xbyt
 
 // W4: the model's attention / FFN linears hold 4-bit codes (a separate
 // instantiation, so the int8 step carries no 4-bit code)
-template <int DH, bool W4, int RM>
+template <int DH, bool W4, int RM, int FL>
 __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcParams *__restrict__ Pp) {
     // Launched as a programmatic dependent of the previous step's vocabulary
     // kernel: everything up to dc_grid_wait() reads only data that no kernel
@@ -503,6 +503,11 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         asm volatile("barrier.cluster.arrive.release;\n" ::: "memory");
     }
     const DcParams &P = *reinterpret_cast<const DcParams *>(smem);
+    // FL >= 0: the model's pre-LN (bit 0) and factorised-embedding (bit 1)
+    // flags fixed at compile time, so the other variants' code is not in the
+    // kernel; FL < 0: read from the parameter block
+    const bool pre_ln = FL < 0 ? P.pre_ln != 0 : (FL & 1) != 0;
+    const bool factorised = FL < 0 ? P.factorised != 0 : (FL & 2) != 0;
     const uint32_t bars = dc_smem_u32(smem + P.off_bar), xbars = bars + 8u * DC_NB;
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
@@ -652,7 +657,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         const int8_t *A = a_full;
         int K = d;
         if (kind == K_EMB) {
-            if (P.factorised)
+            if (factorised)
                 for (int i = threadIdx.x; i < R * P.E; i += DC_THREADS)
                 for (int m = 0; m < R; m++)
                     if (i >= m * P.E && i < (m + 1) * P.E) a_full[i] = P.emb_q[(size_t)tok_s[m] * P.E + (i - m * P.E)];
@@ -662,7 +667,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // residual (written back), or plain quantisation for the first one
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float inv_in = kind == K_QKV ? Y.inv_in1 : (kind == K_Q2 ? Y.inv_in2 : Y.inv_in3);
-            if (P.pre_ln) {
+            if (pre_ln) {
                 dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], inv_in);
@@ -690,7 +695,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         uint8_t *stage = stage2 + (ph & 1) * P.stage_bytes;
         float *stf = reinterpret_cast<float *>(stage);
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
-        if (kind == K_EMB && !P.factorised) {
+        if (kind == K_EMB && !factorised) {
             for (int i = threadIdx.x; i < R * rows; i += DC_THREADS) {
                 const int m = dc_row_of(i, rows, R), nl = i - m * rows, n = n0 + nl, id = tok_s[m];
                 const float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
@@ -826,7 +831,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         if (!mbar_wait(xbar, (uint32_t)(ph >> 1) & 1u)) set_status(P.status, MNMT_ETIMEOUT);
         if (threadIdx.x == 0 && ph + 2 < nphase) mbar_expect_tx(xbar, dc_xbytes(P, ph + 2));
         DC_STAMP(stamp, 7 + 4 * ph);
-        if (kind == K_W2 && !P.pre_ln) {
+        if (kind == K_W2 && !pre_ln) {
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? P.inv_dout : P.layer[l + 1].inv_in1;
@@ -835,7 +840,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
     DC_STAMP(stamp, 100);
     // ---- final LayerNorm + quantisation -> vocabulary input ----
-    if (P.pre_ln)
+    if (pre_ln)
         dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
                      P.inv_dout, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
     __syncthreads();
@@ -1104,18 +1109,24 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
 // the step kernel of a head width, weight format and row count: int8 single-row
 // steps (greedy batch 1) run an instantiation whose slice GEMV keeps one row
 // of accumulators (a smaller kernel; the step is sensitive to its code size)
-static const void *dc_kernel(int dh, bool w4, bool one_row) {
+// (flags: the model's pre-LN / factorised-embedding bits, or -1; the
+// single-row d_h = 64 step of a pre-LN model -- every measured model -- has
+// them compiled in)
+static const void *dc_kernel(int dh, bool w4, bool one_row, int flags = -1) {
     if (w4)
-        return dh == 32 ? (const void *)decode_cluster_kernel<32, true, DC_RMAX>
-                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, true, DC_RMAX>
-                                    : (const void *)decode_cluster_kernel<128, true, DC_RMAX>);
-    if (one_row)
-        return dh == 32 ? (const void *)decode_cluster_kernel<32, false, 1>
-                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, 1>
-                                    : (const void *)decode_cluster_kernel<128, false, 1>);
-    return dh == 32 ? (const void *)decode_cluster_kernel<32, false, DC_RMAX>
-                    : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, DC_RMAX>
-                                : (const void *)decode_cluster_kernel<128, false, DC_RMAX>);
+        return dh == 32 ? (const void *)decode_cluster_kernel<32, true, DC_RMAX, -1>
+                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, true, DC_RMAX, -1>
+                                    : (const void *)decode_cluster_kernel<128, true, DC_RMAX, -1>);
+    if (one_row) {
+        if (dh == 64 && flags == 3) return (const void *)decode_cluster_kernel<64, false, 1, 3>;
+        if (dh == 64 && flags == 1) return (const void *)decode_cluster_kernel<64, false, 1, 1>;
+        return dh == 32 ? (const void *)decode_cluster_kernel<32, false, 1, -1>
+                        : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, 1, -1>
+                                    : (const void *)decode_cluster_kernel<128, false, 1, -1>);
+    }
+    return dh == 32 ? (const void *)decode_cluster_kernel<32, false, DC_RMAX, -1>
+                    : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, DC_RMAX, -1>
+                                : (const void *)decode_cluster_kernel<128, false, DC_RMAX, -1>);
 }
 
 cudaError_t decode_cluster_init() {
@@ -1127,6 +1138,8 @@ cudaError_t decode_cluster_init() {
     };
     for (int dh : {32, 64, 128})
         for (int v = 0; v < 3; v++) setk(dc_kernel(dh, v == 1, v == 2));
+    setk(dc_kernel(64, false, true, 1));
+    setk(dc_kernel(64, false, true, 3));
     // the vocabulary kernel keeps its SMs in the largest shared-memory
     // configuration, so the next step's cluster (about 200 KB per CTA) can
     // become resident beside it as soon as it is allowed to launch
@@ -1141,9 +1154,9 @@ cudaError_t decode_cluster_init() {
 }
 
 // can one cluster of nc CTAs with smem bytes each be resident?
-bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row) {
+bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row, int flags) {
     if (smem > 227 * 1024) return false;
-    const void *k = dc_kernel(dh, w4, one_row);
+    const void *k = dc_kernel(dh, w4, one_row, flags);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -1166,7 +1179,7 @@ bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row) {
 }
 
 cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, bool one_row,
-                                  cudaStream_t st) {
+                                  int flags, cudaStream_t st) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(nc);
     cfg.blockDim = dim3(DC_THREADS);
@@ -1186,7 +1199,7 @@ cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t sme
     cfg.numAttrs = 2;
     if (dh != 32 && dh != 64 && dh != 128) return cudaErrorInvalidValue;
     void *args[] = {(void *)&dP};
-    return cudaLaunchKernelExC(&cfg, dc_kernel(dh, w4, one_row), args);
+    return cudaLaunchKernelExC(&cfg, dc_kernel(dh, w4, one_row, flags), args);
 }
 
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,

@@ -299,10 +299,12 @@ static_assert(sizeof(DcParams) % 16 == 0, "the parameter block is copied in 16-b
 int dc_cluster_size(int d, int F, int E);
 size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
-// one_row: a single-row int8 step (greedy batch 1) takes its own smaller kernel
-bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row);
+// one_row: a single-row int8 step (greedy batch 1) takes its own smaller
+// kernel; flags: the model's pre-LN (bit 0) / factorised-embedding (bit 1)
+// bits, which such a kernel may have compiled in
+bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row, int flags);
 cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, bool one_row,
-                                  cudaStream_t st);
+                                  int flags, cudaStream_t st);
 // reserved_sms: SMs the step kernel that precedes the launch occupies
 cudaError_t launch_vocab_greedy(const int8_t *A, const int8_t *W, const float *s_w, const float *bias, float s_x,
                                 int M, int N, int K, unsigned long long *keys, int *ticket, const GreedyArgs &g,
