@@ -924,6 +924,12 @@ int run_encoder(mnmt_session *s, int B, int S) {
     return MNMT_OK;
 }
 
+// the model bits the single-row step kernels may have compiled in: pre-LN,
+// factorised embedding, R * d above 256
+static int dc_flags(const mnmt_config &c, const mnmt_model *m, int R) {
+    return (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0) | (R * c.d_model > 256 ? 4 : 0);
+}
+
 // one decoder step for all B*k hypotheses (captured into a graph)
 int issue_decode_step(mnmt_session *s) {
     mnmt_model *m = s->m;
@@ -935,8 +941,7 @@ int issue_decode_step(mnmt_session *s) {
     int *t_ptr = s->state + ST_T;
     int *status = s->state + ST_STATUS;
     if (s->use_cluster) {
-        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1,
-                                 (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0), st));
+        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1, dc_flags(c, m, R), st));
         GreedyArgs g;
         g.keys = s->keys;
         g.tok = s->tok;
@@ -1195,8 +1200,7 @@ int setup_cluster_step(mnmt_session *s) {
     P.S = s->Smax;
     size_t smem = dc_layout(P, 227 * 1024);
     P.S = s->S;
-    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1, (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0)))
-        return MNMT_OK;
+    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1, dc_flags(c, m, R))) return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
     s->use_cluster = true;

@@ -135,10 +135,11 @@ MNMT_DEV void dc_copy(void *dst, const void *src, int bytes) {
 // for i, d < 2^16; mg == 0 stands for d == 1), from shifts by powers of two,
 // or from a few compares when the quotient is a row index below DC_RMAX.
 MNMT_DEV int dc_udiv(int i, uint32_t mg) { return mg ? (int)__umulhi((uint32_t)i, mg) : i; }
-MNMT_DEV int dc_row_of(int i, int d, int R) {  // i / d for i < R d, R <= DC_RMAX
+template <int RM = DC_RMAX>
+MNMT_DEV int dc_row_of(int i, int d, int R) {  // i / d for i < R d, R <= RM
     int r = 0;
 #pragma unroll
-    for (int k = 1; k < DC_RMAX; k++) r += (k < R && i >= k * d) ? 1 : 0;
+    for (int k = 1; k < RM; k++) r += (k < R && i >= k * d) ? 1 : 0;
     return r;
 }
 
@@ -245,6 +246,9 @@ MNMT_DEV void dc_row_extremes(const unsigned *mm, int row, int nc, float &hi, fl
     lo = from_ordered_bits(__reduce_min_sync(0xFFFFFFFFu, kl));
 }
 
+// RM: the kernel's row bound; TWO: 0 / 1 when the row width is known to be at
+// most / more than 256 (else -1: decided at run time)
+template <int RM, int TWO>
 __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g, const float *b, float inv,
                                           int8_t *a, int write_back, int *status, const unsigned *mm, int nc,
                                           long long *part_l, int kd, int dodd, unsigned long long zm) {
@@ -252,13 +256,13 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     // a warp takes chunks of cw elements of one row: 32 (one per lane) up to
     // 256 elements, else 64 (two per lane, independent chains), so rows of up
     // to 512 elements still take one round per pass
-    const int n = R * d, two = n > DC_THREADS ? 1 : 0, cs = 5 + two, cw = 32 << two;
+    const int n = R * d, two = TWO >= 0 ? TWO : (n > DC_THREADS ? 1 : 0), cs = 5 + two, cw = 32 << two;
     const int spr = d >> cs;  // partial slots (chunks) per row
     // pass 1: exact sum of x on the grid of max |x|
 #pragma unroll 1
     for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
         float hi, lo;
-        dc_row_extremes(mm, dc_row_of(e0, d, R), nc, hi, lo);
+        dc_row_extremes(mm, dc_row_of<RM>(e0, d, R), nc, hi, lo);
         const float am = fmaxf(fabsf(hi), fabsf(lo));
         if (!(am < 0x1p32f) && lane == 0) set_status(status, MNMT_EOVERFLOW);
         const int sh = 52 - exp_bound(am);
@@ -271,7 +275,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     // pass 2: exact sum of c^2 = fl(x - mean)^2 on the grid of max |c|
 #pragma unroll 1
     for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
-        const int row = dc_row_of(e0, d, R);
+        const int row = dc_row_of<RM>(e0, d, R);
         float hi, lo;
         dc_row_extremes(mm, row, nc, hi, lo);
         const int ea = exp_bound(fmaxf(fabsf(hi), fabsf(lo)));
@@ -295,7 +299,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
     // pass 3: normalise, scale, shift, quantise
 #pragma unroll 1
     for (int e0 = warp * cw; e0 < n; e0 += DC_WARPS * cw) {
-        const int row = dc_row_of(e0, d, R), e = e0 + lane, i = e - row * d;
+        const int row = dc_row_of<RM>(e0, d, R), e = e0 + lane, i = e - row * d;
         const float mu = reinterpret_cast<const float *>(part_l + 128)[2 * row];
         const int eb = reinterpret_cast<const int *>(part_l + 128)[2 * row + 1];
         const float var = dc_rn32_scaled(dc_row_sum(part_l + 64, row, spr), 2 * eb - 52, kd, dodd, zm);
@@ -319,7 +323,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
 // per range; the partials are exact integers, so they combine in any order.
 // self: keys 0..t-1 from the layer's cache (staged or global), key t from the
 // step's own k/v rows; cross: keys j < src_len of the row's sentence.
-template <int DH>
+template <int DH, int RM>
 __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
                                           const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx,
                                           int *att, float *red_f, long long *pz, long long *pn,
@@ -335,7 +339,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
     for (int base = 0; base < items; base += ip) {
         const int it = base + (warp >> lw), part = warp & (wpi - 1);
         const bool live = it < items;
-        const int m = live ? dc_row_of(it, H, R) : 0, h = live ? it - m * H : 0;
+        const int m = live ? dc_row_of<RM>(it, H, R) : 0, h = live ? it - m * H : 0;
         int n;
         const int8_t *kb, *vb;
         if (cross) {
@@ -436,7 +440,7 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                     N += pn[(ii * wpi + w) * DH + e];
                     Z += pz[ii * wpi + w];
                 }
-                const int m2 = dc_row_of(it2, H, R), h2 = it2 - m2 * H;
+                const int m2 = dc_row_of<RM>(it2, H, R), h2 = it2 - m2 * H;
                 ctx[(size_t)m2 * P.d + h2 * DH + e] = q8_quotient(N, Z, rho, dc_rn32_div);
             }
         }
@@ -504,10 +508,11 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     }
     const DcParams &P = *reinterpret_cast<const DcParams *>(smem);
     // FL >= 0: the model's pre-LN (bit 0) and factorised-embedding (bit 1)
-    // flags fixed at compile time, so the other variants' code is not in the
-    // kernel; FL < 0: read from the parameter block
+    // flags and R * d > 256 (bit 2) fixed at compile time, so the other
+    // variants' code is not in the kernel; FL < 0: read from the parameters
     const bool pre_ln = FL < 0 ? P.pre_ln != 0 : (FL & 1) != 0;
     const bool factorised = FL < 0 ? P.factorised != 0 : (FL & 2) != 0;
+    constexpr int TW = FL < 0 ? -1 : ((FL >> 2) & 1);  // row width above 256 (bit 2)
     const uint32_t bars = dc_smem_u32(smem + P.off_bar), xbars = bars + 8u * DC_NB;
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
@@ -668,16 +673,16 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             const int w = kind == K_QKV ? 0 : (kind == K_Q2 ? 2 : 4);
             const float inv_in = kind == K_QKV ? Y.inv_in1 : (kind == K_Q2 ? Y.inv_in2 : Y.inv_in3);
             if (pre_ln) {
-                dc_layernorm(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
+                dc_layernorm<RM, TW>(r_full, R, d, lnl + w * d, lnl + (w + 1) * d, inv_in, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
             } else if (kind == K_QKV) {
                 for (int i = threadIdx.x; i < R * d; i += DC_THREADS) a_full[i] = q8(r_full[i], inv_in);
             } else {
-                dc_layernorm(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, inv_in, a_full, 1, P.status, mm, nc,
+                dc_layernorm<RM, TW>(r_full, R, d, lnl + (w - 2) * d, lnl + (w - 1) * d, inv_in, a_full, 1, P.status, mm, nc,
                              part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
-            dc_attention<DH>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
+            dc_attention<DH, RM>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
                              qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn, smem, src_len_s);
             A = ctx_full;
         } else {  // K_W2
@@ -697,7 +702,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
         int8_t *sti = reinterpret_cast<int8_t *>(stage);
         if (kind == K_EMB && !factorised) {
             for (int i = threadIdx.x; i < R * rows; i += DC_THREADS) {
-                const int m = dc_row_of(i, rows, R), nl = i - m * rows, n = n0 + nl, id = tok_s[m];
+                const int m = dc_row_of<RM>(i, rows, R), nl = i - m * rows, n = n0 + nl, id = tok_s[m];
                 const float v = __fmul_rn(__fmul_rn((float)P.emb_q[(size_t)id * P.E + n], P.emb_s[id]), P.emb_scale);
                 stf[i] = __fadd_rn(v, P.pe[(size_t)t * d + n]);
             }
@@ -835,13 +840,13 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             // post-LN: the FFN's LayerNorm normalises the stream in place
             const bool last = l + 1 == P.n_dec;
             const float inv = last ? P.inv_dout : P.layer[l + 1].inv_in1;
-            dc_layernorm(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
+            dc_layernorm<RM, TW>(r_full, R, d, lnl + 4 * d, lnl + 5 * d, inv, a_full, 1, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
         }
     }
     DC_STAMP(stamp, 100);
     // ---- final LayerNorm + quantisation -> vocabulary input ----
     if (pre_ln)
-        dc_layernorm(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
+        dc_layernorm<RM, TW>(r_full, R, d, lnp + (size_t)6 * P.n_dec * d, lnp + (size_t)(6 * P.n_dec + 1) * d,
                      P.inv_dout, a_full, 0, P.status, mm, nc, part_l, P.ln_kd, P.ln_dodd, P.ln_zm);
     __syncthreads();
     if (c == 0) {
@@ -1109,10 +1114,11 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
 // the step kernel of a head width, weight format and row count: int8 single-row
 // steps (greedy batch 1) run an instantiation whose slice GEMV keeps one row
 // of accumulators (a smaller kernel; the step is sensitive to its code size)
-// (flags: the model's pre-LN / factorised-embedding bits, or -1; the
-// single-row d_h = 64 step of a pre-LN model -- every measured model -- has
-// them compiled in)
+// (flags: the model's pre-LN / factorised-embedding / width > 256 bits, or
+// -1; the single-row d_h = 64 steps of the measured models have them
+// compiled in)
 static const void *dc_kernel(int dh, bool w4, bool one_row, int flags = -1) {
+    if (w4 && one_row && dh == 64 && flags == 3) return (const void *)decode_cluster_kernel<64, true, 1, 3>;
     if (w4)
         return dh == 32 ? (const void *)decode_cluster_kernel<32, true, DC_RMAX, -1>
                         : (dh == 64 ? (const void *)decode_cluster_kernel<64, true, DC_RMAX, -1>
@@ -1120,6 +1126,7 @@ static const void *dc_kernel(int dh, bool w4, bool one_row, int flags = -1) {
     if (one_row) {
         if (dh == 64 && flags == 3) return (const void *)decode_cluster_kernel<64, false, 1, 3>;
         if (dh == 64 && flags == 1) return (const void *)decode_cluster_kernel<64, false, 1, 1>;
+        if (dh == 64 && flags == 5) return (const void *)decode_cluster_kernel<64, false, 1, 5>;
         return dh == 32 ? (const void *)decode_cluster_kernel<32, false, 1, -1>
                         : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, 1, -1>
                                     : (const void *)decode_cluster_kernel<128, false, 1, -1>);
@@ -1138,8 +1145,8 @@ cudaError_t decode_cluster_init() {
     };
     for (int dh : {32, 64, 128})
         for (int v = 0; v < 3; v++) setk(dc_kernel(dh, v == 1, v == 2));
-    setk(dc_kernel(64, false, true, 1));
-    setk(dc_kernel(64, false, true, 3));
+    for (int fl : {1, 3, 5}) setk(dc_kernel(64, false, true, fl));
+    setk(dc_kernel(64, true, true, 3));
     // the vocabulary kernel keeps its SMs in the largest shared-memory
     // configuration, so the next step's cluster (about 200 KB per CTA) can
     // become resident beside it as soon as it is allowed to launch

@@ -300,8 +300,8 @@ int dc_cluster_size(int d, int F, int E);
 size_t dc_layout(DcParams &P, size_t max_smem);
 cudaError_t decode_cluster_init();
 // one_row: a single-row int8 step (greedy batch 1) takes its own smaller
-// kernel; flags: the model's pre-LN (bit 0) / factorised-embedding (bit 1)
-// bits, which such a kernel may have compiled in
+// kernel; flags: the model's pre-LN (bit 0), factorised-embedding (bit 1) and
+// R * d > 256 (bit 2) bits, which such a kernel may have compiled in
 bool decode_cluster_fits(int dh, int nc, size_t smem, bool w4, bool one_row, int flags);
 cudaError_t launch_decode_cluster(const DcParams *dP, int dh, int nc, size_t smem, bool w4, bool one_row,
                                   int flags, cudaStream_t st);
