@@ -590,6 +590,7 @@ struct mnmt_session {
     int dc_S = 0;  // host source of the parameter block's S when it is updated
     int dc_nc = 0;
     size_t dc_smem = 0;
+    int dc_flags = -1;  // the compiled-in model bits of its step kernel (dc_flags)
 };
 
 static int poison(mnmt_session *s, int code) {
@@ -925,9 +926,10 @@ int run_encoder(mnmt_session *s, int B, int S) {
 }
 
 // the model bits the single-row step kernels may have compiled in: pre-LN,
-// factorised embedding, R * d above 256
-static int dc_flags(const mnmt_config &c, const mnmt_model *m, int R) {
-    return (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0) | (R * c.d_model > 256 ? 4 : 0);
+// factorised embedding, R * d above 256, log2 of the attention's warps per
+// item (bits 3-4, from the parameter block's layout)
+static int dc_flags(const mnmt_config &c, const mnmt_model *m, int R, int att_lw) {
+    return (c.pre_ln ? 1 : 0) | (m->factorised ? 2 : 0) | (R * c.d_model > 256 ? 4 : 0) | (att_lw << 3);
 }
 
 // one decoder step for all B*k hypotheses (captured into a graph)
@@ -941,7 +943,7 @@ int issue_decode_step(mnmt_session *s) {
     int *t_ptr = s->state + ST_T;
     int *status = s->state + ST_STATUS;
     if (s->use_cluster) {
-        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1, dc_flags(c, m, R), st));
+        LK(launch_decode_cluster(s->d_dc, dh, s->dc_nc, s->dc_smem, m->wq != 8, R == 1, s->dc_flags, st));
         GreedyArgs g;
         g.keys = s->keys;
         g.tok = s->tok;
@@ -1200,12 +1202,14 @@ int setup_cluster_step(mnmt_session *s) {
     P.S = s->Smax;
     size_t smem = dc_layout(P, 227 * 1024);
     P.S = s->S;
-    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1, dc_flags(c, m, R))) return MNMT_OK;
+    const int flags = dc_flags(c, m, R, P.att_lw);
+    if (!decode_cluster_fits(dh, nc, smem, m->wq != 8, R == 1, flags)) return MNMT_OK;
     CK(cudaMemcpyAsync(s->d_dc, &P, sizeof(P), cudaMemcpyHostToDevice, m->stream));
     CK(cudaStreamSynchronize(m->stream));  // P lives on this stack frame
     s->use_cluster = true;
     s->dc_nc = nc;
     s->dc_smem = smem;
+    s->dc_flags = flags;
     return MNMT_OK;
 }
 

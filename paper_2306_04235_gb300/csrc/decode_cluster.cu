@@ -323,7 +323,9 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
 // per range; the partials are exact integers, so they combine in any order.
 // self: keys 0..t-1 from the layer's cache (staged or global), key t from the
 // step's own k/v rows; cross: keys j < src_len of the row's sentence.
-template <int DH, int RM>
+// LW >= 0: 2^LW warps per item fixed at compile time (LW = 0: each warp holds
+// a whole item -- no cross-warp maximum, and it writes its context itself)
+template <int DH, int RM, int LW>
 __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
                                           const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx,
                                           int *att, float *red_f, long long *pz, long long *pn,
@@ -333,7 +335,8 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
     const int H = P.H, T = P.T, S = P.S, R = P.R;
     const float sigma = cross ? Y.sigma2 : Y.sigma1, rho = cross ? Y.rho2 : Y.rho1;
     const int items = R * H;
-    const int ip = P.att_ip, lw = P.att_lw;  // items per round; 2^lw warps per item
+    const int lw = LW >= 0 ? LW : P.att_lw;                 // 2^lw warps per item
+    const int ip = LW >= 0 ? (DC_WARPS >> LW) : P.att_ip;  // items per round
     const int wpi = 1 << lw;
     constexpr int QC = DH / 16;
     for (int base = 0; base < items; base += ip) {
@@ -385,10 +388,12 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
             }
         }
         mx = warp_max_f(mx);
-        if (lane == 0) red_f[warp] = mx;
-        __syncthreads();
-        mx = -INFINITY;
-        for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp >> lw) * wpi + w]);
+        if (LW != 0) {  // the item's maximum over its warps
+            if (lane == 0) red_f[warp] = mx;
+            __syncthreads();
+            mx = -INFINITY;
+            for (int w = 0; w < wpi; w++) mx = fmaxf(mx, red_f[(warp >> lw) * wpi + w]);
+        }
         int zl = 0;
         if (live)
             for (int j = j0 + lane; j < j1; j += 32) {
@@ -426,6 +431,20 @@ __device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, c
                 hi[u] += __shfl_xor_sync(0xFFFFFFFFu, hi[u], o);
                 lo[u] += __shfl_xor_sync(0xFFFFFFFFu, lo[u], o);
             }
+        if (LW == 0) {
+            // the warp holds its item's whole sums: its lanes write the
+            // context, the KPI lanes of a group sharing its 4 elements
+            if (live) {
+                constexpr int UPL = 4 / KPI;
+#pragma unroll
+                for (int u = 0; u < 4; u++)
+                    if (u / UPL == kg)
+                        ctx[(size_t)m * P.d + h * DH + el + u] =
+                            q8_quotient((long long)hi[u] * 4096 + lo[u], z, rho, dc_rn32_div);
+            }
+            __syncthreads();
+            continue;
+        }
         if (kg == 0)
 #pragma unroll
             for (int u = 0; u < 4; u++) pn[warp * DH + el + u] = (long long)hi[u] * 4096 + lo[u];
@@ -512,7 +531,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
     // variants' code is not in the kernel; FL < 0: read from the parameters
     const bool pre_ln = FL < 0 ? P.pre_ln != 0 : (FL & 1) != 0;
     const bool factorised = FL < 0 ? P.factorised != 0 : (FL & 2) != 0;
-    constexpr int TW = FL < 0 ? -1 : ((FL >> 2) & 1);  // row width above 256 (bit 2)
+    constexpr int TW = FL < 0 ? -1 : ((FL >> 2) & 1);  // row width above 256 (bit 2); bits 3-4: log2 warps per attention item
     const uint32_t bars = dc_smem_u32(smem + P.off_bar), xbars = bars + 8u * DC_NB;
     cg::cluster_group cl = cg::this_cluster();
     const int c = (int)cl.block_rank();
@@ -682,7 +701,7 @@ __global__ void __launch_bounds__(DC_THREADS, 1) decode_cluster_kernel(const DcP
             }
         } else if (kind == K_O || kind == K_O2) {
             const int cross = kind == K_O2;
-            dc_attention<DH, RM>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
+            dc_attention<DH, RM, (FL < 0 ? -1 : ((FL >> 3) & 3))>(P, l, cross, cross ? q2_full : qkv_full, cross ? d : 3 * d, qkv_full + d,
                              qkv_full + 2 * d, 3 * d, t, ctx_full, att, red_f, red_l, pn, smem, src_len_s);
             A = ctx_full;
         } else {  // K_W2
@@ -1114,18 +1133,20 @@ size_t dc_layout(DcParams &P, size_t max_smem) {
 // the step kernel of a head width, weight format and row count: int8 single-row
 // steps (greedy batch 1) run an instantiation whose slice GEMV keeps one row
 // of accumulators (a smaller kernel; the step is sensitive to its code size)
-// (flags: the model's pre-LN / factorised-embedding / width > 256 bits, or
-// -1; the single-row d_h = 64 steps of the measured models have them
-// compiled in)
+// (flags: the model's pre-LN / factorised-embedding / width > 256 bits and
+// the attention's log2 warps per item, or -1; the single-row d_h = 64 steps
+// of the measured models have them compiled in)
 static const void *dc_kernel(int dh, bool w4, bool one_row, int flags = -1) {
-    if (w4 && one_row && dh == 64 && flags == 3) return (const void *)decode_cluster_kernel<64, true, 1, 3>;
+    if (w4 && one_row && dh == 64 && flags == 11) return (const void *)decode_cluster_kernel<64, true, 1, 11>;
     if (w4)
         return dh == 32 ? (const void *)decode_cluster_kernel<32, true, DC_RMAX, -1>
                         : (dh == 64 ? (const void *)decode_cluster_kernel<64, true, DC_RMAX, -1>
                                     : (const void *)decode_cluster_kernel<128, true, DC_RMAX, -1>);
     if (one_row) {
-        if (dh == 64 && flags == 3) return (const void *)decode_cluster_kernel<64, false, 1, 3>;
-        if (dh == 64 && flags == 1) return (const void *)decode_cluster_kernel<64, false, 1, 1>;
+        // small (pre-LN, factorised, 2 warps per head), 10MB (pre-LN, 2 warps
+        // per head), 20MB (pre-LN, d > 256, one warp per head)
+        if (dh == 64 && flags == 11) return (const void *)decode_cluster_kernel<64, false, 1, 11>;
+        if (dh == 64 && flags == 9) return (const void *)decode_cluster_kernel<64, false, 1, 9>;
         if (dh == 64 && flags == 5) return (const void *)decode_cluster_kernel<64, false, 1, 5>;
         return dh == 32 ? (const void *)decode_cluster_kernel<32, false, 1, -1>
                         : (dh == 64 ? (const void *)decode_cluster_kernel<64, false, 1, -1>
@@ -1145,8 +1166,8 @@ cudaError_t decode_cluster_init() {
     };
     for (int dh : {32, 64, 128})
         for (int v = 0; v < 3; v++) setk(dc_kernel(dh, v == 1, v == 2));
-    for (int fl : {1, 3, 5}) setk(dc_kernel(64, false, true, fl));
-    setk(dc_kernel(64, true, true, 3));
+    for (int fl : {5, 9, 11}) setk(dc_kernel(64, false, true, fl));
+    setk(dc_kernel(64, true, true, 11));
     // the vocabulary kernel keeps its SMs in the largest shared-memory
     // configuration, so the next step's cluster (about 200 KB per CTA) can
     // become resident beside it as soon as it is allowed to launch
