@@ -326,7 +326,7 @@ __device__ __noinline__ void dc_layernorm(float *r, int R, int d, const float *g
 // LW >= 0: 2^LW warps per item fixed at compile time (LW = 0: each warp holds
 // a whole item -- no cross-warp maximum, and it writes its context itself)
 template <int DH, int RM, int LW>
-__device__ __noinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
+__device__ __forceinline__ void dc_attention(const DcParams &P, int l, int cross, const int8_t *q, int q_ld,
                                           const int8_t *knew, const int8_t *vnew, int kv_ld, int t, int8_t *ctx,
                                           int *att, float *red_f, long long *pz, long long *pn,
                                           const uint8_t *smem, const int *src_len_s) {
